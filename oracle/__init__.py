@@ -1,0 +1,179 @@
+"""The parity oracle for the GradLev scans (test infrastructure).
+
+A plain fp64 CPU implementation of the sequential online learner
+(GradLev Sec. 3, Eqs. 2-4, and the online MLP of Appendix A), written in C
+(``gradlev_oracle.c``) and loaded through ctypes.  Only ``tests/``,
+``__graft_entry__.smoke()`` and the ``cpu_baseline`` / ``--impl reference``
+legs of ``bench.py`` may import this package.  It shares no code with the CUDA
+library and never calls it.
+
+Every function here takes numpy fp64 arrays (the caller upcasts the exact
+bf16/fp32 tensors fed to the GPU) and returns fp64 arrays.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import sys
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "gradlev_oracle.c")
+_LIB_PATH = os.path.join(_HERE, "_build", "liboracle.so")
+_lib = None
+
+ACT_NONE, ACT_GELU_TANH, ACT_GELU_ERF, ACT_TANH = 0, 1, 2, 3
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (-O2, OpenMP) into oracle/_build/."""
+    os.makedirs(os.path.dirname(_LIB_PATH), exist_ok=True)
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".{os.getpid()}.tmp"
+    # -ffp-contract=off: no fused multiply-add, so every product and sum is a
+    # separately rounded fp64 operation, as written.
+    cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-ffp-contract=off",
+           "-o", tmp, _SRC, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    if _lib is not None:
+        return _lib
+    build()
+    lib = ctypes.CDLL(_LIB_PATH)
+    P = ctypes.c_void_p
+    I = ctypes.c_int
+    lib.oracle_linear_batch.argtypes = [I, I, I, I, P, P, P, P, P, P, P, P, I]
+    lib.oracle_linear_batch.restype = I
+    lib.oracle_mlp_batch.argtypes = [I, I, I, I, I, I, P, P, P, P, P, P, P, P, P,
+                                     P, P, P, P, P, P, I]
+    lib.oracle_mlp_batch.restype = I
+    lib.oracle_act.argtypes = [I, ctypes.c_double]
+    lib.oracle_act.restype = ctypes.c_double
+    lib.oracle_act_deriv.argtypes = [I, ctypes.c_double]
+    lib.oracle_act_deriv.restype = ctypes.c_double
+    lib.oracle_max_threads.argtypes = []
+    lib.oracle_max_threads.restype = I
+    _lib = lib
+    return lib
+
+
+def _f64(a):
+    return np.ascontiguousarray(a, dtype=np.float64)
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _steps(v, T):
+    """A scalar or [T] per-token coefficient as a contiguous fp64 [T] array."""
+    a = np.asarray(v, dtype=np.float64)
+    if a.ndim == 0:
+        a = np.full((T,), float(a))
+    if a.shape != (T,):
+        raise ValueError(f"per-token coefficient must be scalar or [{T}], got {a.shape}")
+    return np.ascontiguousarray(a)
+
+
+def max_threads() -> int:
+    return int(_load().oracle_max_threads())
+
+
+def linear_scan(x, ghat, W0, eta, alpha=None, gout=None, want_y=True, nthreads=0):
+    """Sequential learner for U independent linear maps (Sec. 3, Eqs. 2-4).
+
+    x [U,T,d], ghat [U,T,m], W0 [U,m,d] (or [m,d], shared), eta scalar or [T],
+    alpha None (= 1) or scalar/[T], gout [U,T,m] or None.
+    Returns (y [U,T,m] or None, gin [U,T,d] or None): y_t = W_t x_t and
+    gin_t = W_t^T gout_t, each read before the token-t write.
+    """
+    lib = _load()
+    x = _f64(x)
+    ghat = _f64(ghat)
+    U, T, d = x.shape
+    m = ghat.shape[2]
+    if ghat.shape != (U, T, m):
+        raise ValueError("ghat shape mismatch")
+    W0 = _f64(W0)
+    if W0.shape == (m, d):
+        W0 = np.ascontiguousarray(np.broadcast_to(W0, (U, m, d)))
+    if W0.shape != (U, m, d):
+        raise ValueError("W0 shape mismatch")
+    eta_a = _steps(eta, T)
+    alpha_a = None if alpha is None else _steps(alpha, T)
+    gout_a = None if gout is None else _f64(gout)
+    if gout_a is not None and gout_a.shape != (U, T, m):
+        raise ValueError("gout shape mismatch")
+    y = np.empty((U, T, m)) if want_y else None
+    gin = np.empty((U, T, d)) if gout_a is not None else None
+    rc = lib.oracle_linear_batch(U, T, d, m, _ptr(x), _ptr(ghat), _ptr(W0), _ptr(eta_a),
+                                 _ptr(alpha_a), _ptr(gout_a), _ptr(y), _ptr(gin), int(nthreads))
+    if rc != 0:
+        raise MemoryError("oracle_linear_batch could not allocate scratch")
+    return y, gin
+
+
+def mlp_scan(x, ghz, ghy, W10, W20, eta1, eta2, act=ACT_GELU_TANH, alpha=None, gout=None,
+             nthreads=0):
+    """Sequential online MLP (Appendix A) for U independent sequences.
+
+    Widths: input d, hidden m, output k.  x [U,T,d], ghz [U,T,m], ghy [U,T,k],
+    W10 [m,d], W20 [k,m], gout [U,T,k] or None.
+    Returns a dict with z, h [U,T,m], y [U,T,k] and, when gout is given,
+    gh (= W2_t^T gout), gz (= sigma'(z) * gh) [U,T,m] and gx (= W1_t^T gz) [U,T,d].
+    """
+    lib = _load()
+    x = _f64(x)
+    ghz = _f64(ghz)
+    ghy = _f64(ghy)
+    U, T, d = x.shape
+    m = ghz.shape[2]
+    W10 = _f64(W10)
+    W20 = _f64(W20)
+    k = W20.shape[0]
+    if W10.shape != (m, d) or W20.shape != (k, m) or ghy.shape != (U, T, k):
+        raise ValueError("mlp shape mismatch")
+    e1 = _steps(eta1, T)
+    e2 = _steps(eta2, T)
+    al = None if alpha is None else _steps(alpha, T)
+    go = None if gout is None else _f64(gout)
+    if go is not None and go.shape != (U, T, k):
+        raise ValueError("gout shape mismatch")
+    out = {"z": np.empty((U, T, m)), "h": np.empty((U, T, m)), "y": np.empty((U, T, k))}
+    if go is not None:
+        out.update(gh=np.empty((U, T, m)), gz=np.empty((U, T, m)), gx=np.empty((U, T, d)))
+    rc = lib.oracle_mlp_batch(U, T, d, m, k, int(act), _ptr(x), _ptr(ghz), _ptr(ghy), _ptr(W10),
+                              _ptr(W20), _ptr(e1), _ptr(e2), _ptr(al), _ptr(go),
+                              _ptr(out["z"]), _ptr(out["h"]), _ptr(out["y"]),
+                              _ptr(out.get("gh")), _ptr(out.get("gz")), _ptr(out.get("gx")),
+                              int(nthreads))
+    if rc != 0:
+        raise MemoryError("oracle_mlp_batch could not allocate scratch")
+    return out
+
+
+def act(code, z):
+    """sigma(z) elementwise in fp64 (the oracle's activation)."""
+    lib = _load()
+    f = np.vectorize(lambda v: lib.oracle_act(int(code), float(v)), otypes=[np.float64])
+    return f(np.asarray(z, dtype=np.float64))
+
+
+def act_deriv(code, z):
+    """sigma'(z) elementwise in fp64 (the oracle's derivative)."""
+    lib = _load()
+    f = np.vectorize(lambda v: lib.oracle_act_deriv(int(code), float(v)), otypes=[np.float64])
+    return f(np.asarray(z, dtype=np.float64))
+
+
+if __name__ == "__main__":  # pragma: no cover
+    print(build(force="--force" in sys.argv))

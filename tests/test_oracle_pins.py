@@ -1,0 +1,338 @@
+"""Pins for the fp64 oracle against what the paper and the mathematics fix.
+
+Each test checks the sequential learner in ``oracle/`` against something other
+than itself: the closed form of Eq. 2, the dense scan-read identity of
+Appendix C, plain GEMMs in the degenerate cases, linearity, Theorem 1
+recovery from an independently written serial learner, the Sec. 4.1
+experiment, and finite differences for the activation derivatives.
+"""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rng(seed):
+    return np.random.default_rng(seed)
+
+
+def _rand_problem(seed, U, T, d, m, scale_g=1.0):
+    r = _rng(seed)
+    x = r.standard_normal((U, T, d)) / np.sqrt(d)
+    ghat = r.standard_normal((U, T, m)) * scale_g
+    W0 = r.standard_normal((U, m, d)) / np.sqrt(d)
+    gout = r.standard_normal((U, T, m))
+    return x, ghat, W0, gout
+
+
+# --------------------------------------------------------------------------- Eq. 2
+def _closed_form_delta(t, x, g, eta, alpha):
+    """Delta_t = -sum_{i<t} eta_i (prod_{j=i+1}^{t-1} alpha_j) g_i x_i^T (Eq. 2),
+    with empty sums zero and empty products one."""
+    m, d = g.shape[1], x.shape[1]
+    D = np.zeros((m, d))
+    for i in range(t):
+        prod = 1.0
+        for j in range(i + 1, t):
+            prod *= alpha[j]
+        D -= eta[i] * prod * np.outer(g[i], x[i])
+    return D
+
+
+@pytest.mark.parametrize("T,d,m", [(1, 3, 2), (2, 4, 3), (5, 3, 4), (8, 6, 5)])
+def test_closed_form_eq2_with_gates(T, d, m):
+    x, ghat, W0, gout = _rand_problem(100 + T, 1, T, d, m)
+    r = _rng(7 + T)
+    eta = r.uniform(0.05, 0.5, T)
+    alpha = r.uniform(0.3, 1.0, T)
+    y, gin = oracle.linear_scan(x, ghat, W0, eta, alpha=alpha, gout=gout)
+    for t in range(T):
+        W_t = W0[0] + _closed_form_delta(t, x[0], ghat[0], eta, alpha)
+        np.testing.assert_allclose(y[0, t], W_t @ x[0, t], rtol=0, atol=1e-14)
+        np.testing.assert_allclose(gin[0, t], W_t.T @ gout[0, t], rtol=0, atol=1e-14)
+
+
+def test_first_read_is_slow_weights():
+    """W_hat_0 = W_0 (Delta_0 = 0; read before write): row t=0 is a plain GEMV."""
+    x, ghat, W0, gout = _rand_problem(3, 4, 6, 16, 8)
+    y, gin = oracle.linear_scan(x, ghat, W0, 0.3, gout=gout)
+    for u in range(4):
+        np.testing.assert_allclose(y[u, 0], W0[u] @ x[u, 0], rtol=0, atol=1e-15)
+        np.testing.assert_allclose(gin[u, 0], W0[u].T @ gout[u, 0], rtol=0, atol=1e-15)
+
+
+# ------------------------------------------------------------ App. C scan reads
+def _dense_scan_reads(x, ghat, W0, eta, alpha, gout):
+    """Appendix C: Delta_t a_t = -sum_{i<t} eta_i (prod alpha) ghat_i (x_i^T a_t) and
+    Delta_t^T b_t = -sum_{i<t} eta_i (prod alpha) x_i (ghat_i^T b_t), written as
+    masked products of whole matrices (queries a_t = x_t, b_t = gout_t)."""
+    T = x.shape[0]
+    la = np.concatenate([[0.0], np.cumsum(np.log(alpha))])  # la[k] = sum_{j<k} log alpha_j
+    gamma = np.zeros((T, T))
+    for t in range(T):
+        for i in range(t):
+            # prod_{j=i+1}^{t-1} alpha_j = exp(la[t] - la[i+1])
+            gamma[t, i] = eta[i] * np.exp(la[t] - la[i + 1])
+    Y = x @ W0.T - (gamma * (x @ x.T)) @ ghat
+    G = gout @ W0 - (gamma * (gout @ ghat.T)) @ x
+    return Y, G
+
+
+@pytest.mark.parametrize("T,d,m,gated", [(64, 16, 24, False), (300, 32, 32, False),
+                                         (512, 64, 64, False), (200, 12, 20, True)])
+def test_dense_scan_read_identity(T, d, m, gated):
+    x, ghat, W0, gout = _rand_problem(11 + T, 1, T, d, m)
+    r = _rng(T)
+    eta = r.uniform(0.01, 0.2, T)
+    alpha = r.uniform(0.9, 1.0, T) if gated else np.ones(T)
+    y, gin = oracle.linear_scan(x, ghat, W0, eta, alpha=alpha if gated else None, gout=gout)
+    Yd, Gd = _dense_scan_reads(x[0], ghat[0], W0[0], eta, alpha, gout[0])
+    scale_y = np.abs(Yd).max()
+    scale_g = np.abs(Gd).max()
+    assert np.abs(y[0] - Yd).max() <= 1e-12 * scale_y
+    assert np.abs(gin[0] - Gd).max() <= 1e-12 * scale_g
+
+
+def test_exclusive_not_inclusive():
+    """The read at t excludes the write at t: with one nonzero write at token 3,
+    y_3 is still W0 x_3 while y_4 sees the write."""
+    T, d, m = 6, 5, 4
+    x, ghat, W0, _ = _rand_problem(5, 1, T, d, m)
+    g = np.zeros_like(ghat)
+    g[0, 3] = ghat[0, 3]
+    y, _ = oracle.linear_scan(x, g, W0, 0.7)
+    np.testing.assert_allclose(y[0, 3], W0[0] @ x[0, 3], atol=1e-15)
+    expect4 = (W0[0] - 0.7 * np.outer(g[0, 3], x[0, 3])) @ x[0, 4]
+    np.testing.assert_allclose(y[0, 4], expect4, atol=1e-15)
+    assert np.abs(y[0, 4] - W0[0] @ x[0, 4]).max() > 1e-3
+
+
+# ---------------------------------------------------------- degenerate cases
+@pytest.mark.parametrize("which", ["eta0", "ghat0"])
+def test_degenerate_is_plain_gemm(which):
+    x, ghat, W0, gout = _rand_problem(21, 3, 40, 32, 16)
+    eta = 0.0 if which == "eta0" else 0.4
+    if which == "ghat0":
+        ghat = np.zeros_like(ghat)
+    y, gin = oracle.linear_scan(x, ghat, W0, eta, gout=gout)
+    np.testing.assert_allclose(y, np.einsum("umd,utd->utm", W0, x), rtol=0, atol=1e-13)
+    np.testing.assert_allclose(gin, np.einsum("umd,utm->utd", W0, gout), rtol=0, atol=1e-13)
+
+
+def test_linearity_in_ghat_and_eta():
+    U, T, d, m = 2, 50, 16, 12
+    x, g1, W0, gout = _rand_problem(31, U, T, d, m)
+    g2 = _rng(32).standard_normal((U, T, m))
+    base_y = np.einsum("umd,utd->utm", W0, x)
+    base_g = np.einsum("umd,utm->utd", W0, gout)
+
+    def corr(g, eta):
+        y, gi = oracle.linear_scan(x, g, W0, eta, gout=gout)
+        return y - base_y, gi - base_g
+
+    a, b = 0.7, -1.3
+    y12, g12 = corr(a * g1 + b * g2, 0.2)
+    y1, gg1 = corr(g1, 0.2)
+    y2, gg2 = corr(g2, 0.2)
+    np.testing.assert_allclose(y12, a * y1 + b * y2, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(g12, a * gg1 + b * gg2, rtol=0, atol=1e-12)
+    y3, g3 = corr(g1, 0.6)
+    np.testing.assert_allclose(y3, 3.0 * y1, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(g3, 3.0 * gg1, rtol=0, atol=1e-12)
+
+
+def test_units_are_independent():
+    """Each unit uses only its own W0 and its own history."""
+    x, ghat, W0, gout = _rand_problem(41, 3, 20, 8, 8)
+    y, gin = oracle.linear_scan(x, ghat, W0, 0.3, gout=gout)
+    for u in range(3):
+        yu, gu = oracle.linear_scan(x[u:u + 1], ghat[u:u + 1], W0[u:u + 1], 0.3,
+                                    gout=gout[u:u + 1])
+        np.testing.assert_array_equal(yu[0], y[u])
+        np.testing.assert_array_equal(gu[0], gin[u])
+
+
+# --------------------------------------------------------------- Theorem 1
+def test_theorem1_recovery_linear():
+    """A true serial learner with l_t = 1/2 ||y_t - c_t||^2 (so g_t = y_t - c_t),
+    written independently here, is reproduced when its costates are supplied."""
+    T, d, m = 64, 10, 6
+    r = _rng(77)
+    x = r.standard_normal((T, d))
+    c = r.standard_normal((T, m))
+    W0 = r.standard_normal((m, d)) * 0.3
+    eta = 0.05
+    W = W0.copy()
+    ys, gs, gxs = [], [], []
+    for t in range(T):
+        yt = W @ x[t]
+        gt = yt - c[t]
+        ys.append(yt)
+        gs.append(gt)
+        gxs.append(W.T @ gt)       # dl_t/dx_t at the pre-update weights
+        W = W - eta * np.outer(gt, x[t])
+    g = np.array(gs)
+    y, gin = oracle.linear_scan(x[None], g[None], W0, eta, gout=g[None])
+    assert np.abs(y[0] - np.array(ys)).max() < 1e-13
+    assert np.abs(gin[0] - np.array(gxs)).max() < 1e-13
+    # Consistency residual ghat - g_tilde is zero at the fixed point (Theorem 1).
+    assert np.abs(y[0] - c - g).max() < 1e-13
+
+
+def _read_golden(name):
+    vals = {}
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                k, v = line.split()
+                vals[k] = float(v)
+    return vals
+
+
+def _sigmoid(v):
+    return 1.0 / (1.0 + np.exp(-v))
+
+
+def _e1_serial(seed):
+    """Sec. 4.1 / Appendix B protocol: serial TTT of y = W2 tanh(W1 x), l = 1/2||y-c||^2,
+    both matrices updated after every token with centered decay.  Manual backprop."""
+    r = np.random.default_rng(seed)
+    T, d, m, k = 32, 4, 7, 3
+    W10 = r.standard_normal((m, d)) * (0.5 / np.sqrt(4))
+    W20 = r.standard_normal((k, m)) * (0.5 / np.sqrt(7))
+    va = r.standard_normal(d) * 0.25
+    vm = r.standard_normal(d) * 0.25
+    x = r.standard_normal((T, d))
+    c = r.standard_normal((T, k))
+    alpha = _sigmoid(x @ va + 1.5)
+    mu = _sigmoid(x @ vm - 0.2)
+    eta1, eta2 = mu / 4.0, mu / 7.0
+    W1, W2 = W10.copy(), W20.copy()
+    rec = {k_: [] for k_ in ("y", "gy", "gz", "gW1", "gz_ctrl", "gW1_ctrl")}
+    for t in range(T):
+        z = W1 @ x[t]
+        h = np.tanh(z)
+        y = W2 @ h
+        gy = y - c[t]
+        gz = (1.0 - h * h) * (W2.T @ gy)
+        gz_ctrl = (1.0 - h * h) * (W20.T @ gy)     # "slow transpose only" control
+        rec["y"].append(y)
+        rec["gy"].append(gy)
+        rec["gz"].append(gz)
+        rec["gW1"].append(np.outer(gz, x[t]))
+        rec["gz_ctrl"].append(gz_ctrl)
+        rec["gW1_ctrl"].append(np.outer(gz_ctrl, x[t]))
+        W1n = W10 + alpha[t] * (W1 - W10) - eta1[t] * np.outer(gz, x[t])
+        W2n = W20 + alpha[t] * (W2 - W20) - eta2[t] * np.outer(gy, h)
+        W1, W2 = W1n, W2n
+    rec = {k_: np.array(v) for k_, v in rec.items()}
+    return dict(x=x, W10=W10, W20=W20, alpha=alpha, eta1=eta1, eta2=eta2, **rec)
+
+
+def _e1_parallel(p):
+    """Appendix C explicit causal sums (the parallel construction) for the same MLP,
+    fed the serial learner's costates (Appendix A eqs. scan1-reconstructed-reverse)."""
+    x, alpha = p["x"], p["alpha"]
+    T = x.shape[0]
+    la = np.concatenate([[0.0], np.cumsum(np.log(alpha))])
+    disc = np.zeros((T, T))
+    for t in range(T):
+        for i in range(t):
+            disc[t, i] = np.exp(la[t] - la[i + 1])
+    G1 = disc * p["eta1"][None, :]
+    G2 = disc * p["eta2"][None, :]
+    z = x @ p["W10"].T - (G1 * (x @ x.T)) @ p["gz"]
+    h = np.tanh(z)
+    y = h @ p["W20"].T - (G2 * (h @ h.T)) @ p["gy"]
+    gh = p["gy"] @ p["W20"] - (G2 * (p["gy"] @ p["gy"].T)) @ h
+    gz = (1.0 - h * h) * gh
+    return y, gz
+
+
+@pytest.mark.parametrize("seed", [17, 42, 123])
+def test_e1_mlp_recovery_sec41(seed):
+    gold = _read_golden("e1_recovery.txt")
+    p = _e1_serial(seed)
+    # (a) the dense causal-sum construction recovers serial TTT at rounding level
+    y_par, gz_par = _e1_parallel(p)
+    err_y = np.abs(y_par - p["y"]).max()
+    err_gz = np.abs(gz_par - p["gz"]).max()
+    err_gw = np.abs(gz_par[:, :, None] * p["x"][:, None, :] - p["gW1"]).max()
+    assert max(err_y, err_gz, err_gw) < gold["rounding_bound"]
+    # (b) the oracle, fed the same costates, recovers it too
+    o = oracle.mlp_scan(p["x"][None], p["gz"][None], p["gy"][None], p["W10"], p["W20"],
+                        p["eta1"], p["eta2"], act=oracle.ACT_TANH, alpha=p["alpha"],
+                        gout=p["gy"][None])
+    assert np.abs(o["y"][0] - p["y"]).max() < gold["rounding_bound"]
+    assert np.abs(o["gz"][0] - p["gz"]).max() < gold["rounding_bound"]
+    gw = o["gz"][0][:, :, None] * p["x"][:, None, :]
+    assert np.abs(gw - p["gW1"]).max() < gold["rounding_bound"]
+    # (c) the slow-transpose control changes the reverse by O(0.1-1)
+    ctrl_gz = np.abs(p["gz_ctrl"] - p["gz"]).max()
+    ctrl_gw = np.abs(p["gW1_ctrl"] - p["gW1"]).max()
+    assert gold["control_min"] < max(ctrl_gz, ctrl_gw) < gold["control_max"]
+
+
+def test_e1_control_over_three_seeds():
+    """Maxima over the three seeds, as Fig. 2 reports them."""
+    gold = _read_golden("e1_recovery.txt")
+    cg, cw = 0.0, 0.0
+    for seed in (17, 42, 123):
+        p = _e1_serial(seed)
+        cg = max(cg, np.abs(p["gz_ctrl"] - p["gz"]).max())
+        cw = max(cw, np.abs(p["gW1_ctrl"] - p["gW1"]).max())
+    assert gold["control_min"] < cg < gold["control_max"]
+    assert gold["control_min"] < cw < gold["control_max"]
+
+
+# ------------------------------------------------------------ MLP chaining
+@pytest.mark.parametrize("act", [oracle.ACT_GELU_TANH, oracle.ACT_GELU_ERF, oracle.ACT_TANH])
+def test_mlp_equals_two_chained_linear_maps(act):
+    """Appendix A: layer 1 then sigma then layer 2 forward; costate through layer 2,
+    sigma', then layer 1.  Composing the single-map oracle reproduces the MLP oracle."""
+    U, T, d, m = 2, 40, 6, 10
+    r = _rng(90 + act)
+    x = r.standard_normal((U, T, d))
+    ghz = r.standard_normal((U, T, m)) * 0.2
+    ghy = r.standard_normal((U, T, d)) * 0.2
+    W10 = r.standard_normal((m, d)) / np.sqrt(d)
+    W20 = r.standard_normal((d, m)) / np.sqrt(m)
+    gout = r.standard_normal((U, T, d))
+    o = oracle.mlp_scan(x, ghz, ghy, W10, W20, 0.1, 0.05, act=act, gout=gout)
+    z, _ = oracle.linear_scan(x, ghz, W10, 0.1)
+    h = oracle.act(act, z)
+    y, gh = oracle.linear_scan(h, ghy, W20, 0.05, gout=gout)
+    gz = oracle.act_deriv(act, z) * gh
+    _, gx = oracle.linear_scan(x, ghz, W10, 0.1, gout=gz)
+    for a, b in ((o["z"], z), (o["h"], h), (o["y"], y), (o["gh"], gh), (o["gz"], gz),
+                 (o["gx"], gx)):
+        np.testing.assert_allclose(a, b, rtol=0, atol=1e-12)
+
+
+# ------------------------------------------------------------- activations
+@pytest.mark.parametrize("act", [oracle.ACT_GELU_TANH, oracle.ACT_GELU_ERF, oracle.ACT_TANH])
+def test_activation_derivative_matches_finite_differences(act):
+    z = np.linspace(-6, 6, 241)
+    h = 1e-5
+    fd = (oracle.act(act, z + h) - oracle.act(act, z - h)) / (2 * h)
+    np.testing.assert_allclose(oracle.act_deriv(act, z), fd, rtol=0, atol=1e-8)
+
+
+def test_activation_values():
+    from scipy.special import erf
+    z = np.linspace(-5, 5, 101)
+    # GELU with the exact Gaussian CDF: z * Phi(z) (library erf).
+    np.testing.assert_allclose(oracle.act(oracle.ACT_GELU_ERF, z),
+                               z * 0.5 * (1 + erf(z / np.sqrt(2))), rtol=0, atol=1e-14)
+    np.testing.assert_allclose(oracle.act(oracle.ACT_TANH, z), np.tanh(z), rtol=0, atol=1e-15)
+    # The tanh approximation stays within 1e-3 of the exact GELU (a known bound).
+    assert np.abs(oracle.act(oracle.ACT_GELU_TANH, z) - oracle.act(oracle.ACT_GELU_ERF, z)).max() < 1e-3
+    assert oracle.act(oracle.ACT_GELU_TANH, np.array([0.0]))[0] == 0.0
+    assert abs(oracle.act_deriv(oracle.ACT_GELU_TANH, np.array([0.0]))[0] - 0.5) < 1e-15
+    np.testing.assert_allclose(oracle.act(oracle.ACT_NONE, z), z)
+    np.testing.assert_allclose(oracle.act_deriv(oracle.ACT_NONE, z), np.ones_like(z))
