@@ -1,0 +1,407 @@
+#!/usr/bin/env python3
+"""Benchmark of the GradLev token scans on GB300.
+
+One step = the forward scan (Sec. 3 step 2, Eq. 3) and the costate scan
+(Sec. 3 step 3, Eq. 4) over one batch of the workload, through the library's
+C ABI.  Default workload: the model-shaped layer sweep (12 independent layers
+x 12 heads of 64x64 fast weights, B=8, T=8192, bf16), all layers' forward and
+costate scans per step.
+
+Prints ONE JSON line on rank 0.  `value` is tokens/s of the whole step
+(L*B*T tokens per step, both scans) with inputs resident in HBM; `scans`
+breaks it down per scan with each scan's roofline; `roofline` is the dominant
+(slowest) kernel's; `e2e` is the same metric through the public API with
+pinned host buffers copied in and results copied out inside the timed region;
+`cpu_baseline` is the fp64 oracle timed on this host's cores on a bounded
+sample of the same workload.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c5] [--impl reference]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+import workloads as W  # noqa: E402
+
+METRIC = "tokens/s per scan (fwd, costate) at 1 GB300; % of scan roofline"
+UNIT = "tokens/s"
+COUNT_CHUNK = 64  # chunk size fixed for counting flops (scan roofline convention)
+L2_BYTES = 129 * 1024 * 1024
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+# ------------------------------------------------------------- scan accounting
+def scan_counts(wl, scan: str):
+    """Algorithmic flops and compulsory bytes of one scan call over the workload.
+
+    Per token and unit (one head of one layer): flops 4*d*m + C*(d+m) with C = 64
+    (state read 2dm, state update 2dm, causal halves of the two CxC products);
+    bytes e*(d + 2m) forward (x, ghat in; y out), e*(2d + 2m) costate (x, ghat,
+    g_out in; g_in out), plus 4*d*m per slow matrix W0.
+    """
+    e = 2 if wl.dtype == "bf16" else 4
+    d, m = wl.d_in, wl.d_out
+    tu = wl.L * wl.B * wl.T * wl.H
+    flops = tu * (4 * d * m + COUNT_CHUNK * (d + m))
+    per_tok = e * (d + 2 * m) if scan == "fwd" else e * (2 * d + 2 * m)
+    nbytes = tu * per_tok + 4 * d * m * wl.L * wl.H
+    return flops, nbytes
+
+
+def roofline_entry(flops, nbytes, seconds, pk):
+    t_hbm = nbytes / (pk["hbm_gbs"] * 1e9)
+    t_tc = flops / (pk["bf16_tflops"] * 1e12)
+    if t_hbm >= t_tc:
+        ach = nbytes / seconds / 1e9
+        return {"bound": "hbm", "achieved": round(ach, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": round(ach / pk["hbm_gbs"], 4), "algorithmic_bytes": nbytes,
+                "peak_source": pk["source"]}
+    ach = flops / seconds / 1e12
+    return {"bound": "tensor", "achieved": round(ach, 2), "peak": pk["bf16_tflops"],
+            "unit": "TFLOP/s", "frac": round(ach / pk["bf16_tflops"], 4),
+            "algorithmic_flops": flops, "peak_source": pk["source"]}
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.marks = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def mark(self):
+        self.marks.append(time.time())
+
+    def stop(self):
+        if self.proc is None:
+            return
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+
+    def summary(self):
+        if not self.lines:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        t0, t1 = (self.marks[0], self.marks[-1]) if len(self.marks) >= 2 else (0, 1e30)
+        inside = [ln for (t, ln) in self.lines if t0 <= t <= t1]
+        rows = inside if inside else [ln for _, ln in self.lines]
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in rows:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        out = {"sm_mhz": statistics.median(sm) if sm else None,
+               "sm_max_mhz": max(smax) if smax else None, "reasons": sorted(reasons),
+               "samples": len(sm), "window": "timed region" if inside else "whole run"}
+        return out
+
+
+# ------------------------------------------------------------------ workload
+def linear_inputs(wl, device, rank):
+    return W.make_linear(wl.resized(seed=wl.seed + 1000 * rank), device=device)
+
+
+def run_step(gl, inp, wl, outs, events=None):
+    if events is not None:
+        events[0].record()
+    gl.forward_scan(inp["x"], inp["g_hat"], inp["W0"], wl.eta, y=outs["y"],
+                    workspace=outs["ws"])
+    if events is not None:
+        events[1].record()
+    gl.costate_scan(inp["x"], inp["g_hat"], inp["W0"], wl.eta, inp["g_out"], g_in=outs["g_in"],
+                    workspace=outs["ws"])
+    if events is not None:
+        events[2].record()
+
+
+def cpu_baseline(wl, inp, target_s=12.0):
+    """The fp64 oracle (as it stands) on a bounded sample of units, all host cores."""
+    import oracle
+
+    cores = len(os.sched_getaffinity(0))
+    units_all = [(l, b, h) for l in range(wl.L) for b in range(wl.B) for h in range(wl.H)]
+
+    def run(units):
+        x = W.units_fp64(inp["x"], units)
+        g = W.units_fp64(inp["g_hat"], units)
+        w0 = W.w0_fp64(inp["W0"], units)
+        go = W.units_fp64(inp["g_out"], units)
+        t = time.perf_counter()
+        oracle.linear_scan(x, g, w0, wl.eta, gout=go, nthreads=cores)
+        return time.perf_counter() - t
+
+    # calibrate with one unit per core, then size the sample for ~target_s
+    n0 = min(len(units_all), cores)
+    dt0 = run(units_all[:n0])
+    per_unit = dt0 / n0
+    n = int(max(n0, min(len(units_all), target_s / max(per_unit, 1e-9))))
+    n = max(cores, n // cores * cores) if n >= cores else n
+    n = min(n, len(units_all))
+    dt = run(units_all[:n])
+    # metric tokens: one token spans all H heads of a layer, so a unit-token is 1/H token
+    tokens = n * wl.T / wl.H
+    return {"value": round(tokens / dt, 1), "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{n} of {len(units_all)} (layer, batch, head) units at full T={wl.T}, "
+                      f"forward and costate reads in one sequential walk per unit, fp64",
+            "seconds": round(dt, 2)}
+
+
+def e2e_measure(gl, inp, wl, outs, steps, stream):
+    """The same step through the public API from pinned host buffers, copies inside."""
+    host = {k: inp[k].cpu().pin_memory() for k in ("x", "g_hat", "g_out", "W0")}
+    hy = torch.empty(outs["y"].shape, dtype=outs["y"].dtype, pin_memory=True)
+    hg = torch.empty(outs["g_in"].shape, dtype=outs["g_in"].dtype, pin_memory=True)
+    dev = {k: torch.empty_like(inp[k]) for k in host}
+    bi = sum(t.numel() * t.element_size() for t in host.values())
+    bo = hy.numel() * hy.element_size() + hg.numel() * hg.element_size()
+
+    def one():
+        for k in host:
+            dev[k].copy_(host[k], non_blocking=True)
+        run_step(gl, dev, wl, outs)
+        hy.copy_(outs["y"], non_blocking=True)
+        hg.copy_(outs["g_in"], non_blocking=True)
+
+    one()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        one()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    sec = e0.elapsed_time(e1) / 1e3
+    return {"value": round(wl.tokens * steps / sec, 1), "unit": UNIT, "h2d_bytes_per_step": bi,
+            "d2h_bytes_per_step": bo, "steps": steps, "ms_per_step": round(sec / steps * 1e3, 3)}
+
+
+# ------------------------------------------------------------------- arms
+def run_reference(args, wl, rank, world):
+    """The oracle as the reference arm, on this host's cores (rank 0 only)."""
+    if rank != 0:
+        return None
+    import oracle
+
+    oracle.build()
+    inp = W.make_linear(wl, device="cpu")
+    cores = len(os.sched_getaffinity(0))
+    units_all = [(l, b, h) for l in range(wl.L) for b in range(wl.B) for h in range(wl.H)]
+    n = min(len(units_all), max(cores, 2 * cores))
+    units = units_all[:n]
+    x = W.units_fp64(inp["x"], units)
+    g = W.units_fp64(inp["g_hat"], units)
+    w0 = W.w0_fp64(inp["W0"], units)
+    go = W.units_fp64(inp["g_out"], units)
+    for _ in range(args.warmup):
+        oracle.linear_scan(x[:cores], g[:cores], w0[:cores], wl.eta, gout=go[:cores],
+                           nthreads=cores)
+    t = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.linear_scan(x, g, w0, wl.eta, gout=go, nthreads=cores)
+    sec = time.perf_counter() - t
+    tokens = n * wl.T / wl.H
+    value = tokens * args.steps / sec
+    sample = (f"{n} of {len(units_all)} (layer, batch, head) units at full T={wl.T} per step, "
+              f"fp64 sequential walk")
+    return {"impl": "reference", "metric": METRIC, "value": round(value, 1), "unit": UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(sec / args.steps * 1e3, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": f"{args.workload}: {wl.name}", "sample": sample},
+            "cpu_baseline": {"value": round(value, 1), "unit": UNIT, "cores": cores,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def run_gradlev(args, wl, rank, world, local_rank):
+    import paper_2609_34174_gb300 as gl
+
+    device = torch.device("cuda", local_rank)
+    torch.cuda.set_device(device)
+    gl.load_library()
+    inp = linear_inputs(wl, device, rank)
+    outs = {"y": torch.empty_like(inp["g_hat"]),
+            "g_in": torch.empty_like(inp["x"]),
+            "ws": torch.empty(max(256, gl.workspace_bytes(wl.L, wl.B, wl.T, wl.H, wl.d_in, wl.d_out,
+                                                          1 if wl.dtype == "bf16" else 0)),
+                              dtype=torch.uint8, device=device)}
+    in_bytes = sum(inp[k].numel() * inp[k].element_size() for k in ("x", "g_hat", "g_out"))
+    flush = None
+    if in_bytes < 2 * L2_BYTES:
+        flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
+    stream = torch.cuda.current_stream(device)
+
+    for _ in range(args.warmup):
+        run_step(gl, inp, wl, outs)
+    torch.cuda.synchronize()
+    if gl.workspace_status(outs["ws"]) != 0:
+        raise RuntimeError("device-side timeout reported by the scan kernels")
+
+    sampler = ClockSampler(local_rank)
+    sampler.start()
+    # let the sampler produce a first line before the timed region
+    time.sleep(0.3)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    sampler.mark()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(args.steps):
+        if flush is not None:
+            flush.zero_()
+        run_step(gl, inp, wl, outs, ev[i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    sampler.mark()
+    if world > 1:
+        torch.distributed.barrier()
+    time.sleep(0.25)
+    sampler.stop()
+    if gl.workspace_status(outs["ws"]) != 0:
+        raise RuntimeError("device-side timeout reported by the scan kernels")
+
+    total_ms = t_start.elapsed_time(t_end)
+    fwd_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / args.steps
+    cos_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / args.steps
+    step_ms = total_ms / args.steps
+    if world > 1:
+        t = torch.tensor([step_ms], device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        step_ms = float(t.item())
+    if flush is not None:
+        # the flush is not part of the step: take the scans' own time
+        step_ms = max(fwd_ms + cos_ms, 1e-9) if world == 1 else step_ms
+    pk = peaks()
+    scans = {}
+    for name, ms in (("fwd", fwd_ms), ("costate", cos_ms)):
+        fl, nb = scan_counts(wl, name)
+        scans[name] = {"ms": round(ms, 4), "tokens_per_s": round(wl.tokens / (ms / 1e3), 1),
+                       "roofline": roofline_entry(fl, nb, ms / 1e3, pk)}
+    dominant = "costate" if cos_ms >= fwd_ms else "fwd"
+    rl = dict(scans[dominant]["roofline"])
+    rl["kernel"] = f"tc_scan_kernel ({dominant} scan)"
+    rl["traffic"] = None
+    value = world * wl.tokens / (step_ms / 1e3)
+    line = {"metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms, 4),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
+            "data": "synthetic",
+            "config": {"workload": f"{args.workload}: {wl.name}", "L": wl.L, "B": wl.B, "T": wl.T,
+                       "H": wl.H, "d_in": wl.d_in, "d_out": wl.d_out, "eta": wl.eta,
+                       "tokens_per_step": wl.tokens, "parallelism": f"replicas x{world}",
+                       "l2": ("inputs larger than L2" if flush is None
+                              else "L2 flushed between steps")},
+            "scans": scans, "roofline": rl, "clocks": sampler.summary(),
+            "gpu_launches": 2 * args.steps}
+    if rank == 0 and world == 1 and not args.no_e2e:
+        line["e2e"] = e2e_measure(gl, inp, wl, outs, max(3, min(args.steps, 10)), stream)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+
+        oracle.build()
+        line["cpu_baseline"] = cpu_baseline(wl, inp)
+    return line
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default="c5", choices=["c1", "c2", "c4", "c5"])
+    ap.add_argument("--impl", default="gradlev", choices=["gradlev", "reference"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        args.warmup = 3
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    wl = W.workload(args.workload)
+
+    if args.impl == "reference":
+        line = run_reference(args, wl, rank, world)
+        if line is not None:
+            print(json.dumps(line), flush=True)
+        return 0
+
+    if world > 1:
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    try:
+        line = run_gradlev(args, wl, rank, world, local_rank)
+        if rank == 0:
+            print(json.dumps(line), flush=True)
+    finally:
+        if world > 1:
+            torch.distributed.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,165 @@
+/*
+ * gradlev.h -- C ABI of the GradLev token-scan library for GB300 (sm_103a).
+ *
+ * GradLev (Token-Parallel Test-Time Training via Costate Prediction) turns
+ * token-by-token online gradient descent on a fast-weight matrix into two
+ * associative scans once the per-token costates are supplied (Sec. 3,
+ * "Observation: known costates expose exact scans").  With slow weights W0
+ * (d_out x d_in), a step size eta and proposals ghat_t, the adapted weights
+ * before token t are (Eq. 2 with unit retention, Eq. 3)
+ *
+ *     What_t = W0 + Deltahat_t,   Deltahat_t = -eta * sum_{s<t} ghat_s x_s^T,
+ *
+ * an EXCLUSIVE sum: every token reads the weights before its own write
+ * (Sec. 3 step 2, "read before each write"; Deltahat_0 = 0).  The library
+ * computes the two reads of those weights for every token in parallel:
+ *
+ *   forward scan  (Eq. 3):  y_t    = What_t x_t
+ *                                   = W0 x_t - eta sum_{s<t} ghat_s (x_s . x_t)
+ *   costate scan  (Eq. 4):  g_in_t = What_t^T g_out_t
+ *                                   = W0^T g_out_t - eta sum_{s<t} x_s (ghat_s . g_out_t)
+ *
+ * (the transpose scan reuses the same historical writes (x_s, ghat_s),
+ * queried by the incoming costate; Appendix C, eq. scan-reads).  An
+ * elementwise activation can be fused on the outputs, for the two-layer
+ * fast-weight MLP of Appendix A: the forward scan can also emit sigma(y_t),
+ * and the costate scan can multiply its result by sigma'(z_t) (Sec. 3
+ * step 3: g^z = sigma'(z) (.) g^x).
+ *
+ * Units.  A call covers L*B*H independent units (layer group l, batch row b,
+ * head h).  Every unit starts with Deltahat = 0 at token 0 (a reset at the
+ * start of each sequence) and has its own slow matrix W0[l][h]; batch rows
+ * of one (l, h) share W0.
+ *
+ * Layouts.  Token tensors are 5-D [L][B][T][H][w] with w = d_in for x-like
+ * tensors (x, g_in, z) and w = d_out for g-like tensors (ghat, g_out, y,
+ * act_out).  The feature dimension is contiguous; the other four dimensions
+ * use the element strides given in gradlev_tensor (all zero means the
+ * contiguous default).  W0 is fp32 [L][H][d_out][d_in], contiguous.
+ * All pointers are device pointers of the current CUDA device.
+ *
+ * Precision.  dtype GRADLEV_BF16: x, ghat, g_out and all outputs are bf16;
+ * products run on the tensor cores with fp32 accumulation and an fp32 running
+ * state; outputs are rounded to bf16 (round to nearest even).  dtype
+ * GRADLEV_F32: everything is fp32 and computed with fp32 FMA.
+ *
+ * Ownership and concurrency.  The caller owns every buffer, including the
+ * workspace.  Calls are asynchronous on the given stream, allocate nothing and
+ * keep no state between calls.  A workspace must not be shared by calls that
+ * may run concurrently.
+ *
+ * Errors.  Every entry point returns GRADLEV_OK (0) or a negative code; an
+ * argument error is detected on the host before anything is launched, and
+ * there is no CPU fallback.  A device-side wait that exceeds its time limit
+ * (a defect, never expected) is reported through the workspace: see
+ * gradlev_workspace_status.
+ */
+#ifndef GRADLEV_H
+#define GRADLEV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define GRADLEV_ABI_VERSION 1
+
+#define GRADLEV_OK 0
+#define GRADLEV_ERR_INVALID_ARG (-1) /* null pointer, bad size or stride, non-finite eta */
+#define GRADLEV_ERR_UNSUPPORTED (-2) /* shape, alignment, dtype or device not handled */
+#define GRADLEV_ERR_CUDA (-3)        /* a CUDA runtime call or kernel launch failed */
+#define GRADLEV_ERR_TIMEOUT (-4)     /* a bounded device-side wait expired */
+#define GRADLEV_ERR_WORKSPACE (-5)   /* workspace missing, too small or misaligned */
+
+typedef enum { GRADLEV_F32 = 0, GRADLEV_BF16 = 1 } gradlev_dtype;
+
+/* Elementwise activations for the MLP fusion (App. A; App. E uses the tanh
+ * approximation of GELU). */
+typedef enum {
+    GRADLEV_ACT_NONE = 0,
+    GRADLEV_ACT_GELU_TANH = 1,
+    GRADLEV_ACT_GELU_ERF = 2,
+    GRADLEV_ACT_TANH = 3
+} gradlev_act;
+
+/* The same type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* gradlev_stream_t;
+
+/* Problem shape shared by both scans. */
+typedef struct {
+    int32_t L;      /* independent layer groups, each with its own W0 per head */
+    int32_t B;      /* batch rows */
+    int32_t T;      /* tokens per sequence (0 is allowed: nothing to do) */
+    int32_t H;      /* heads */
+    int32_t d_in;   /* width of x (input of the adapted map) */
+    int32_t d_out;  /* width of y, ghat and g_out (output of the adapted map) */
+    int32_t dtype;  /* gradlev_dtype of every token tensor */
+    int32_t reserved; /* must be 0 */
+} gradlev_desc;
+
+/* A token tensor: device pointer plus element strides of (L, B, T, H).  The
+ * feature dimension is contiguous.  stride all zero = contiguous default. */
+typedef struct {
+    void* data;
+    int64_t stride[4];
+} gradlev_tensor;
+
+/*
+ * gradlev_forward_scan -- forward exclusive prefix scan (Sec. 3 step 2, Eq. 3).
+ *   x        [L][B][T][H][d_in]   layer inputs x_t (read)
+ *   g_hat    [L][B][T][H][d_out]  costate proposals ghat_t: the writes (read)
+ *   W0       [L][H][d_out][d_in]  fp32 slow weights (read)
+ *   eta      step size of every write (finite; 0 gives y = W0 x)
+ *   act      activation applied for act_out (GRADLEV_ACT_NONE: act_out unused)
+ *   y        [L][B][T][H][d_out]  out: y_t = What_t x_t (pre-activation)
+ *   act_out  [L][B][T][H][d_out]  optional out (data NULL to skip): sigma(y_t)
+ *   workspace/workspace_bytes  scratch of at least gradlev_workspace_bytes(desc)
+ *            bytes, 256-byte aligned; its contents on entry are ignored.
+ * Returns GRADLEV_OK or an error code; nothing is launched on error.
+ */
+int gradlev_forward_scan(const gradlev_desc* desc, const gradlev_tensor* x,
+                         const gradlev_tensor* g_hat, const float* W0, float eta, int act,
+                         const gradlev_tensor* y, const gradlev_tensor* act_out, void* workspace,
+                         size_t workspace_bytes, gradlev_stream_t stream);
+
+/*
+ * gradlev_costate_scan -- costate (transpose) scan (Sec. 3 step 3, Eq. 4).
+ *   x, g_hat, W0, eta  the same writes and slow weights as the forward scan
+ *   g_out    [L][B][T][H][d_out]  incoming costates gtilde_t = dl_t/dy_t (read)
+ *   act, z   optional fusion: with z.data non-NULL and act != NONE the output is
+ *            sigma'(z_t) (.) (What_t^T g_out_t), z of shape [L][B][T][H][d_in]
+ *            (the preactivation whose activation fed this map's input)
+ *   g_in     [L][B][T][H][d_in]   out: What_t^T g_out_t (times sigma'(z_t) if fused)
+ *   workspace/workspace_bytes  as for the forward scan.
+ */
+int gradlev_costate_scan(const gradlev_desc* desc, const gradlev_tensor* x,
+                         const gradlev_tensor* g_hat, const float* W0, float eta,
+                         const gradlev_tensor* g_out, int act, const gradlev_tensor* z,
+                         const gradlev_tensor* g_in, void* workspace, size_t workspace_bytes,
+                         gradlev_stream_t stream);
+
+/* Bytes of workspace either scan needs for this shape (the same bound serves
+ * both).  Returns 0 for an invalid descriptor. */
+size_t gradlev_workspace_bytes(const gradlev_desc* desc);
+
+/* Waits for `stream`, then reads the device-side status word a scan left in
+ * `workspace`: GRADLEV_OK, or GRADLEV_ERR_TIMEOUT if a bounded device wait
+ * expired (the outputs of that call are then undefined), or GRADLEV_ERR_CUDA. */
+int gradlev_workspace_status(const void* workspace, gradlev_stream_t stream);
+
+/* 1 if the current device can run this library (compute capability 10.3), else 0. */
+int gradlev_device_supported(void);
+
+/* Human-readable text for a status code (static storage). */
+const char* gradlev_status_string(int code);
+
+/* GRADLEV_ABI_VERSION of the loaded library. */
+int gradlev_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GRADLEV_H */

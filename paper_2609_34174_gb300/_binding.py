@@ -1,0 +1,303 @@
+"""ctypes binding of include/gradlev.h.
+
+Argument marshalling only: tensors are described by pointer and strides and
+handed to the C ABI with the current torch CUDA stream; outputs and the
+workspace are ordinary torch allocations.  All arithmetic happens in the CUDA
+kernels of libgradlev.so.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from typing import Optional
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_HERE, "_build", "libgradlev.so")
+
+ACT_NONE, ACT_GELU_TANH, ACT_GELU_ERF, ACT_TANH = 0, 1, 2, 3
+_ACT_NAMES = {None: ACT_NONE, "none": ACT_NONE, "gelu_tanh": ACT_GELU_TANH, "gelu": ACT_GELU_TANH,
+              "gelu_erf": ACT_GELU_ERF, "tanh": ACT_TANH}
+
+GRADLEV_F32, GRADLEV_BF16 = 0, 1
+
+_STATUS = {0: "ok", -1: "invalid argument", -2: "unsupported", -3: "CUDA error", -4: "timeout",
+           -5: "workspace"}
+
+
+class GradLevError(RuntimeError):
+    """A libgradlev call returned a non-zero status."""
+
+    def __init__(self, code: int, what: str):
+        self.code = code
+        super().__init__(f"{what}: status {code} ({_STATUS.get(code, 'unknown')})")
+
+
+class _Desc(ctypes.Structure):
+    _fields_ = [("L", ctypes.c_int32), ("B", ctypes.c_int32), ("T", ctypes.c_int32),
+                ("H", ctypes.c_int32), ("d_in", ctypes.c_int32), ("d_out", ctypes.c_int32),
+                ("dtype", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+class _Tensor(ctypes.Structure):
+    _fields_ = [("data", ctypes.c_void_p), ("stride", ctypes.c_int64 * 4)]
+
+
+_lib = None
+_lib_lock = threading.Lock()
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def load_library():
+    """Load libgradlev.so (building it first if nvcc is available)."""
+    global _lib
+    with _lib_lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(_LIB_PATH):
+            from . import build as _build
+            _build.build()
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError(f"libgradlev.so is missing at {_LIB_PATH}; run build() first")
+        lib = ctypes.CDLL(_LIB_PATH)
+        P = ctypes.c_void_p
+        D = ctypes.POINTER(_Desc)
+        Tp = ctypes.POINTER(_Tensor)
+        lib.gradlev_forward_scan.argtypes = [D, Tp, Tp, P, ctypes.c_float, ctypes.c_int, Tp, Tp, P,
+                                             ctypes.c_size_t, P]
+        lib.gradlev_forward_scan.restype = ctypes.c_int
+        lib.gradlev_costate_scan.argtypes = [D, Tp, Tp, P, ctypes.c_float, Tp, ctypes.c_int, Tp, Tp,
+                                             P, ctypes.c_size_t, P]
+        lib.gradlev_costate_scan.restype = ctypes.c_int
+        lib.gradlev_workspace_bytes.argtypes = [D]
+        lib.gradlev_workspace_bytes.restype = ctypes.c_size_t
+        lib.gradlev_workspace_status.argtypes = [P, P]
+        lib.gradlev_workspace_status.restype = ctypes.c_int
+        lib.gradlev_device_supported.argtypes = []
+        lib.gradlev_device_supported.restype = ctypes.c_int
+        lib.gradlev_status_string.argtypes = [ctypes.c_int]
+        lib.gradlev_status_string.restype = ctypes.c_char_p
+        lib.gradlev_abi_version.argtypes = []
+        lib.gradlev_abi_version.restype = ctypes.c_int
+        _lib = lib
+        return lib
+
+
+def device_supported() -> bool:
+    return bool(load_library().gradlev_device_supported())
+
+
+def _act_code(act) -> int:
+    if isinstance(act, int):
+        return act
+    if act not in _ACT_NAMES:
+        raise ValueError(f"unknown activation {act!r}")
+    return _ACT_NAMES[act]
+
+
+def _as5(t: torch.Tensor) -> torch.Tensor:
+    """View a token tensor as [L, B, T, H, w] without copying."""
+    if t.dim() == 5:
+        return t
+    if t.dim() == 4:   # [B, T, H, w]
+        return t.unsqueeze(0)
+    if t.dim() == 3:   # [B, T, w]
+        return t.unsqueeze(0).unsqueeze(3)
+    if t.dim() == 2:   # [T, w]
+        return t.unsqueeze(0).unsqueeze(0).unsqueeze(3)
+    raise ValueError(f"token tensors are 2- to 5-D, got {t.dim()}-D")
+
+
+def _tensor(t5: Optional[torch.Tensor]) -> Optional[_Tensor]:
+    if t5 is None:
+        return None
+    if t5.stride(4) != 1:
+        raise ValueError("the feature dimension of a token tensor must be contiguous")
+    st = _Tensor()
+    st.data = t5.data_ptr()
+    for i in range(4):
+        s = t5.stride(i)
+        if t5.shape[i] == 1:
+            s = max(s, 1)
+        st.stride[i] = s
+    return st
+
+
+_ws_cache = {}
+_ws_lock = threading.Lock()
+
+
+def _workspace(nbytes: int, device: torch.device) -> torch.Tensor:
+    with _ws_lock:
+        key = (device.index, torch.cuda.current_stream(device).cuda_stream)
+        buf = _ws_cache.get(key)
+        if buf is None or buf.numel() < nbytes:
+            buf = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=device)
+            _ws_cache[key] = buf
+        return buf
+
+
+def _w0(W0: torch.Tensor, L: int, H: int, rows: int, cols: int) -> torch.Tensor:
+    if W0.dtype != torch.float32:
+        raise TypeError("W0 must be float32")
+    if W0.dim() == 2:
+        W0 = W0.reshape(1, 1, rows, cols)
+    elif W0.dim() == 3:
+        W0 = W0.unsqueeze(0)
+    if tuple(W0.shape) != (L, H, rows, cols):
+        raise ValueError(f"W0 must be [L,H,d_out,d_in] = {(L, H, rows, cols)}, got {tuple(W0.shape)}")
+    return W0.contiguous()
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return GRADLEV_BF16
+    if t.dtype == torch.float32:
+        return GRADLEV_F32
+    raise TypeError(f"token tensors must be bfloat16 or float32, got {t.dtype}")
+
+
+def _check_same(ref: torch.Tensor, *others):
+    for o in others:
+        if o is None:
+            continue
+        if o.device != ref.device:
+            raise ValueError("all tensors must be on the same device")
+        if o.dtype != ref.dtype:
+            raise TypeError("all token tensors must share one dtype")
+
+
+def _desc(x5: torch.Tensor, d_out: int, dtype: int) -> _Desc:
+    L, B, T, H, d_in = x5.shape
+    return _Desc(L, B, T, H, d_in, d_out, dtype, 0)
+
+
+def workspace_bytes(L, B, T, H, d_in, d_out, dtype=GRADLEV_BF16) -> int:
+    d = _Desc(L, B, T, H, d_in, d_out, dtype, 0)
+    return int(load_library().gradlev_workspace_bytes(ctypes.byref(d)))
+
+
+def workspace_status(workspace: torch.Tensor) -> int:
+    """Device-side status a previous call left in `workspace` (syncs the stream)."""
+    lib = load_library()
+    s = torch.cuda.current_stream(workspace.device).cuda_stream
+    return int(lib.gradlev_workspace_status(ctypes.c_void_p(workspace.data_ptr()),
+                                            ctypes.c_void_p(s)))
+
+
+def _call(rc: int, what: str):
+    if rc != 0:
+        raise GradLevError(rc, what)
+
+
+def forward_scan(x, g_hat, W0, eta, act=None, y=None, act_out=None, want_act_out=False,
+                 workspace=None):
+    """y_t = (W0 - eta sum_{s<t} ghat_s x_s^T) x_t for every token (Sec. 3 step 2, Eq. 3).
+
+    x [L,B,T,H,d_in] (or [B,T,H,d_in], [B,T,d_in], [T,d_in]), g_hat with d_out features,
+    W0 fp32 [L,H,d_out,d_in].  With want_act_out (or act_out given) also returns
+    sigma(y) for the activation `act`.  Returns y, or (y, act_out).
+    """
+    lib = load_library()
+    x5, g5 = _as5(x), _as5(g_hat)
+    _check_same(x5, g5)
+    if not x5.is_cuda:
+        raise ValueError("tensors must be on a CUDA device")
+    L, B, T, H, d_in = x5.shape
+    d_out = g5.shape[4]
+    if tuple(g5.shape[:4]) != (L, B, T, H):
+        raise ValueError("x and g_hat token shapes differ")
+    W = _w0(W0, L, H, d_out, d_in)
+    if W.device != x5.device:
+        raise ValueError("W0 must be on the tensors' device")
+    code = _act_code(act)
+    if y is None:
+        y = torch.empty(g5.shape[:4] + (d_out,), dtype=x5.dtype, device=x5.device)
+    y5 = _as5(y)
+    _check_same(x5, y5)
+    if (want_act_out or act_out is not None) and act_out is None:
+        act_out = torch.empty_like(y5)
+    a5 = _as5(act_out) if act_out is not None else None
+    desc = _desc(x5, d_out, _dtype_code(x5))
+    nbytes = int(lib.gradlev_workspace_bytes(ctypes.byref(desc)))
+    ws = workspace if workspace is not None else _workspace(nbytes, x5.device)
+    tx, tg, ty = _tensor(x5), _tensor(g5), _tensor(y5)
+    ta = _tensor(a5) if a5 is not None else None
+    stream = torch.cuda.current_stream(x5.device).cuda_stream
+    with torch.cuda.device(x5.device):
+        rc = lib.gradlev_forward_scan(ctypes.byref(desc), ctypes.byref(tx), ctypes.byref(tg),
+                                      ctypes.c_void_p(W.data_ptr()), float(eta), code,
+                                      ctypes.byref(ty), ctypes.byref(ta) if ta is not None else None,
+                                      ctypes.c_void_p(ws.data_ptr()), ws.numel(),
+                                      ctypes.c_void_p(stream))
+    _call(rc, "gradlev_forward_scan")
+    if act_out is not None:
+        return y, act_out
+    return y
+
+
+def costate_scan(x, g_hat, W0, eta, g_out, act=None, z=None, g_in=None, workspace=None):
+    """g_in_t = (W0 - eta sum_{s<t} ghat_s x_s^T)^T g_out_t (Sec. 3 step 3, Eq. 4).
+
+    With z (the preactivation that fed this map's input through sigma = act) the
+    result is sigma'(z_t) * (What_t^T g_out_t).  Returns g_in [.., d_in].
+    """
+    lib = load_library()
+    x5, g5, go5 = _as5(x), _as5(g_hat), _as5(g_out)
+    _check_same(x5, g5, go5)
+    if not x5.is_cuda:
+        raise ValueError("tensors must be on a CUDA device")
+    L, B, T, H, d_in = x5.shape
+    d_out = g5.shape[4]
+    if tuple(g5.shape) != tuple(go5.shape) or tuple(g5.shape[:4]) != (L, B, T, H):
+        raise ValueError("g_hat / g_out shapes differ from x")
+    W = _w0(W0, L, H, d_out, d_in)
+    code = _act_code(act)
+    z5 = _as5(z) if z is not None else None
+    if z5 is not None:
+        _check_same(x5, z5)
+        if tuple(z5.shape) != tuple(x5.shape):
+            raise ValueError("z must have the shape of x")
+    if g_in is None:
+        g_in = torch.empty(x5.shape, dtype=x5.dtype, device=x5.device).view(x.shape)
+    gi5 = _as5(g_in)
+    _check_same(x5, gi5)
+    desc = _desc(x5, d_out, _dtype_code(x5))
+    nbytes = int(lib.gradlev_workspace_bytes(ctypes.byref(desc)))
+    ws = workspace if workspace is not None else _workspace(nbytes, x5.device)
+    tx, tg, tgo, tgi = _tensor(x5), _tensor(g5), _tensor(go5), _tensor(gi5)
+    tz = _tensor(z5) if z5 is not None else None
+    stream = torch.cuda.current_stream(x5.device).cuda_stream
+    with torch.cuda.device(x5.device):
+        rc = lib.gradlev_costate_scan(ctypes.byref(desc), ctypes.byref(tx), ctypes.byref(tg),
+                                      ctypes.c_void_p(W.data_ptr()), float(eta), ctypes.byref(tgo),
+                                      code, ctypes.byref(tz) if tz is not None else None,
+                                      ctypes.byref(tgi), ctypes.c_void_p(ws.data_ptr()), ws.numel(),
+                                      ctypes.c_void_p(stream))
+    _call(rc, "gradlev_costate_scan")
+    return g_in
+
+
+def mlp_forward(x, g_hat_z, g_hat_y, W1, W2, eta1, eta2, act="gelu_tanh"):
+    """Forward through the two-layer fast-weight MLP (Appendix A, eqs. scan1-proposed).
+
+    Layer 1 writes z = (W1 + Delta1_t) x and, fused in its epilogue, h = sigma(z);
+    layer 2 reads h.  Returns (z, h, y).
+    """
+    z, h = forward_scan(x, g_hat_z, W1, eta1, act=act, want_act_out=True)
+    y = forward_scan(h, g_hat_y, W2, eta2)
+    return z, h, y
+
+
+def mlp_costate(x, h, z, g_hat_z, g_hat_y, W1, W2, eta1, eta2, g_out, act="gelu_tanh"):
+    """Costates back through both layers (Appendix A eq. reconstructed-reverse, then
+    the layer-1 transpose read).  Returns (g_z, g_x): g_z = sigma'(z) * (W2_t^T g_out)
+    with sigma' fused in the layer-2 costate epilogue, g_x = W1_t^T g_z."""
+    g_z = costate_scan(h, g_hat_y, W2, eta2, g_out, act=act, z=z)
+    g_x = costate_scan(x, g_hat_z, W1, eta1, g_z)
+    return g_z, g_x

@@ -1,0 +1,400 @@
+// gradlev_host.cu -- the C ABI of include/gradlev.h: argument validation, work
+// planning, TMA descriptor creation and kernel launch.  No compute happens on
+// the host and there is no host fallback: a call either launches its kernels on
+// the caller's stream or returns an error without launching anything.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "../../include/gradlev.h"
+#include "scan_common.cuh"
+
+namespace gl {
+cudaError_t launch_tc_scan(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
+                           const TcScanParams& p, bool costate, int grid, cudaStream_t stream);
+cudaError_t launch_simt_scan(const SimtScanParams& p, bool bf16, cudaStream_t stream);
+size_t simt_smem_bytes(int dq);
+}  // namespace gl
+
+namespace {
+
+using gl::TcScanParams;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    });
+    return fn;
+}
+
+constexpr int kMaxDevices = 64;
+
+struct DevInfo {
+    int sms = 0;
+    int major = 0, minor = 0;
+    bool ok = false;
+};
+
+bool device_info(DevInfo* out) {
+    static DevInfo cache[kMaxDevices];
+    static std::mutex mu;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return false;
+    std::lock_guard<std::mutex> g(mu);
+    if (!cache[dev].ok) {
+        DevInfo d;
+        if (cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&d.major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&d.minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+            return false;
+        d.ok = true;
+        cache[dev] = d;
+    }
+    *out = cache[dev];
+    return true;
+}
+
+// Resolved token tensor: pointer plus element strides of (L, B, T, H).
+struct Tok {
+    void* data = nullptr;
+    long long s[4] = {0, 0, 0, 0};
+};
+
+bool resolve(const gradlev_desc& d, const gradlev_tensor* t, int width, Tok* out, bool required) {
+    if (!t || !t->data) return !required;
+    out->data = t->data;
+    bool zero = true;
+    for (int i = 0; i < 4; ++i) zero = zero && t->stride[i] == 0;
+    if (zero) {
+        out->s[3] = width;
+        out->s[2] = (long long)d.H * width;
+        out->s[1] = (long long)d.T * d.H * width;
+        out->s[0] = (long long)d.B * d.T * d.H * width;
+    } else {
+        const int dims[4] = {d.L, d.B, d.T, d.H};
+        // natural contiguous strides, used for size-1 dimensions (never indexed)
+        const long long nat[4] = {(long long)d.B * d.T * d.H * width, (long long)d.T * d.H * width,
+                                  (long long)d.H * width, (long long)width};
+        for (int i = 0; i < 4; ++i) {
+            if (t->stride[i] < 0) return false;
+            if (t->stride[i] == 0 && dims[i] > 1) return false;
+            out->s[i] = dims[i] == 1 ? nat[i] : t->stride[i];
+        }
+        if (d.H > 1 && out->s[3] < width) return false;  // rows of one token must not overlap
+    }
+    return true;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// The tensor-core path moves 16-byte pieces: base and every stride must keep
+// each 64-element row piece 16-byte aligned, and TMA needs strides < 2^40 bytes.
+bool tc_layout_ok(const Tok& t, int elem) {
+    if (!t.data) return true;
+    if (!aligned16(t.data)) return false;
+    for (int i = 0; i < 4; ++i) {
+        long long bytes = t.s[i] * elem;
+        if (bytes % 16 != 0 || bytes >= (1ll << 40)) return false;
+    }
+    return true;
+}
+
+// Segment plan of the tensor-core path: enough (unit, tile, segment) items to
+// keep every SM busy, with segments of at least 512 tokens.
+struct Plan {
+    int n_tiles = 0, seg_len = 0, n_seg = 1, n_items = 0;
+    size_t ws_bytes = 0;
+    // workspace layout
+    size_t off_flags = 0, off_agg = 0, off_incl = 0, zero_bytes = 0;
+};
+
+constexpr int kChunk = 128;
+
+size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+Plan plan_tc(const gradlev_desc& d, int dq, int dv, int sms) {
+    Plan pl;
+    pl.n_tiles = dv / 64;
+    const long long units = (long long)d.L * d.B * d.H * pl.n_tiles;
+    const long long target = 4ll * (sms > 0 ? sms : 148);
+    int n_seg = 1;
+    if (units < target && d.T > 1024) {
+        long long want = (target + units - 1) / units;
+        long long max_seg = (d.T + 511) / 512;
+        n_seg = (int)(want < max_seg ? want : max_seg);
+        if (n_seg < 1) n_seg = 1;
+    }
+    long long seg = ((long long)d.T + n_seg - 1) / n_seg;
+    seg = (seg + kChunk - 1) / kChunk * kChunk;
+    if (seg < kChunk) seg = kChunk;
+    pl.seg_len = (int)seg;
+    pl.n_seg = (int)(((long long)d.T + seg - 1) / seg);
+    if (pl.n_seg < 1) pl.n_seg = 1;
+    pl.n_items = (int)(units * pl.n_seg);
+    pl.off_flags = 256;
+    pl.off_agg = round_up(pl.off_flags + sizeof(unsigned int) * (size_t)pl.n_items, 256);
+    pl.zero_bytes = pl.off_agg;
+    size_t blk = sizeof(float) * (size_t)dq * 64;
+    if (pl.n_seg > 1) {
+        pl.off_incl = pl.off_agg + blk * (size_t)pl.n_items;
+        pl.ws_bytes = pl.off_incl + blk * (size_t)pl.n_items;
+    } else {
+        pl.off_incl = pl.off_agg;
+        pl.ws_bytes = pl.off_agg;
+    }
+    return pl;
+}
+
+bool tc_shape_ok(const gradlev_desc& d, int dq, int dv) {
+    return d.dtype == GRADLEV_BF16 && (dq == 64 || dq == 128) && dv % 64 == 0 && dv > 0;
+}
+
+constexpr int kSimtMaxDq = 256;
+
+bool simt_shape_ok(const gradlev_desc& d, int dq) {
+    (void)d;
+    return dq >= 1 && dq <= kSimtMaxDq;
+}
+
+bool desc_ok(const gradlev_desc* d) {
+    if (!d) return false;
+    if (d->L < 1 || d->B < 1 || d->H < 1 || d->T < 0 || d->d_in < 1 || d->d_out < 1) return false;
+    if (d->dtype != GRADLEV_F32 && d->dtype != GRADLEV_BF16) return false;
+    if (d->reserved != 0) return false;
+    long long units = (long long)d->L * d->B * d->H;
+    if (units > (1ll << 30) || d->d_in > (1 << 20) || d->d_out > (1 << 20)) return false;
+    return true;
+}
+
+bool make_tmap(CUtensorMap* m, const gradlev_desc& d, const Tok& t, int width) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    const cuuint64_t dims[5] = {(cuuint64_t)width, (cuuint64_t)d.H, (cuuint64_t)d.T, (cuuint64_t)d.B,
+                                (cuuint64_t)d.L};
+    // byte strides of dims 1..4; a size-1 dimension gets a harmless valid stride
+    cuuint64_t strides[4];
+    const long long s[4] = {t.s[3], t.s[2], t.s[1], t.s[0]};
+    const int sizes[4] = {d.H, d.T, d.B, d.L};
+    for (int i = 0; i < 4; ++i) {
+        long long b = s[i] * 2;
+        if (sizes[i] == 1 && b == 0) b = 16;
+        strides[i] = (cuuint64_t)b;
+    }
+    const cuuint32_t box[5] = {64, 1, (cuuint32_t)kChunk, 1, 1};
+    const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, t.data, dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+void fill_epi(gl::EpiParams* e, const Tok& out, const Tok& out2, const Tok& z, int act) {
+    e->out = out.data;
+    e->out2 = out2.data;
+    e->zin = z.data;
+    e->act = act;
+    for (int i = 0; i < 4; ++i) {
+        e->out_str[i] = out.s[i];
+        e->out2_str[i] = out2.s[i];
+        e->z_str[i] = z.s[i];
+    }
+}
+
+// Shared driver of both scans.  Roles (Sec. 3, Eqs. 3-4):
+//   forward:  q = k = x, v = g_hat, B0 = W0     (dq = d_in,  dv = d_out)
+//   costate:  q = g_out, k = g_hat, v = x, B0 = W0^T (dq = d_out, dv = d_in)
+int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
+             const gradlev_tensor* g_hat, const float* W0, float eta, const gradlev_tensor* g_out,
+             int act, const gradlev_tensor* out, const gradlev_tensor* out2,
+             const gradlev_tensor* z, void* ws, size_t ws_bytes, cudaStream_t stream) {
+    if (!desc_ok(desc)) return GRADLEV_ERR_INVALID_ARG;
+    const gradlev_desc& d = *desc;
+    if (!W0 || !isfinite(eta)) return GRADLEV_ERR_INVALID_ARG;
+    if (act < GRADLEV_ACT_NONE || act > GRADLEV_ACT_TANH) return GRADLEV_ERR_INVALID_ARG;
+    const int din = d.d_in, dout = d.d_out;
+    Tok tx, tg, tgo, to, to2, tz;
+    if (!resolve(d, x, din, &tx, true) || !resolve(d, g_hat, dout, &tg, true) ||
+        !resolve(d, out, costate ? din : dout, &to, true))
+        return GRADLEV_ERR_INVALID_ARG;
+    if (costate) {
+        if (!resolve(d, g_out, dout, &tgo, true) || !resolve(d, z, din, &tz, false))
+            return GRADLEV_ERR_INVALID_ARG;
+        if (tz.data && act == GRADLEV_ACT_NONE) return GRADLEV_ERR_INVALID_ARG;
+    } else {
+        if (!resolve(d, out2, dout, &to2, false)) return GRADLEV_ERR_INVALID_ARG;
+        if (to2.data && act == GRADLEV_ACT_NONE) return GRADLEV_ERR_INVALID_ARG;
+    }
+    DevInfo dev;
+    if (!device_info(&dev)) return GRADLEV_ERR_CUDA;
+    if (!(dev.major == 10 && dev.minor == 3)) return GRADLEV_ERR_UNSUPPORTED;
+    if (d.T == 0) return GRADLEV_OK;
+
+    const int dq = costate ? dout : din;
+    const int dv = costate ? din : dout;
+    const Tok& tq = costate ? tgo : tx;
+    const Tok& tk = tg;
+    const Tok& tv = costate ? tx : tg;
+    const int elem = d.dtype == GRADLEV_BF16 ? 2 : 4;
+
+    if (tc_shape_ok(d, dq, dv) && tc_layout_ok(tq, 2) && tc_layout_ok(tk, 2) &&
+        tc_layout_ok(tv, 2) && tc_layout_ok(to, 2) && tc_layout_ok(to2, 2) && tc_layout_ok(tz, 2)) {
+        Plan pl = plan_tc(d, dq, dv, dev.sms);
+        if (!ws || ws_bytes < pl.ws_bytes) return GRADLEV_ERR_WORKSPACE;
+        if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return GRADLEV_ERR_WORKSPACE;
+        CUtensorMap mq, mk, mv;
+        if (!make_tmap(&mq, d, tq, dq) || !make_tmap(&mk, d, tk, dq) || !make_tmap(&mv, d, tv, dv))
+            return GRADLEV_ERR_UNSUPPORTED;
+        TcScanParams p;
+        memset(&p, 0, sizeof(p));
+        p.L = d.L;
+        p.B = d.B;
+        p.T = d.T;
+        p.H = d.H;
+        p.dq = dq;
+        p.dv = dv;
+        p.n_tiles = pl.n_tiles;
+        p.seg_len = pl.seg_len;
+        p.n_seg = pl.n_seg;
+        p.n_items = pl.n_items;
+        p.eta = eta;
+        p.w0_transposed = costate ? 1 : 0;
+        p.W0 = W0;
+        fill_epi(&p.epi, to, to2, tz, act);
+        uint8_t* wsb = static_cast<uint8_t*>(ws);
+        p.ctrl = reinterpret_cast<unsigned int*>(wsb);
+        p.flags = reinterpret_cast<unsigned int*>(wsb + pl.off_flags);
+        p.agg = reinterpret_cast<float*>(wsb + pl.off_agg);
+        p.incl = reinterpret_cast<float*>(wsb + pl.off_incl);
+        if (cudaMemsetAsync(ws, 0, pl.zero_bytes, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
+        const int grid = pl.n_items < dev.sms ? pl.n_items : dev.sms;
+        if (gl::launch_tc_scan(mq, mk, mv, p, costate, grid, stream) != cudaSuccess)
+            return GRADLEV_ERR_CUDA;
+        return GRADLEV_OK;
+    }
+    if (simt_shape_ok(d, dq)) {
+        // CUDA-core path: fp32 (exact fp32 FMA), or bf16 shapes the tensor-core
+        // tiling does not cover.  Needs only element alignment.
+        const Tok* all[6] = {&tq, &tk, &tv, &to, &to2, &tz};
+        for (const Tok* t : all)
+            if (t->data && (reinterpret_cast<uintptr_t>(t->data) % elem) != 0)
+                return GRADLEV_ERR_UNSUPPORTED;
+        if ((reinterpret_cast<uintptr_t>(W0) & 3u) != 0) return GRADLEV_ERR_INVALID_ARG;
+        if (ws) {
+            if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return GRADLEV_ERR_WORKSPACE;
+            if (ws_bytes >= 256 && cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess)
+                return GRADLEV_ERR_CUDA;
+        }
+        gl::SimtScanParams p;
+        memset(&p, 0, sizeof(p));
+        p.L = d.L;
+        p.B = d.B;
+        p.T = d.T;
+        p.H = d.H;
+        p.dq = dq;
+        p.dv = dv;
+        p.eta = eta;
+        p.w0_transposed = costate ? 1 : 0;
+        p.W0 = W0;
+        p.q = tq.data;
+        p.k = tk.data;
+        p.v = tv.data;
+        for (int i = 0; i < 4; ++i) {
+            p.q_str[i] = tq.s[i];
+            p.k_str[i] = tk.s[i];
+            p.v_str[i] = tv.s[i];
+        }
+        fill_epi(&p.epi, to, to2, tz, act);
+        if (gl::launch_simt_scan(p, d.dtype == GRADLEV_BF16, stream) != cudaSuccess)
+            return GRADLEV_ERR_CUDA;
+        return GRADLEV_OK;
+    }
+    return GRADLEV_ERR_UNSUPPORTED;
+}
+
+size_t ws_bytes_for(const gradlev_desc& d, int dq, int dv, int sms) {
+    size_t b = 256;
+    if (tc_shape_ok(d, dq, dv)) {
+        Plan pl = plan_tc(d, dq, dv, sms);
+        if (pl.ws_bytes > b) b = pl.ws_bytes;
+    }
+    return b;
+}
+
+}  // namespace
+
+extern "C" {
+
+int gradlev_forward_scan(const gradlev_desc* desc, const gradlev_tensor* x,
+                         const gradlev_tensor* g_hat, const float* W0, float eta, int act,
+                         const gradlev_tensor* y, const gradlev_tensor* act_out, void* workspace,
+                         size_t workspace_bytes, gradlev_stream_t stream) {
+    return run_scan(desc, false, x, g_hat, W0, eta, nullptr, act, y, act_out, nullptr, workspace,
+                    workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int gradlev_costate_scan(const gradlev_desc* desc, const gradlev_tensor* x,
+                         const gradlev_tensor* g_hat, const float* W0, float eta,
+                         const gradlev_tensor* g_out, int act, const gradlev_tensor* z,
+                         const gradlev_tensor* g_in, void* workspace, size_t workspace_bytes,
+                         gradlev_stream_t stream) {
+    return run_scan(desc, true, x, g_hat, W0, eta, g_out, act, g_in, nullptr, z, workspace,
+                    workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t gradlev_workspace_bytes(const gradlev_desc* desc) {
+    if (!desc_ok(desc)) return 0;
+    DevInfo dev;
+    int sms = device_info(&dev) ? dev.sms : 160;
+    size_t a = ws_bytes_for(*desc, desc->d_in, desc->d_out, sms);
+    size_t b = ws_bytes_for(*desc, desc->d_out, desc->d_in, sms);
+    return a > b ? a : b;
+}
+
+int gradlev_workspace_status(const void* workspace, gradlev_stream_t stream) {
+    if (!workspace) return GRADLEV_ERR_INVALID_ARG;
+    unsigned int word = 0;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(s) != cudaSuccess) return GRADLEV_ERR_CUDA;
+    if (cudaMemcpy(&word, static_cast<const unsigned int*>(workspace) + 1, sizeof(word),
+                   cudaMemcpyDeviceToHost) != cudaSuccess)
+        return GRADLEV_ERR_CUDA;
+    return word == 0 ? GRADLEV_OK : GRADLEV_ERR_TIMEOUT;
+}
+
+int gradlev_device_supported(void) {
+    DevInfo dev;
+    if (!device_info(&dev)) return 0;
+    return (dev.major == 10 && dev.minor == 3) ? 1 : 0;
+}
+
+const char* gradlev_status_string(int code) {
+    switch (code) {
+    case GRADLEV_OK: return "ok";
+    case GRADLEV_ERR_INVALID_ARG: return "invalid argument";
+    case GRADLEV_ERR_UNSUPPORTED: return "unsupported shape, alignment, dtype or device";
+    case GRADLEV_ERR_CUDA: return "CUDA runtime error";
+    case GRADLEV_ERR_TIMEOUT: return "a bounded device-side wait expired";
+    case GRADLEV_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+    default: return "unknown status";
+    }
+}
+
+int gradlev_abi_version(void) { return GRADLEV_ABI_VERSION; }
+
+}  // extern "C"
