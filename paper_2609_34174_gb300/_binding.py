@@ -217,11 +217,13 @@ def forward_scan(x, g_hat, W0, eta, act=None, y=None, act_out=None, want_act_out
         raise ValueError("W0 must be on the tensors' device")
     code = _act_code(act)
     if y is None:
-        y = torch.empty(g5.shape[:4] + (d_out,), dtype=x5.dtype, device=x5.device)
+        y = torch.empty(tuple(x.shape[:-1]) + (d_out,), dtype=x5.dtype, device=x5.device)
     y5 = _as5(y)
     _check_same(x5, y5)
-    if (want_act_out or act_out is not None) and act_out is None:
-        act_out = torch.empty_like(y5)
+    if tuple(y5.shape) != (L, B, T, H, d_out):
+        raise ValueError("y has the wrong shape")
+    if want_act_out and act_out is None:
+        act_out = torch.empty_like(y)
     a5 = _as5(act_out) if act_out is not None else None
     desc = _desc(x5, d_out, _dtype_code(x5))
     nbytes = int(lib.gradlev_workspace_bytes(ctypes.byref(desc)))

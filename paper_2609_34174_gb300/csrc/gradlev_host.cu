@@ -248,7 +248,7 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
     const int dq = costate ? dout : din;
     const int dv = costate ? din : dout;
     const Tok& tq = costate ? tgo : tx;
-    const Tok& tk = tg;
+    const Tok& tk = costate ? tg : tx;
     const Tok& tv = costate ? tx : tg;
     const int elem = d.dtype == GRADLEV_BF16 ? 2 : 4;
 
