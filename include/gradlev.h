@@ -140,6 +140,35 @@ int gradlev_costate_scan(const gradlev_desc* desc, const gradlev_tensor* x,
                          const gradlev_tensor* g_in, void* workspace, size_t workspace_bytes,
                          gradlev_stream_t stream);
 
+/* Size of the fixed device array used by gradlev_forward_scan_noalloc (4 MiB). */
+#define GRADLEV_NOALLOC_SCRATCH_BYTES (4u << 20)
+
+/*
+ * gradlev_forward_scan_noalloc -- the forward scan without a caller workspace.
+ * (The paper has no counterpart: this is a calling convention of this library.)
+ *
+ * For callers that cannot allocate device memory when they call and have no
+ * workspace to pass, such as a plugin behind a fixed "inputs, outputs, stream"
+ * signature, or a serving loop whose device memory is budgeted once at start-up.
+ * Arguments and results are those of gradlev_forward_scan; the scratch
+ * the kernel needs lives in a GRADLEV_NOALLOC_SCRATCH_BYTES array inside the
+ * library, which every GPU that loads the library holds until the process
+ * exits.  The call allocates nothing.
+ *   - A shape whose scratch would exceed that array returns
+ *     GRADLEV_ERR_WORKSPACE (gradlev_workspace_bytes(desc) tells the need);
+ *     nothing is launched.  Long sequences over few units need the most.
+ *   - The first call on each device looks up the array's device address with
+ *     that device current; make that first call before any stream capture.
+ *   - All calls on a device share the array and it keeps the last call's
+ *     contents; each call clears what must start at zero on its own stream.
+ *     Calls that may overlap on the GPU race on it and must not be issued.
+ *   - gradlev_workspace_status does not apply (there is no caller workspace).
+ */
+int gradlev_forward_scan_noalloc(const gradlev_desc* desc, const gradlev_tensor* x,
+                                 const gradlev_tensor* g_hat, const float* W0, float eta, int act,
+                                 const gradlev_tensor* y, const gradlev_tensor* act_out,
+                                 gradlev_stream_t stream);
+
 /* Bytes of workspace either scan needs for this shape (the same bound serves
  * both).  Returns 0 for an invalid descriptor. */
 size_t gradlev_workspace_bytes(const gradlev_desc* desc);
