@@ -373,6 +373,9 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--workload", default="c5", choices=["c1", "c2", "c4", "c5"])
     ap.add_argument("--impl", default="gradlev", choices=["gradlev", "reference"])
+    ap.add_argument("--resize", default="",
+                    help="comma-separated K=V overrides of the workload's sizes (e.g. L=2), "
+                         "for small profiling captures; the headline uses the full workload")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args(argv)
@@ -383,6 +386,13 @@ def main(argv=None):
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     wl = W.workload(args.workload)
+    if args.resize:
+        kw = {}
+        for item in args.resize.split(","):
+            k, v = item.split("=")
+            kw[k.strip()] = int(v) if v.strip().lstrip("-").isdigit() else float(v)
+        wl = wl.resized(**kw)
+        args.workload = f"{args.workload}[{args.resize}]"
 
     if args.impl == "reference":
         line = run_reference(args, wl, rank, world)

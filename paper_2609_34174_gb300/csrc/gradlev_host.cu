@@ -15,7 +15,8 @@
 
 namespace gl {
 cudaError_t launch_tc_scan(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
-                           const TcScanParams& p, bool costate, int grid, cudaStream_t stream);
+                           const CUtensorMap& o, const TcScanParams& p, bool costate, int grid,
+                           cudaStream_t stream);
 cudaError_t launch_simt_scan(const SimtScanParams& p, bool bf16, cudaStream_t stream);
 size_t simt_smem_bytes(int dq);
 }  // namespace gl
@@ -200,7 +201,7 @@ bool make_tmap(CUtensorMap* m, const gradlev_desc& d, const Tok& t, int width) {
     const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
     CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, t.data, dims, strides, box, estr,
                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
 
@@ -257,8 +258,9 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
         Plan pl = plan_tc(d, dq, dv, dev.sms);
         if (!ws || ws_bytes < pl.ws_bytes) return GRADLEV_ERR_WORKSPACE;
         if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return GRADLEV_ERR_WORKSPACE;
-        CUtensorMap mq, mk, mv;
-        if (!make_tmap(&mq, d, tq, dq) || !make_tmap(&mk, d, tk, dq) || !make_tmap(&mv, d, tv, dv))
+        CUtensorMap mq, mk, mv, mo;
+        if (!make_tmap(&mq, d, tq, dq) || !make_tmap(&mk, d, tk, dq) || !make_tmap(&mv, d, tv, dv) ||
+            !make_tmap(&mo, d, to, dv))
             return GRADLEV_ERR_UNSUPPORTED;
         TcScanParams p;
         memset(&p, 0, sizeof(p));
@@ -283,7 +285,7 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
         p.incl = reinterpret_cast<float*>(wsb + pl.off_incl);
         if (cudaMemsetAsync(ws, 0, pl.zero_bytes, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
         const int grid = pl.n_items < dev.sms ? pl.n_items : dev.sms;
-        if (gl::launch_tc_scan(mq, mk, mv, p, costate, grid, stream) != cudaSuccess)
+        if (gl::launch_tc_scan(mq, mk, mv, mo, p, costate, grid, stream) != cudaSuccess)
             return GRADLEV_ERR_CUDA;
         return GRADLEV_OK;
     }

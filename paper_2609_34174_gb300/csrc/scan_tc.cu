@@ -17,15 +17,27 @@
 // (phase 1), publishes it, looks back, publishes its inclusive prefix, then runs
 // the full chunk loop (phase 2, which re-reads the same tiles, mostly from L2).
 //
-// Warp roles (14 warps, one CTA per SM):
+// Warp roles (15 warps, one CTA per SM):
 //   warp 0      TMA producer: tickets, item queue, chunk tiles into a stage ring
-//   warp 1      TMEM allocator and single-thread tcgen05.mma issuer
-//   warps 2-5   score -> P: TMEM score tile, causal mask, scale by -eta, bf16 into smem
-//   warps 6-9   output epilogue: TMEM O tile, optional activation, bf16 stores
+//   warp 1      TMEM allocator; its lane 0 issues the "front" MMAs of every chunk
+//               (score Q K^T and state increment K^T V), up to two chunks ahead
+//   warp 14     lane 0 issues the "back" MMAs (O = Q S^T, then O += P V); the two
+//               issuers run independent in-order loops, so the output product of
+//               chunk c never waits behind the score of chunk c+1
+//   warps 2-5   score -> P: TMEM score tile, causal mask, scale by -eta, bf16 P
+//               written back over the same TMEM columns (the PV product reads its A
+//               operand from tensor memory, so P never touches shared memory)
+//   warps 6-9   output epilogue: TMEM O tile -> bf16 staging tile in shared memory ->
+//               one TMA tensor store per chunk (whole 128-byte rows, no scattered
+//               per-thread stores competing with the other roles for the LSU path)
 //   warps 10-13 state: fp32 state rows in registers, dZ from TMEM, S^T tile into smem,
 //               look-back carry
 //
-// Tensor memory (512 columns): score x2 (128 each), O x2 (64), dZ x2 (64).
+// Tensor memory (512 columns): score/P x2 (128 each), O x2 (64), dZ x2 (64).
+//
+// Every MMA operand descriptor is built once per stage; a K-step only adds a
+// compile-time constant to its low word, which keeps the single issuing thread
+// ahead of the tensor pipe.
 #include <cuda.h>
 
 #include "scan_common.cuh"
@@ -35,10 +47,11 @@ namespace gl {
 
 constexpr int kChunk = 128;
 constexpr int kTile = 16384;  // one [128 rows][64 bf16] 128B-swizzled tile
-constexpr int kWarps = 14;
+constexpr int kWarps = 15;
 constexpr int kThreads = kWarps * 32;
 constexpr int kWarpO0 = 6, kWarpZ0 = 10;  // score->P warps are 2..5
-constexpr int kItemConsumers = 1 + 4 + 4 + 4;  // MMA thread + lane 0 of every other role warp
+constexpr int kWarpBack = 14;             // back-MMA issuer
+constexpr int kItemConsumers = 2 + 4 + 4 + 4;  // two MMA issuers + lane 0 of every other role warp
 
 // TMEM column map.
 constexpr uint32_t kTmemCols = 512;
@@ -53,13 +66,14 @@ struct TcLayout {
     static constexpr int kKOff = COSTATE ? kQkBlocks * kTile : 0;
     static constexpr int kVOff = kKOff + kQkBlocks * kTile;
     static constexpr int kStageBytes = kVOff + kTile;
-    // Stage count: fill what is left of the 227 KB opt-in budget after P, the two
-    // S^T tiles, the barrier block and the alignment slack.
-    static constexpr int kFixed = 2 * kTile + 2 * DQ * 128;
-    static constexpr int kStages0 = (232448 - kFixed - 1024 - 1024) / kStageBytes;
-    static constexpr int kStages = kStages0 > 4 ? 4 : kStages0;
-    static constexpr int kPOff = kStages * kStageBytes;
-    static constexpr int kStOff = kPOff + 2 * kTile;
+    // Stage ring: what is left of the 227 KB opt-in budget after the two S^T
+    // tiles, the two output staging tiles, the barrier block and the alignment
+    // slack (at most 6 stages).
+    static constexpr int kAvail = 232448 - 2 * DQ * 128 - 2 * kTile - 1024 - 1024;
+    static constexpr int kStages0 = kAvail / kStageBytes;
+    static constexpr int kStages = kStages0 > 6 ? 6 : kStages0;
+    static constexpr int kOOff = kStages * kStageBytes;  // two [128 t][64] output tiles
+    static constexpr int kStOff = kOOff + 2 * kTile;
     static constexpr int kStBytes = DQ * 128;
     static constexpr int kBarOff = kStOff + 2 * kStBytes;
     static constexpr int kBarBytes = 1024;
@@ -119,10 +133,20 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
     return ok != 0;
 }
 
+// K-step offsets (in the 16-byte units of a descriptor's low word).
+// K-major operand, 64-wide K blocks 16 KB apart: step kk starts 32 B further in
+// its 128-byte swizzled row, and every 4 steps moves to the next block.
+__host__ __device__ constexpr uint32_t kmaj_step(int kk) {
+    return (uint32_t)(((kk >> 2) * kTile + (kk & 3) * 32) >> 4);
+}
+// MN-major operand: step kk starts 16 rows (two 8-row groups of 1024 B) further.
+__host__ __device__ constexpr uint32_t mnmaj_step(int kk) { return (uint32_t)((kk * 2048) >> 4); }
+
 template <int DQ, bool COSTATE>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_scan_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                   const __grid_constant__ CUtensorMap tm_v, const TcScanParams p) {
+                   const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
+                   const TcScanParams p) {
     using Lay = TcLayout<DQ, COSTATE>;
     constexpr int NS = Lay::kStages;
     extern __shared__ uint8_t smem_raw[];
@@ -133,8 +157,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Lay::kBarOff);
     uint64_t* full = bars;                 // [NS]
     uint64_t* empty = bars + 8;            // [NS]
-    uint64_t* sc_full = bars + 16;         // [2]
-    uint64_t* sc_free = bars + 18;         // [2]
+    uint64_t* sc_full = bars + 16;         // [2] score in TMEM (front commit)
+    uint64_t* sc_free = bars + 18;         // [2] score/P buffer reusable (back commit after PV)
     uint64_t* o_full = bars + 20;          // [2]
     uint64_t* o_free = bars + 22;          // [2]
     uint64_t* dz_full = bars + 24;         // [2]
@@ -143,13 +167,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* st_free = bars + 30;         // [2]
     uint64_t* item_full = bars + 32;       // [2]
     uint64_t* item_empty = bars + 34;      // [2]
-    uint64_t* p_ready = bars + 36;
-    uint64_t* p_free = bars + 37;
-    uint64_t* z_pub = bars + 38;           // state warps: all rows written before a flag
-    uint64_t* z_lb = bars + 39;            // state warps: look-back result broadcast
-    uint64_t* z_ack = bars + 40;           // state warps: broadcast consumed
-    uint64_t* drain = bars + 41;
-    int* misc = reinterpret_cast<int*>(bars + 48);
+    uint64_t* p_ready = bars + 36;         // [2] P written over the score buffer (P warps)
+    uint64_t* o_staged = bars + 44;        // [2] output tile staged by all 4 epilogue warps
+    uint64_t* o_buf_free = bars + 46;      // [2] output staging tile read by its TMA store
+    uint64_t* z_pub = bars + 40;           // state warps: all rows written before a flag
+    uint64_t* z_lb = bars + 41;            // state warps: look-back result broadcast
+    uint64_t* z_ack = bars + 42;           // state warps: broadcast consumed
+    uint64_t* drain = bars + 38;
+    uint64_t* drain2 = bars + 39;
+    int* misc = reinterpret_cast<int*>(bars + 56);
     volatile int* abort_flag = misc + 0;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(misc + 1);
     volatile int* item_slot = misc + 2;    // [2]
@@ -162,11 +188,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < NS; ++i) {
             mbar_init(&full[i], 1);
-            mbar_init(&empty[i], 1);
+            mbar_init(&empty[i], 2);  // released by both MMA issuers
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&sc_full[i], 1);
-            mbar_init(&sc_free[i], 4);
+            mbar_init(&sc_free[i], 1);
+            mbar_init(&p_ready[i], 4);
+            mbar_init(&o_staged[i], 4);
+            mbar_init(&o_buf_free[i], 1);
             mbar_init(&o_full[i], 1);
             mbar_init(&o_free[i], 4);
             mbar_init(&dz_full[i], 1);
@@ -176,12 +205,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&item_full[i], 1);
             mbar_init(&item_empty[i], kItemConsumers);
         }
-        mbar_init(p_ready, 4);
-        mbar_init(p_free, 1);
         mbar_init(z_pub, kZActiveWarps);
         mbar_init(z_lb, 1);
         mbar_init(z_ack, kZActiveWarps);
         mbar_init(drain, 1);
+        mbar_init(drain2, 1);
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -194,6 +222,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         prefetch_tmap(&tm_q);
         prefetch_tmap(&tm_k);
         prefetch_tmap(&tm_v);
+        prefetch_tmap(&tm_o);
     }
     __syncthreads();
     tc_fence_after();
@@ -253,29 +282,28 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------- MMA issuer
+        // ------------------------------------------------- front MMA issuer
         if (lane == 0) {
-            constexpr uint32_t ID_SC = idesc_bf16(128, 128, false, false);
-            constexpr uint32_t ID_O = idesc_bf16(128, 64, false, true);
-            constexpr uint32_t ID_DZ = idesc_bf16(128, 64, true, true);
-            const uint32_t p_addr = sbase + Lay::kPOff;
+            constexpr uint32_t ID_SC = idesc_bf16(128, 128, false, false);  // Q K^T
+            constexpr uint32_t ID_DZ = idesc_bf16(128, 64, true, true);     // K^T V
             uint32_t n = 0, c2 = 0, dzc = 0;
             bool ok = true;
-            // dZ += K^T V over one stage (A = K^T: MN-major, 64-wide M blocks 16 KB apart;
-            // for DQ = 64 the second M block is the V tile, whose rows land in unused lanes).
-            auto issue_dz = [&](int s, uint32_t dcol, bool first) {
-                const uint32_t st = sbase + s * Lay::kStageBytes;
-#pragma unroll
-                for (int kk = 0; kk < kChunk / 16; ++kk) {
-                    uint64_t a = sdesc_sw128(st + Lay::kKOff + kk * 2048, kTile, 1024);
-                    uint64_t b = sdesc_sw128(st + Lay::kVOff + kk * 2048, kTile, 1024);
-                    mma_bf16_ss(tmem + dcol, a, b, ID_DZ, (first && kk == 0) ? 0u : 1u);
-                }
-            };
             auto wait_or_fail = [&](uint64_t* bar, uint32_t par) -> bool {
                 if (mbar_wait(bar, par, abort_flag)) return true;
                 raise_error(p, kErrWaitTimeout, abort_flag);
                 return false;
+            };
+            // dZ += K^T V over one stage.  A = K^T is MN-major with 64-wide M blocks
+            // 16 KB apart; for DQ = 64 the second M block is the V tile, whose rows
+            // land in TMEM lanes 64..127 that nobody reads.
+            auto issue_dz = [&](uint32_t st, uint32_t dcol, bool first) {
+                const uint32_t a_lo = sdesc_lo(st + Lay::kKOff, kTile);
+                const uint32_t b_lo = sdesc_lo(st + Lay::kVOff, kTile);
+#pragma unroll
+                for (int kk = 0; kk < kChunk / 16; ++kk)
+                    mma_bf16_ss(tmem + dcol, sdesc_from_lo(a_lo + mnmaj_step(kk)),
+                                sdesc_from_lo(b_lo + mnmaj_step(kk)), ID_DZ,
+                                (first && kk == 0) ? 0u : 1u);
             };
             for (int it = 0; ok; ++it) {
                 const int slot = it & 1;
@@ -292,88 +320,101 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const int s = n % NS;
                         if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
                         tc_fence_after();
-                        issue_dz(s, col_dz(b), c == 0);
+                        issue_dz(sbase + s * Lay::kStageBytes, col_dz(b), c == 0);
                         mma_commit(&empty[s]);
+                        mma_commit(&empty[s]);  // the back issuer skips phase-1 stages
                     }
                     if (!ok) break;
                     mma_commit(&dz_full[b]);
                     ++dzc;
                 }
-                // Phase 2.  front(c): score and dZ of chunk c; back(c): O of chunk c.
-                const uint32_t n0 = n;
-                auto front = [&](int c) -> bool {
-                    const uint32_t nn = n0 + c;
-                    const int s = nn % NS;
-                    if (!wait_or_fail(&full[s], (nn / NS) & 1)) return false;
-                    const uint32_t cc = c2 + c, sb = cc & 1;
-                    if (!wait_or_fail(&sc_free[sb], ((cc >> 1) & 1) ^ 1)) return false;
+                // Phase 2: score and dZ of every chunk (dZ of the last one is not needed).
+                for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
+                    const int s = n % NS;
+                    if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
+                    const uint32_t sb = c2 & 1;
+                    // the score/P buffer is free once the PV product two chunks back is done
+                    if (!(ok = wait_or_fail(&sc_free[sb], ((c2 >> 1) & 1) ^ 1))) break;
                     tc_fence_after();
                     const uint32_t st = sbase + s * Lay::kStageBytes;
+                    const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
+                    const uint32_t k_lo = sdesc_lo(st + Lay::kKOff, 16);
 #pragma unroll
-                    for (int kk = 0; kk < DQ / 16; ++kk) {
-                        const uint32_t off = (kk >> 2) * kTile + (kk & 3) * 32;
-                        uint64_t a = sdesc_sw128(st + Lay::kQOff + off, 16, 1024);
-                        uint64_t b = sdesc_sw128(st + Lay::kKOff + off, 16, 1024);
-                        mma_bf16_ss(tmem + col_sc(sb), a, b, ID_SC, kk > 0 ? 1u : 0u);
-                    }
+                    for (int kk = 0; kk < DQ / 16; ++kk)
+                        mma_bf16_ss(tmem + col_sc(sb), sdesc_from_lo(q_lo + kmaj_step(kk)),
+                                    sdesc_from_lo(k_lo + kmaj_step(kk)), ID_SC, kk > 0 ? 1u : 0u);
                     mma_commit(&sc_full[sb]);
                     if (c < I.nch - 1) {
                         const uint32_t b = dzc & 1;
-                        if (!wait_or_fail(&dz_free[b], ((dzc >> 1) & 1) ^ 1)) return false;
+                        if (!(ok = wait_or_fail(&dz_free[b], ((dzc >> 1) & 1) ^ 1))) break;
                         tc_fence_after();
-                        issue_dz(s, col_dz(b), true);
+                        issue_dz(st, col_dz(b), true);
                         mma_commit(&dz_full[b]);
                         ++dzc;
                     }
-                    return true;
-                };
-                if (!(ok = front(0))) break;
-                for (int c = 0; c < I.nch && ok; ++c) {
-                    if (c + 1 < I.nch && !(ok = front(c + 1))) break;
-                    const uint32_t nn = n0 + c;
-                    const int s = nn % NS;
-                    const uint32_t cc = c2 + c, ob = cc & 1, oph = (cc >> 1) & 1;
+                    mma_commit(&empty[s]);
+                }
+            }
+            // Every MMA this thread issued has completed before TMEM is released.
+            mma_commit(drain);
+            mbar_drain(drain, 0);
+        }
+    } else if (warp == kWarpBack) {
+        // -------------------------------------------------- back MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t ID_O = idesc_bf16(128, 64, false, true);  // Q S^T, P V
+            uint32_t n = 0, c2 = 0;
+            bool ok = true;
+            auto wait_or_fail = [&](uint64_t* bar, uint32_t par) -> bool {
+                if (mbar_wait(bar, par, abort_flag)) return true;
+                raise_error(p, kErrWaitTimeout, abort_flag);
+                return false;
+            };
+            for (int it = 0; ok; ++it) {
+                const int slot = it & 1;
+                if (!wait_or_fail(&item_full[slot], (it >> 1) & 1)) break;
+                const int item = item_slot[slot];
+                mbar_arrive(&item_empty[slot]);
+                if (item < 0) break;
+                const Item I = decode_item(item, p);
+                if (I.phase1) n += I.nch;  // phase-1 stages are released by the front issuer
+                for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
+                    const int s = n % NS;
+                    const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
+                    if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
                     if (!(ok = wait_or_fail(&o_free[ob], oph ^ 1))) break;
                     if (!(ok = wait_or_fail(&st_ready[ob], oph))) break;
                     tc_fence_after();
                     const uint32_t st = sbase + s * Lay::kStageBytes;
-                    const uint32_t st_tile = sbase + Lay::kStOff + ob * Lay::kStBytes;
                     // O = Q S^T  (B = S^T tile [dq][64]: MN-major)
+                    const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
+                    const uint32_t s_lo = sdesc_lo(sbase + Lay::kStOff + ob * Lay::kStBytes, kTile);
 #pragma unroll
-                    for (int kk = 0; kk < DQ / 16; ++kk) {
-                        const uint32_t off = (kk >> 2) * kTile + (kk & 3) * 32;
-                        uint64_t a = sdesc_sw128(st + Lay::kQOff + off, 16, 1024);
-                        uint64_t b = sdesc_sw128(st_tile + kk * 2048, kTile, 1024);
-                        mma_bf16_ss(tmem + col_o(ob), a, b, ID_O, kk > 0 ? 1u : 0u);
-                    }
+                    for (int kk = 0; kk < DQ / 16; ++kk)
+                        mma_bf16_ss(tmem + col_o(ob), sdesc_from_lo(q_lo + kmaj_step(kk)),
+                                    sdesc_from_lo(s_lo + mnmaj_step(kk)), ID_O, kk > 0 ? 1u : 0u);
                     mma_commit(&st_free[ob]);
-                    if (!(ok = wait_or_fail(p_ready, cc & 1))) break;
+                    if (!(ok = wait_or_fail(&p_ready[ob], oph))) break;
                     tc_fence_after();
-                    // O += P V  (A = P [128][128] K-major, B = V [128 tokens][64]: MN-major)
+                    // O += P V  (A = P in TMEM over the score buffer; B = V [128 t][64]: MN-major)
+                    const uint32_t v_lo = sdesc_lo(st + Lay::kVOff, kTile);
 #pragma unroll
-                    for (int kk = 0; kk < kChunk / 16; ++kk) {
-                        const uint32_t off = (kk >> 2) * kTile + (kk & 3) * 32;
-                        uint64_t a = sdesc_sw128(p_addr + off, 16, 1024);
-                        uint64_t b = sdesc_sw128(st + Lay::kVOff + kk * 2048, kTile, 1024);
-                        mma_bf16_ss(tmem + col_o(ob), a, b, ID_O, 1u);
-                    }
+                    for (int kk = 0; kk < kChunk / 16; ++kk)
+                        mma_bf16_ts(tmem + col_o(ob), tmem + col_sc(ob) + kk * 8,
+                                    sdesc_from_lo(v_lo + mnmaj_step(kk)), ID_O, 1u);
                     mma_commit(&o_full[ob]);
-                    mma_commit(p_free);
+                    mma_commit(&sc_free[ob]);
                     mma_commit(&empty[s]);
                 }
-                n = n0 + I.nch;
-                c2 += I.nch;
             }
-            // Every MMA has completed before TMEM is released.
-            mma_commit(drain);
-            mbar_drain(drain, 0);
+            mma_commit(drain2);
+            mbar_drain(drain2, 0);
         }
     } else if (warp < kWarpO0) {
         // ------------------------------------------------------ score -> P
         const int q4 = warp & 3;
         const int row = q4 * 32 + lane;
         const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
-        const uint32_t p_addr = sbase + Lay::kPOff;
         const float neg_eta = -p.eta;
         uint32_t c2 = 0;
         for (int it = 0;; ++it) {
@@ -390,45 +431,39 @@ __global__ void __launch_bounds__(kThreads, 1)
             bool ok = true;
             for (int c = 0; c < I.nch; ++c, ++c2) {
                 const uint32_t sb = c2 & 1;
-                if (!warp_wait(&sc_full[sb], (c2 >> 1) & 1, abort_flag) ||
-                    !warp_wait(p_free, (c2 & 1) ^ 1, abort_flag)) {
+                if (!warp_wait(&sc_full[sb], (c2 >> 1) & 1, abort_flag)) {
                     raise_error(p, kErrWaitTimeout, abort_flag);
                     ok = false;
                     break;
                 }
                 tc_fence_after();
+                // Rows of this warp are 32*q4 .. 32*q4+31, so only columns s < 32*(q4+1)
+                // survive the strict causal mask: warps 0-1 read 64 score columns, 2-3
+                // read 128.  P row t packs (s, s+1) pairs as bf16x2 into column s/2 of
+                // the same buffer.  Columns 0..63 of the score have been read before
+                // P columns 0..31 overwrite them, and likewise for the second half.
+                const uint32_t base = tmem + col_sc(sb) + lane_off;
 #pragma unroll 1
-                for (int piece = 0; piece < 4; ++piece) {
-                    uint32_t w[16];
-                    if (piece <= q4) {
-                        float v[32];
-                        tmem_ld32(tmem + col_sc(sb) + lane_off + piece * 32, v);
+                for (int half = 0; half < 2; ++half) {
+                    uint32_t w[32];
+                    if (half == 0 || q4 >= 2) {
+                        float v[64];
+                        tmem_ld64(base + half * 64, v);
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            const int s0 = piece * 32 + 2 * i;
-                            float a = (s0 < row) ? neg_eta * v[2 * i] : 0.0f;
-                            float b2 = (s0 + 1 < row) ? neg_eta * v[2 * i + 1] : 0.0f;
-                            w[i] = pack_bf16x2(a, b2);
+                        for (int i = 0; i < 32; ++i) {
+                            const int s0 = half * 64 + 2 * i;
+                            w[i] = pack_bf16x2(s0 < row ? neg_eta * v[2 * i] : 0.0f,
+                                               s0 + 1 < row ? neg_eta * v[2 * i + 1] : 0.0f);
                         }
                     } else {
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) w[i] = 0u;
+                        for (int i = 0; i < 32; ++i) w[i] = 0u;
                     }
-                    const uint32_t blk = p_addr + (piece >> 1) * kTile;
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const uint32_t chunk = (piece & 1) * 4 + q;
-                        st_shared_v4(blk + sw128_off(row, chunk), w[4 * q], w[4 * q + 1],
-                                     w[4 * q + 2], w[4 * q + 3]);
-                    }
+                    tmem_st32(base + half * 32, w);
                 }
                 tc_fence_before();
-                fence_proxy_async_smem();
                 __syncwarp();
-                if (lane == 0) {
-                    mbar_arrive(&sc_free[sb]);
-                    mbar_arrive(p_ready);
-                }
+                if (lane == 0) mbar_arrive(&p_ready[sb]);
             }
             if (!ok) break;
         }
@@ -437,6 +472,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int q4 = warp & 3;
         const int row = q4 * 32 + lane;
         const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
+        const bool storer = (warp == kWarpO0) && (lane == 0);  // issues the TMA stores
         const EpiParams& e = p.epi;
         uint32_t c2 = 0;
         for (int it = 0;; ++it) {
@@ -452,69 +488,82 @@ __global__ void __launch_bounds__(kThreads, 1)
             const Item I = decode_item(item, p);
             bool ok = true;
             for (int c = 0; c < I.nch; ++c, ++c2) {
-                const uint32_t ob = c2 & 1;
-                if (!warp_wait(&o_full[ob], (c2 >> 1) & 1, abort_flag)) {
+                const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
+                if (!warp_wait(&o_full[ob], oph, abort_flag)) {
                     raise_error(p, kErrWaitTimeout, abort_flag);
                     ok = false;
                     break;
                 }
                 tc_fence_after();
                 float v[64];
-                {
-                    float a[32];
-                    tmem_ld32(tmem + col_o(ob) + lane_off, a);
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] = a[i];
-                    tmem_ld32(tmem + col_o(ob) + lane_off + 32, a);
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) v[32 + i] = a[i];
-                }
+                tmem_ld64(tmem + col_o(ob) + lane_off, v);
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&o_free[ob]);
-                const int t = I.t_begin + c * kChunk + row;
-                if (t < I.t_end) {
-                    const int col0 = I.j * 64;
-                    if (e.zin) {
-                        const __nv_bfloat16* zp = static_cast<const __nv_bfloat16*>(e.zin) +
-                                                  tok_off(e.z_str, I.l, I.b, t, I.h) + col0;
+                const int t0 = I.t_begin + c * kChunk;
+                const int t = t0 + row;
+                const int col0 = I.j * 64;
+                if (e.zin && t < I.t_end) {
+                    const __nv_bfloat16* zp = static_cast<const __nv_bfloat16*>(e.zin) +
+                                              tok_off(e.z_str, I.l, I.b, t, I.h) + col0;
 #pragma unroll
-                        for (int q = 0; q < 8; ++q) {
-                            uint4 zz = *reinterpret_cast<const uint4*>(zp + 8 * q);
-                            const __nv_bfloat16* zb = reinterpret_cast<const __nv_bfloat16*>(&zz);
+                    for (int q = 0; q < 8; ++q) {
+                        uint4 zz = *reinterpret_cast<const uint4*>(zp + 8 * q);
+                        const __nv_bfloat16* zb = reinterpret_cast<const __nv_bfloat16*>(&zz);
 #pragma unroll
-                            for (int i = 0; i < 8; ++i)
-                                v[8 * q + i] *= act_df(e.act, __bfloat162float(zb[i]));
-                        }
+                        for (int i = 0; i < 8; ++i) v[8 * q + i] *= act_df(e.act, __bfloat162float(zb[i]));
                     }
-                    __nv_bfloat16* op = static_cast<__nv_bfloat16*>(e.out) +
-                                        tok_off(e.out_str, I.l, I.b, t, I.h) + col0;
+                }
+                if (e.out2 && t < I.t_end) {
+                    __nv_bfloat16* op2 = static_cast<__nv_bfloat16*>(e.out2) +
+                                         tok_off(e.out2_str, I.l, I.b, t, I.h) + col0;
 #pragma unroll
                     for (int q = 0; q < 8; ++q) {
                         uint4 w;
-                        w.x = pack_bf16x2(v[8 * q + 0], v[8 * q + 1]);
-                        w.y = pack_bf16x2(v[8 * q + 2], v[8 * q + 3]);
-                        w.z = pack_bf16x2(v[8 * q + 4], v[8 * q + 5]);
-                        w.w = pack_bf16x2(v[8 * q + 6], v[8 * q + 7]);
-                        *reinterpret_cast<uint4*>(op + 8 * q) = w;
+                        w.x = pack_bf16x2(act_f(e.act, v[8 * q + 0]), act_f(e.act, v[8 * q + 1]));
+                        w.y = pack_bf16x2(act_f(e.act, v[8 * q + 2]), act_f(e.act, v[8 * q + 3]));
+                        w.z = pack_bf16x2(act_f(e.act, v[8 * q + 4]), act_f(e.act, v[8 * q + 5]));
+                        w.w = pack_bf16x2(act_f(e.act, v[8 * q + 6]), act_f(e.act, v[8 * q + 7]));
+                        *reinterpret_cast<uint4*>(op2 + 8 * q) = w;
                     }
-                    if (e.out2) {
-                        __nv_bfloat16* op2 = static_cast<__nv_bfloat16*>(e.out2) +
-                                             tok_off(e.out2_str, I.l, I.b, t, I.h) + col0;
+                }
+                // Stage the bf16 row in the 128B-swizzled output tile (the TMA store
+                // clips rows past the end of the sequence).
+                if (!warp_wait(&o_buf_free[ob], oph ^ 1, abort_flag)) {
+                    raise_error(p, kErrWaitTimeout, abort_flag);
+                    ok = false;
+                    break;
+                }
+                const uint32_t otile = sbase + Lay::kOOff + ob * kTile;
 #pragma unroll
-                        for (int q = 0; q < 8; ++q) {
-                            uint4 w;
-                            w.x = pack_bf16x2(act_f(e.act, v[8 * q + 0]), act_f(e.act, v[8 * q + 1]));
-                            w.y = pack_bf16x2(act_f(e.act, v[8 * q + 2]), act_f(e.act, v[8 * q + 3]));
-                            w.z = pack_bf16x2(act_f(e.act, v[8 * q + 4]), act_f(e.act, v[8 * q + 5]));
-                            w.w = pack_bf16x2(act_f(e.act, v[8 * q + 6]), act_f(e.act, v[8 * q + 7]));
-                            *reinterpret_cast<uint4*>(op2 + 8 * q) = w;
-                        }
+                for (int q = 0; q < 8; ++q)
+                    st_shared_v4(otile + sw128_off(row, q), pack_bf16x2(v[8 * q], v[8 * q + 1]),
+                                 pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                                 pack_bf16x2(v[8 * q + 4], v[8 * q + 5]),
+                                 pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&o_staged[ob]);
+                if (storer) {
+                    if (!mbar_wait(&o_staged[ob], oph, abort_flag)) {
+                        raise_error(p, kErrWaitTimeout, abort_flag);
+                        ok = false;
+                    } else {
+                        tma_store_5d(&tm_o, smem + Lay::kOOff + ob * kTile, col0, I.h, t0, I.b, I.l);
+                        bulk_commit_group();
+                        // the previous chunk's store (other tile) has finished reading
+                        bulk_wait_group_read<1>();
+                        if (c2 > 0) mbar_arrive(&o_buf_free[ob ^ 1]);
                     }
+                }
+                if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
+                    ok = false;
+                    break;
                 }
             }
             if (!ok) break;
         }
+        if (storer) bulk_wait_group_all();
     } else {
         // ------------------------------------------------------------ state
         const int q4 = warp & 3;
@@ -725,6 +774,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     }
 
+
     __syncthreads();
     if (warp == 1) {
         __syncwarp();
@@ -736,24 +786,26 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ------------------------------------------------------------------ host side
 template <int DQ, bool COSTATE>
 static cudaError_t launch_one(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
-                              const TcScanParams& p, int grid, cudaStream_t stream) {
+                              const CUtensorMap& o, const TcScanParams& p, int grid,
+                              cudaStream_t stream) {
     using Lay = TcLayout<DQ, COSTATE>;
     auto kern = tc_scan_kernel<DQ, COSTATE>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          Lay::kSmemBytes);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kThreads, Lay::kSmemBytes, stream>>>(q, k, v, p);
+    kern<<<grid, kThreads, Lay::kSmemBytes, stream>>>(q, k, v, o, p);
     return cudaGetLastError();
 }
 
 cudaError_t launch_tc_scan(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
-                           const TcScanParams& p, bool costate, int grid, cudaStream_t stream) {
+                           const CUtensorMap& o, const TcScanParams& p, bool costate, int grid,
+                           cudaStream_t stream) {
     if (p.dq == 64)
-        return costate ? launch_one<64, true>(q, k, v, p, grid, stream)
-                       : launch_one<64, false>(q, k, v, p, grid, stream);
+        return costate ? launch_one<64, true>(q, k, v, o, p, grid, stream)
+                       : launch_one<64, false>(q, k, v, o, p, grid, stream);
     if (p.dq == 128)
-        return costate ? launch_one<128, true>(q, k, v, p, grid, stream)
-                       : launch_one<128, false>(q, k, v, p, grid, stream);
+        return costate ? launch_one<128, true>(q, k, v, o, p, grid, stream)
+                       : launch_one<128, false>(q, k, v, o, p, grid, stream);
     return cudaErrorInvalidValue;
 }
 
