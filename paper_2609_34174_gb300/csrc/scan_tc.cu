@@ -31,7 +31,9 @@
 //               one TMA tensor store per chunk (whole 128-byte rows, no scattered
 //               per-thread stores competing with the other roles for the LSU path)
 //   warps 10-13 state: fp32 state rows in registers, dZ from TMEM, S^T tile into smem,
-//               look-back carry
+//               look-back carry.  With 64-wide keys only warps 10-11... hold state
+//               rows (lanes 0..63); the two warps whose lanes are 64..127 then build
+//               the second half of P for those rows instead.
 //
 // Tensor memory (512 columns): score/P x2 (128 each), O x2 (64), dZ x2 (64).
 //
@@ -183,7 +185,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    constexpr int kZActiveWarps = DQ / 32;
+    constexpr int kZActiveWarps = DQ / 32;          // state warps holding rows
+    constexpr int kPHelpers = 4 - kZActiveWarps;    // state-slot warps building P half 1
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < NS; ++i) {
@@ -193,14 +196,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(&sc_full[i], 1);
             mbar_init(&sc_free[i], 1);
-            mbar_init(&p_ready[i], 4);
+            mbar_init(&p_ready[i], 4 + kPHelpers);
             mbar_init(&o_staged[i], 4);
             mbar_init(&o_buf_free[i], 1);
             mbar_init(&o_full[i], 1);
             mbar_init(&o_free[i], 4);
             mbar_init(&dz_full[i], 1);
-            mbar_init(&dz_free[i], 4);
-            mbar_init(&st_ready[i], 4);
+            mbar_init(&dz_free[i], kZActiveWarps);
+            mbar_init(&st_ready[i], kZActiveWarps);
             mbar_init(&st_free[i], 1);
             mbar_init(&item_full[i], 1);
             mbar_init(&item_empty[i], kItemConsumers);
@@ -396,11 +399,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mma_commit(&st_free[ob]);
                     if (!(ok = wait_or_fail(&p_ready[ob], oph))) break;
                     tc_fence_after();
-                    // O += P V  (A = P in TMEM over the score buffer; B = V [128 t][64]: MN-major)
+                    // O += P V  (A = P in TMEM over the score buffer: tokens s < 64 in
+                    // columns 0..31, s >= 64 in columns 64..95; B = V [128 t][64]: MN-major)
                     const uint32_t v_lo = sdesc_lo(st + Lay::kVOff, kTile);
 #pragma unroll
                     for (int kk = 0; kk < kChunk / 16; ++kk)
-                        mma_bf16_ts(tmem + col_o(ob), tmem + col_sc(ob) + kk * 8,
+                        mma_bf16_ts(tmem + col_o(ob),
+                                    tmem + col_sc(ob) + (kk < 4 ? kk * 8 : 64 + (kk - 4) * 8),
                                     sdesc_from_lo(v_lo + mnmaj_step(kk)), ID_O, 1u);
                     mma_commit(&o_full[ob]);
                     mma_commit(&sc_free[ob]);
@@ -410,8 +415,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_commit(drain2);
             mbar_drain(drain2, 0);
         }
-    } else if (warp < kWarpO0) {
+    } else if (warp < kWarpO0 || (warp >= kWarpZ0 && (warp & 3) >= kZActiveWarps)) {
         // ------------------------------------------------------ score -> P
+        // Warps 2-5 build P; with 64-wide keys the two state-slot warps whose
+        // lanes (64..127) hold no state rows build the second half of P for them.
+        const bool helper = warp >= kWarpZ0;
         const int q4 = warp & 3;
         const int row = q4 * 32 + lane;
         const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
@@ -438,29 +446,33 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_after();
                 // Rows of this warp are 32*q4 .. 32*q4+31, so only columns s < 32*(q4+1)
-                // survive the strict causal mask: warps 0-1 read 64 score columns, 2-3
-                // read 128.  P row t packs (s, s+1) pairs as bf16x2 into column s/2 of
-                // the same buffer.  Columns 0..63 of the score have been read before
-                // P columns 0..31 overwrite them, and likewise for the second half.
+                // survive the strict causal mask.  P row t packs (s, s+1) pairs as
+                // bf16x2: tokens s < 64 into columns s/2 (0..31), tokens s >= 64 into
+                // columns 64 + (s-64)/2 (64..95), each written only after the same
+                // warp has read the score columns it overwrites.  Rows below 64 have
+                // an all-zero second half; with 64-wide keys the second half of rows
+                // 64..127 is built by the two spare state-slot warps.
                 const uint32_t base = tmem + col_sc(sb) + lane_off;
 #pragma unroll 1
                 for (int half = 0; half < 2; ++half) {
-                    uint32_t w[32];
-                    if (half == 0 || q4 >= 2) {
-                        float v[64];
-                        tmem_ld64(base + half * 64, v);
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const int s0 = half * 64 + 2 * i;
-                            w[i] = pack_bf16x2(s0 < row ? neg_eta * v[2 * i] : 0.0f,
-                                               s0 + 1 < row ? neg_eta * v[2 * i + 1] : 0.0f);
-                        }
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) w[i] = 0u;
+                    const bool mine = half == 0 ? !helper : (q4 < 2 ? !helper : (helper || kPHelpers == 0));
+                    if (!mine) continue;
+                    if (half == 1 && q4 < 2) {
+                        tmem_zero32_async(base + 64);  // rows < 64: tokens >= 64 all masked
+                        continue;
                     }
-                    tmem_st32(base + half * 32, w);
+                    float v[64];
+                    uint32_t w[32];
+                    tmem_ld64(base + half * 64, v);
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        const int s0 = half * 64 + 2 * i;
+                        w[i] = pack_bf16x2(s0 < row ? neg_eta * v[2 * i] : 0.0f,
+                                           s0 + 1 < row ? neg_eta * v[2 * i + 1] : 0.0f);
+                    }
+                    tmem_st32_async(base + half * 64, w);
                 }
+                tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&p_ready[sb]);
@@ -565,8 +577,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (storer) bulk_wait_group_all();
     } else {
-        // ------------------------------------------------------------ state
         const int q4 = warp & 3;
+        {
+        // ------------------------------------------------------------ state
         const int row = q4 * 32 + lane;         // contraction index q of this thread's state row
         const bool active = row < DQ;           // warp-uniform
         const bool leader = (q4 == 0) && (lane == 0);
@@ -772,8 +785,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (!ok) break;
         }
+        }
     }
-
 
     __syncthreads();
     if (warp == 1) {
