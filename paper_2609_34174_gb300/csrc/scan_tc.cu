@@ -14,8 +14,11 @@
 // is a decoupled look-back over per-segment aggregates sum_{s in seg} k_s v_s^T
 // (the additive scan is associative, Sec. 3 "Observation", Eq. 2).  A segment
 // that has successors first streams its keys/values once to form its aggregate
-// (phase 1), publishes it, looks back, publishes its inclusive prefix, then runs
-// the full chunk loop (phase 2, which re-reads the same tiles, mostly from L2).
+// (phase 1) and publishes it, then later looks back, publishes its inclusive prefix
+// and runs the full chunk loop (phase 2, which re-reads the same tiles, mostly
+// from L2).  A CTA runs phase 1 of the item it has just taken BEFORE phase 2 of
+// its previous item, so an aggregate is published right after its ticket is
+// taken and successors in other CTAs rarely wait in their look-back.
 //
 // Warp roles (15 warps, one CTA per SM):
 //   warp 0      TMA producer: tickets, item queue, chunk tiles into a stage ring
@@ -54,6 +57,7 @@ constexpr int kThreads = kWarps * 32;
 constexpr int kWarpO0 = 6, kWarpZ0 = 10;  // score->P warps are 2..5
 constexpr int kWarpBack = 14;             // back-MMA issuer
 constexpr int kItemConsumers = 2 + 4 + 4 + 4;  // two MMA issuers + lane 0 of every other role warp
+constexpr int kRing = 4;                        // item queue depth
 
 // TMEM column map.
 constexpr uint32_t kTmemCols = 512;
@@ -167,8 +171,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* dz_free = bars + 26;         // [2]
     uint64_t* st_ready = bars + 28;        // [2]
     uint64_t* st_free = bars + 30;         // [2]
-    uint64_t* item_full = bars + 32;       // [2]
-    uint64_t* item_empty = bars + 34;      // [2]
+    uint64_t* item_full = bars + 48;       // [kRing]
+    uint64_t* item_empty = bars + 52;      // [kRing]
     uint64_t* p_ready = bars + 36;         // [2] P written over the score buffer (P warps)
     uint64_t* o_staged = bars + 44;        // [2] output tile staged by all 4 epilogue warps
     uint64_t* o_buf_free = bars + 46;      // [2] output staging tile read by its TMA store
@@ -180,8 +184,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     int* misc = reinterpret_cast<int*>(bars + 56);
     volatile int* abort_flag = misc + 0;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(misc + 1);
-    volatile int* item_slot = misc + 2;    // [2]
-    volatile unsigned int* lb_word = reinterpret_cast<volatile unsigned int*>(misc + 4);
+    volatile unsigned int* lb_word = reinterpret_cast<volatile unsigned int*>(misc + 2);
+    volatile int* item_slot = misc + 4;    // [kRing]
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -205,6 +209,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&dz_free[i], kZActiveWarps);
             mbar_init(&st_ready[i], kZActiveWarps);
             mbar_init(&st_free[i], 1);
+        }
+        for (int i = 0; i < kRing; ++i) {
             mbar_init(&item_full[i], 1);
             mbar_init(&item_empty[i], kItemConsumers);
         }
@@ -235,9 +241,38 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------ producer
         if (lane == 0) {
             uint32_t n = 0;
-            for (int it = 0;; ++it) {
-                const int slot = it & 1;
-                if (!mbar_wait(&item_empty[slot], ((it >> 1) & 1) ^ 1, abort_flag)) {
+            bool ok = true;
+            // Stream the stages of one pass of an item into the ring.
+            auto load_pass = [&](const Item& I, int pass) {
+                for (int c = 0; c < I.nch && ok; ++c, ++n) {
+                    const int s = n % NS;
+                    if (!mbar_wait(&empty[s], ((n / NS) & 1) ^ 1, abort_flag)) {
+                        raise_error(p, kErrWaitTimeout, abort_flag);
+                        ok = false;
+                        break;
+                    }
+                    uint8_t* st = smem + s * Lay::kStageBytes;
+                    const int t0 = I.t_begin + c * kChunk;
+                    mbar_arrive_expect_tx(&full[s], pass == 1 ? Lay::kTxPass1 : Lay::kTxPass2);
+                    if (COSTATE && pass == 2) {
+#pragma unroll
+                        for (int kb = 0; kb < Lay::kQkBlocks; ++kb)
+                            tma_load_5d(st + Lay::kQOff + kb * kTile, &tm_q, &full[s], kb * 64, I.h,
+                                        t0, I.b, I.l);
+                    }
+#pragma unroll
+                    for (int kb = 0; kb < Lay::kQkBlocks; ++kb)
+                        tma_load_5d(st + Lay::kKOff + kb * kTile, &tm_k, &full[s], kb * 64, I.h, t0,
+                                    I.b, I.l);
+                    tma_load_5d(st + Lay::kVOff, &tm_v, &full[s], I.j * 64, I.h, t0, I.b, I.l);
+                }
+            };
+            // Stage order: P1(i0), P1(i1), P2(i0), P1(i2), P2(i1), ...: phase 1 of a new
+            // item is loaded before phase 2 of the previous one.
+            int pending = -1;
+            for (int it = 0; ok; ++it) {
+                const int slot = it % kRing;
+                if (!mbar_wait(&item_empty[slot], ((it / kRing) & 1) ^ 1, abort_flag)) {
                     raise_error(p, kErrWaitTimeout, abort_flag);
                     break;
                 }
@@ -245,34 +280,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (item >= p.n_items) item = -1;
                 item_slot[slot] = item;
                 mbar_arrive(&item_full[slot]);
-                if (item < 0) break;
-                const Item I = decode_item(item, p);
-                bool ok = true;
-                for (int pass = I.phase1 ? 1 : 2; pass <= 2 && ok; ++pass) {
-                    for (int c = 0; c < I.nch; ++c, ++n) {
-                        const int s = n % NS;
-                        if (!mbar_wait(&empty[s], ((n / NS) & 1) ^ 1, abort_flag)) {
-                            raise_error(p, kErrWaitTimeout, abort_flag);
-                            ok = false;
-                            break;
-                        }
-                        uint8_t* st = smem + s * Lay::kStageBytes;
-                        const int t0 = I.t_begin + c * kChunk;
-                        mbar_arrive_expect_tx(&full[s], pass == 1 ? Lay::kTxPass1 : Lay::kTxPass2);
-                        if (COSTATE && pass == 2) {
-#pragma unroll
-                            for (int kb = 0; kb < Lay::kQkBlocks; ++kb)
-                                tma_load_5d(st + Lay::kQOff + kb * kTile, &tm_q, &full[s], kb * 64,
-                                            I.h, t0, I.b, I.l);
-                        }
-#pragma unroll
-                        for (int kb = 0; kb < Lay::kQkBlocks; ++kb)
-                            tma_load_5d(st + Lay::kKOff + kb * kTile, &tm_k, &full[s], kb * 64, I.h,
-                                        t0, I.b, I.l);
-                        tma_load_5d(st + Lay::kVOff, &tm_v, &full[s], I.j * 64, I.h, t0, I.b, I.l);
-                    }
+                if (item >= 0) {
+                    const Item I = decode_item(item, p);
+                    if (I.phase1) load_pass(I, 1);
                 }
-                if (!ok) break;
+                if (pending >= 0) load_pass(decode_item(pending, p), 2);
+                pending = item;
+                if (item < 0) break;
             }
             // Drain: every issued load has landed before the CTA can exit.
             if (*abort_flag) {
@@ -308,55 +322,64 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 sdesc_from_lo(b_lo + mnmaj_step(kk)), ID_DZ,
                                 (first && kk == 0) ? 0u : 1u);
             };
+            int pending = -1;
             for (int it = 0; ok; ++it) {
-                const int slot = it & 1;
-                if (!wait_or_fail(&item_full[slot], (it >> 1) & 1)) break;
+                const int slot = it % kRing;
+                if (!wait_or_fail(&item_full[slot], (it / kRing) & 1)) break;
                 const int item = item_slot[slot];
                 mbar_arrive(&item_empty[slot]);
-                if (item < 0) break;
-                const Item I = decode_item(item, p);
-                if (I.phase1) {
-                    const uint32_t b = dzc & 1;
-                    if (!wait_or_fail(&dz_free[b], ((dzc >> 1) & 1) ^ 1)) break;
-                    tc_fence_after();
-                    for (int c = 0; c < I.nch; ++c, ++n) {
-                        const int s = n % NS;
-                        if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
-                        tc_fence_after();
-                        issue_dz(sbase + s * Lay::kStageBytes, col_dz(b), c == 0);
-                        mma_commit(&empty[s]);
-                        mma_commit(&empty[s]);  // the back issuer skips phase-1 stages
-                    }
-                    if (!ok) break;
-                    mma_commit(&dz_full[b]);
-                    ++dzc;
-                }
-                // Phase 2: score and dZ of every chunk (dZ of the last one is not needed).
-                for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
-                    const int s = n % NS;
-                    if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
-                    const uint32_t sb = c2 & 1;
-                    // the score/P buffer is free once the PV product two chunks back is done
-                    if (!(ok = wait_or_fail(&sc_free[sb], ((c2 >> 1) & 1) ^ 1))) break;
-                    tc_fence_after();
-                    const uint32_t st = sbase + s * Lay::kStageBytes;
-                    const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
-                    const uint32_t k_lo = sdesc_lo(st + Lay::kKOff, 16);
-#pragma unroll
-                    for (int kk = 0; kk < DQ / 16; ++kk)
-                        mma_bf16_ss(tmem + col_sc(sb), sdesc_from_lo(q_lo + kmaj_step(kk)),
-                                    sdesc_from_lo(k_lo + kmaj_step(kk)), ID_SC, kk > 0 ? 1u : 0u);
-                    mma_commit(&sc_full[sb]);
-                    if (c < I.nch - 1) {
+                // phase 1 of the new item: its segment aggregate sum K^T V
+                if (item >= 0) {
+                    const Item I = decode_item(item, p);
+                    if (I.phase1) {
                         const uint32_t b = dzc & 1;
                         if (!(ok = wait_or_fail(&dz_free[b], ((dzc >> 1) & 1) ^ 1))) break;
                         tc_fence_after();
-                        issue_dz(st, col_dz(b), true);
+                        for (int c = 0; c < I.nch; ++c, ++n) {
+                            const int s = n % NS;
+                            if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
+                            tc_fence_after();
+                            issue_dz(sbase + s * Lay::kStageBytes, col_dz(b), c == 0);
+                            mma_commit(&empty[s]);
+                            mma_commit(&empty[s]);  // the back issuer skips phase-1 stages
+                        }
+                        if (!ok) break;
                         mma_commit(&dz_full[b]);
                         ++dzc;
                     }
-                    mma_commit(&empty[s]);
                 }
+                // phase 2 of the previous item: score and dZ of every chunk (dZ of the
+                // last chunk is not needed)
+                if (pending >= 0) {
+                    const Item I = decode_item(pending, p);
+                    for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
+                        const int s = n % NS;
+                        if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
+                        const uint32_t sb = c2 & 1;
+                        // the score/P buffer is free once the PV product two chunks back is done
+                        if (!(ok = wait_or_fail(&sc_free[sb], ((c2 >> 1) & 1) ^ 1))) break;
+                        tc_fence_after();
+                        const uint32_t st = sbase + s * Lay::kStageBytes;
+                        const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
+                        const uint32_t k_lo = sdesc_lo(st + Lay::kKOff, 16);
+#pragma unroll
+                        for (int kk = 0; kk < DQ / 16; ++kk)
+                            mma_bf16_ss(tmem + col_sc(sb), sdesc_from_lo(q_lo + kmaj_step(kk)),
+                                        sdesc_from_lo(k_lo + kmaj_step(kk)), ID_SC, kk > 0 ? 1u : 0u);
+                        mma_commit(&sc_full[sb]);
+                        if (c < I.nch - 1) {
+                            const uint32_t b = dzc & 1;
+                            if (!(ok = wait_or_fail(&dz_free[b], ((dzc >> 1) & 1) ^ 1))) break;
+                            tc_fence_after();
+                            issue_dz(st, col_dz(b), true);
+                            mma_commit(&dz_full[b]);
+                            ++dzc;
+                        }
+                        mma_commit(&empty[s]);
+                    }
+                }
+                pending = item;
+                if (item < 0) break;
             }
             // Every MMA this thread issued has completed before TMEM is released.
             mma_commit(drain);
@@ -373,44 +396,53 @@ __global__ void __launch_bounds__(kThreads, 1)
                 raise_error(p, kErrWaitTimeout, abort_flag);
                 return false;
             };
+            int pending = -1;
             for (int it = 0; ok; ++it) {
-                const int slot = it & 1;
-                if (!wait_or_fail(&item_full[slot], (it >> 1) & 1)) break;
+                const int slot = it % kRing;
+                if (!wait_or_fail(&item_full[slot], (it / kRing) & 1)) break;
                 const int item = item_slot[slot];
                 mbar_arrive(&item_empty[slot]);
-                if (item < 0) break;
-                const Item I = decode_item(item, p);
-                if (I.phase1) n += I.nch;  // phase-1 stages are released by the front issuer
-                for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
-                    const int s = n % NS;
-                    const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
-                    if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
-                    if (!(ok = wait_or_fail(&o_free[ob], oph ^ 1))) break;
-                    if (!(ok = wait_or_fail(&st_ready[ob], oph))) break;
-                    tc_fence_after();
-                    const uint32_t st = sbase + s * Lay::kStageBytes;
-                    // O = Q S^T  (B = S^T tile [dq][64]: MN-major)
-                    const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
-                    const uint32_t s_lo = sdesc_lo(sbase + Lay::kStOff + ob * Lay::kStBytes, kTile);
-#pragma unroll
-                    for (int kk = 0; kk < DQ / 16; ++kk)
-                        mma_bf16_ss(tmem + col_o(ob), sdesc_from_lo(q_lo + kmaj_step(kk)),
-                                    sdesc_from_lo(s_lo + mnmaj_step(kk)), ID_O, kk > 0 ? 1u : 0u);
-                    mma_commit(&st_free[ob]);
-                    if (!(ok = wait_or_fail(&p_ready[ob], oph))) break;
-                    tc_fence_after();
-                    // O += P V  (A = P in TMEM over the score buffer: tokens s < 64 in
-                    // columns 0..31, s >= 64 in columns 64..95; B = V [128 t][64]: MN-major)
-                    const uint32_t v_lo = sdesc_lo(st + Lay::kVOff, kTile);
-#pragma unroll
-                    for (int kk = 0; kk < kChunk / 16; ++kk)
-                        mma_bf16_ts(tmem + col_o(ob),
-                                    tmem + col_sc(ob) + (kk < 4 ? kk * 8 : 64 + (kk - 4) * 8),
-                                    sdesc_from_lo(v_lo + mnmaj_step(kk)), ID_O, 1u);
-                    mma_commit(&o_full[ob]);
-                    mma_commit(&sc_free[ob]);
-                    mma_commit(&empty[s]);
+                // the new item's phase-1 stages precede the previous item's phase 2 and
+                // are released by the front issuer
+                if (item >= 0) {
+                    const Item In = decode_item(item, p);
+                    if (In.phase1) n += In.nch;
                 }
+                if (pending >= 0) {
+                    const Item I = decode_item(pending, p);
+                    for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
+                        const int s = n % NS;
+                        const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
+                        if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
+                        if (!(ok = wait_or_fail(&o_free[ob], oph ^ 1))) break;
+                        if (!(ok = wait_or_fail(&st_ready[ob], oph))) break;
+                        tc_fence_after();
+                        const uint32_t st = sbase + s * Lay::kStageBytes;
+                        // O = Q S^T  (B = S^T tile [dq][64]: MN-major)
+                        const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
+                        const uint32_t s_lo = sdesc_lo(sbase + Lay::kStOff + ob * Lay::kStBytes, kTile);
+#pragma unroll
+                        for (int kk = 0; kk < DQ / 16; ++kk)
+                            mma_bf16_ss(tmem + col_o(ob), sdesc_from_lo(q_lo + kmaj_step(kk)),
+                                        sdesc_from_lo(s_lo + mnmaj_step(kk)), ID_O, kk > 0 ? 1u : 0u);
+                        mma_commit(&st_free[ob]);
+                        if (!(ok = wait_or_fail(&p_ready[ob], oph))) break;
+                        tc_fence_after();
+                        // O += P V  (A = P in TMEM over the score buffer: tokens s < 64 in
+                        // columns 0..31, s >= 64 in columns 64..95; B = V [128 t][64]: MN-major)
+                        const uint32_t v_lo = sdesc_lo(st + Lay::kVOff, kTile);
+#pragma unroll
+                        for (int kk = 0; kk < kChunk / 16; ++kk)
+                            mma_bf16_ts(tmem + col_o(ob),
+                                        tmem + col_sc(ob) + (kk < 4 ? kk * 8 : 64 + (kk - 4) * 8),
+                                        sdesc_from_lo(v_lo + mnmaj_step(kk)), ID_O, 1u);
+                        mma_commit(&o_full[ob]);
+                        mma_commit(&sc_free[ob]);
+                        mma_commit(&empty[s]);
+                    }
+                }
+                pending = item;
+                if (item < 0) break;
             }
             mma_commit(drain2);
             mbar_drain(drain2, 0);
@@ -426,8 +458,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float neg_eta = -p.eta;
         uint32_t c2 = 0;
         for (int it = 0;; ++it) {
-            const int slot = it & 1;
-            if (!warp_wait(&item_full[slot], (it >> 1) & 1, abort_flag)) {
+            const int slot = it % kRing;
+            if (!warp_wait(&item_full[slot], (it / kRing) & 1, abort_flag)) {
                 raise_error(p, kErrWaitTimeout, abort_flag);
                 break;
             }
@@ -488,8 +520,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const EpiParams& e = p.epi;
         uint32_t c2 = 0;
         for (int it = 0;; ++it) {
-            const int slot = it & 1;
-            if (!warp_wait(&item_full[slot], (it >> 1) & 1, abort_flag)) {
+            const int slot = it % kRing;
+            if (!warp_wait(&item_full[slot], (it / kRing) & 1, abort_flag)) {
                 raise_error(p, kErrWaitTimeout, abort_flag);
                 break;
             }
@@ -588,22 +620,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t c2 = 0, dzc = 0, pubc = 0, lbc = 0;
         float st[64];
         const size_t blk = (size_t)DQ * 64;
+        int pending = -1;
         for (int it = 0;; ++it) {
-            const int slot = it & 1;
-            if (!warp_wait(&item_full[slot], (it >> 1) & 1, abort_flag)) {
+            const int slot = it % kRing;
+            if (!warp_wait(&item_full[slot], (it / kRing) & 1, abort_flag)) {
                 raise_error(p, kErrWaitTimeout, abort_flag);
                 break;
             }
-            const int item = item_slot[slot];
+            const int new_item = item_slot[slot];
             __syncwarp();
             if (lane == 0) mbar_arrive(&item_empty[slot]);
-            if (item < 0) break;
-            const Item I = decode_item(item, p);
             bool ok = true;
-            // Publish this item's look-back status once every active state thread's
+            // Publish an item's look-back status once every active state thread's
             // rows are globally visible: all arrive and all wait (a full barrier),
             // then the leader releases the flag.
-            auto publish = [&](unsigned int flag) -> bool {
+            auto publish = [&](int item, unsigned int flag) -> bool {
                 __threadfence();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(z_pub);
@@ -616,174 +647,201 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (leader) st_release_gpu(p.flags + item, flag);
                 return true;
             };
-            // ---- phase 1: this segment's aggregate sum_{s in seg} k_s v_s^T.  The
-            // first segment's aggregate is already its inclusive prefix (flag 2);
-            // later segments publish the aggregate (flag 1) and look back.
-            if (I.phase1) {
-                const uint32_t b = dzc & 1;
-                if (!warp_wait(&dz_full[b], (dzc >> 1) & 1, abort_flag)) {
-                    raise_error(p, kErrWaitTimeout, abort_flag);
-                    break;
-                }
-                tc_fence_after();
-                if (active) {
-                    float* dst = (I.k == 0 ? p.incl : p.agg) + (size_t)item * blk + (size_t)row * 64;
-                    float a[32];
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        tmem_ld32(tmem + col_dz(b) + lane_off + h * 32, a);
-#pragma unroll
-                        for (int i = 0; i < 32; i += 4)
-                            *reinterpret_cast<float4*>(dst + h * 32 + i) =
-                                make_float4(a[i], a[i + 1], a[i + 2], a[i + 3]);
-                    }
-                }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&dz_free[b]);
-                ++dzc;
-                if (active && !publish(I.k == 0 ? 2u : 1u)) break;
-            }
-            // ---- look-back: E = sum of the earlier segments' aggregates, stopping at
-            // the nearest inclusive prefix.  The leader walks the flags; one broadcast
-            // (count << 1 | ends-at-inclusive) tells every state thread what to sum.
-#pragma unroll
-            for (int i = 0; i < 64; ++i) st[i] = 0.0f;
-            if (active && I.k > 0) {
-                if (leader) {
-                    unsigned int word = 0xFFFFFFFFu;
-                    unsigned int cnt = 0;
-                    const uint64_t t0 = globaltimer_ns();
-                    bool timed_out = false;
-                    for (int pred = item - 1, kk = I.k - 1; kk >= 0 && !timed_out; --pred, --kk) {
-                        unsigned int f;
-                        while ((f = ld_acquire_gpu(p.flags + pred)) == 0u) {
-                            if (globaltimer_ns() - t0 > kWaitLimitNs) {
-                                timed_out = true;
-                                break;
-                            }
-                            __nanosleep(64);
-                        }
-                        if (timed_out) break;
-                        ++cnt;
-                        if (f == 2u) {
-                            word = (cnt << 1) | 1u;
-                            break;
-                        }
-                    }
-                    if (timed_out) {
-                        word = 0xFFFFFFFFu;
-                        raise_error(p, kErrLookbackTimeout, nullptr);
-                    }
-                    // the previous broadcast has been read by every state thread
-                    if (!mbar_wait(z_ack, (lbc & 1) ^ 1, abort_flag))
-                        raise_error(p, kErrWaitTimeout, abort_flag);
-                    *lb_word = word;
-                    mbar_arrive(z_lb);
-                }
-                if (!warp_wait(z_lb, lbc & 1, abort_flag)) {
-                    raise_error(p, kErrWaitTimeout, abort_flag);
-                    break;
-                }
-                const unsigned int word = *lb_word;
-                __syncwarp();
-                if (lane == 0) mbar_arrive(z_ack);
-                ++lbc;
-                if (word != 0xFFFFFFFFu) {
-                    const int cnt = static_cast<int>(word >> 1);
-                    const bool ends_incl = (word & 1u) != 0;
-                    __threadfence();
-                    for (int i = 0; i < cnt; ++i) {
-                        const int pred = item - 1 - i;
-                        const float* src = ((i == cnt - 1 && ends_incl) ? p.incl : p.agg) +
-                                           (size_t)pred * blk + (size_t)row * 64;
-#pragma unroll
-                        for (int e4 = 0; e4 < 64; e4 += 4) {
-                            float4 a = __ldcg(reinterpret_cast<const float4*>(src + e4));
-                            st[e4] += a.x;
-                            st[e4 + 1] += a.y;
-                            st[e4 + 2] += a.z;
-                            st[e4 + 3] += a.w;
-                        }
-                    }
-                }
-            }
-            // ---- publish the inclusive prefix E + aggregate (flag 2)
-            if (active && I.phase1 && I.k > 0) {
-                const float* own = p.agg + (size_t)item * blk + (size_t)row * 64;
-                float* dst = p.incl + (size_t)item * blk + (size_t)row * 64;
-#pragma unroll
-                for (int i = 0; i < 64; i += 4) {
-                    float4 a = __ldcg(reinterpret_cast<const float4*>(own + i));
-                    *reinterpret_cast<float4*>(dst + i) =
-                        make_float4(st[i] + a.x, st[i + 1] + a.y, st[i + 2] + a.z, st[i + 3] + a.w);
-                }
-                if (!publish(2u)) break;
-            }
-            // ---- starting state S^T row = B0^T row - eta * E
-            if (active) {
-                const float* w0 = p.W0 + (size_t)(I.l * p.H + I.h) * p.dq * p.dv;
-                const int v0 = I.j * 64;
-                if (p.w0_transposed) {
-                    const float* r = w0 + (size_t)row * p.dv + v0;  // W0 [dq][dv]
-#pragma unroll
-                    for (int i = 0; i < 64; i += 4) {
-                        float4 a = *reinterpret_cast<const float4*>(r + i);
-                        st[i] = a.x - eta * st[i];
-                        st[i + 1] = a.y - eta * st[i + 1];
-                        st[i + 2] = a.z - eta * st[i + 2];
-                        st[i + 3] = a.w - eta * st[i + 3];
-                    }
-                } else {
-#pragma unroll
-                    for (int i = 0; i < 64; ++i)  // W0 [dv][dq]: column `row`
-                        st[i] = w0[(size_t)(v0 + i) * p.dq + row] - eta * st[i];
-                }
-            }
-            // ---- phase 2: S^T tile for every chunk, state advanced by dZ
-            for (int c = 0; c < I.nch; ++c, ++c2) {
-                const uint32_t sb = c2 & 1;
-                if (!warp_wait(&st_free[sb], ((c2 >> 1) & 1) ^ 1, abort_flag)) {
-                    raise_error(p, kErrWaitTimeout, abort_flag);
-                    ok = false;
-                    break;
-                }
-                if (active) {
-                    const uint32_t tile = sbase + Lay::kStOff + sb * Lay::kStBytes;
-#pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        st_shared_v4(tile + sw128_off(row, q), pack_bf16x2(st[8 * q], st[8 * q + 1]),
-                                     pack_bf16x2(st[8 * q + 2], st[8 * q + 3]),
-                                     pack_bf16x2(st[8 * q + 4], st[8 * q + 5]),
-                                     pack_bf16x2(st[8 * q + 6], st[8 * q + 7]));
-                    fence_proxy_async_smem();
-                }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&st_ready[sb]);
-                if (c < I.nch - 1) {
+            // ---- phase 1 of the newly taken item (before phase 2 of the previous one)
+            if (new_item >= 0) {
+                const int item = new_item;
+                const Item I = decode_item(item, p);
+                // ---- phase 1: this segment's aggregate sum_{s in seg} k_s v_s^T.  The
+                // first segment's aggregate is already its inclusive prefix (flag 2);
+                // later segments publish the aggregate (flag 1) and look back.
+                if (I.phase1) {
                     const uint32_t b = dzc & 1;
                     if (!warp_wait(&dz_full[b], (dzc >> 1) & 1, abort_flag)) {
                         raise_error(p, kErrWaitTimeout, abort_flag);
-                        ok = false;
                         break;
                     }
                     tc_fence_after();
                     if (active) {
+                        float* dst = (I.k == 0 ? p.incl : p.agg) + (size_t)item * blk + (size_t)row * 64;
                         float a[32];
-#pragma unroll
+    #pragma unroll
                         for (int h = 0; h < 2; ++h) {
                             tmem_ld32(tmem + col_dz(b) + lane_off + h * 32, a);
-#pragma unroll
-                            for (int i = 0; i < 32; ++i) st[h * 32 + i] -= eta * a[i];
+    #pragma unroll
+                            for (int i = 0; i < 32; i += 4)
+                                *reinterpret_cast<float4*>(dst + h * 32 + i) =
+                                    make_float4(a[i], a[i + 1], a[i + 2], a[i + 3]);
                         }
                     }
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&dz_free[b]);
                     ++dzc;
+                    if (active && !publish(item, I.k == 0 ? 2u : 1u)) break;
+                }
+            }
+            // ---- look-back and phase 2 of the previous item
+            if (pending >= 0) {
+                const int item = pending;
+                const Item I = decode_item(item, p);
+                // ---- look-back: E = sum of the earlier segments' aggregates, stopping at
+                // the nearest inclusive prefix.  The lead state warp polls up to 32
+                // predecessor flags at once (lane i: segment k-1-i) and a ballot finds
+                // the nearest inclusive prefix; one broadcast (count << 1 |
+                // ends-at-inclusive) tells every state thread what to sum.
+#pragma unroll
+                for (int i = 0; i < 64; ++i) st[i] = 0.0f;
+                if (active && I.k > 0) {
+                    if (q4 == 0) {
+                        int total = 0, base_pred = item - 1, remaining = I.k;
+                        bool found = false, timed_out = false;
+                        const uint64_t t0 = globaltimer_ns();
+                        while (!found && !timed_out && remaining > 0) {
+                            const int n = remaining < 32 ? remaining : 32;
+                            unsigned int f = 1u;
+                            if (lane < n) {
+                                while ((f = ld_acquire_gpu(p.flags + (base_pred - lane))) == 0u) {
+                                    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                                        f = 0xFFFFFFFFu;
+                                        break;
+                                    }
+                                    __nanosleep(32);
+                                }
+                            }
+                            if (__ballot_sync(0xffffffffu, f == 0xFFFFFFFFu)) {
+                                timed_out = true;
+                                break;
+                            }
+                            const unsigned int incl = __ballot_sync(0xffffffffu, lane < n && f == 2u);
+                            if (incl) {
+                                total += __ffs(incl);  // up to and including the nearest inclusive
+                                found = true;
+                            } else {
+                                total += n;
+                                base_pred -= n;
+                                remaining -= n;
+                            }
+                        }
+                        if (lane == 0) {
+                            unsigned int word = ((unsigned int)total << 1) | (found ? 1u : 0u);
+                            if (timed_out) {
+                                word = 0xFFFFFFFFu;
+                                raise_error(p, kErrLookbackTimeout, nullptr);
+                            }
+                            // the previous broadcast has been read by every state thread
+                            if (!mbar_wait(z_ack, (lbc & 1) ^ 1, abort_flag))
+                                raise_error(p, kErrWaitTimeout, abort_flag);
+                            *lb_word = word;
+                            mbar_arrive(z_lb);
+                        }
+                        __syncwarp();
+                    }
+                    if (!warp_wait(z_lb, lbc & 1, abort_flag)) {
+                        raise_error(p, kErrWaitTimeout, abort_flag);
+                        break;
+                    }
+                    const unsigned int word = *lb_word;
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(z_ack);
+                    ++lbc;
+                    if (word != 0xFFFFFFFFu) {
+                        const int cnt = static_cast<int>(word >> 1);
+                        const bool ends_incl = (word & 1u) != 0;
+                        __threadfence();
+                        for (int i = 0; i < cnt; ++i) {
+                            const int pred = item - 1 - i;
+                            const float* src = ((i == cnt - 1 && ends_incl) ? p.incl : p.agg) +
+                                               (size_t)pred * blk + (size_t)row * 64;
+    #pragma unroll
+                            for (int e4 = 0; e4 < 64; e4 += 4) {
+                                float4 a = __ldcg(reinterpret_cast<const float4*>(src + e4));
+                                st[e4] += a.x;
+                                st[e4 + 1] += a.y;
+                                st[e4 + 2] += a.z;
+                                st[e4 + 3] += a.w;
+                            }
+                        }
+                    }
+                }
+                // ---- publish the inclusive prefix E + aggregate (flag 2)
+                if (active && I.phase1 && I.k > 0) {
+                    const float* own = p.agg + (size_t)item * blk + (size_t)row * 64;
+                    float* dst = p.incl + (size_t)item * blk + (size_t)row * 64;
+    #pragma unroll
+                    for (int i = 0; i < 64; i += 4) {
+                        float4 a = __ldcg(reinterpret_cast<const float4*>(own + i));
+                        *reinterpret_cast<float4*>(dst + i) =
+                            make_float4(st[i] + a.x, st[i + 1] + a.y, st[i + 2] + a.z, st[i + 3] + a.w);
+                    }
+                    if (!publish(item, 2u)) break;
+                }
+                // ---- starting state S^T row = B0^T row - eta * E
+                if (active) {
+                    const float* w0 = p.W0 + (size_t)(I.l * p.H + I.h) * p.dq * p.dv;
+                    const int v0 = I.j * 64;
+                    if (p.w0_transposed) {
+                        const float* r = w0 + (size_t)row * p.dv + v0;  // W0 [dq][dv]
+    #pragma unroll
+                        for (int i = 0; i < 64; i += 4) {
+                            float4 a = *reinterpret_cast<const float4*>(r + i);
+                            st[i] = a.x - eta * st[i];
+                            st[i + 1] = a.y - eta * st[i + 1];
+                            st[i + 2] = a.z - eta * st[i + 2];
+                            st[i + 3] = a.w - eta * st[i + 3];
+                        }
+                    } else {
+    #pragma unroll
+                        for (int i = 0; i < 64; ++i)  // W0 [dv][dq]: column `row`
+                            st[i] = w0[(size_t)(v0 + i) * p.dq + row] - eta * st[i];
+                    }
+                }
+                // ---- phase 2: S^T tile for every chunk, state advanced by dZ
+                for (int c = 0; c < I.nch; ++c, ++c2) {
+                    const uint32_t sb = c2 & 1;
+                    if (!warp_wait(&st_free[sb], ((c2 >> 1) & 1) ^ 1, abort_flag)) {
+                        raise_error(p, kErrWaitTimeout, abort_flag);
+                        ok = false;
+                        break;
+                    }
+                    if (active) {
+                        const uint32_t tile = sbase + Lay::kStOff + sb * Lay::kStBytes;
+    #pragma unroll
+                        for (int q = 0; q < 8; ++q)
+                            st_shared_v4(tile + sw128_off(row, q), pack_bf16x2(st[8 * q], st[8 * q + 1]),
+                                         pack_bf16x2(st[8 * q + 2], st[8 * q + 3]),
+                                         pack_bf16x2(st[8 * q + 4], st[8 * q + 5]),
+                                         pack_bf16x2(st[8 * q + 6], st[8 * q + 7]));
+                        fence_proxy_async_smem();
+                    }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&st_ready[sb]);
+                    if (c < I.nch - 1) {
+                        const uint32_t b = dzc & 1;
+                        if (!warp_wait(&dz_full[b], (dzc >> 1) & 1, abort_flag)) {
+                            raise_error(p, kErrWaitTimeout, abort_flag);
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        if (active) {
+                            float a[32];
+    #pragma unroll
+                            for (int h = 0; h < 2; ++h) {
+                                tmem_ld32(tmem + col_dz(b) + lane_off + h * 32, a);
+    #pragma unroll
+                                for (int i = 0; i < 32; ++i) st[h * 32 + i] -= eta * a[i];
+                            }
+                        }
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&dz_free[b]);
+                        ++dzc;
+                    }
                 }
             }
             if (!ok) break;
+            pending = new_item;
+            if (new_item < 0) break;
         }
         }
     }
