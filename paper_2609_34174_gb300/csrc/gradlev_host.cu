@@ -18,6 +18,9 @@ cudaError_t launch_tc_scan(const CUtensorMap& q, const CUtensorMap& k, const CUt
                            const CUtensorMap& o, const TcScanParams& p, bool costate, int grid,
                            cudaStream_t stream);
 cudaError_t launch_simt_scan(const SimtScanParams& p, bool bf16, cudaStream_t stream);
+cudaError_t launch_seg_gemm(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b,
+                            const CUtensorMap& a2, const CUtensorMap& b2, const SegGemmParams& p,
+                            int grid, cudaStream_t stream);
 size_t simt_smem_bytes(int dq);
 }  // namespace gl
 
@@ -133,7 +136,7 @@ Plan plan_tc(const gradlev_desc& d, int dq, int dv, int sms) {
     Plan pl;
     pl.n_tiles = dv / 64;
     const long long units = (long long)d.L * d.B * d.H * pl.n_tiles;
-    const long long target = 4ll * (sms > 0 ? sms : 148);
+    const long long target = 2ll * (sms > 0 ? sms : 148);
     int n_seg = 1;
     if (units < target && d.T > 1024) {
         long long want = (target + units - 1) / units;
@@ -183,7 +186,7 @@ bool desc_ok(const gradlev_desc* d) {
     return true;
 }
 
-bool make_tmap(CUtensorMap* m, const gradlev_desc& d, const Tok& t, int width) {
+bool make_tmap(CUtensorMap* m, const gradlev_desc& d, const Tok& t, int width, int box_t = kChunk) {
     EncodeTiledFn enc = encode_fn();
     if (!enc) return false;
     const cuuint64_t dims[5] = {(cuuint64_t)width, (cuuint64_t)d.H, (cuuint64_t)d.T, (cuuint64_t)d.B,
@@ -197,12 +200,57 @@ bool make_tmap(CUtensorMap* m, const gradlev_desc& d, const Tok& t, int width) {
         if (sizes[i] == 1 && b == 0) b = 16;
         strides[i] = (cuuint64_t)b;
     }
-    const cuuint32_t box[5] = {64, 1, (cuuint32_t)kChunk, 1, 1};
+    const cuuint32_t box[5] = {64, 1, (cuuint32_t)box_t, 1, 1};
     const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
     CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, t.data, dims, strides, box, estr,
                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
+}
+
+// 3-D bf16 map over a contiguous workspace tensor [n2][n1][n0] with a {64, box1, 1} box.
+bool make_tmap_3d(CUtensorMap* m, void* base, long long n0, long long n1, long long n2, int box1) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    const cuuint64_t dims[3] = {(cuuint64_t)n0, (cuuint64_t)n1, (cuuint64_t)n2};
+    const cuuint64_t strides[2] = {(cuuint64_t)(n0 * 2), (cuuint64_t)(n0 * n1 * 2)};
+    const cuuint32_t box[3] = {64, (cuuint32_t)box1, 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+// Wide layers (dq a multiple of 128 and at least 256): the scan split at segment
+// boundaries into a state pass, a score pass and an output pass (seg_gemm_tc.cu).
+struct SegPlan {
+    int seg_len = 0, n_seg = 0, bn = 0;
+    long long tiles_state = 0, tiles_score = 0, tiles_out = 0;
+    size_t off_sbuf = 0, off_pbuf = 0, ws_bytes = 0;
+};
+
+bool seg_shape_ok(const gradlev_desc& d, int dq, int dv) {
+    return d.dtype == GRADLEV_BF16 && dq >= 256 && dq % 128 == 0 && dv % 64 == 0 && dv > 0;
+}
+
+SegPlan plan_seg(const gradlev_desc& d, int dq, int dv) {
+    SegPlan sp;
+    const long long T = d.T > 0 ? d.T : 1;
+    long long ls = (T + kChunk - 1) / kChunk * kChunk;
+    if (ls > 512) ls = 512;
+    sp.seg_len = (int)ls;
+    sp.n_seg = (int)((T + ls - 1) / ls);
+    sp.bn = dv % 256 == 0 ? 256 : (dv % 128 == 0 ? 128 : 64);
+    const long long U = (long long)d.L * d.B * d.H;
+    const long long R = ls / kChunk;
+    sp.tiles_state = U * (dq / 128) * (dv / sp.bn);
+    sp.tiles_score = U * sp.n_seg * (R * (R + 1) / 2);
+    sp.tiles_out = U * sp.n_seg * R * (dv / sp.bn);
+    sp.off_sbuf = 1024;
+    sp.off_pbuf = round_up(sp.off_sbuf + (size_t)U * sp.n_seg * dq * dv * 2, 1024);
+    sp.ws_bytes = sp.off_pbuf + (size_t)U * sp.n_seg * ls * ls * 2;
+    return sp;
 }
 
 void fill_epi(gl::EpiParams* e, const Tok& out, const Tok& out2, const Tok& z, int act) {
@@ -289,6 +337,58 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
             return GRADLEV_ERR_CUDA;
         return GRADLEV_OK;
     }
+    if (seg_shape_ok(d, dq, dv) && tc_layout_ok(tq, 2) && tc_layout_ok(tk, 2) &&
+        tc_layout_ok(tv, 2) && tc_layout_ok(to, 2) && tc_layout_ok(to2, 2) && tc_layout_ok(tz, 2)) {
+        SegPlan sp = plan_seg(d, dq, dv);
+        const long long lim = 0x7fffffffll;
+        if (sp.tiles_state > lim || sp.tiles_score > lim || sp.tiles_out > lim ||
+            (long long)d.L * d.B * d.H * sp.n_seg > lim)
+            return GRADLEV_ERR_UNSUPPORTED;
+        if (!ws || ws_bytes < sp.ws_bytes) return GRADLEV_ERR_WORKSPACE;
+        if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return GRADLEV_ERR_WORKSPACE;
+        if (!aligned16(W0)) return GRADLEV_ERR_INVALID_ARG;
+        uint8_t* wsb = static_cast<uint8_t*>(ws);
+        const long long us = (long long)d.L * d.B * d.H * sp.n_seg;
+        CUtensorMap mq, mk, mk64, mv64, msb, mpb;
+        if (!make_tmap(&mq, d, tq, dq) || !make_tmap(&mk, d, tk, dq) ||
+            !make_tmap(&mk64, d, tk, dq, 64) || !make_tmap(&mv64, d, tv, dv, 64) ||
+            !make_tmap_3d(&msb, wsb + sp.off_sbuf, dv, dq, us, 64) ||
+            !make_tmap_3d(&mpb, wsb + sp.off_pbuf, sp.seg_len, sp.seg_len, us, kChunk))
+            return GRADLEV_ERR_UNSUPPORTED;
+        gl::SegGemmParams p;
+        memset(&p, 0, sizeof(p));
+        p.L = d.L;
+        p.B = d.B;
+        p.T = d.T;
+        p.H = d.H;
+        p.dq = dq;
+        p.dv = dv;
+        p.seg_len = sp.seg_len;
+        p.n_seg = sp.n_seg;
+        p.eta = eta;
+        p.w0_transposed = costate ? 1 : 0;
+        p.W0 = W0;
+        p.sbuf = reinterpret_cast<__nv_bfloat16*>(wsb + sp.off_sbuf);
+        p.pbuf = reinterpret_cast<__nv_bfloat16*>(wsb + sp.off_pbuf);
+        fill_epi(&p.epi, to, to2, tz, act);
+        p.ctrl = reinterpret_cast<unsigned int*>(wsb);
+        if (cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
+        const long long tiles[3] = {sp.tiles_state, sp.tiles_score, sp.tiles_out};
+        for (int mode = 0; mode < 3; ++mode) {
+            p.n_tiles = (int)tiles[mode];
+            const int grid = p.n_tiles < dev.sms ? p.n_tiles : dev.sms;
+            if (grid < 1) continue;
+            cudaError_t e;
+            if (mode == 0)
+                e = gl::launch_seg_gemm(0, sp.bn, mk64, mv64, mk64, mv64, p, grid, stream);
+            else if (mode == 1)
+                e = gl::launch_seg_gemm(1, sp.bn, mq, mk, mq, mk, p, grid, stream);
+            else
+                e = gl::launch_seg_gemm(2, sp.bn, mq, msb, mpb, mv64, p, grid, stream);
+            if (e != cudaSuccess) return GRADLEV_ERR_CUDA;
+        }
+        return GRADLEV_OK;
+    }
     if (simt_shape_ok(d, dq)) {
         // CUDA-core path: fp32 (exact fp32 FMA), or bf16 shapes the tensor-core
         // tiling does not cover.  Needs only element alignment.
@@ -334,6 +434,9 @@ size_t ws_bytes_for(const gradlev_desc& d, int dq, int dv, int sms) {
     if (tc_shape_ok(d, dq, dv)) {
         Plan pl = plan_tc(d, dq, dv, sms);
         if (pl.ws_bytes > b) b = pl.ws_bytes;
+    } else if (seg_shape_ok(d, dq, dv)) {
+        SegPlan sp = plan_seg(d, dq, dv);
+        if (sp.ws_bytes > b) b = sp.ws_bytes;
     }
     return b;
 }

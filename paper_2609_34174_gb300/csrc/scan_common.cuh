@@ -87,6 +87,23 @@ struct TcScanParams {
     float* incl;          // [n_items][dq][64] inclusive prefix of the aggregates
 };
 
+// Parameters of the wide-layer passes (bf16, dq % 128 == 0, dv % 64 == 0): the
+// scan split at segment boundaries into three GEMM-shaped passes.
+struct SegGemmParams {
+    int L, B, T, H;
+    int dq, dv;
+    int seg_len;             // Ls, tokens per segment (multiple of 128)
+    int n_seg;               // segments per unit
+    int n_tiles;             // output tiles of the pass being launched
+    float eta;
+    int w0_transposed;       // as in TcScanParams
+    const float* W0;
+    __nv_bfloat16* sbuf;     // [U][n_seg][dq][dv]  S_k^T at every segment start
+    __nv_bfloat16* pbuf;     // [U][n_seg][Ls][Ls]  -eta * strict_lower(Q_k K_k^T)
+    EpiParams epi;
+    unsigned int* ctrl;      // [1] error bits
+};
+
 // Parameters of the fp32 SIMT scan kernel.
 struct SimtScanParams {
     int L, B, T, H;

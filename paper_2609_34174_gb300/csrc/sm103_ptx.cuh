@@ -97,6 +97,16 @@ __device__ __forceinline__ void tma_load_5d(void* dst, const void* tmap, uint64_
         : "memory");
 }
 
+// 3-D tiled load global -> shared (workspace tensors), completing on `bar`.
+__device__ __forceinline__ void tma_load_3d(void* dst, const void* tmap, uint64_t* bar, int c0,
+                                            int c1, int c2) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
+        : "memory");
+}
+
 // 5-D tiled store shared -> global of a TMA box (out-of-range rows are clipped),
 // tracked by the issuing thread's bulk async-group.
 __device__ __forceinline__ void tma_store_5d(const void* tmap, const void* src, int c0, int c1,
