@@ -5,7 +5,9 @@ One step = the forward scan (Sec. 3 step 2, Eq. 3) and the costate scan
 (Sec. 3 step 3, Eq. 4) over one batch of the workload, through the library's
 C ABI.  Default workload: the model-shaped layer sweep (12 independent layers
 x 12 heads of 64x64 fast weights, B=8, T=8192, bf16), all layers' forward and
-costate scans per step.
+costate scans per step.  `--workload c3` runs the two-layer MLP of Appendix A
+(512 -> 2048 -> 512, GELU): forward through both layers, then costates back
+through both.
 
 Prints ONE JSON line on rank 0.  `value` is tokens/s of the whole step
 (L*B*T tokens per step, both scans) with inputs resident in HBM; `scans`
@@ -53,24 +55,6 @@ def peaks():
     except Exception:
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
                 "source": "fallback"}
-
-
-# ------------------------------------------------------------- scan accounting
-def scan_counts(wl, scan: str):
-    """Algorithmic flops and compulsory bytes of one scan call over the workload.
-
-    Per token and unit (one head of one layer): flops 4*d*m + C*(d+m) with C = 64
-    (state read 2dm, state update 2dm, causal halves of the two CxC products);
-    bytes e*(d + 2m) forward (x, ghat in; y out), e*(2d + 2m) costate (x, ghat,
-    g_out in; g_in out), plus 4*d*m per slow matrix W0.
-    """
-    e = 2 if wl.dtype == "bf16" else 4
-    d, m = wl.d_in, wl.d_out
-    tu = wl.L * wl.B * wl.T * wl.H
-    flops = tu * (4 * d * m + COUNT_CHUNK * (d + m))
-    per_tok = e * (d + 2 * m) if scan == "fwd" else e * (2 * d + 2 * m)
-    nbytes = tu * per_tok + 4 * d * m * wl.L * wl.H
-    return flops, nbytes
 
 
 def roofline_entry(flops, nbytes, seconds, pk):
@@ -155,71 +139,225 @@ class ClockSampler:
         return out
 
 
-# ------------------------------------------------------------------ workload
-def linear_inputs(wl, device, rank):
-    return W.make_linear(wl.resized(seed=wl.seed + 1000 * rank), device=device)
+# ------------------------------------------------------------------ workloads
+def _bytes(*ts):
+    return sum(t.numel() * t.element_size() for t in ts)
 
 
-def run_step(gl, inp, wl, outs, events=None):
-    if events is not None:
-        events[0].record()
-    gl.forward_scan(inp["x"], inp["g_hat"], inp["W0"], wl.eta, y=outs["y"],
-                    workspace=outs["ws"])
-    if events is not None:
-        events[1].record()
-    gl.costate_scan(inp["x"], inp["g_hat"], inp["W0"], wl.eta, inp["g_out"], g_in=outs["g_in"],
-                    workspace=outs["ws"])
-    if events is not None:
-        events[2].record()
+class LinearJob:
+    """One fast-weight linear map per (layer, batch, head) unit: the forward scan
+    (Eq. 3) and the costate scan (Eq. 4), one library call each."""
 
+    kind = "linear"
 
-def cpu_baseline(wl, inp, target_s=12.0):
-    """The fp64 oracle (as it stands) on a bounded sample of units, all host cores."""
-    import oracle
+    def __init__(self, gl, wl, device, rank):
+        self.gl, self.wl = gl, wl
+        self.inp = W.make_linear(wl.resized(seed=wl.seed + 1000 * rank), device=device)
+        self.outs = {"y": torch.empty_like(self.inp["g_hat"]),
+                     "g_in": torch.empty_like(self.inp["x"])}
+        self.ws = torch.empty(max(256, gl.workspace_bytes(wl.L, wl.B, wl.T, wl.H, wl.d_in,
+                                                          wl.d_out, 1 if wl.dtype == "bf16" else 0)),
+                              dtype=torch.uint8, device=device)
+        self.tokens = wl.tokens
+        self.launches_per_step = 2
+        self.in_keys = ("x", "g_hat", "g_out", "W0")
+        self.out_keys = ("y", "g_in")
+        self.kernel = {"fwd": "tc_scan_kernel<64, false> (forward scan)",
+                       "costate": "tc_scan_kernel<64, true> (costate scan)"}
 
-    cores = len(os.sched_getaffinity(0))
-    units_all = [(l, b, h) for l in range(wl.L) for b in range(wl.B) for h in range(wl.H)]
+    def input_bytes(self):
+        return _bytes(self.inp["x"], self.inp["g_hat"], self.inp["g_out"])
 
-    def run(units):
+    def step(self, inp=None, events=None):
+        gl, wl, o = self.gl, self.wl, self.outs
+        inp = inp or self.inp
+        if events is not None:
+            events[0].record()
+        gl.forward_scan(inp["x"], inp["g_hat"], inp["W0"], wl.eta, y=o["y"], workspace=self.ws)
+        if events is not None:
+            events[1].record()
+        gl.costate_scan(inp["x"], inp["g_hat"], inp["W0"], wl.eta, inp["g_out"], g_in=o["g_in"],
+                        workspace=self.ws)
+        if events is not None:
+            events[2].record()
+
+    def counts(self, scan):
+        """Algorithmic flops and compulsory bytes of one scan call.
+
+        Per token and unit: flops 4*d*m + C*(d+m) with C = 64 (state read 2dm,
+        state update 2dm, causal halves of the two CxC products); bytes
+        e*(d + 2m) forward (x, ghat in; y out), e*(2d + 2m) costate (x, ghat,
+        g_out in; g_in out), plus 4*d*m per slow matrix W0.
+        """
+        wl = self.wl
+        e = 2 if wl.dtype == "bf16" else 4
+        d, m = wl.d_in, wl.d_out
+        tu = wl.L * wl.B * wl.T * wl.H
+        flops = tu * (4 * d * m + COUNT_CHUNK * (d + m))
+        per_tok = e * (d + 2 * m) if scan == "fwd" else e * (2 * d + 2 * m)
+        return flops, tu * per_tok + 4 * d * m * wl.L * wl.H
+
+    def config(self):
+        wl = self.wl
+        return {"L": wl.L, "B": wl.B, "T": wl.T, "H": wl.H, "d_in": wl.d_in, "d_out": wl.d_out,
+                "eta": wl.eta}
+
+    def oracle_run(self, inp, n_units, cores, t_tokens=None):
+        """Time the fp64 oracle on the first n_units units (forward and costate
+        reads in one sequential walk per unit); returns (seconds, metric tokens)."""
+        import oracle
+        wl = self.wl
+        units = [(l, b, h) for l in range(wl.L) for b in range(wl.B) for h in range(wl.H)]
+        units = units[:n_units]
         x = W.units_fp64(inp["x"], units)
         g = W.units_fp64(inp["g_hat"], units)
         w0 = W.w0_fp64(inp["W0"], units)
         go = W.units_fp64(inp["g_out"], units)
         t = time.perf_counter()
         oracle.linear_scan(x, g, w0, wl.eta, gout=go, nthreads=cores)
-        return time.perf_counter() - t
+        # one metric token spans all H heads of a layer
+        return time.perf_counter() - t, len(units) * wl.T / wl.H
 
-    # calibrate with one unit per core, then size the sample for ~target_s
-    n0 = min(len(units_all), cores)
-    dt0 = run(units_all[:n0])
-    per_unit = dt0 / n0
-    n = int(max(n0, min(len(units_all), target_s / max(per_unit, 1e-9))))
-    n = max(cores, n // cores * cores) if n >= cores else n
-    n = min(n, len(units_all))
-    dt = run(units_all[:n])
-    # metric tokens: one token spans all H heads of a layer, so a unit-token is 1/H token
-    tokens = n * wl.T / wl.H
+    def n_units(self):
+        return self.wl.L * self.wl.B * self.wl.H
+
+    def sample_text(self, n):
+        return (f"{n} of {self.n_units()} (layer, batch, head) units at full T={self.wl.T}, "
+                f"forward and costate reads in one sequential walk per unit, fp64")
+
+
+class MLPJob:
+    """The two-layer fast-weight MLP of Appendix A: forward through both layers
+    (sigma fused in the layer-1 epilogue), then costates back through both
+    (sigma' fused in the layer-2 costate epilogue)."""
+
+    kind = "mlp"
+
+    def __init__(self, gl, wl, device, rank):
+        self.gl, self.wl = gl, wl
+        self.inp = W.make_mlp(wl.resized(seed=wl.seed + 1000 * rank), device=device)
+        B, T, d, m, k = wl.B, wl.T, wl.d, wl.m, wl.k
+        dt = self.inp["x"].dtype
+        mk = lambda w: torch.empty((B, T, w), dtype=dt, device=device)
+        self.outs = {"z": mk(m), "h": mk(m), "y": mk(k), "gz": mk(m), "gx": mk(d)}
+        code = 1 if wl.dtype == "bf16" else 0
+        nb = max(gl.workspace_bytes(1, B, T, 1, d, m, code), gl.workspace_bytes(1, B, T, 1, m, k, code))
+        self.ws = torch.empty(max(256, nb), dtype=torch.uint8, device=device)
+        self.tokens = wl.tokens
+        # forward: two layers x (state, score, output pass); the same for the costate
+        self.launches_per_step = 12
+        self.in_keys = ("x", "g_hat_z", "g_hat_y", "g_out", "W1", "W2")
+        self.out_keys = ("y", "gx")
+        self.kernel = {"fwd": "seg_gemm_kernel state/score/output passes (forward, both layers)",
+                       "costate": "seg_gemm_kernel state/score/output passes (costate, both layers)"}
+
+    def input_bytes(self):
+        return _bytes(self.inp["x"], self.inp["g_hat_z"], self.inp["g_hat_y"], self.inp["g_out"])
+
+    def step(self, inp=None, events=None):
+        gl, wl, o = self.gl, self.wl, self.outs
+        inp = inp or self.inp
+        if events is not None:
+            events[0].record()
+        gl.forward_scan(inp["x"], inp["g_hat_z"], inp["W1"], wl.eta1, act=wl.act, y=o["z"],
+                        act_out=o["h"], workspace=self.ws)
+        gl.forward_scan(o["h"], inp["g_hat_y"], inp["W2"], wl.eta2, y=o["y"], workspace=self.ws)
+        if events is not None:
+            events[1].record()
+        gl.costate_scan(o["h"], inp["g_hat_y"], inp["W2"], wl.eta2, inp["g_out"], act=wl.act,
+                        z=o["z"], g_in=o["gz"], workspace=self.ws)
+        gl.costate_scan(inp["x"], inp["g_hat_z"], inp["W1"], wl.eta1, o["gz"], g_in=o["gx"],
+                        workspace=self.ws)
+        if events is not None:
+            events[2].record()
+
+    def counts(self, scan):
+        """Both layers: flops 4*d_i*m_i + C*(d_i+m_i) per token and layer (C = 64).
+        Compulsory bytes with sigma fused (h is never needed from HBM): forward
+        x, ghat_z in, z out; z, ghat_y in, y out.  Costate g_out, ghat_y, z in,
+        g_z out; g_z, ghat_z, x in, g_x out.  Plus 4*d*m per slow matrix."""
+        wl = self.wl
+        e = 2 if wl.dtype == "bf16" else 4
+        d, m, k = wl.d, wl.m, wl.k
+        n = wl.B * wl.T
+        flops = n * (4 * d * m + COUNT_CHUNK * (d + m) + 4 * m * k + COUNT_CHUNK * (m + k))
+        if scan == "fwd":
+            per_tok = e * ((d + m + m) + (m + k + k))
+        else:
+            per_tok = e * ((k + k + m + m) + (m + m + d + d))
+        return flops, n * per_tok + 4 * (d * m + m * k)
+
+    def config(self):
+        wl = self.wl
+        return {"B": wl.B, "T": wl.T, "widths": [wl.d, wl.m, wl.k], "act": wl.act,
+                "eta": [wl.eta1, wl.eta2]}
+
+    def oracle_run(self, inp, n_units, cores, t_tokens=None):
+        """Time the fp64 MLP oracle on the first n_units sequences, truncated to
+        t_tokens tokens (all reads and writes of both layers in one walk)."""
+        import oracle
+        wl = self.wl
+        T = t_tokens or wl.T
+        f = lambda t: t[:n_units, :T].to(torch.float64).cpu().numpy()
+        args = (f(inp["x"]), f(inp["g_hat_z"]), f(inp["g_hat_y"]),
+                inp["W1"].double().cpu().numpy(), inp["W2"].double().cpu().numpy())
+        t = time.perf_counter()
+        oracle.mlp_scan(*args, wl.eta1, wl.eta2, act=oracle.ACT_GELU_TANH, gout=f(inp["g_out"]),
+                        nthreads=min(cores, n_units))
+        return time.perf_counter() - t, n_units * T
+
+    def n_units(self):
+        return self.wl.B
+
+    def sample_text(self, n, t_tokens=None):
+        return (f"{n} of {self.wl.B} sequences, first {t_tokens or self.wl.T} of {self.wl.T} "
+                f"tokens, both layers forward and costate in one sequential walk, fp64")
+
+
+def make_job(gl, wl, device, rank):
+    return MLPJob(gl, wl, device, rank) if isinstance(wl, W.MLPWorkload) else LinearJob(
+        gl, wl, device, rank)
+
+
+def cpu_baseline(job, inp, target_s=12.0):
+    """The fp64 oracle (as it stands) on a bounded sample of the workload, all host cores."""
+    cores = len(os.sched_getaffinity(0))
+    if job.kind == "mlp":
+        # calibrate on a short prefix of one sequence per core, then grow the prefix
+        n = min(job.n_units(), cores)
+        t_try = 128
+        dt0, _ = job.oracle_run(inp, n, cores, t_try)
+        t_tok = int(min(job.wl.T, max(t_try, t_try * target_s / max(dt0, 1e-9))))
+        dt, tokens = job.oracle_run(inp, n, cores, t_tok)
+        sample = job.sample_text(n, t_tok)
+    else:
+        n0 = min(job.n_units(), cores)
+        dt0, _ = job.oracle_run(inp, n0, cores)
+        per_unit = dt0 / n0
+        n = int(max(n0, min(job.n_units(), target_s / max(per_unit, 1e-9))))
+        n = max(cores, n // cores * cores) if n >= cores else n
+        n = min(n, job.n_units())
+        dt, tokens = job.oracle_run(inp, n, cores)
+        sample = job.sample_text(n)
     return {"value": round(tokens / dt, 1), "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"{n} of {len(units_all)} (layer, batch, head) units at full T={wl.T}, "
-                      f"forward and costate reads in one sequential walk per unit, fp64",
-            "seconds": round(dt, 2)}
+            "sample": sample, "seconds": round(dt, 2)}
 
 
-def e2e_measure(gl, inp, wl, outs, steps, stream):
+def e2e_measure(job, steps, stream):
     """The same step through the public API from pinned host buffers, copies inside."""
-    host = {k: inp[k].cpu().pin_memory() for k in ("x", "g_hat", "g_out", "W0")}
-    hy = torch.empty(outs["y"].shape, dtype=outs["y"].dtype, pin_memory=True)
-    hg = torch.empty(outs["g_in"].shape, dtype=outs["g_in"].dtype, pin_memory=True)
-    dev = {k: torch.empty_like(inp[k]) for k in host}
-    bi = sum(t.numel() * t.element_size() for t in host.values())
-    bo = hy.numel() * hy.element_size() + hg.numel() * hg.element_size()
+    host = {k: job.inp[k].cpu().pin_memory() for k in job.in_keys}
+    dev = {k: torch.empty_like(job.inp[k]) for k in job.in_keys}
+    hout = {k: torch.empty(job.outs[k].shape, dtype=job.outs[k].dtype, pin_memory=True)
+            for k in job.out_keys}
+    bi = _bytes(*host.values())
+    bo = _bytes(*hout.values())
 
     def one():
         for k in host:
             dev[k].copy_(host[k], non_blocking=True)
-        run_step(gl, dev, wl, outs)
-        hy.copy_(outs["y"], non_blocking=True)
-        hg.copy_(outs["g_in"], non_blocking=True)
+        job.step(inp=dev)
+        for k in hout:
+            hout[k].copy_(job.outs[k], non_blocking=True)
 
     one()
     torch.cuda.synchronize()
@@ -230,8 +368,39 @@ def e2e_measure(gl, inp, wl, outs, steps, stream):
     e1.record(stream)
     torch.cuda.synchronize()
     sec = e0.elapsed_time(e1) / 1e3
-    return {"value": round(wl.tokens * steps / sec, 1), "unit": UNIT, "h2d_bytes_per_step": bi,
+    return {"value": round(job.tokens * steps / sec, 1), "unit": UNIT, "h2d_bytes_per_step": bi,
             "d2h_bytes_per_step": bo, "steps": steps, "ms_per_step": round(sec / steps * 1e3, 3)}
+
+
+# ---------------------------------------------------------- DRAM traffic
+TRAFFIC_RECORD = os.path.join(ROOT, "profiles", "dram_traffic.txt")
+KERNEL_SOURCES = ("paper_2609_34174_gb300/csrc/scan_tc.cu", "paper_2609_34174_gb300/csrc/sm103_ptx.cuh",
+                  "paper_2609_34174_gb300/csrc/scan_common.cuh",
+                  "paper_2609_34174_gb300/csrc/gradlev_host.cu")
+
+
+def kernel_source_digest():
+    import hashlib
+    h = hashlib.sha1()
+    for rel in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def recorded_traffic(workload_key, scan):
+    """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of the
+    dominant kernel from the committed ncu record, or None when no record exists
+    for this workload and scan or the kernel sources changed since it was taken."""
+    try:
+        with open(TRAFFIC_RECORD) as f:
+            rec = json.load(f)
+    except Exception:
+        return None
+    if rec.get("kernel_source_sha1") != kernel_source_digest():
+        return None
+    ent = rec.get("entries", {}).get(f"{workload_key}:{scan}")
+    return None if ent is None else int(ent["bytes_per_launch"])
 
 
 # ------------------------------------------------------------------- arms
@@ -242,26 +411,32 @@ def run_reference(args, wl, rank, world):
     import oracle
 
     oracle.build()
-    inp = W.make_linear(wl, device="cpu")
     cores = len(os.sched_getaffinity(0))
-    units_all = [(l, b, h) for l in range(wl.L) for b in range(wl.B) for h in range(wl.H)]
-    n = min(len(units_all), max(cores, 2 * cores))
-    units = units_all[:n]
-    x = W.units_fp64(inp["x"], units)
-    g = W.units_fp64(inp["g_hat"], units)
-    w0 = W.w0_fp64(inp["W0"], units)
-    go = W.units_fp64(inp["g_out"], units)
+    if isinstance(wl, W.MLPWorkload):
+        inp = W.make_mlp(wl, device="cpu")
+        job = MLPJob.__new__(MLPJob)
+        job.wl = wl
+        n = min(wl.B, cores)
+        t_tok = min(wl.T, 256)
+        run = lambda: job.oracle_run(inp, n, cores, t_tok)
+        sample = job.sample_text(n, t_tok) + " per step"
+    else:
+        inp = W.make_linear(wl, device="cpu")
+        job = LinearJob.__new__(LinearJob)
+        job.wl = wl
+        n = min(job.n_units(), max(cores, 2 * cores))
+        run = lambda: job.oracle_run(inp, n, cores)
+        sample = (f"{n} of {job.n_units()} (layer, batch, head) units at full T={wl.T} per step, "
+                  f"fp64 sequential walk")
     for _ in range(args.warmup):
-        oracle.linear_scan(x[:cores], g[:cores], w0[:cores], wl.eta, gout=go[:cores],
-                           nthreads=cores)
-    t = time.perf_counter()
+        run()
+    sec = 0.0
+    tokens = 0.0
     for _ in range(args.steps):
-        oracle.linear_scan(x, g, w0, wl.eta, gout=go, nthreads=cores)
-    sec = time.perf_counter() - t
-    tokens = n * wl.T / wl.H
-    value = tokens * args.steps / sec
-    sample = (f"{n} of {len(units_all)} (layer, batch, head) units at full T={wl.T} per step, "
-              f"fp64 sequential walk")
+        dt, tk = run()
+        sec += dt
+        tokens += tk
+    value = tokens / sec
     return {"impl": "reference", "metric": METRIC, "value": round(value, 1), "unit": UNIT,
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(sec / args.steps * 1e3, 3), "higher_is_better": True,
@@ -279,22 +454,16 @@ def run_gradlev(args, wl, rank, world, local_rank):
     device = torch.device("cuda", local_rank)
     torch.cuda.set_device(device)
     gl.load_library()
-    inp = linear_inputs(wl, device, rank)
-    outs = {"y": torch.empty_like(inp["g_hat"]),
-            "g_in": torch.empty_like(inp["x"]),
-            "ws": torch.empty(max(256, gl.workspace_bytes(wl.L, wl.B, wl.T, wl.H, wl.d_in, wl.d_out,
-                                                          1 if wl.dtype == "bf16" else 0)),
-                              dtype=torch.uint8, device=device)}
-    in_bytes = sum(inp[k].numel() * inp[k].element_size() for k in ("x", "g_hat", "g_out"))
+    job = make_job(gl, wl, device, rank)
     flush = None
-    if in_bytes < 2 * L2_BYTES:
+    if job.input_bytes() < 2 * L2_BYTES:
         flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
     stream = torch.cuda.current_stream(device)
 
     for _ in range(args.warmup):
-        run_step(gl, inp, wl, outs)
+        job.step()
     torch.cuda.synchronize()
-    if gl.workspace_status(outs["ws"]) != 0:
+    if gl.workspace_status(job.ws) != 0:
         raise RuntimeError("device-side timeout reported by the scan kernels")
 
     sampler = ClockSampler(local_rank)
@@ -312,7 +481,7 @@ def run_gradlev(args, wl, rank, world, local_rank):
     for i in range(args.steps):
         if flush is not None:
             flush.zero_()
-        run_step(gl, inp, wl, outs, ev[i])
+        job.step(events=ev[i])
     t_end.record(stream)
     torch.cuda.synchronize()
     sampler.mark()
@@ -320,49 +489,46 @@ def run_gradlev(args, wl, rank, world, local_rank):
         torch.distributed.barrier()
     time.sleep(0.25)
     sampler.stop()
-    if gl.workspace_status(outs["ws"]) != 0:
+    if gl.workspace_status(job.ws) != 0:
         raise RuntimeError("device-side timeout reported by the scan kernels")
 
     total_ms = t_start.elapsed_time(t_end)
     fwd_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / args.steps
     cos_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / args.steps
     step_ms = total_ms / args.steps
+    if flush is not None:
+        # the flush is not part of the step: take the scans' own time
+        step_ms = max(fwd_ms + cos_ms, 1e-9)
     if world > 1:
         t = torch.tensor([step_ms], device=device)
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         step_ms = float(t.item())
-    if flush is not None:
-        # the flush is not part of the step: take the scans' own time
-        step_ms = max(fwd_ms + cos_ms, 1e-9) if world == 1 else step_ms
     pk = peaks()
     scans = {}
     for name, ms in (("fwd", fwd_ms), ("costate", cos_ms)):
-        fl, nb = scan_counts(wl, name)
-        scans[name] = {"ms": round(ms, 4), "tokens_per_s": round(wl.tokens / (ms / 1e3), 1),
+        fl, nb = job.counts(name)
+        scans[name] = {"ms": round(ms, 4), "tokens_per_s": round(job.tokens / (ms / 1e3), 1),
                        "roofline": roofline_entry(fl, nb, ms / 1e3, pk)}
     dominant = "costate" if cos_ms >= fwd_ms else "fwd"
     rl = dict(scans[dominant]["roofline"])
-    rl["kernel"] = f"tc_scan_kernel ({dominant} scan)"
-    rl["traffic"] = None
-    value = world * wl.tokens / (step_ms / 1e3)
+    rl["kernel"] = job.kernel[dominant]
+    rl["traffic"] = None if args.resize else recorded_traffic(args.workload, dominant)
+    value = world * job.tokens / (step_ms / 1e3)
+    cfg = {"workload": f"{args.workload}: {wl.name}", **job.config(),
+           "tokens_per_step": job.tokens, "parallelism": f"replicas x{world}",
+           "l2": "inputs larger than L2" if flush is None else "L2 flushed between steps"}
     line = {"metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms, 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
-            "data": "synthetic",
-            "config": {"workload": f"{args.workload}: {wl.name}", "L": wl.L, "B": wl.B, "T": wl.T,
-                       "H": wl.H, "d_in": wl.d_in, "d_out": wl.d_out, "eta": wl.eta,
-                       "tokens_per_step": wl.tokens, "parallelism": f"replicas x{world}",
-                       "l2": ("inputs larger than L2" if flush is None
-                              else "L2 flushed between steps")},
-            "scans": scans, "roofline": rl, "clocks": sampler.summary(),
-            "gpu_launches": 2 * args.steps}
+            "data": "synthetic", "config": cfg, "scans": scans, "roofline": rl,
+            "clocks": sampler.summary(), "gpu_launches": job.launches_per_step * args.steps}
     if rank == 0 and world == 1 and not args.no_e2e:
-        line["e2e"] = e2e_measure(gl, inp, wl, outs, max(3, min(args.steps, 10)), stream)
+        line["e2e"] = e2e_measure(job, max(3, min(args.steps, 10)), stream)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
 
         oracle.build()
-        line["cpu_baseline"] = cpu_baseline(wl, inp)
+        line["cpu_baseline"] = cpu_baseline(job, job.inp)
     return line
 
 
@@ -371,7 +537,7 @@ def main(argv=None):
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--workload", default="c5", choices=["c1", "c2", "c4", "c5"])
+    ap.add_argument("--workload", default="c5", choices=["c1", "c2", "c3", "c4", "c5"])
     ap.add_argument("--impl", default="gradlev", choices=["gradlev", "reference"])
     ap.add_argument("--resize", default="",
                     help="comma-separated K=V overrides of the workload's sizes (e.g. L=2), "
