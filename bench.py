@@ -403,6 +403,18 @@ def recorded_traffic(workload_key, scan):
     return None if ent is None else int(ent["bytes_per_launch"])
 
 
+# ------------------------------------------------------------- multi-rank
+def combine_ranks(step_ms, tokens_per_rank, world, device):
+    """Whole-job step time and throughput over N replicas: every rank processes
+    its own copy of the workload, the step time is the maximum over ranks, and
+    the value counts all ranks' tokens.  Returns (step_ms, tokens/s)."""
+    if world > 1:
+        t = torch.tensor([float(step_ms)], dtype=torch.float64, device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        step_ms = float(t.item())
+    return step_ms, world * tokens_per_rank / (step_ms / 1e3)
+
+
 # ------------------------------------------------------------------- arms
 def run_reference(args, wl, rank, world):
     """The oracle as the reference arm, on this host's cores (rank 0 only)."""
@@ -499,10 +511,7 @@ def run_gradlev(args, wl, rank, world, local_rank):
     if flush is not None:
         # the flush is not part of the step: take the scans' own time
         step_ms = max(fwd_ms + cos_ms, 1e-9)
-    if world > 1:
-        t = torch.tensor([step_ms], device=device)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        step_ms = float(t.item())
+    step_ms, value = combine_ranks(step_ms, job.tokens, world, device)
     pk = peaks()
     scans = {}
     for name, ms in (("fwd", fwd_ms), ("costate", cos_ms)):
@@ -513,7 +522,6 @@ def run_gradlev(args, wl, rank, world, local_rank):
     rl = dict(scans[dominant]["roofline"])
     rl["kernel"] = job.kernel[dominant]
     rl["traffic"] = None if args.resize else recorded_traffic(args.workload, dominant)
-    value = world * job.tokens / (step_ms / 1e3)
     cfg = {"workload": f"{args.workload}: {wl.name}", **job.config(),
            "tokens_per_step": job.tokens, "parallelism": f"replicas x{world}",
            "l2": "inputs larger than L2" if flush is None else "L2 flushed between steps"}
