@@ -136,16 +136,31 @@ Plan plan_tc(const gradlev_desc& d, int dq, int dv, int sms) {
     Plan pl;
     pl.n_tiles = dv / 64;
     const long long units = (long long)d.L * d.B * d.H * pl.n_tiles;
-    const long long target = 2ll * (sms > 0 ? sms : 148);
-    int n_seg = 1;
-    if (units < target && d.T > 1024) {
-        long long want = (target + units - 1) / units;
-        long long max_seg = (d.T + 511) / 512;
-        n_seg = (int)(want < max_seg ? want : max_seg);
-        if (n_seg < 1) n_seg = 1;
+    const long long nsm = sms > 0 ? sms : 148;
+    // Segment count: with fewer (unit, tile) pairs than two per SM and a long
+    // sequence, split it so every SM gets work.  Pick the count that minimises
+    // the chunks the busiest SM processes: waves x chunks per segment, with the
+    // phase-1 re-stream of every segment but the last (about 0.55 of a full chunk)
+    // and a look-back (about 0.7 of a chunk) per item.  Ties go to fewer segments.
+    long long best_seg = ((long long)d.T + kChunk - 1) / kChunk * kChunk;
+    if (units < 2 * nsm && d.T > 1024) {
+        const long long max_seg = (d.T + 511) / 512;
+        double best = 1e300;
+        for (long long n = 1; n <= max_seg; ++n) {
+            long long seg = ((long long)d.T + n - 1) / n;
+            seg = (seg + kChunk - 1) / kChunk * kChunk;
+            const long long n_eff = ((long long)d.T + seg - 1) / seg;
+            const long long waves = (units * n_eff + nsm - 1) / nsm;
+            const double chunks = (double)(seg / kChunk);
+            const double p1 = n_eff > 1 ? 0.55 * (double)(n_eff - 1) / (double)n_eff : 0.0;
+            const double cost = (double)waves * (chunks * (1.0 + p1) + (n_eff > 1 ? 0.7 : 0.0));
+            if (cost < best * (1.0 - 1e-9)) {
+                best = cost;
+                best_seg = seg;
+            }
+        }
     }
-    long long seg = ((long long)d.T + n_seg - 1) / n_seg;
-    seg = (seg + kChunk - 1) / kChunk * kChunk;
+    long long seg = best_seg;
     if (seg < kChunk) seg = kChunk;
     pl.seg_len = (int)seg;
     pl.n_seg = (int)(((long long)d.T + seg - 1) / seg);
@@ -322,6 +337,7 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
         p.seg_len = pl.seg_len;
         p.n_seg = pl.n_seg;
         p.n_items = pl.n_items;
+        p.n_ut = pl.n_items / pl.n_seg;
         p.eta = eta;
         p.w0_transposed = costate ? 1 : 0;
         p.W0 = W0;

@@ -77,6 +77,7 @@ struct TcScanParams {
     int seg_len;          // tokens per segment (multiple of 128)
     int n_seg;            // segments per (unit, tile)
     int n_items;          // units * n_tiles * n_seg
+    int n_ut;             // units * n_tiles: items per segment index (segment-major order)
     float eta;
     int w0_transposed;    // 0: B0 = W0 ([dv][dq], forward); 1: B0 = W0^T (W0 is [dq][dv])
     const float* W0;      // [L][H][rows][cols] fp32 contiguous

@@ -9,14 +9,14 @@
 // and the state advances by Z_{c+1} = Z_c + K_c^T V_c.
 //
 // Work decomposition.  One item = (unit, 64-wide output tile, token segment).
-// A persistent CTA per SM takes items in ticket order.  Segments after the first
+// A persistent CTA per SM takes items in ticket order, segment-major (segment k of
+// every (unit, tile) pair before any segment k+1).  Segments after the first
 // need the state carried in from the earlier segments of their unit; that carry
 // is a decoupled look-back over per-segment aggregates sum_{s in seg} k_s v_s^T
 // (the additive scan is associative, Sec. 3 "Observation", Eq. 2).  A segment
 // that has successors first streams its keys/values once to form its aggregate
 // (phase 1) and publishes it, then later looks back, publishes its inclusive prefix
-// and runs the full chunk loop (phase 2, which re-reads the same tiles, mostly
-// from L2).  A CTA runs phase 1 of the item it has just taken BEFORE phase 2 of
+// and runs the full chunk loop (phase 2, which re-reads the same tiles).  A CTA runs phase 1 of the item it has just taken BEFORE phase 2 of
 // its previous item, so an aggregate is published right after its ticket is
 // taken and successors in other CTAs rarely wait in their look-back.
 //
@@ -97,10 +97,13 @@ struct Item {
     bool phase1;
 };
 
+// Items are numbered segment-major: every (unit, tile) pair's segment k comes
+// before any segment k+1, so segment k's predecessor is item - n_ut and a
+// look-back mostly finds inclusive prefixes published by earlier waves.
 __device__ __forceinline__ Item decode_item(int item, const TcScanParams& p) {
     Item I;
-    I.k = item % p.n_seg;
-    int r = item / p.n_seg;
+    I.k = item / p.n_ut;
+    int r = item - I.k * p.n_ut;
     I.j = r % p.n_tiles;
     int u = r / p.n_tiles;
     I.h = u % p.H;
@@ -684,6 +687,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (pending >= 0) {
                 const int item = pending;
                 const Item I = decode_item(item, p);
+                const int n_ut = p.n_ut;
+                const int r_ut = item - I.k * n_ut;
                 // ---- look-back: E = sum of the earlier segments' aggregates, stopping at
                 // the nearest inclusive prefix.  The lead state warp polls up to 32
                 // predecessor flags at once (lane i: segment k-1-i) and a ballot finds
@@ -693,14 +698,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int i = 0; i < 64; ++i) st[i] = 0.0f;
                 if (active && I.k > 0) {
                     if (q4 == 0) {
-                        int total = 0, base_pred = item - 1, remaining = I.k;
+                        // predecessor segment sk of this (unit, tile) is item sk * n_ut + r_ut
+                        int total = 0, base_pred = I.k - 1, remaining = I.k;
                         bool found = false, timed_out = false;
                         const uint64_t t0 = globaltimer_ns();
                         while (!found && !timed_out && remaining > 0) {
                             const int n = remaining < 32 ? remaining : 32;
                             unsigned int f = 1u;
                             if (lane < n) {
-                                while ((f = ld_acquire_gpu(p.flags + (base_pred - lane))) == 0u) {
+                                while ((f = ld_acquire_gpu(p.flags + (base_pred - lane) * n_ut + r_ut)) == 0u) {
                                     if (globaltimer_ns() - t0 > kWaitLimitNs) {
                                         f = 0xFFFFFFFFu;
                                         break;
@@ -749,7 +755,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const bool ends_incl = (word & 1u) != 0;
                         __threadfence();
                         for (int i = 0; i < cnt; ++i) {
-                            const int pred = item - 1 - i;
+                            const int pred = (I.k - 1 - i) * n_ut + r_ut;
                             const float* src = ((i == cnt - 1 && ends_incl) ? p.incl : p.agg) +
                                                (size_t)pred * blk + (size_t)row * 64;
     #pragma unroll
