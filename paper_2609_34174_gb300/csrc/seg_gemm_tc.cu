@@ -15,9 +15,10 @@
 // which is Eq. 3 (forward: q = k = x, v = g_hat, B0 = W0) and Eq. 4 (costate:
 // q = g_out, k = g_hat, v = x, B0 = W0^T) with the exclusive sum over s < t split
 // at the segment start.  Each pass is a persistent warp-specialised kernel: a TMA
-// producer warp, a tcgen05.mma issuer warp that owns the tensor memory, and four
+// producer warp, a tcgen05.mma issuer warp that owns the tensor memory, and eight
 // epilogue warps that read the fp32 accumulator out of TMEM (warp w reads lanes
-// 32*(w%4)..+31, so warps 2-5 cover all 128 lanes).
+// 32*(w%4)..+31; warps 2-5 take the left half of the tile's columns and warps
+// 6-9 the right half).
 //
 // Operand tiles are 128B-swizzled [rows][64 bf16] atoms written by TMA:
 //   K-major  (A = Q or P; B = K in the score pass): 128 rows x 64 K, 16 KB
@@ -31,7 +32,8 @@
 namespace gl {
 namespace sg {
 
-constexpr int kWarps = 6;
+constexpr int kWarps = 10;   // producer, MMA issuer, eight epilogue warps
+constexpr int kEpiWarps = 8;
 constexpr int kThreads = kWarps * 32;
 constexpr int kStages = 4;
 constexpr int kAtom = 8192;                         // [64 rows][64 bf16]
@@ -160,7 +162,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&acc_full[i], 1);
-            mbar_init(&acc_free[i], 4);
+            mbar_init(&acc_free[i], kEpiWarps);
         }
         *abort_flag = 0;
         fence_mbar_init();
@@ -320,61 +322,76 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
         // --------------------------------------------------------- epilogue
         const int q4 = warp & 3;
+        const int half = (warp - 2) >> 2;
         const int row = q4 * 32 + lane;
         const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
         const float eta = p.eta;
+        constexpr int W = (MODE == SCORE) ? 128 : BN;  // accumulator columns of a tile
+        constexpr int HW = W / 2;                       // columns this warp handles
+        const int cb = half * HW;                       // first of them
         uint32_t e = 0;
         int it = 0;
         for (int tile = blockIdx.x; tile < p.n_tiles; tile += gridDim.x, ++it) {
             const Tile t = decode<MODE, BN>(tile, p);
             bool ok = true;
             if (MODE == STATE) {
+                // B0^T for this tile goes to TMEM columns 256.. once (the accumulator
+                // uses columns 0..BN-1), and is also segment 0's starting state.
                 const int dq_row = t.mi * 128 + row;
                 const float* w0 = p.W0 + (size_t)(t.l * p.H + t.h) * p.dq * p.dv;
-                for (int k = 0; k < p.n_seg; ++k) {
-                    if (k > 0) {
-                        if (!warp_wait(&acc_full[0], e & 1, abort_flag)) {
-                            raise_error(p, abort_flag);
-                            ok = false;
-                            break;
+                const uint32_t b0_t = tmem + lane_off + 256;
+                __nv_bfloat16* dst0 = p.sbuf + ((size_t)(t.u * p.n_seg) * p.dq + dq_row) * p.dv + t.ni * BN;
+#pragma unroll 1
+                for (int c0 = cb; c0 < cb + HW; c0 += 32) {
+                    float a[32];
+                    const int col0 = t.ni * BN + c0;
+                    if (p.w0_transposed) {
+                        const float* src = w0 + (size_t)dq_row * p.dv + col0;  // W0 [dq][dv]
+#pragma unroll
+                        for (int j = 0; j < 32; j += 4) {
+                            const float4 b = *reinterpret_cast<const float4*>(src + j);
+                            a[j] = b.x;
+                            a[j + 1] = b.y;
+                            a[j + 2] = b.z;
+                            a[j + 3] = b.w;
                         }
-                        tc_fence_after();
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)  // W0 [dv][dq]: column dq_row
+                            a[j] = w0[(size_t)(col0 + j) * p.dq + dq_row];
                     }
+                    uint32_t r[32];
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(a[j]);
+                    tmem_st32_async(b0_t + c0, r);
+                    store_bf16x32(dst0 + c0, a);
+                }
+                tmem_wait_st();
+                for (int k = 1; k < p.n_seg; ++k) {
+                    if (!warp_wait(&acc_full[0], e & 1, abort_flag)) {
+                        raise_error(p, abort_flag);
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
                     __nv_bfloat16* dst = p.sbuf + ((size_t)(t.u * p.n_seg + k) * p.dq + dq_row) * p.dv +
                                          t.ni * BN;
 #pragma unroll 1
-                    for (int c0 = 0; c0 < BN; c0 += 32) {
-                        float a[32];
-                        if (k > 0) {
-                            tmem_ld32(tmem + lane_off + c0, a);
-                        } else {
-#pragma unroll
-                            for (int j = 0; j < 32; ++j) a[j] = 0.0f;
+                    for (int c0 = cb; c0 < cb + HW; c0 += 32) {
+                        float a[32], b[32];
+                        tmem_ld32(tmem + lane_off + c0, a);
+                        if (c0 + 32 == cb + HW) {
+                            // last accumulator read of this segment: let the next one start
+                            tc_fence_before();
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(&acc_free[0]);
                         }
-                        const int col0 = t.ni * BN + c0;
-                        if (p.w0_transposed) {
-                            const float* src = w0 + (size_t)dq_row * p.dv + col0;  // W0 [dq][dv]
+                        tmem_ld32(b0_t + c0, b);
 #pragma unroll
-                            for (int j = 0; j < 32; j += 4) {
-                                const float4 b = *reinterpret_cast<const float4*>(src + j);
-                                a[j] = b.x - eta * a[j];
-                                a[j + 1] = b.y - eta * a[j + 1];
-                                a[j + 2] = b.z - eta * a[j + 2];
-                                a[j + 3] = b.w - eta * a[j + 3];
-                            }
-                        } else {
-#pragma unroll
-                            for (int j = 0; j < 32; ++j)  // W0 [dv][dq]: column dq_row
-                                a[j] = w0[(size_t)(col0 + j) * p.dq + dq_row] - eta * a[j];
-                        }
+                        for (int j = 0; j < 32; ++j) a[j] = b[j] - eta * a[j];
                         store_bf16x32(dst + c0, a);
                     }
-                    if (k > 0) {
-                        tc_fence_before();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(&acc_free[0]);
-                        ++e;
-                    }
+                    ++e;
                 }
             } else {
                 const uint32_t buf = it & 1;
@@ -389,7 +406,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     __nv_bfloat16* dst = p.pbuf + ((size_t)(t.u * p.n_seg + t.k) * Ls + t_seg) * Ls +
                                          t.c * 128;
 #pragma unroll 1
-                    for (int c0 = 0; c0 < 128; c0 += 32) {
+                    for (int c0 = cb; c0 < cb + HW; c0 += 32) {
                         float a[32];
                         tmem_ld32(acc + c0, a);
                         const int s0 = t.c * 128 + c0;
@@ -402,7 +419,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int tok = t.k * Ls + t.r * 128 + row;
                     const bool valid = tok < p.T;
 #pragma unroll 1
-                    for (int c0 = 0; c0 < BN; c0 += 32) {
+                    for (int c0 = cb; c0 < cb + HW; c0 += 32) {
                         float a[32];
                         tmem_ld32(acc + c0, a);
                         if (!valid) continue;
