@@ -339,6 +339,9 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
         p.n_items = pl.n_items;
         p.n_ut = pl.n_items / pl.n_seg;
         p.eta = eta;
+        p.lam = eta != 0.0f ? -eta : 1.0f;
+        p.inv_lam = 1.0f / p.lam;
+        p.mu = eta != 0.0f ? 1.0f : 0.0f;
         p.w0_transposed = costate ? 1 : 0;
         p.W0 = W0;
         fill_epi(&p.epi, to, to2, tz, act);

@@ -79,6 +79,9 @@ struct TcScanParams {
     int n_items;          // units * n_tiles * n_seg
     int n_ut;             // units * n_tiles: items per segment index (segment-major order)
     float eta;
+    // State units of the chunk kernel: lam = -eta (1 when eta = 0), inv_lam = 1 / lam,
+    // mu = -eta / lam (1, or 0 when eta = 0).
+    float lam, inv_lam, mu;
     int w0_transposed;    // 0: B0 = W0 ([dv][dq], forward); 1: B0 = W0^T (W0 is [dq][dv])
     const float* W0;      // [L][H][rows][cols] fp32 contiguous
     EpiParams epi;

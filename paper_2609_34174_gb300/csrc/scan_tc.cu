@@ -27,9 +27,11 @@
 //   warp 14     lane 0 issues the "back" MMAs (O = Q S^T, then O += P V); the two
 //               issuers run independent in-order loops, so the output product of
 //               chunk c never waits behind the score of chunk c+1
-//   warps 2-5   score -> P: TMEM score tile, causal mask, scale by -eta, bf16 P
-//               written back over the same TMEM columns (the PV product reads its A
-//               operand from tensor memory, so P never touches shared memory)
+//   warps 2-5   score -> P: TMEM score tile, causal mask, bf16 P written back over
+//               the same TMEM columns (the PV product reads its A operand from
+//               tensor memory, so P never touches shared memory).  P is left
+//               unscaled: the state is kept in units of lam = -eta, so the S^T tile
+//               carries the factor and the epilogue multiplies O by lam once.
 //   warps 6-9   output epilogue: TMEM O tile -> bf16 staging tile in shared memory ->
 //               one TMA tensor store per chunk (whole 128-byte rows, no scattered
 //               per-thread stores competing with the other roles for the LSU path)
@@ -140,6 +142,30 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
     ok = __shfl_sync(0xffffffffu, ok, 0);
     __syncwarp();
     return ok != 0;
+}
+
+// v *= sigma'(z) for one 64-wide output row piece (costate MLP fusion).
+__device__ __noinline__ void epi_apply_dact(const EpiParams& e, long long z_off, float* v) {
+    const __nv_bfloat16* zp = static_cast<const __nv_bfloat16*>(e.zin) + z_off;
+    for (int q = 0; q < 8; ++q) {
+        const uint4 zz = *reinterpret_cast<const uint4*>(zp + 8 * q);
+        const __nv_bfloat16* zb = reinterpret_cast<const __nv_bfloat16*>(&zz);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[8 * q + i] *= act_df(e.act, __bfloat162float(zb[i]));
+    }
+}
+
+// out2 = sigma(v) for one 64-wide output row piece (forward MLP fusion).
+__device__ __noinline__ void epi_store_act(const EpiParams& e, long long o_off, const float* v) {
+    __nv_bfloat16* op2 = static_cast<__nv_bfloat16*>(e.out2) + o_off;
+    for (int q = 0; q < 8; ++q) {
+        uint4 w;
+        w.x = pack_bf16x2(act_f(e.act, v[8 * q + 0]), act_f(e.act, v[8 * q + 1]));
+        w.y = pack_bf16x2(act_f(e.act, v[8 * q + 2]), act_f(e.act, v[8 * q + 3]));
+        w.z = pack_bf16x2(act_f(e.act, v[8 * q + 4]), act_f(e.act, v[8 * q + 5]));
+        w.w = pack_bf16x2(act_f(e.act, v[8 * q + 6]), act_f(e.act, v[8 * q + 7]));
+        *reinterpret_cast<uint4*>(op2 + 8 * q) = w;
+    }
 }
 
 // K-step offsets (in the 16-byte units of a descriptor's low word).
@@ -458,7 +484,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int q4 = warp & 3;
         const int row = q4 * 32 + lane;
         const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
-        const float neg_eta = -p.eta;
         uint32_t c2 = 0;
         for (int it = 0;; ++it) {
             const int slot = it % kRing;
@@ -492,20 +517,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int half = 0; half < 2; ++half) {
                     const bool mine = half == 0 ? !helper : (q4 < 2 ? !helper : (helper || kPHelpers == 0));
                     if (!mine) continue;
-                    if (half == 1 && q4 < 2) {
-                        tmem_zero32_async(base + 64);  // rows < 64: tokens >= 64 all masked
+                    if ((half == 1 && q4 < 2) || p.mu == 0.0f) {
+                        // rows < 64: tokens >= 64 all masked; eta = 0: no P at all
+                        tmem_zero32_async(base + half * 64);
                         continue;
                     }
-                    float v[64];
-                    uint32_t w[32];
-                    tmem_ld64(base + half * 64, v);
+#pragma unroll 1
+                    for (int sub = 0; sub < 2; ++sub) {
+                        float v[32];
+                        uint32_t w[16];
+                        tmem_ld32(base + half * 64 + sub * 32, v);
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        const int s0 = half * 64 + 2 * i;
-                        w[i] = pack_bf16x2(s0 < row ? neg_eta * v[2 * i] : 0.0f,
-                                           s0 + 1 < row ? neg_eta * v[2 * i + 1] : 0.0f);
+                        for (int i = 0; i < 16; ++i) {
+                            const int s0 = half * 64 + sub * 32 + 2 * i;
+                            w[i] = pack_bf16x2(s0 < row ? v[2 * i] : 0.0f,
+                                               s0 + 1 < row ? v[2 * i + 1] : 0.0f);
+                        }
+                        tmem_st16_async(base + half * 64 + sub * 16, w);
                     }
-                    tmem_st32_async(base + half * 64, w);
                 }
                 tmem_wait_st();
                 tc_fence_before();
@@ -547,32 +576,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&o_free[ob]);
+#pragma unroll
+                for (int i = 0; i < 64; ++i) v[i] *= p.lam;  // O = lam * (Q S'^T + L(Q K^T) V)
                 const int t0 = I.t_begin + c * kChunk;
                 const int t = t0 + row;
                 const int col0 = I.j * 64;
+                // The activation paths (MLP layers only) run out of line, so the hot
+                // loop of the plain scans stays small in the instruction cache.
                 if (e.zin && t < I.t_end) {
-                    const __nv_bfloat16* zp = static_cast<const __nv_bfloat16*>(e.zin) +
-                                              tok_off(e.z_str, I.l, I.b, t, I.h) + col0;
+                    float tmp[64];
 #pragma unroll
-                    for (int q = 0; q < 8; ++q) {
-                        uint4 zz = *reinterpret_cast<const uint4*>(zp + 8 * q);
-                        const __nv_bfloat16* zb = reinterpret_cast<const __nv_bfloat16*>(&zz);
+                    for (int i = 0; i < 64; ++i) tmp[i] = v[i];
+                    epi_apply_dact(e, tok_off(e.z_str, I.l, I.b, t, I.h) + col0, tmp);
 #pragma unroll
-                        for (int i = 0; i < 8; ++i) v[8 * q + i] *= act_df(e.act, __bfloat162float(zb[i]));
-                    }
+                    for (int i = 0; i < 64; ++i) v[i] = tmp[i];
                 }
                 if (e.out2 && t < I.t_end) {
-                    __nv_bfloat16* op2 = static_cast<__nv_bfloat16*>(e.out2) +
-                                         tok_off(e.out2_str, I.l, I.b, t, I.h) + col0;
+                    float tmp[64];
 #pragma unroll
-                    for (int q = 0; q < 8; ++q) {
-                        uint4 w;
-                        w.x = pack_bf16x2(act_f(e.act, v[8 * q + 0]), act_f(e.act, v[8 * q + 1]));
-                        w.y = pack_bf16x2(act_f(e.act, v[8 * q + 2]), act_f(e.act, v[8 * q + 3]));
-                        w.z = pack_bf16x2(act_f(e.act, v[8 * q + 4]), act_f(e.act, v[8 * q + 5]));
-                        w.w = pack_bf16x2(act_f(e.act, v[8 * q + 6]), act_f(e.act, v[8 * q + 7]));
-                        *reinterpret_cast<uint4*>(op2 + 8 * q) = w;
-                    }
+                    for (int i = 0; i < 64; ++i) tmp[i] = v[i];
+                    epi_store_act(e, tok_off(e.out2_str, I.l, I.b, t, I.h) + col0, tmp);
                 }
                 // Stage the bf16 row in the 128B-swizzled output tile (the TMA store
                 // clips rows past the end of the sequence).
@@ -619,7 +642,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool active = row < DQ;           // warp-uniform
         const bool leader = (q4 == 0) && (lane == 0);
         const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
-        const float eta = p.eta;
+        // The state is kept in units of lam = -eta (1 when eta = 0): the rows hold
+        // S' = S / lam, so the S^T tile carries the -eta of P and the update is
+        // S' += mu * dZ with mu = -eta / lam (1, or 0 when eta = 0).
         uint32_t c2 = 0, dzc = 0, pubc = 0, lbc = 0;
         float st[64];
         const size_t blk = (size_t)DQ * 64;
@@ -781,7 +806,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     if (!publish(item, 2u)) break;
                 }
-                // ---- starting state S^T row = B0^T row - eta * E
+                // ---- starting state S'^T row = (B0^T row - eta * E) / lam
                 if (active) {
                     const float* w0 = p.W0 + (size_t)(I.l * p.H + I.h) * p.dq * p.dv;
                     const int v0 = I.j * 64;
@@ -790,15 +815,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     #pragma unroll
                         for (int i = 0; i < 64; i += 4) {
                             float4 a = *reinterpret_cast<const float4*>(r + i);
-                            st[i] = a.x - eta * st[i];
-                            st[i + 1] = a.y - eta * st[i + 1];
-                            st[i + 2] = a.z - eta * st[i + 2];
-                            st[i + 3] = a.w - eta * st[i + 3];
+                            st[i] = a.x * p.inv_lam + p.mu * st[i];
+                            st[i + 1] = a.y * p.inv_lam + p.mu * st[i + 1];
+                            st[i + 2] = a.z * p.inv_lam + p.mu * st[i + 2];
+                            st[i + 3] = a.w * p.inv_lam + p.mu * st[i + 3];
                         }
                     } else {
     #pragma unroll
                         for (int i = 0; i < 64; ++i)  // W0 [dv][dq]: column `row`
-                            st[i] = w0[(size_t)(v0 + i) * p.dq + row] - eta * st[i];
+                            st[i] = w0[(size_t)(v0 + i) * p.dq + row] * p.inv_lam + p.mu * st[i];
                     }
                 }
                 // ---- phase 2: S^T tile for every chunk, state advanced by dZ
@@ -835,7 +860,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             for (int h = 0; h < 2; ++h) {
                                 tmem_ld32(tmem + col_dz(b) + lane_off + h * 32, a);
     #pragma unroll
-                                for (int i = 0; i < 32; ++i) st[h * 32 + i] -= eta * a[i];
+                                for (int i = 0; i < 32; ++i) st[h * 32 + i] += p.mu * a[i];
                             }
                         }
                         tc_fence_before();
