@@ -140,6 +140,38 @@ int gradlev_costate_scan(const gradlev_desc* desc, const gradlev_tensor* x,
                          const gradlev_tensor* g_in, void* workspace, size_t workspace_bytes,
                          gradlev_stream_t stream);
 
+/*
+ * gradlev_forward_scan_gated / gradlev_costate_scan_gated -- the scans with the
+ * general gates of Sec. 3 ("Observation", Eq. 2): a step size eta_t >= 0 per token
+ * and, optionally, a retention alpha_t in [0, 1] with decay centred at W0,
+ *     W_{t+1} = W0 + alpha_t (W_t - W0) - eta_t ghat_t x_t^T,   read before write.
+ * alpha_t = 0 resets the fast weights to W0 (a document boundary).
+ *   eta_t    fp32 [L][B][T][H], contiguous device array (read)
+ *   alpha_t  fp32 [L][B][T][H], contiguous, or NULL for alpha = 1 (read)
+ *   other arguments as in gradlev_forward_scan / gradlev_costate_scan (the scalar
+ *   eta is replaced by eta_t).
+ * Without alpha_t the proposals are scaled by eta_t into the workspace (one
+ * elementwise pass, rounded to the input dtype) and the chunked scan runs with
+ * eta = 1.  With alpha_t a token-serial kernel runs the recurrence as written
+ * (state W - W0 in fp32 shared memory; the read width, d_in forward and d_out
+ * costate, must be at most 256, else GRADLEV_ERR_UNSUPPORTED).
+ * Workspace: at least gradlev_workspace_bytes_gated(desc) bytes, 256-byte aligned.
+ */
+int gradlev_forward_scan_gated(const gradlev_desc* desc, const gradlev_tensor* x,
+                               const gradlev_tensor* g_hat, const float* W0, const float* eta_t,
+                               const float* alpha_t, int act, const gradlev_tensor* y,
+                               const gradlev_tensor* act_out, void* workspace,
+                               size_t workspace_bytes, gradlev_stream_t stream);
+int gradlev_costate_scan_gated(const gradlev_desc* desc, const gradlev_tensor* x,
+                               const gradlev_tensor* g_hat, const float* W0, const float* eta_t,
+                               const float* alpha_t, const gradlev_tensor* g_out, int act,
+                               const gradlev_tensor* z, const gradlev_tensor* g_in, void* workspace,
+                               size_t workspace_bytes, gradlev_stream_t stream);
+
+/* Bytes of workspace the gated scans need for this shape (0 for an invalid
+ * descriptor). */
+size_t gradlev_workspace_bytes_gated(const gradlev_desc* desc);
+
 /* Size of the fixed device array used by gradlev_forward_scan_noalloc (4 MiB). */
 #define GRADLEV_NOALLOC_SCRATCH_BYTES (4u << 20)
 

@@ -74,6 +74,14 @@ def load_library():
         lib.gradlev_costate_scan.argtypes = [D, Tp, Tp, P, ctypes.c_float, Tp, ctypes.c_int, Tp, Tp,
                                              P, ctypes.c_size_t, P]
         lib.gradlev_costate_scan.restype = ctypes.c_int
+        lib.gradlev_forward_scan_gated.argtypes = [D, Tp, Tp, P, P, P, ctypes.c_int, Tp, Tp, P,
+                                                   ctypes.c_size_t, P]
+        lib.gradlev_forward_scan_gated.restype = ctypes.c_int
+        lib.gradlev_costate_scan_gated.argtypes = [D, Tp, Tp, P, P, P, Tp, ctypes.c_int, Tp, Tp, P,
+                                                   ctypes.c_size_t, P]
+        lib.gradlev_costate_scan_gated.restype = ctypes.c_int
+        lib.gradlev_workspace_bytes_gated.argtypes = [D]
+        lib.gradlev_workspace_bytes_gated.restype = ctypes.c_size_t
         lib.gradlev_workspace_bytes.argtypes = [D]
         lib.gradlev_workspace_bytes.restype = ctypes.c_size_t
         lib.gradlev_workspace_status.argtypes = [P, P]
@@ -190,18 +198,38 @@ def workspace_status(workspace: torch.Tensor) -> int:
                                             ctypes.c_void_p(s)))
 
 
+def _gates(eta, alpha, x5):
+    """Per-token gate arrays for the gated entry points, or None for a plain scalar
+    eta: fp32 [L,B,T,H] contiguous on the tensors' device."""
+    if not isinstance(eta, torch.Tensor) and alpha is None:
+        return None
+    shape = tuple(x5.shape[:4])
+
+    def norm(v):
+        if isinstance(v, torch.Tensor):
+            t = v.to(device=x5.device, dtype=torch.float32)
+            return t.reshape(shape).contiguous()
+        return torch.full(shape, float(v), dtype=torch.float32, device=x5.device)
+
+    return norm(eta), (norm(alpha) if alpha is not None else None)
+
+
 def _call(rc: int, what: str):
     if rc != 0:
         raise GradLevError(rc, what)
 
 
 def forward_scan(x, g_hat, W0, eta, act=None, y=None, act_out=None, want_act_out=False,
-                 workspace=None):
+                 workspace=None, alpha=None):
     """y_t = (W0 - eta sum_{s<t} ghat_s x_s^T) x_t for every token (Sec. 3 step 2, Eq. 3).
 
     x [L,B,T,H,d_in] (or [B,T,H,d_in], [B,T,d_in], [T,d_in]), g_hat with d_out features,
     W0 fp32 [L,H,d_out,d_in].  With want_act_out (or act_out given) also returns
     sigma(y) for the activation `act`.  Returns y, or (y, act_out).
+
+    Gates (Eq. 2): `eta` may be a tensor of per-token step sizes with the token
+    shape of x, and `alpha` an optional per-token retention (decay centred at W0;
+    alpha = 0 resets to W0).
     """
     lib = load_library()
     x5, g5 = _as5(x), _as5(g_hat)
@@ -226,11 +254,27 @@ def forward_scan(x, g_hat, W0, eta, act=None, y=None, act_out=None, want_act_out
         act_out = torch.empty_like(y)
     a5 = _as5(act_out) if act_out is not None else None
     desc = _desc(x5, d_out, _dtype_code(x5))
-    nbytes = int(lib.gradlev_workspace_bytes(ctypes.byref(desc)))
+    gates = _gates(eta, alpha, x5)
+    if gates is not None:
+        nbytes = int(lib.gradlev_workspace_bytes_gated(ctypes.byref(desc)))
+    else:
+        nbytes = int(lib.gradlev_workspace_bytes(ctypes.byref(desc)))
     ws = workspace if workspace is not None else _workspace(nbytes, x5.device)
     tx, tg, ty = _tensor(x5), _tensor(g5), _tensor(y5)
     ta = _tensor(a5) if a5 is not None else None
     stream = torch.cuda.current_stream(x5.device).cuda_stream
+    if gates is not None:
+        et, al = gates
+        with torch.cuda.device(x5.device):
+            rc = lib.gradlev_forward_scan_gated(
+                ctypes.byref(desc), ctypes.byref(tx), ctypes.byref(tg), ctypes.c_void_p(W.data_ptr()),
+                ctypes.c_void_p(et.data_ptr()), ctypes.c_void_p(al.data_ptr()) if al is not None else None,
+                code, ctypes.byref(ty), ctypes.byref(ta) if ta is not None else None,
+                ctypes.c_void_p(ws.data_ptr()), ws.numel(), ctypes.c_void_p(stream))
+        _call(rc, "gradlev_forward_scan_gated")
+        if act_out is not None:
+            return y, act_out
+        return y
     with torch.cuda.device(x5.device):
         rc = lib.gradlev_forward_scan(ctypes.byref(desc), ctypes.byref(tx), ctypes.byref(tg),
                                       ctypes.c_void_p(W.data_ptr()), float(eta), code,
@@ -243,11 +287,13 @@ def forward_scan(x, g_hat, W0, eta, act=None, y=None, act_out=None, want_act_out
     return y
 
 
-def costate_scan(x, g_hat, W0, eta, g_out, act=None, z=None, g_in=None, workspace=None):
+def costate_scan(x, g_hat, W0, eta, g_out, act=None, z=None, g_in=None, workspace=None,
+                 alpha=None):
     """g_in_t = (W0 - eta sum_{s<t} ghat_s x_s^T)^T g_out_t (Sec. 3 step 3, Eq. 4).
 
     With z (the preactivation that fed this map's input through sigma = act) the
     result is sigma'(z_t) * (What_t^T g_out_t).  Returns g_in [.., d_in].
+    Gates as for forward_scan.
     """
     lib = load_library()
     x5, g5, go5 = _as5(x), _as5(g_hat), _as5(g_out)
@@ -270,11 +316,25 @@ def costate_scan(x, g_hat, W0, eta, g_out, act=None, z=None, g_in=None, workspac
     gi5 = _as5(g_in)
     _check_same(x5, gi5)
     desc = _desc(x5, d_out, _dtype_code(x5))
-    nbytes = int(lib.gradlev_workspace_bytes(ctypes.byref(desc)))
+    gates = _gates(eta, alpha, x5)
+    if gates is not None:
+        nbytes = int(lib.gradlev_workspace_bytes_gated(ctypes.byref(desc)))
+    else:
+        nbytes = int(lib.gradlev_workspace_bytes(ctypes.byref(desc)))
     ws = workspace if workspace is not None else _workspace(nbytes, x5.device)
     tx, tg, tgo, tgi = _tensor(x5), _tensor(g5), _tensor(go5), _tensor(gi5)
     tz = _tensor(z5) if z5 is not None else None
     stream = torch.cuda.current_stream(x5.device).cuda_stream
+    if gates is not None:
+        et, al = gates
+        with torch.cuda.device(x5.device):
+            rc = lib.gradlev_costate_scan_gated(
+                ctypes.byref(desc), ctypes.byref(tx), ctypes.byref(tg), ctypes.c_void_p(W.data_ptr()),
+                ctypes.c_void_p(et.data_ptr()), ctypes.c_void_p(al.data_ptr()) if al is not None else None,
+                ctypes.byref(tgo), code, ctypes.byref(tz) if tz is not None else None,
+                ctypes.byref(tgi), ctypes.c_void_p(ws.data_ptr()), ws.numel(), ctypes.c_void_p(stream))
+        _call(rc, "gradlev_costate_scan_gated")
+        return g_in
     with torch.cuda.device(x5.device):
         rc = lib.gradlev_costate_scan(ctypes.byref(desc), ctypes.byref(tx), ctypes.byref(tg),
                                       ctypes.c_void_p(W.data_ptr()), float(eta), ctypes.byref(tgo),

@@ -22,6 +22,10 @@ cudaError_t launch_seg_gemm(int mode, int bn, const CUtensorMap& a, const CUtens
                             const CUtensorMap& a2, const CUtensorMap& b2, const SegGemmParams& p,
                             int grid, cudaStream_t stream);
 size_t simt_smem_bytes(int dq);
+size_t gated_serial_smem(int din, int dout, bool costate);
+cudaError_t launch_gated_serial(const GatedParams& p, bool costate, bool bf16, cudaStream_t stream);
+cudaError_t launch_gated_prescale(const void* g, const TokStr& gs, const float* eta, void* out, int L,
+                                  int B, int T, int H, int w, bool bf16, cudaStream_t stream);
 }  // namespace gl
 
 namespace {
@@ -460,6 +464,97 @@ size_t ws_bytes_for(const gradlev_desc& d, int dq, int dv, int sms) {
     return b;
 }
 
+// Gated scans (Eq. 2 with per-token eta_t and optional retention alpha_t).
+constexpr int kGatedSerialMaxWidth = 256;
+
+size_t gated_ws_bytes(const gradlev_desc& d, int sms) {
+    const size_t a = ws_bytes_for(d, d.d_in, d.d_out, sms);
+    const size_t b = ws_bytes_for(d, d.d_out, d.d_in, sms);
+    const size_t base = round_up(a > b ? a : b, 256);
+    const size_t elem = d.dtype == GRADLEV_BF16 ? 2 : 4;
+    return base + (size_t)d.L * d.B * d.T * d.H * d.d_out * elem;
+}
+
+int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
+              const gradlev_tensor* g_hat, const float* W0, const float* eta_t,
+              const float* alpha_t, const gradlev_tensor* g_out, int act, const gradlev_tensor* out,
+              const gradlev_tensor* out2, const gradlev_tensor* z, void* ws, size_t ws_bytes,
+              cudaStream_t stream) {
+    if (!desc_ok(desc)) return GRADLEV_ERR_INVALID_ARG;
+    const gradlev_desc& d = *desc;
+    if (!W0 || !eta_t || (reinterpret_cast<uintptr_t>(eta_t) & 3u) ||
+        (alpha_t && (reinterpret_cast<uintptr_t>(alpha_t) & 3u)))
+        return GRADLEV_ERR_INVALID_ARG;
+    if (act < GRADLEV_ACT_NONE || act > GRADLEV_ACT_TANH) return GRADLEV_ERR_INVALID_ARG;
+    DevInfo dev;
+    if (!device_info(&dev)) return GRADLEV_ERR_CUDA;
+    if (!(dev.major == 10 && dev.minor == 3)) return GRADLEV_ERR_UNSUPPORTED;
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return GRADLEV_ERR_WORKSPACE;
+    if (ws_bytes < gated_ws_bytes(d, dev.sms)) return GRADLEV_ERR_WORKSPACE;
+    if (d.T == 0) return GRADLEV_OK;
+    const bool bf16 = d.dtype == GRADLEV_BF16;
+    Tok tx, tg;
+    if (!resolve(d, x, d.d_in, &tx, true) || !resolve(d, g_hat, d.d_out, &tg, true))
+        return GRADLEV_ERR_INVALID_ARG;
+    if (!alpha_t) {
+        // eta_t only: scale the writes' proposals, then the ungated scan with eta = 1
+        const size_t a = ws_bytes_for(d, d.d_in, d.d_out, dev.sms);
+        const size_t b = ws_bytes_for(d, d.d_out, d.d_in, dev.sms);
+        const size_t base = round_up(a > b ? a : b, 256);
+        void* gp = static_cast<uint8_t*>(ws) + base;
+        gl::TokStr gs;
+        for (int i = 0; i < 4; ++i) gs.s[i] = tg.s[i];
+        if (gl::launch_gated_prescale(tg.data, gs, eta_t, gp, d.L, d.B, d.T, d.H, d.d_out, bf16,
+                                      stream) != cudaSuccess)
+            return GRADLEV_ERR_CUDA;
+        gradlev_tensor gpt;
+        gpt.data = gp;
+        for (int i = 0; i < 4; ++i) gpt.stride[i] = 0;
+        return run_scan(desc, costate, x, &gpt, W0, 1.0f, g_out, act, out, out2, z, ws, base, stream);
+    }
+    // with retention: the token-serial kernel
+    const int J = costate ? d.d_out : d.d_in;
+    if (J > kGatedSerialMaxWidth) return GRADLEV_ERR_UNSUPPORTED;
+    Tok tgo, to, to2, tz;
+    if (!resolve(d, out, costate ? d.d_in : d.d_out, &to, true)) return GRADLEV_ERR_INVALID_ARG;
+    if (costate) {
+        if (!resolve(d, g_out, d.d_out, &tgo, true) || !resolve(d, z, d.d_in, &tz, false))
+            return GRADLEV_ERR_INVALID_ARG;
+        if (tz.data && act == GRADLEV_ACT_NONE) return GRADLEV_ERR_INVALID_ARG;
+    } else {
+        if (!resolve(d, out2, d.d_out, &to2, false)) return GRADLEV_ERR_INVALID_ARG;
+        if (to2.data && act == GRADLEV_ACT_NONE) return GRADLEV_ERR_INVALID_ARG;
+    }
+    const int elem = bf16 ? 2 : 4;
+    const Tok* all[6] = {&tx, &tg, &tgo, &to, &to2, &tz};
+    for (const Tok* t : all)
+        if (t->data && (reinterpret_cast<uintptr_t>(t->data) % elem) != 0) return GRADLEV_ERR_UNSUPPORTED;
+    if ((reinterpret_cast<uintptr_t>(W0) & 3u) != 0) return GRADLEV_ERR_INVALID_ARG;
+    if (cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
+    gl::GatedParams p;
+    memset(&p, 0, sizeof(p));
+    p.L = d.L;
+    p.B = d.B;
+    p.T = d.T;
+    p.H = d.H;
+    p.din = d.d_in;
+    p.dout = d.d_out;
+    p.W0 = W0;
+    p.eta = eta_t;
+    p.alpha = alpha_t;
+    p.x = tx.data;
+    p.g = tg.data;
+    p.q = costate ? tgo.data : tx.data;
+    for (int i = 0; i < 4; ++i) {
+        p.x_s[i] = tx.s[i];
+        p.g_s[i] = tg.s[i];
+        p.q_s[i] = costate ? tgo.s[i] : tx.s[i];
+    }
+    fill_epi(&p.epi, to, to2, tz, act);
+    if (gl::launch_gated_serial(p, costate, bf16, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
+    return GRADLEV_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -479,6 +574,31 @@ int gradlev_costate_scan(const gradlev_desc* desc, const gradlev_tensor* x,
                          gradlev_stream_t stream) {
     return run_scan(desc, true, x, g_hat, W0, eta, g_out, act, g_in, nullptr, z, workspace,
                     workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int gradlev_forward_scan_gated(const gradlev_desc* desc, const gradlev_tensor* x,
+                               const gradlev_tensor* g_hat, const float* W0, const float* eta_t,
+                               const float* alpha_t, int act, const gradlev_tensor* y,
+                               const gradlev_tensor* act_out, void* workspace,
+                               size_t workspace_bytes, gradlev_stream_t stream) {
+    return run_gated(desc, false, x, g_hat, W0, eta_t, alpha_t, nullptr, act, y, act_out, nullptr,
+                     workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int gradlev_costate_scan_gated(const gradlev_desc* desc, const gradlev_tensor* x,
+                               const gradlev_tensor* g_hat, const float* W0, const float* eta_t,
+                               const float* alpha_t, const gradlev_tensor* g_out, int act,
+                               const gradlev_tensor* z, const gradlev_tensor* g_in, void* workspace,
+                               size_t workspace_bytes, gradlev_stream_t stream) {
+    return run_gated(desc, true, x, g_hat, W0, eta_t, alpha_t, g_out, act, g_in, nullptr, z,
+                     workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t gradlev_workspace_bytes_gated(const gradlev_desc* desc) {
+    if (!desc_ok(desc)) return 0;
+    DevInfo dev;
+    int sms = device_info(&dev) ? dev.sms : 160;
+    return gated_ws_bytes(*desc, sms);
 }
 
 size_t gradlev_workspace_bytes(const gradlev_desc* desc) {

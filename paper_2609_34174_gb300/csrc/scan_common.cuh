@@ -121,6 +121,23 @@ struct SimtScanParams {
     EpiParams epi;
 };
 
+// Element strides of (L, B, T, H) of a token tensor.
+struct TokStr {
+    long long s[4];
+};
+
+// Parameters of the gated token-serial kernel (gated.cu).
+struct GatedParams {
+    int L, B, T, H, din, dout;
+    const float* W0;       // [L][H][dout][din]
+    const float* eta;      // [L][B][T][H] per-token step sizes
+    const float* alpha;    // [L][B][T][H] retention, or null (= 1)
+    const void* x; long long x_s[4];   // layer inputs (the writes' right factor)
+    const void* g; long long g_s[4];   // proposals ghat (the writes' left factor)
+    const void* q; long long q_s[4];   // read vector: x (forward) or g_out (costate)
+    EpiParams epi;
+};
+
 // Error bits written to ctrl[1].
 constexpr unsigned int kErrWaitTimeout = 1u;
 constexpr unsigned int kErrLookbackTimeout = 2u;

@@ -1,0 +1,120 @@
+"""GPU parity of the gated scans (Sec. 3 "Observation", Eq. 2 with per-token step
+sizes eta_t and retention alpha_t, decay centred at W0) against the fp64 oracle,
+which runs the same recurrence token by token.
+
+Per-token eta_t alone takes the chunked kernels on eta-scaled proposals;
+with alpha_t the token-serial kernel runs.  alpha_t = 0 marks resets (the fast
+weights return to W0, as at a document boundary).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads as W
+from parity_util import TOL, rel_l2
+
+gl = pytest.importorskip("paper_2609_34174_gb300")
+
+pytestmark = pytest.mark.gpu
+
+
+def _gates(wl, seed, with_alpha, resets=True):
+    g = torch.Generator().manual_seed(seed)
+    shape = (wl.L, wl.B, wl.T, wl.H)
+    eta = torch.rand(shape, generator=g, dtype=torch.float64) * (2 * wl.eta)
+    alpha = None
+    if with_alpha:
+        alpha = 0.9 + 0.1 * torch.rand(shape, generator=g, dtype=torch.float64)
+        if resets:
+            alpha[..., wl.T // 3, :] = 0.0      # a document boundary
+            alpha[..., (2 * wl.T) // 3, :] = 0.0
+    return eta.float(), (alpha.float() if alpha is not None else None)
+
+
+def _oracle(inputs, eta, alpha, wl):
+    """fp64 oracle per unit with that unit's gate sequences."""
+    f64 = lambda t: t.double().cpu().numpy()
+    x, g, go, W0 = f64(inputs["x"]), f64(inputs["g_hat"]), f64(inputs["g_out"]), f64(inputs["W0"])
+    e, a = f64(eta), (f64(alpha) if alpha is not None else None)
+    ys, gs = np.zeros(x.shape[:-1] + (g.shape[-1],)), np.zeros(x.shape)
+    for l in range(wl.L):
+        for b in range(wl.B):
+            for h in range(wl.H):
+                y, gin = oracle.linear_scan(x[l, b, :, h][None], g[l, b, :, h][None], W0[l, h],
+                                            e[l, b, :, h], alpha=None if a is None else a[l, b, :, h],
+                                            gout=go[l, b, :, h][None])
+                ys[l, b, :, h] = y[0]
+                gs[l, b, :, h] = gin[0]
+    return ys, gs
+
+
+def _check(name, out, ref, tol):
+    out = out.double().cpu().numpy()
+    assert np.isfinite(out).all(), f"{name}: non-finite output"
+    err = rel_l2(out, ref)
+    assert err <= tol, f"{name}: rel-L2 {err:.3e} > {tol:.1e}"
+
+
+CASES = {
+    # (workload, resize, alpha?)
+    "eta_t-chunked-64": ("c5", dict(L=1, B=2, H=2, T=700), False),
+    "eta_t-segmented-64": ("c4", dict(B=1, H=2, T=3000), False),
+    "eta_t-chunked-128": ("c2", dict(B=1, H=2, T=900), False),
+    "eta_t-wide-256x512": ("c2", dict(B=1, H=1, T=600, d_in=256, d_out=512, w_std=1 / 16), False),
+    "alpha-serial-64": ("c5", dict(L=1, B=2, H=2, T=700), True),
+    "alpha-serial-128x64": ("c2", dict(B=1, H=2, T=500, d_in=128, d_out=64), True),
+    "alpha-serial-fp32": ("c1", dict(T=300), True),
+}
+
+
+@pytest.mark.parametrize("case", sorted(CASES))
+def test_gated_scans(case):
+    key, kw, with_alpha = CASES[case]
+    wl = W.workload(key).resized(**kw)
+    inputs = W.make_linear(wl)
+    eta, alpha = _gates(wl, 4242 + wl.T, with_alpha)
+    dev = {k: (v.cuda() if isinstance(v, torch.Tensor) else v) for k, v in inputs.items()}
+    y = gl.forward_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(),
+                        alpha=alpha.cuda() if alpha is not None else None)
+    gin = gl.costate_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), dev["g_out"],
+                          alpha=alpha.cuda() if alpha is not None else None)
+    torch.cuda.synchronize()
+    yr, gr = _oracle(inputs, eta, alpha, wl)
+    tol = TOL["f32"] if wl.dtype == "f32" else TOL["bf16"]
+    _check(f"{case} forward", y, yr, tol)
+    _check(f"{case} costate", gin, gr, tol)
+
+
+def test_reset_restarts_from_slow_weights():
+    """Right after a reset (alpha = 0 at token r) the fast weights are
+    W0 - eta_r ghat_r x_r^T, so the read at r+1 sees only that one write: the
+    outputs after the reset do not depend on any token before r."""
+    wl = W.workload("c5").resized(L=1, B=1, H=1, T=400)
+    inputs = W.make_linear(wl)
+    eta, alpha = _gates(wl, 7, True, resets=False)
+    alpha[..., 200, :] = 0.0
+    dev = {k: (v.cuda() if isinstance(v, torch.Tensor) else v) for k, v in inputs.items()}
+    y1 = gl.forward_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), alpha=alpha.cuda())
+    x2 = dev["x"].clone()
+    g2 = dev["g_hat"].clone()
+    x2[:, :, :200] = torch.randn_like(x2[:, :, :200].float()).to(x2.dtype)
+    g2[:, :, :200] = torch.randn_like(g2[:, :, :200].float()).to(g2.dtype)
+    y2 = gl.forward_scan(x2, g2, dev["W0"], eta.cuda(), alpha=alpha.cuda())
+    torch.cuda.synchronize()
+    assert torch.equal(y1[:, :, 201:], y2[:, :, 201:])
+    assert not torch.equal(y1[:, :, 150:200], y2[:, :, 150:200])
+
+
+def test_constant_gates_match_plain_scan():
+    """eta_t = eta everywhere and alpha = 1 is the plain scan (Eq. 3)."""
+    wl = W.workload("c5").resized(L=1, B=1, H=2, T=500)
+    inputs = W.make_linear(wl)
+    dev = {k: (v.cuda() if isinstance(v, torch.Tensor) else v) for k, v in inputs.items()}
+    shape = (wl.L, wl.B, wl.T, wl.H)
+    y_plain = gl.forward_scan(dev["x"], dev["g_hat"], dev["W0"], wl.eta)
+    y_serial = gl.forward_scan(dev["x"], dev["g_hat"], dev["W0"], wl.eta,
+                               alpha=torch.ones(shape, device="cuda"))
+    torch.cuda.synchronize()
+    err = rel_l2(y_serial.double().cpu().numpy(), y_plain.double().cpu().numpy())
+    assert err <= TOL["bf16"], f"serial vs chunked rel-L2 {err:.3e}"
