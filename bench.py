@@ -22,6 +22,7 @@ sample of the same workload.
 from __future__ import annotations
 
 import argparse
+import ctypes
 import json
 import os
 import statistics
@@ -150,20 +151,40 @@ class LinearJob:
 
     kind = "linear"
 
-    def __init__(self, gl, wl, device, rank):
+    def __init__(self, gl, wl, device, rank, gates=None):
         self.gl, self.wl = gl, wl
         self.inp = W.make_linear(wl.resized(seed=wl.seed + 1000 * rank), device=device)
         self.outs = {"y": torch.empty_like(self.inp["g_hat"]),
                      "g_in": torch.empty_like(self.inp["x"])}
-        self.ws = torch.empty(max(256, gl.workspace_bytes(wl.L, wl.B, wl.T, wl.H, wl.d_in,
-                                                          wl.d_out, 1 if wl.dtype == "bf16" else 0)),
-                              dtype=torch.uint8, device=device)
+        # Gated scans (Eq. 2): per-token eta_t in [0, 2 eta] and, for "alpha",
+        # retention alpha_t in [0.9, 1]; tensors [L, B, T, H] drawn once.
+        self.gates = gates
+        self.eta_t = self.alpha_t = None
+        code = 1 if wl.dtype == "bf16" else 0
+        nb = gl.workspace_bytes(wl.L, wl.B, wl.T, wl.H, wl.d_in, wl.d_out, code)
+        if gates:
+            gen = torch.Generator(device=device)
+            gen.manual_seed(wl.seed * 1000 + 17)
+            shape = (wl.L, wl.B, wl.T, wl.H)
+            self.eta_t = torch.rand(shape, generator=gen, device=device) * (2 * wl.eta)
+            if gates == "alpha":
+                self.alpha_t = 0.9 + 0.1 * torch.rand(shape, generator=gen, device=device)
+                self.inp["alpha_t"] = self.alpha_t
+            self.inp["eta_t"] = self.eta_t
+            from paper_2609_34174_gb300 import _binding as _B
+            d = _B._Desc(wl.L, wl.B, wl.T, wl.H, wl.d_in, wl.d_out, code, 0)
+            nb = int(_B.load_library().gradlev_workspace_bytes_gated(ctypes.byref(d)))
+        self.ws = torch.empty(max(256, nb), dtype=torch.uint8, device=device)
         self.tokens = wl.tokens
         self.launches_per_step = 2
-        self.in_keys = ("x", "g_hat", "g_out", "W0")
+        self.in_keys = ("x", "g_hat", "g_out", "W0") + (
+            ("eta_t",) if gates else ()) + (("alpha_t",) if gates == "alpha" else ())
         self.out_keys = ("y", "g_in")
         self.kernel = {"fwd": "tc_scan_kernel<64, false> (forward scan)",
                        "costate": "tc_scan_kernel<64, true> (costate scan)"}
+        if gates == "alpha":
+            self.kernel = {"fwd": "gated serial_kernel (forward scan)",
+                           "costate": "gated serial_kernel (costate scan)"}
 
     def input_bytes(self):
         return _bytes(self.inp["x"], self.inp["g_hat"], self.inp["g_out"])
@@ -173,11 +194,14 @@ class LinearJob:
         inp = inp or self.inp
         if events is not None:
             events[0].record()
-        gl.forward_scan(inp["x"], inp["g_hat"], inp["W0"], wl.eta, y=o["y"], workspace=self.ws)
+        eta = inp["eta_t"] if self.gates else wl.eta
+        alpha = inp.get("alpha_t")
+        gl.forward_scan(inp["x"], inp["g_hat"], inp["W0"], eta, y=o["y"], workspace=self.ws,
+                        alpha=alpha)
         if events is not None:
             events[1].record()
-        gl.costate_scan(inp["x"], inp["g_hat"], inp["W0"], wl.eta, inp["g_out"], g_in=o["g_in"],
-                        workspace=self.ws)
+        gl.costate_scan(inp["x"], inp["g_hat"], inp["W0"], eta, inp["g_out"], g_in=o["g_in"],
+                        workspace=self.ws, alpha=alpha)
         if events is not None:
             events[2].record()
 
@@ -199,8 +223,12 @@ class LinearJob:
 
     def config(self):
         wl = self.wl
-        return {"L": wl.L, "B": wl.B, "T": wl.T, "H": wl.H, "d_in": wl.d_in, "d_out": wl.d_out,
-                "eta": wl.eta}
+        c = {"L": wl.L, "B": wl.B, "T": wl.T, "H": wl.H, "d_in": wl.d_in, "d_out": wl.d_out,
+             "eta": wl.eta}
+        if self.gates:
+            c["gates"] = ("per-token eta_t" if self.gates == "eta"
+                          else "per-token eta_t and retention alpha_t (token-serial kernel)")
+        return c
 
     def oracle_run(self, inp, n_units, cores, t_tokens=None):
         """Time the fp64 oracle on the first n_units units (forward and costate
@@ -314,9 +342,12 @@ class MLPJob:
                 f"tokens, both layers forward and costate in one sequential walk, fp64")
 
 
-def make_job(gl, wl, device, rank):
-    return MLPJob(gl, wl, device, rank) if isinstance(wl, W.MLPWorkload) else LinearJob(
-        gl, wl, device, rank)
+def make_job(gl, wl, device, rank, gates=None):
+    if isinstance(wl, W.MLPWorkload):
+        if gates:
+            raise SystemExit("--gates applies to the linear workloads")
+        return MLPJob(gl, wl, device, rank)
+    return LinearJob(gl, wl, device, rank, gates)
 
 
 def cpu_baseline(job, inp, target_s=12.0):
@@ -466,7 +497,7 @@ def run_gradlev(args, wl, rank, world, local_rank):
     device = torch.device("cuda", local_rank)
     torch.cuda.set_device(device)
     gl.load_library()
-    job = make_job(gl, wl, device, rank)
+    job = make_job(gl, wl, device, rank, args.gates)
     flush = None
     if job.input_bytes() < 2 * L2_BYTES:
         flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
@@ -521,7 +552,7 @@ def run_gradlev(args, wl, rank, world, local_rank):
     dominant = "costate" if cos_ms >= fwd_ms else "fwd"
     rl = dict(scans[dominant]["roofline"])
     rl["kernel"] = job.kernel[dominant]
-    rl["traffic"] = None if args.resize else recorded_traffic(args.workload, dominant)
+    rl["traffic"] = None if (args.resize or args.gates) else recorded_traffic(args.workload, dominant)
     cfg = {"workload": f"{args.workload}: {wl.name}", **job.config(),
            "tokens_per_step": job.tokens, "parallelism": f"replicas x{world}",
            "l2": "inputs larger than L2" if flush is None else "L2 flushed between steps"}
@@ -550,6 +581,8 @@ def main(argv=None):
     ap.add_argument("--resize", default="",
                     help="comma-separated K=V overrides of the workload's sizes (e.g. L=2), "
                          "for small profiling captures; the headline uses the full workload")
+    ap.add_argument("--gates", default=None, choices=["eta", "alpha"],
+                    help="time the gated scans of Eq. 2: per-token eta_t, or eta_t with retention")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args(argv)

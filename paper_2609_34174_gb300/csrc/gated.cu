@@ -43,24 +43,50 @@ __device__ __forceinline__ void st(void* p, long long i, float v) {
         static_cast<float*>(p)[i] = v;
 }
 
-// ghat'[l,b,t,h,:] = eta_t[l,b,t,h] * ghat[l,b,t,h,:], written contiguous.
+// ghat'[l,b,t,h,:] = eta_t[l,b,t,h] * ghat[l,b,t,h,:], written contiguous.  One
+// thread per 16-byte piece of a token row (w a multiple of 16 bytes / element).
 template <bool BF16>
 __global__ void prescale_kernel(const void* __restrict__ g, TokStr gs, const float* __restrict__ eta,
                                 void* __restrict__ out, int L, int B, int T, int H, int w) {
-    const long long n = (long long)L * B * T * H * w;
-    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n;
-         i += (long long)gridDim.x * blockDim.x) {
-        const long long tok = i / w;
-        const int f = (int)(i - tok * w);
+    constexpr int kPer = BF16 ? 8 : 4;  // elements per 16 bytes
+    const int vpr = w / kPer;           // pieces per token row
+    const long long tokens = (long long)L * B * T * H;
+    const long long n = tokens * vpr;
+    for (long long v = (long long)blockIdx.x * blockDim.x + threadIdx.x; v < n;
+         v += (long long)gridDim.x * blockDim.x) {
+        const long long tok = v / vpr;
+        const int f = (int)(v - tok * vpr) * kPer;
         const int h = (int)(tok % H);
-        long long r = tok / H;
+        const long long r = tok / H;
         const int t = (int)(r % T);
-        r /= T;
-        const int b = (int)(r % B);
-        const int l = (int)(r / B);
+        const long long r2 = r / T;
+        const int b = (int)(r2 % B);
+        const int l = (int)(r2 / B);
         const long long src = (long long)l * gs.s[0] + (long long)b * gs.s[1] + (long long)t * gs.s[2] +
                               (long long)h * gs.s[3] + f;
-        st<BF16>(out, i, eta[tok] * ld<BF16>(g, src));
+        const float e = eta[tok];
+        uint4 in;
+        if constexpr (BF16)
+            in = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(g) + src);
+        else
+            in = *reinterpret_cast<const uint4*>(static_cast<const float*>(g) + src);
+        uint4 o;
+        if constexpr (BF16) {
+            const __nv_bfloat162* pi = reinterpret_cast<const __nv_bfloat162*>(&in);
+            __nv_bfloat162* po = reinterpret_cast<__nv_bfloat162*>(&o);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float2 x = __bfloat1622float2(pi[k]);
+                po[k] = __floats2bfloat162_rn(e * x.x, e * x.y);
+            }
+            *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(out) + tok * w + f) = o;
+        } else {
+            const float* pi = reinterpret_cast<const float*>(&in);
+            float* po = reinterpret_cast<float*>(&o);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) po[k] = e * pi[k];
+            *reinterpret_cast<uint4*>(static_cast<float*>(out) + tok * w + f) = o;
+        }
     }
 }
 
@@ -69,20 +95,24 @@ __global__ void prescale_kernel(const void* __restrict__ g, TokStr gs, const flo
 //            a = ghat (row-indexed), bvec = x (column-indexed)
 //   costate  (COSTATE = true):  outputs are columns d of W; q = g_out (length m),
 //            a = x (column-indexed), bvec = ghat (row-indexed)
-// Held per CTA (fp32): Wt[i][j] = W0 entry and Dt[i][j] = (W_t - W0) entry for output
-// i of the tile and input j (J = d forward, m costate).
+// Held per CTA (fp32): W0t[i][j] = W0 entry and Dt[i][j] = (W_t - W0) entry for
+// output i of the tile and input j (J = d forward, m costate).  Thread 4i+p owns
+// entries (i, j) with j = p mod 4: it both reads and writes exactly those, so a
+// token needs one barrier (its staged vectors, double-buffered).  The next
+// token's vectors are loaded into registers while this token is computed.
 template <bool COSTATE, bool BF16>
 __global__ void __launch_bounds__(kThreads)
     serial_kernel(GatedParams p) {
     extern __shared__ float sm[];
-    const int J = COSTATE ? p.dout : p.din;   // inputs of the read
+    const int J = COSTATE ? p.dout : p.din;   // inputs of the read (at most kThreads)
     const int NO = COSTATE ? p.din : p.dout;  // outputs of the read
-    float* W0t = sm;                          // [64][J]
-    float* Dt = W0t + kTile * J;              // [64][J]
-    float* qv = Dt + kTile * J;               // [J]  read vector
-    float* bv = qv + J;                       // [J]  write vector on the input side
-    float* av = bv + J;                       // [64] write vector on the output side
-    float* gate = av + kTile;                 // [2]  eta_t, alpha_t
+    // rows padded to J + 4 floats: the 8 rows x 4 parts a warp touches then fall in
+    // 32 distinct banks (row stride = 4 banks)
+    const int JS = J + 4;
+    float* W0t = sm;                          // [64][JS]
+    float* Dt = W0t + kTile * JS;             // [64][JS]
+    float* stage = Dt + kTile * JS;           // 2 x { q [J], b [J], a [64], eta, alpha }
+    const int sstride = 2 * J + kTile + 2;
 
     const int tiles = (NO + kTile - 1) / kTile;
     const int tile = blockIdx.x % tiles;
@@ -98,58 +128,90 @@ __global__ void __launch_bounds__(kThreads)
         const int o = o0 + i;
         float w = 0.0f;
         if (o < NO) w = COSTATE ? w0[(size_t)j * p.din + o] : w0[(size_t)o * p.din + j];
-        W0t[e] = w;
-        Dt[e] = 0.0f;
+        W0t[i * JS + j] = w;
+        Dt[i * JS + j] = 0.0f;
     }
-    const int i_own = threadIdx.x >> 2;  // output index of this thread's group of 4
-    const int part = threadIdx.x & 3;
-    for (int t = 0; t < p.T; ++t) {
-        const long long tok = ((long long)l * p.B + b) * p.T * p.H + (long long)t * p.H + h;
-        // stage this token's vectors
+    // what this thread stages: q[tid], b[tid] (tid < J), a[tid] (tid < 64), gates (tid 0)
+    const int tid = threadIdx.x;
+    auto fetch = [&](int t, float& qv, float& bv, float& av, float& ev, float& alv) {
         const long long xo = tok_off(p.x_s, l, b, t, h);
         const long long go = tok_off(p.g_s, l, b, t, h);
         const long long qo = tok_off(p.q_s, l, b, t, h);
-        for (int j = threadIdx.x; j < J; j += kThreads) {
-            qv[j] = ld<BF16>(p.q, qo + j);
-            bv[j] = COSTATE ? ld<BF16>(p.g, go + j) : ld<BF16>(p.x, xo + j);
+        if (tid < J) {
+            qv = ld<BF16>(p.q, qo + tid);
+            bv = COSTATE ? ld<BF16>(p.g, go + tid) : ld<BF16>(p.x, xo + tid);
         }
-        for (int i = threadIdx.x; i < kTile; i += kThreads) {
-            const int o = o0 + i;
-            av[i] = o < NO ? (COSTATE ? ld<BF16>(p.x, xo + o) : ld<BF16>(p.g, go + o)) : 0.0f;
+        if (tid < kTile) {
+            const int o = o0 + tid;
+            av = o < NO ? (COSTATE ? ld<BF16>(p.x, xo + o) : ld<BF16>(p.g, go + o)) : 0.0f;
         }
-        if (threadIdx.x == 0) {
-            gate[0] = p.eta[tok];
-            gate[1] = p.alpha ? p.alpha[tok] : 1.0f;
+        if (tid == 0) {
+            const long long tok = ((long long)l * p.B + b) * p.T * p.H + (long long)t * p.H + h;
+            ev = p.eta[tok];
+            alv = p.alpha ? p.alpha[tok] : 1.0f;
         }
-        __syncthreads();
-        // read before write: out_i = sum_j (W0 + D)[i][j] q_j
-        float acc = 0.0f;
-        const float* w_row = W0t + i_own * J;
-        const float* d_row = Dt + i_own * J;
-        for (int j = part; j < J; j += 4) acc += (w_row[j] + d_row[j]) * qv[j];
-        acc += __shfl_xor_sync(0xffffffffu, acc, 1);
-        acc += __shfl_xor_sync(0xffffffffu, acc, 2);
-        const int o = o0 + i_own;
-        if (part == 0 && o < NO) {
-            const EpiParams& e = p.epi;
-            const long long oo = tok_off(e.out_str, l, b, t, h) + o;
-            float v = acc;
-            if (e.zin) {
-                const long long zo = tok_off(e.z_str, l, b, t, h) + o;
-                v *= act_df(e.act, ld<BF16>(e.zin, zo));
+    };
+    auto put = [&](int buf, float qv, float bv, float av, float ev, float alv) {
+        float* s = stage + buf * sstride;
+        if (tid < J) {
+            s[tid] = qv;
+            s[J + tid] = bv;
+        }
+        if (tid < kTile) s[2 * J + tid] = av;
+        if (tid == 0) {
+            s[2 * J + kTile] = ev;
+            s[2 * J + kTile + 1] = alv;
+        }
+    };
+    // register ring of the next kAhead tokens' vectors (slots indexed by t mod kAhead)
+    constexpr int kAhead = 4;
+    float qv[kAhead], bv[kAhead], av[kAhead], ev[kAhead], alv[kAhead];
+#pragma unroll
+    for (int u = 0; u < kAhead; ++u) {
+        qv[u] = bv[u] = av[u] = ev[u] = 0.0f;
+        alv[u] = 1.0f;
+        if (u < p.T) fetch(u, qv[u], bv[u], av[u], ev[u], alv[u]);
+    }
+    if (p.T > 0) put(0, qv[0], bv[0], av[0], ev[0], alv[0]);
+    const int i_own = threadIdx.x >> 2;  // output index of this thread's group of 4
+    const int part = threadIdx.x & 3;
+    const int o = o0 + i_own;
+    float* w_row = W0t + i_own * JS;
+    float* d_row = Dt + i_own * JS;
+    for (int t0 = 0; t0 < p.T; t0 += kAhead) {
+#pragma unroll
+        for (int u = 0; u < kAhead; ++u) {
+            const int t = t0 + u;
+            if (t >= p.T) break;
+            __syncthreads();  // token t staged; token t-1's buffer no longer read
+            const float* s = stage + (t & 1) * sstride;
+            const float* q = s;
+            const float* bw = s + J;
+            const float a_i = s[2 * J + i_own];
+            const float eta = s[2 * J + kTile], alpha = s[2 * J + kTile + 1];
+            // read before write: out_i = sum_j (W0 + D)[i][j] q_j, then
+            // write D[i][j] = alpha D[i][j] - eta a_i b_j on the same entries
+            float acc = 0.0f;
+            for (int j = part; j < J; j += 4) {
+                const float dv = d_row[j];
+                acc += (w_row[j] + dv) * q[j];
+                d_row[j] = alpha * dv - eta * a_i * bw[j];
             }
-            st<BF16>(e.out, oo, v);
-            if (e.out2) st<BF16>(e.out2, tok_off(e.out2_str, l, b, t, h) + o, act_f(e.act, acc));
+            acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+            acc += __shfl_xor_sync(0xffffffffu, acc, 2);
+            if (part == 0 && o < NO) {
+                const EpiParams& e = p.epi;
+                const long long oo = tok_off(e.out_str, l, b, t, h) + o;
+                float v = acc;
+                if (e.zin) v *= act_df(e.act, ld<BF16>(e.zin, tok_off(e.z_str, l, b, t, h) + o));
+                st<BF16>(e.out, oo, v);
+                if (e.out2) st<BF16>(e.out2, tok_off(e.out2_str, l, b, t, h) + o, act_f(e.act, acc));
+            }
+            // stage token t+1 (fetched kAhead-1 tokens ago), then refill this slot
+            const int un = (u + 1) % kAhead;
+            if (t + 1 < p.T) put((t + 1) & 1, qv[un], bv[un], av[un], ev[un], alv[un]);
+            if (t + kAhead < p.T) fetch(t + kAhead, qv[u], bv[u], av[u], ev[u], alv[u]);
         }
-        // every read of D for this token is done before the write
-        __syncthreads();
-        // write: D = alpha D - eta a b^T
-        const float eta = gate[0], alpha = gate[1];
-        for (int e = threadIdx.x; e < kTile * J; e += kThreads) {
-            const int i = e / J, j = e - i * J;
-            Dt[e] = alpha * Dt[e] - eta * av[i] * bv[j];
-        }
-        __syncthreads();
     }
 }
 
@@ -166,7 +228,7 @@ cudaError_t launch_serial(const GatedParams& p, int blocks, size_t smem, cudaStr
 
 size_t gated_serial_smem(int din, int dout, bool costate) {
     const int J = costate ? dout : din;
-    return sizeof(float) * ((size_t)2 * gated::kTile * J + 2 * (size_t)J + gated::kTile + 2);
+    return sizeof(float) * ((size_t)2 * gated::kTile * (J + 4) + 2 * (2 * (size_t)J + gated::kTile + 2));
 }
 
 cudaError_t launch_gated_serial(const GatedParams& p, bool costate, bool bf16, cudaStream_t stream) {
@@ -184,7 +246,7 @@ cudaError_t launch_gated_serial(const GatedParams& p, bool costate, bool bf16, c
 
 cudaError_t launch_gated_prescale(const void* g, const TokStr& gs, const float* eta, void* out, int L,
                                   int B, int T, int H, int w, bool bf16, cudaStream_t stream) {
-    const long long n = (long long)L * B * T * H * w;
+    const long long n = (long long)L * B * T * H * (w / (bf16 ? 8 : 4));
     if (n <= 0) return cudaSuccess;
     long long blocks = (n + 255) / 256;
     if (blocks > 152 * 16) blocks = 152 * 16;

@@ -497,7 +497,10 @@ int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
     if (!resolve(d, x, d.d_in, &tx, true) || !resolve(d, g_hat, d.d_out, &tg, true))
         return GRADLEV_ERR_INVALID_ARG;
     if (!alpha_t) {
-        // eta_t only: scale the writes' proposals, then the ungated scan with eta = 1
+        // eta_t only: scale the writes' proposals, then the ungated scan with eta = 1.
+        // The scaling pass moves 16-byte pieces of each token row.
+        if (d.d_out % (bf16 ? 8 : 4) != 0 || !tc_layout_ok(tg, bf16 ? 2 : 4))
+            return GRADLEV_ERR_UNSUPPORTED;
         const size_t a = ws_bytes_for(d, d.d_in, d.d_out, dev.sms);
         const size_t b = ws_bytes_for(d, d.d_out, d.d_in, dev.sms);
         const size_t base = round_up(a > b ? a : b, 256);
