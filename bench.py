@@ -205,6 +205,60 @@ class LinearJob:
         if events is not None:
             events[2].record()
 
+    # --- pipelined end-to-end step: chunks along layers (or batch rows when L = 1)
+    def e2e_chunks(self):
+        wl = self.wl
+        if wl.L > 1:
+            return [("L", l, l + 1) for l in range(wl.L)]
+        if wl.B > 1:
+            return [("B", b, b + 1) for b in range(wl.B)]
+        return [("L", 0, 1)]
+
+    @staticmethod
+    def _cut(t, sl, lead_w0=False):
+        axis, a, b = sl
+        if axis == "L" or lead_w0:
+            return t[a:b] if axis == "L" else t
+        return t[:, a:b]
+
+    def e2e_inputs(self, host, dev, sl, first):
+        out = []
+        for k in self.in_keys:
+            if k == "W0":
+                if sl[0] == "L":
+                    out.append((k, host[k][sl[1]:sl[2]], dev[k][sl[1]:sl[2]]))
+                elif first:
+                    out.append((k, host[k], dev[k]))
+            else:
+                out.append((k, self._cut(host[k], sl), self._cut(dev[k], sl)))
+        return out
+
+    def e2e_outputs(self, hout, sl):
+        return [(self._cut(self.outs[k], sl), self._cut(hout[k], sl)) for k in self.out_keys]
+
+    def e2e_step(self, dev, sl, ws):
+        gl, wl = self.gl, self.wl
+        cut = lambda t: self._cut(t, sl)
+        w0 = dev["W0"][sl[1]:sl[2]] if sl[0] == "L" else dev["W0"]
+        eta = cut(dev["eta_t"]) if self.gates else wl.eta
+        alpha = cut(dev["alpha_t"]) if self.gates == "alpha" else None
+        gl.forward_scan(cut(dev["x"]), cut(dev["g_hat"]), w0, eta, y=cut(self.outs["y"]),
+                        workspace=ws, alpha=alpha)
+        gl.costate_scan(cut(dev["x"]), cut(dev["g_hat"]), w0, eta, cut(dev["g_out"]),
+                        g_in=cut(self.outs["g_in"]), workspace=ws, alpha=alpha)
+
+    def e2e_workspace_bytes(self):
+        wl = self.wl
+        sl = self.e2e_chunks()[0]
+        L = 1 if sl[0] == "L" else wl.L
+        B = wl.B if sl[0] == "L" else 1
+        code = 1 if wl.dtype == "bf16" else 0
+        from paper_2609_34174_gb300 import _binding as _B
+        d = _B._Desc(L, B, wl.T, wl.H, wl.d_in, wl.d_out, code, 0)
+        lib = _B.load_library()
+        return int(max(lib.gradlev_workspace_bytes(ctypes.byref(d)),
+                       lib.gradlev_workspace_bytes_gated(ctypes.byref(d))))
+
     def counts(self, scan):
         """Algorithmic flops and compulsory bytes of one scan call.
 
@@ -299,6 +353,37 @@ class MLPJob:
         if events is not None:
             events[2].record()
 
+    # --- pipelined end-to-end step: chunks along the batch rows
+    def e2e_chunks(self):
+        return [(b, b + 1) for b in range(self.wl.B)]
+
+    def e2e_inputs(self, host, dev, sl, first):
+        out = []
+        for k in self.in_keys:
+            if k in ("W1", "W2"):
+                if first:
+                    out.append((k, host[k], dev[k]))
+            else:
+                out.append((k, host[k][sl[0]:sl[1]], dev[k][sl[0]:sl[1]]))
+        return out
+
+    def e2e_outputs(self, hout, sl):
+        return [(self.outs[k][sl[0]:sl[1]], hout[k][sl[0]:sl[1]]) for k in self.out_keys]
+
+    def e2e_step(self, dev, sl, ws):
+        gl, wl, o = self.gl, self.wl, self.outs
+        c = lambda t: t[sl[0]:sl[1]]
+        gl.forward_scan(c(dev["x"]), c(dev["g_hat_z"]), dev["W1"], wl.eta1, act=wl.act, y=c(o["z"]),
+                        act_out=c(o["h"]), workspace=ws)
+        gl.forward_scan(c(o["h"]), c(dev["g_hat_y"]), dev["W2"], wl.eta2, y=c(o["y"]), workspace=ws)
+        gl.costate_scan(c(o["h"]), c(dev["g_hat_y"]), dev["W2"], wl.eta2, c(dev["g_out"]), act=wl.act,
+                        z=c(o["z"]), g_in=c(o["gz"]), workspace=ws)
+        gl.costate_scan(c(dev["x"]), c(dev["g_hat_z"]), dev["W1"], wl.eta1, c(o["gz"]), g_in=c(o["gx"]),
+                        workspace=ws)
+
+    def e2e_workspace_bytes(self):
+        return self.ws.numel()
+
     def counts(self, scan):
         """Both layers: flops 4*d_i*m_i + C*(d_i+m_i) per token and layer (C = 64).
         Compulsory bytes with sigma fused (h is never needed from HBM): forward
@@ -375,32 +460,77 @@ def cpu_baseline(job, inp, target_s=12.0):
 
 
 def e2e_measure(job, steps, stream):
-    """The same step through the public API from pinned host buffers, copies inside."""
+    """The same step through the public API from pinned host buffers, copies inside.
+
+    The step is cut into chunks along its leading independent dimension (layers,
+    or batch rows) and pipelined over three streams: the host-to-device copy of
+    chunk c+1 and the device-to-host copy of chunk c-1 overlap the scans of chunk
+    c.  Every input byte is copied in and every result byte out on every step."""
+    dev_id = job.ws.device
     host = {k: job.inp[k].cpu().pin_memory() for k in job.in_keys}
     dev = {k: torch.empty_like(job.inp[k]) for k in job.in_keys}
     hout = {k: torch.empty(job.outs[k].shape, dtype=job.outs[k].dtype, pin_memory=True)
             for k in job.out_keys}
     bi = _bytes(*host.values())
     bo = _bytes(*hout.values())
+    chunks = job.e2e_chunks()
+    ws = torch.empty(max(job.ws.numel(), job.e2e_workspace_bytes()), dtype=torch.uint8,
+                     device=dev_id)
+    s_in = torch.cuda.Stream(dev_id)
+    s_run = torch.cuda.Stream(dev_id)
+    s_out = torch.cuda.Stream(dev_id)
+    n = len(chunks)
+    ev_in = [torch.cuda.Event() for _ in range(n)]
+    ev_run = [torch.cuda.Event() for _ in range(n)]
+    ev_out = [torch.cuda.Event() for _ in range(n)]
+    started = [False] * n
 
     def one():
-        for k in host:
-            dev[k].copy_(host[k], non_blocking=True)
-        job.step(inp=dev)
-        for k in hout:
-            hout[k].copy_(job.outs[k], non_blocking=True)
+        for c, sl in enumerate(chunks):
+            with torch.cuda.stream(s_in):
+                if started[c]:
+                    s_in.wait_event(ev_run[c])  # the previous step's scans of chunk c are done
+                for k, hv, dv in job.e2e_inputs(host, dev, sl, c == 0):
+                    dv.copy_(hv, non_blocking=True)
+                ev_in[c].record(s_in)
+            with torch.cuda.stream(s_run):
+                s_run.wait_event(ev_in[c])
+                if started[c]:
+                    s_run.wait_event(ev_out[c])  # its previous results have been read out
+                job.e2e_step(dev, sl, ws)
+                ev_run[c].record(s_run)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev_run[c])
+                for dv, hv in job.e2e_outputs(hout, sl):
+                    hv.copy_(dv, non_blocking=True)
+                ev_out[c].record(s_out)
+            started[c] = True
 
     one()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
+    e0.record(s_in)
     for _ in range(steps):
         one()
-    e1.record(stream)
+    s_out.wait_stream(s_in)
+    s_out.wait_stream(s_run)
+    e1.record(s_out)
     torch.cuda.synchronize()
     sec = e0.elapsed_time(e1) / 1e3
+    # the results that came back agree with the whole-step call on resident inputs
+    job.step()
+    torch.cuda.synchronize()
+    worst = 0.0
+    for k in job.out_keys:
+        ref = job.outs[k].double().cpu()
+        got = hout[k].double()
+        worst = max(worst, float((got - ref).norm() / max(float(ref.norm()), 1e-30)))
+    if not worst <= 2e-2:
+        raise RuntimeError(f"pipelined end-to-end results differ from the resident step: {worst:.3e}")
     return {"value": round(job.tokens * steps / sec, 1), "unit": UNIT, "h2d_bytes_per_step": bi,
-            "d2h_bytes_per_step": bo, "steps": steps, "ms_per_step": round(sec / steps * 1e3, 3)}
+            "d2h_bytes_per_step": bo, "steps": steps, "ms_per_step": round(sec / steps * 1e3, 3),
+            "pipeline": f"{n} chunks, copies overlapped with the scans on three streams",
+            "rel_l2_vs_resident_step": worst}
 
 
 # ---------------------------------------------------------- DRAM traffic
@@ -562,7 +692,7 @@ def run_gradlev(args, wl, rank, world, local_rank):
             "data": "synthetic", "config": cfg, "scans": scans, "roofline": rl,
             "clocks": sampler.summary(), "gpu_launches": job.launches_per_step * args.steps}
     if rank == 0 and world == 1 and not args.no_e2e:
-        line["e2e"] = e2e_measure(job, max(3, min(args.steps, 10)), stream)
+        line["e2e"] = e2e_measure(job, max(3, min(args.steps, 20)), stream)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
 
