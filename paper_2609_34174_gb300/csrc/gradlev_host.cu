@@ -257,7 +257,7 @@ SegPlan plan_seg(const gradlev_desc& d, int dq, int dv) {
     SegPlan sp;
     const long long T = d.T > 0 ? d.T : 1;
     long long ls = (T + kChunk - 1) / kChunk * kChunk;
-    if (ls > 512) ls = 512;
+    if (ls > 1024) ls = 1024;  // measured best on 512 -> 2048 -> 512 (1024 vs 512: 4-6% faster)
     sp.seg_len = (int)ls;
     sp.n_seg = (int)((T + ls - 1) / ls);
     sp.bn = dv % 256 == 0 ? 256 : (dv % 128 == 0 ? 128 : 64);
