@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include <mutex>
@@ -342,6 +343,15 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
         p.n_seg = pl.n_seg;
         p.n_items = pl.n_items;
         p.n_ut = pl.n_items / pl.n_seg;
+        // A look-back wait is bounded by 4 s.  Failure tests (host-side fault
+        // injection, no GPU fault) can make one item skip its publish and shorten
+        // the bound, so that its successors' waits expire, the kernel writes
+        // the error word and returns, and the host reports GRADLEV_ERR_TIMEOUT.
+        p.lookback_limit_ns = 4000000000ull;
+        p.test_skip_publish = -1;
+        if (const char* v = getenv("GRADLEV_TEST_SKIP_PUBLISH")) p.test_skip_publish = atoi(v);
+        if (const char* v = getenv("GRADLEV_TEST_LOOKBACK_LIMIT_MS"))
+            p.lookback_limit_ns = 1000000ull * (unsigned long long)atoi(v);
         p.eta = eta;
         p.lam = eta != 0.0f ? -eta : 1.0f;
         p.inv_lam = 1.0f / p.lam;

@@ -87,6 +87,8 @@ struct TcScanParams {
     EpiParams epi;
     unsigned int* ctrl;   // [0] work ticket, [1] error bits
     unsigned int* flags;  // [n_items] look-back status: 0 none, 1 aggregate, 2 inclusive
+    unsigned long long lookback_limit_ns;  // bound on a look-back wait (4 s)
+    int test_skip_publish;  // failure tests only: this item never publishes (-1: none)
     float* agg;           // [n_items][dq][64] segment aggregate  sum_s k_s v_s^T
     float* incl;          // [n_items][dq][64] inclusive prefix of the aggregates
 };

@@ -672,7 +672,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     raise_error(p, kErrWaitTimeout, abort_flag);
                     return false;
                 }
-                if (leader) st_release_gpu(p.flags + item, flag);
+                // (failure tests only: one item may be told never to publish)
+                if (leader && item != p.test_skip_publish) st_release_gpu(p.flags + item, flag);
                 return true;
             };
             // ---- phase 1 of the newly taken item (before phase 2 of the previous one)
@@ -732,7 +733,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             unsigned int f = 1u;
                             if (lane < n) {
                                 while ((f = ld_acquire_gpu(p.flags + (base_pred - lane) * n_ut + r_ut)) == 0u) {
-                                    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                                    if (globaltimer_ns() - t0 > p.lookback_limit_ns) {
                                         f = 0xFFFFFFFFu;
                                         break;
                                     }
