@@ -229,3 +229,23 @@ def test_full_size_sampled_units(key):
     yr, gr = oracle_linear(inputs, units, wl.eta)
     _assert_close(f"{key} full forward", gpu_units(y, units), yr, TOL["bf16"])
     _assert_close(f"{key} full costate", gpu_units(gin, units), gr, TOL["bf16"])
+
+
+# ------------------------------------------------ pipeline phase bookkeeping
+SWEEP_T = sorted(set(list(range(1, 3 * 128 + 1, 11)) + [63, 64, 65, 127, 128, 129, 191, 192, 193,
+                                                        255, 256, 257, 383, 384]))
+
+
+@pytest.mark.parametrize("dq", [64, 128])
+def test_length_sweep_one_to_three_chunks(dq):
+    """Every sequence length in a dense sweep over 1..3 chunks (128 tokens each),
+    many units per launch, so each CTA walks its stage ring, TMEM buffers and
+    barrier phases through many item boundaries with partial chunks.  Each length
+    is checked against the oracle."""
+    for T in SWEEP_T:
+        wl = W.workload("c2" if dq == 128 else "c5").resized(L=1, B=3, H=5, T=T, d_in=dq, d_out=64,
+                                                            seed=300 + T)
+        inputs = W.make_linear(wl)
+        y, g, yr, gr = _run_linear(wl, inputs)
+        _assert_close(f"T={T} forward", y, yr, TOL["bf16"])
+        _assert_close(f"T={T} costate", g, gr, TOL["bf16"])
