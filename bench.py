@@ -706,7 +706,7 @@ def main(argv=None):
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--workload", default="c5", choices=["c1", "c2", "c3", "c4", "c5"])
+    ap.add_argument("--workload", default="c5", choices=["c1", "c2", "c3", "c4", "c5", "paper_mlp"])
     ap.add_argument("--impl", default="gradlev", choices=["gradlev", "reference"])
     ap.add_argument("--resize", default="",
                     help="comma-separated K=V overrides of the workload's sizes (e.g. L=2), "

@@ -91,3 +91,10 @@ def test_mlp_full_size_sampled_sequences():
     wl = W.workload("c3")
     inp = W.make_mlp(wl, device="cuda")
     _mlp_check(wl, inp, [0, 3])
+
+
+def test_paper_shaped_final_mlp():
+    """The adapted final MLP at the paper's own shape: 1024 -> 4096 -> 1024 with
+    GELU, T = 1024 (the training context), two sequences, checked in full."""
+    wl = W.workload("c3").resized(B=2, T=1024, d=1024, m=4096, k=1024)
+    _mlp_check(wl, W.make_mlp(wl), [0, 1])

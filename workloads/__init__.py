@@ -94,6 +94,11 @@ WORKLOADS = {
     "c3": MLPWorkload("mlp-B4-T4096-512x2048x512-gelu-bf16", B=4, T=4096, d=512, m=2048, k=512,
                       dtype="bf16", eta1=0.01, eta2=0.01, act="gelu_tanh", g_std=0.02,
                       seed=BASE_SEED + 2),
+    # The paper's adapted final MLP at its training context (not one of the five
+    # scan workloads; used by tests and bench --workload paper_mlp).
+    "paper_mlp": MLPWorkload("final-mlp-B2-T1024-1024x4096x1024-gelu-bf16", B=2, T=1024, d=1024,
+                             m=4096, k=1024, dtype="bf16", eta1=0.01, eta2=0.01, act="gelu_tanh",
+                             g_std=0.02, seed=BASE_SEED + 7),
     "c4": LinearWorkload("longctx-B2-H16-T32768-64x64-bf16", L=1, B=2, T=32768, H=16, d_in=64,
                          d_out=64, dtype="bf16", eta=0.02, x_dist="unitnorm", x_std=1.0,
                          g_dist="student_t4", g_std=0.02, w_std=1 / 8, seed=BASE_SEED + 3),
