@@ -130,18 +130,24 @@ def mlp_scan(x, ghz, ghy, W10, W20, eta1, eta2, act=ACT_GELU_TANH, alpha=None, g
     W10 [m,d], W20 [k,m], gout [U,T,k] or None.
     Returns a dict with z, h [U,T,m], y [U,T,k] and, when gout is given,
     gh (= W2_t^T gout), gz (= sigma'(z) * gh) [U,T,m] and gx (= W1_t^T gz) [U,T,d].
+    A proposal of None writes the true costate instead (deployment): ghz None
+    writes gz_t, ghy None writes gout_t.
     """
     lib = _load()
     x = _f64(x)
-    ghz = _f64(ghz)
-    ghy = _f64(ghy)
     U, T, d = x.shape
-    m = ghz.shape[2]
     W10 = _f64(W10)
     W20 = _f64(W20)
+    m = W10.shape[0]
     k = W20.shape[0]
-    if W10.shape != (m, d) or W20.shape != (k, m) or ghy.shape != (U, T, k):
+    ghz = None if ghz is None else _f64(ghz)
+    ghy = None if ghy is None else _f64(ghy)
+    if W10.shape != (m, d) or W20.shape != (k, m):
         raise ValueError("mlp shape mismatch")
+    if (ghz is not None and ghz.shape != (U, T, m)) or (ghy is not None and ghy.shape != (U, T, k)):
+        raise ValueError("mlp proposal shape mismatch")
+    if (ghz is None or ghy is None) and gout is None:
+        raise ValueError("deployment (a proposal of None) needs gout")
     e1 = _steps(eta1, T)
     e2 = _steps(eta2, T)
     al = None if alpha is None else _steps(alpha, T)
@@ -159,6 +165,14 @@ def mlp_scan(x, ghz, ghy, W10, W20, eta1, eta2, act=ACT_GELU_TANH, alpha=None, g
     if rc != 0:
         raise MemoryError("oracle_mlp_batch could not allocate scratch")
     return out
+
+
+def mlp_deploy(x, W10, W20, eta1, eta2, gout, act=ACT_GELU_TANH, alpha=None, nthreads=0):
+    """The deployed online MLP (Sec. 3; Appendix A): after each scored target both
+    layers write their true costates, gout_t at layer 2 and gz_t at layer 1.
+    Same shapes and outputs as mlp_scan."""
+    return mlp_scan(x, None, None, W10, W20, eta1, eta2, act=act, alpha=alpha, gout=gout,
+                    nthreads=nthreads)
 
 
 def act(code, z):

@@ -167,6 +167,9 @@ int oracle_linear_batch(int U, int T, int d, int m, const double* x, const doubl
  *   writes (online-update, with the proposals as the written costates):
  *     W1 <- W10 + alpha (W1 - W10) - eta1_t ghz_t x_t^T
  *     W2 <- W20 + alpha (W2 - W20) - eta2_t ghy_t h_t^T
+ * Deployment (Sec. 3, training objective paragraph; Appendix A: after each scored
+ * target the learner writes true costates): with ghz NULL layer 1 writes its
+ * reconstructed gz_t, and with ghy NULL layer 2 writes gout_t.  Either needs gout.
  * Widths: input d, hidden m, output k (Appendix A has k = d; Sec. 4.1 uses 4->7->3).
  * Shapes: x [T][d], ghz [T][m], ghy [T][k], W10 [m][d], W20 [k][m], gout [T][k].
  * Outputs (each nullable): z, h [T][m]; y [T][k]; gh, gz [T][m]; gx [T][d].
@@ -218,8 +221,10 @@ void oracle_mlp(int T, int d, int m, int k, int act, const double* x, const doub
             }
         }
         double a = alpha ? alpha[t] : 1.0;
-        write_update(m, d, W1s, W10, a, eta1[t], ghz + (size_t)t * m, xt);
-        write_update(k, m, W2s, W20, a, eta2[t], ghy + (size_t)t * k, ht);
+        /* in deployment gz_t is still in ght: it is written before being overwritten */
+        write_update(m, d, W1s, W10, a, eta1[t], ghz ? ghz + (size_t)t * m : ght, xt);
+        write_update(k, m, W2s, W20, a, eta2[t], ghy ? ghy + (size_t)t * k : gout + (size_t)t * k,
+                     ht);
     }
 }
 
@@ -231,6 +236,7 @@ int oracle_mlp_batch(int U, int T, int d, int m, int k, int act, const double* x
                      const double* gout, double* z, double* h, double* y, double* gh, double* gz,
                      double* gx, int nthreads) {
     int err = 0;
+    if ((!ghz || !ghy) && !gout) return -2;
 #ifdef _OPENMP
     if (nthreads > 0) omp_set_num_threads(nthreads);
 #else
@@ -248,7 +254,8 @@ int oracle_mlp_batch(int U, int T, int d, int m, int k, int act, const double* x
 #pragma omp for schedule(dynamic, 1)
             for (int u = 0; u < U; ++u) {
                 size_t tm = (size_t)u * T * m, td = (size_t)u * T * d, tk = (size_t)u * T * k;
-                oracle_mlp(T, d, m, k, act, x + td, ghz + tm, ghy + tk, W10, W20, eta1, eta2,
+                oracle_mlp(T, d, m, k, act, x + td, ghz ? ghz + tm : NULL, ghy ? ghy + tk : NULL,
+                           W10, W20, eta1, eta2,
                            alpha, gout ? gout + tk : NULL, z ? z + tm : NULL, h ? h + tm : NULL,
                            y ? y + tk : NULL, gh ? gh + tm : NULL, gz ? gz + tm : NULL,
                            gx ? gx + td : NULL, W1s, W2s, tmp);

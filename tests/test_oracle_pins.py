@@ -336,3 +336,40 @@ def test_activation_values():
     assert abs(oracle.act_deriv(oracle.ACT_GELU_TANH, np.array([0.0]))[0] - 0.5) < 1e-15
     np.testing.assert_allclose(oracle.act(oracle.ACT_NONE, z), z)
     np.testing.assert_allclose(oracle.act_deriv(oracle.ACT_NONE, z), np.ones_like(z))
+
+
+# -------------------------------------------------------------- deployment
+@pytest.mark.parametrize("seed", [17, 42])
+def test_mlp_deploy_matches_serial_learner(seed):
+    """Deployment writes true costates (Sec. 3; Appendix A): layer 2 writes the
+    supplied gout_t and layer 1 its own reconstructed gz_t.  The hand-written serial
+    learner of Sec. 4.1 does exactly that, so the deployed oracle reproduces it."""
+    p = _e1_serial(seed)
+    o = oracle.mlp_deploy(p["x"][None], p["W10"], p["W20"], p["eta1"], p["eta2"],
+                          gout=p["gy"][None], act=oracle.ACT_TANH, alpha=p["alpha"])
+    assert np.abs(o["y"][0] - p["y"]).max() < 1e-13
+    assert np.abs(o["gz"][0] - p["gz"]).max() < 1e-13
+
+
+def test_mlp_deploy_is_the_fixed_point_of_proposals():
+    """Theorem 1: the reconstructed costate at token t depends only on proposals
+    before t, so sweeping G <- F(G) from zero proposals fixes one more token per
+    sweep and reaches the deployed learner's costates after T sweeps."""
+    U, T, d, m, k = 2, 12, 5, 9, 4
+    r = _rng(321)
+    x = r.standard_normal((U, T, d))
+    gout = r.standard_normal((U, T, k)) * 0.5
+    W10 = r.standard_normal((m, d)) / np.sqrt(d)
+    W20 = r.standard_normal((k, m)) / np.sqrt(m)
+    eta1, eta2 = 0.2, 0.1
+    dep = oracle.mlp_deploy(x, W10, W20, eta1, eta2, gout=gout, act=oracle.ACT_GELU_TANH)
+    ghz = np.zeros((U, T, m))
+    for n in range(1, T + 1):
+        o = oracle.mlp_scan(x, ghz, gout, W10, W20, eta1, eta2, act=oracle.ACT_GELU_TANH,
+                            gout=gout)
+        ghz = o["gz"]
+        assert np.abs(ghz[:, :n] - dep["gz"][:, :n]).max() < 1e-12
+        if n <= 3:  # later tokens still see a wrong history (the gap shrinks every sweep)
+            assert np.abs(ghz[:, n:] - dep["gz"][:, n:]).max() > 1e-9
+    for key in ("z", "h", "y", "gh", "gx"):
+        assert np.abs(o[key] - dep[key]).max() < 1e-12, key
