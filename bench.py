@@ -585,7 +585,23 @@ def run_reference(args, wl, rank, world):
 
     oracle.build()
     cores = len(os.sched_getaffinity(0))
-    if isinstance(wl, W.MLPWorkload):
+    metric = METRIC
+    if args.workload == "decode_mlp":
+        inp = W.make_mlp(wl, device="cpu")
+        f = lambda t, T: t[:, :T].to(torch.float64).numpy()
+        W1, W2 = inp["W1"].double().numpy(), inp["W2"].double().numpy()
+        t_tok = 16
+
+        def run():
+            t0 = time.perf_counter()
+            oracle.mlp_deploy(f(inp["x"], t_tok), W1, W2, wl.eta1, wl.eta2,
+                              gout=f(inp["g_out"], t_tok), act=oracle.ACT_GELU_TANH,
+                              nthreads=min(cores, wl.B))
+            return time.perf_counter() - t0, wl.B * t_tok
+
+        sample = f"{wl.B} sequences x {t_tok} tokens of the deployed MLP per step, fp64"
+        metric = DECODE_METRIC
+    elif isinstance(wl, W.MLPWorkload):
         inp = W.make_mlp(wl, device="cpu")
         job = MLPJob.__new__(MLPJob)
         job.wl = wl
@@ -610,7 +626,7 @@ def run_reference(args, wl, rank, world):
         sec += dt
         tokens += tk
     value = tokens / sec
-    return {"impl": "reference", "metric": METRIC, "value": round(value, 1), "unit": UNIT,
+    return {"impl": "reference", "metric": metric, "value": round(value, 1), "unit": UNIT,
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(sec / args.steps * 1e3, 3), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
@@ -619,6 +635,226 @@ def run_reference(args, wl, rank, world):
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
+
+
+DECODE_METRIC = "deployment tokens/s (one token per sequence per step) at 1 GB300; % of HBM roofline"
+
+
+class DecodeMLPJob:
+    """Deployment of the two-layer MLP (Sec. 3; Appendix A): every step each of the
+    B sequences advances one token.  Layer 1 is read (sigma fused), then layer 2;
+    with the scored token's costate, layer 2 is written together with its costate
+    read (sigma' fused, giving gz) and layer 1 is written with gz.  The fast
+    weights live on the device as Delta = W - W0 in fp32 between steps."""
+
+    kernels = ("read L1", "read L2", "write L2 + g_in", "write L1")
+
+    def __init__(self, gl, wl, device, rank):
+        self.gl, self.wl = gl, wl
+        inp = W.make_mlp(wl.resized(seed=wl.seed + 1000 * rank), device=device)
+        self.inp = inp
+        B, d, m, k = wl.B, wl.d, wl.m, wl.k
+        dt = inp["x"].dtype
+        self.W1 = inp["W1"].reshape(1, 1, m, d)
+        self.W2 = inp["W2"].reshape(1, 1, k, m)
+        self.D1 = torch.zeros(1, B, 1, m, d, device=device)
+        self.D2 = torch.zeros(1, B, 1, k, m, device=device)
+        mk = lambda w: torch.empty(1, B, 1, w, dtype=dt, device=device)
+        self.x, self.g = mk(d), mk(k)           # the token's input and scored costate
+        self.z, self.h, self.y, self.gz = mk(m), mk(m), mk(k), mk(m)
+        self.eta1 = torch.full((1, B, 1), wl.eta1, device=device)
+        self.eta2 = torch.full((1, B, 1), wl.eta2, device=device)
+        self.ws = torch.empty(max(256, gl.decode_workspace_bytes(1, B, 1, m, k)), dtype=torch.uint8,
+                              device=device)
+        self.t = 0
+
+    def load_token(self, t):
+        T = self.wl.T
+        self.x.copy_(self.inp["x"][:, t % T].reshape(self.x.shape))
+        self.g.copy_(self.inp["g_out"][:, t % T].reshape(self.g.shape))
+
+    def launch(self, i):
+        gl, wl = self.gl, self.wl
+        if i == 0:
+            gl.decode_read(self.x, self.W1, self.D1, act=wl.act, y=self.z, act_out=self.h)
+        elif i == 1:
+            gl.decode_read(self.h, self.W2, self.D2, y=self.y)
+        elif i == 2:
+            gl.decode_write(self.h, self.g, self.W2, self.D2, self.eta2, act=wl.act, z=self.z,
+                            g_in=self.gz, workspace=self.ws)
+        else:
+            gl.decode_write(self.x, self.gz, self.W1, self.D1, self.eta1, want_g_in=False)
+
+    def step(self):
+        for i in range(4):
+            self.launch(i)
+
+    def kernel_bytes(self, i):
+        """Algorithmic HBM bytes of kernel i: Delta once per sequence (read, or read
+        and written), W0 once (shared by the B sequences), token vectors."""
+        wl = self.wl
+        B, d, m, k = wl.B, wl.d, wl.m, wl.k
+        e = 2 if wl.dtype == "bf16" else 4
+        if i == 0:
+            return 4 * m * d * (B + 1) + e * B * (d + 2 * m)
+        if i == 1:
+            return 4 * k * m * (B + 1) + e * B * (m + k)
+        if i == 2:
+            return 4 * k * m * (2 * B + 1) + e * B * (m + k + m + m)
+        return 4 * m * d * 2 * B + e * B * (d + m)
+
+    def step_bytes(self):
+        return sum(self.kernel_bytes(i) for i in range(4))
+
+
+def _graph(fn, stream):
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        fn()
+    return g
+
+
+def run_decode(args, wl, rank, world, local_rank):
+    """Deployment steps of the paper-shaped final MLP, replayed as one CUDA graph per
+    step (the four kernels back to back, no host in between)."""
+    import paper_2609_34174_gb300 as gl
+
+    device = torch.device("cuda", local_rank)
+    torch.cuda.set_device(device)
+    gl.load_library()
+    job = DecodeMLPJob(gl, wl, device, rank)
+    cap = torch.cuda.Stream(device)
+    job.load_token(0)
+    with torch.cuda.stream(cap):
+        job.step()  # warm the binding before capture
+    torch.cuda.synchronize()
+    g_step = _graph(job.step, cap)
+    g_kern = [_graph(lambda i=i: job.launch(i), cap) for i in range(4)]
+    # L2 flush between steps: write a buffer larger than L2, then read another one,
+    # so that no dirty lines are left for the timed step to write back
+    fw = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
+    fr = torch.ones(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
+
+    def flush():
+        fw.zero_()
+        fr.sum()
+
+    stream = torch.cuda.current_stream(device)
+    for t in range(args.warmup):
+        job.load_token(t)
+        g_step.replay()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(local_rank)
+    sampler.start()
+    time.sleep(0.3)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    sampler.mark()
+    for i in range(args.steps):
+        job.load_token(args.warmup + i)
+        flush()
+        ev[i][0].record(stream)
+        g_step.replay()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    sampler.mark()
+    # per-kernel times (each kernel alone after a flush), for the roofline of each
+    kev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in range(args.steps)] for _ in range(4)]
+    for j in range(args.steps):
+        for i in range(4):
+            flush()
+            kev[i][j][0].record(stream)
+            g_kern[i].replay()
+            kev[i][j][1].record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    time.sleep(0.25)
+    sampler.stop()
+    step_ms = statistics.median(a.elapsed_time(b) for a, b in ev)
+    step_ms, value = combine_ranks(step_ms, wl.B, world, device)
+    pk = peaks()
+    kern = {}
+    for i, name in enumerate(job.kernels):
+        ms = statistics.median(a.elapsed_time(b) for a, b in kev[i])
+        nb = job.kernel_bytes(i)
+        ach = nb / (ms / 1e3) / 1e9
+        kern[name] = {"ms": round(ms, 4), "bytes": nb, "achieved_gbs": round(ach, 1),
+                      "frac": round(ach / pk["hbm_gbs"], 4)}
+    dom = max(kern, key=lambda n: kern[n]["ms"])
+    rl = {"bound": "hbm", "achieved": kern[dom]["achieved_gbs"], "peak": pk["hbm_gbs"],
+          "unit": "GB/s", "frac": kern[dom]["frac"], "traffic": None,
+          "kernel": f"decode {dom} ({'write_kernel' if 'write' in dom else 'read_kernel'})",
+          "peak_source": pk.get("source", "MEASURED_PEAKS.json"),
+          "step_frac": round(job.step_bytes() / (step_ms / 1e3) / 1e9 / pk["hbm_gbs"], 4)}
+    cfg = {"workload": f"{args.workload}: deployment of {wl.name}", "B": wl.B,
+           "widths": [wl.d, wl.m, wl.k], "act": wl.act, "eta": [wl.eta1, wl.eta2],
+           "state": "Delta fp32 on the device", "tokens_per_step": wl.B,
+           "parallelism": f"replicas x{world}", "l2": "L2 flushed between steps",
+           "launch": "CUDA graph per step"}
+    line = {"metric": DECODE_METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms, 4),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
+            "data": "synthetic", "config": cfg, "kernels": kern, "roofline": rl,
+            "clocks": sampler.summary(), "gpu_launches": 4 * args.steps}
+    if rank == 0 and world == 1 and not args.no_e2e:
+        line["e2e"] = decode_e2e(job, g_step, max(20, min(args.steps, 200)), stream)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+
+        oracle.build()
+        line["cpu_baseline"] = decode_cpu_baseline(wl, job.inp)
+    return line
+
+
+def decode_e2e(job, g_step, steps, stream):
+    """Deployment steps through the public API from pinned host memory: each step
+    copies the token's x and scored costate in and reads y back."""
+    B = job.wl.B
+    hx = job.inp["x"].cpu().pin_memory()
+    hg = job.inp["g_out"].cpu().pin_memory()
+    hy = torch.empty(job.y.shape, dtype=job.y.dtype, pin_memory=True)
+    T = job.wl.T
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for t in range(steps):
+        job.x.copy_(hx[:, t % T].reshape(job.x.shape), non_blocking=True)
+        job.g.copy_(hg[:, t % T].reshape(job.g.shape), non_blocking=True)
+        g_step.replay()
+        hy.copy_(job.y, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    sec = e0.elapsed_time(e1) / 1e3
+    return {"value": round(steps * B / sec, 1), "unit": UNIT,
+            "h2d_bytes_per_step": _bytes(job.x, job.g), "d2h_bytes_per_step": _bytes(hy),
+            "note": "L2 not flushed: consecutive tokens, as in deployment"}
+
+
+def decode_cpu_baseline(wl, inp, target_s=12.0):
+    """The fp64 oracle's deployed MLP on a bounded number of tokens per sequence."""
+    import oracle
+    cores = len(os.sched_getaffinity(0))
+    f = lambda t, T: t[:, :T].to(torch.float64).cpu().numpy()
+    W1 = inp["W1"].double().cpu().numpy()
+    W2 = inp["W2"].double().cpu().numpy()
+
+    def run(T):
+        t0 = time.perf_counter()
+        oracle.mlp_deploy(f(inp["x"], T), W1, W2, wl.eta1, wl.eta2, gout=f(inp["g_out"], T),
+                          act=oracle.ACT_GELU_TANH, nthreads=min(cores, wl.B))
+        return time.perf_counter() - t0
+
+    dt0 = run(4)
+    T = int(min(wl.T, max(4, 4 * target_s / max(dt0, 1e-9))))
+    dt = run(T)
+    return {"value": round(wl.B * T / dt, 1), "unit": UNIT, "cores": min(cores, wl.B),
+            "kind": "oracle", "seconds": round(dt, 2),
+            "sample": f"{wl.B} sequences x first {T} tokens of the deployed MLP, fp64"}
 
 
 def run_gradlev(args, wl, rank, world, local_rank):
@@ -706,7 +942,8 @@ def main(argv=None):
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--workload", default="c5", choices=["c1", "c2", "c3", "c4", "c5", "paper_mlp"])
+    ap.add_argument("--workload", default="c5",
+                    choices=["c1", "c2", "c3", "c4", "c5", "paper_mlp", "decode_mlp"])
     ap.add_argument("--impl", default="gradlev", choices=["gradlev", "reference"])
     ap.add_argument("--resize", default="",
                     help="comma-separated K=V overrides of the workload's sizes (e.g. L=2), "
@@ -722,7 +959,8 @@ def main(argv=None):
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
-    wl = W.workload(args.workload)
+    decode = args.workload == "decode_mlp"
+    wl = W.workload("paper_mlp" if decode else args.workload)
     if args.resize:
         kw = {}
         for item in args.resize.split(","):
@@ -741,7 +979,10 @@ def main(argv=None):
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
     try:
-        line = run_gradlev(args, wl, rank, world, local_rank)
+        if decode:
+            line = run_decode(args, wl, rank, world, local_rank)
+        else:
+            line = run_gradlev(args, wl, rank, world, local_rank)
         if rank == 0:
             print(json.dumps(line), flush=True)
     finally:

@@ -172,6 +172,63 @@ int gradlev_costate_scan_gated(const gradlev_desc* desc, const gradlev_tensor* x
  * descriptor). */
 size_t gradlev_workspace_bytes_gated(const gradlev_desc* desc);
 
+/*
+ * Deployment (decode) -- Sec. 3, training-objective paragraph, and Appendix A:
+ * once deployed, the proposal network is gone and each adapted map updates from
+ * its own costates after the target has been scored, one token at a time.  The
+ * caller keeps each unit's fast weights as Delta = W - W0 (fp32
+ * [L][B][H][d_out][d_in], contiguous, 16-byte aligned; all zero at the start of a
+ * sequence) and calls, per token,
+ *   gradlev_decode_read   y     = (W0 + Delta) x             (the read before the write)
+ *   ... the model scores the target and back-propagates its true costate g ...
+ *   gradlev_decode_write  g_in  = (W0 + Delta)^T g           (optional, pre-write weights)
+ *                         Delta <- alpha Delta - eta g x^T   (Eq. 2, decay centred at W0)
+ * The descriptor has T = 1: token tensors are [L][B][1][H][w] with the usual
+ * strides.  d_in must be a multiple of 4 (GRADLEV_ERR_UNSUPPORTED otherwise), and
+ * L*H at most 65535.  dtype as for the scans; Delta, W0 and every sum stay fp32.
+ * Reads and writes of one Delta must be issued in order on one stream; both
+ * calls are asynchronous and keep no state of their own.
+ */
+
+/*
+ * gradlev_decode_read -- y = (W0 + Delta) x for one token per unit.
+ *   x        [L][B][1][H][d_in]   (read)
+ *   W0       fp32 [L][H][d_out][d_in], 16-byte aligned (read)
+ *   delta    fp32 [L][B][H][d_out][d_in] (read)
+ *   act, act_out  optional sigma(y) (act_out.data NULL to skip), as for the forward scan
+ *   y        [L][B][1][H][d_out]  (out)
+ * x is read four elements at a time: its base must be aligned to four elements
+ * and its strides multiples of four (GRADLEV_ERR_UNSUPPORTED otherwise).
+ */
+int gradlev_decode_read(const gradlev_desc* desc, const gradlev_tensor* x, const float* W0,
+                        const float* delta, int act, const gradlev_tensor* y,
+                        const gradlev_tensor* act_out, gradlev_stream_t stream);
+
+/*
+ * gradlev_decode_write -- the write of one token per unit, with its costate read.
+ *   x        [L][B][1][H][d_in]   the token's input (read)
+ *   g        [L][B][1][H][d_out]  the true costate dl/dy of the scored token (read)
+ *   W0       fp32 slow weights; needed only when g_in is requested (else may be NULL)
+ *   delta    fp32 [L][B][H][d_out][d_in] (read and updated in place)
+ *   eta      fp32 [L][B][H] step size per unit (read)
+ *   alpha    fp32 [L][B][H] retention per unit, or NULL for 1; 0 resets Delta to zero
+ *   g_in     optional [L][B][1][H][d_in] (data NULL to skip): (W0 + Delta)^T g with the
+ *            weights BEFORE this write (Sec. 3 step 3 holds them fixed), times
+ *            sigma'(z) when z is given with act != NONE (z of shape [L][B][1][H][d_in])
+ *   workspace/workspace_bytes  at least gradlev_decode_workspace_bytes(desc) bytes,
+ *            256-byte aligned, when g_in is requested (NULL if that is 0)
+ * The column sums of g_in are combined in a fixed order: results are reproducible.
+ */
+int gradlev_decode_write(const gradlev_desc* desc, const gradlev_tensor* x,
+                         const gradlev_tensor* g, const float* W0, float* delta, const float* eta,
+                         const float* alpha, int act, const gradlev_tensor* z,
+                         const gradlev_tensor* g_in, void* workspace, size_t workspace_bytes,
+                         gradlev_stream_t stream);
+
+/* Workspace bytes of a gradlev_decode_write that returns g_in (0: none needed, or
+ * an invalid descriptor). */
+size_t gradlev_decode_workspace_bytes(const gradlev_desc* desc);
+
 /* Size of the fixed device array used by gradlev_forward_scan_noalloc (4 MiB). */
 #define GRADLEV_NOALLOC_SCRATCH_BYTES (4u << 20)
 

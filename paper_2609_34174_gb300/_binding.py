@@ -82,6 +82,13 @@ def load_library():
         lib.gradlev_costate_scan_gated.restype = ctypes.c_int
         lib.gradlev_workspace_bytes_gated.argtypes = [D]
         lib.gradlev_workspace_bytes_gated.restype = ctypes.c_size_t
+        lib.gradlev_decode_read.argtypes = [D, Tp, P, P, ctypes.c_int, Tp, Tp, P]
+        lib.gradlev_decode_read.restype = ctypes.c_int
+        lib.gradlev_decode_write.argtypes = [D, Tp, Tp, P, P, P, P, ctypes.c_int, Tp, Tp, P,
+                                             ctypes.c_size_t, P]
+        lib.gradlev_decode_write.restype = ctypes.c_int
+        lib.gradlev_decode_workspace_bytes.argtypes = [D]
+        lib.gradlev_decode_workspace_bytes.restype = ctypes.c_size_t
         lib.gradlev_workspace_bytes.argtypes = [D]
         lib.gradlev_workspace_bytes.restype = ctypes.c_size_t
         lib.gradlev_workspace_status.argtypes = [P, P]
@@ -363,3 +370,120 @@ def mlp_costate(x, h, z, g_hat_z, g_hat_y, W1, W2, eta1, eta2, g_out, act="gelu_
     g_z = costate_scan(h, g_hat_y, W2, eta2, g_out, act=act, z=z)
     g_x = costate_scan(x, g_hat_z, W1, eta1, g_z)
     return g_z, g_x
+
+
+# ------------------------------------------------------------------ deployment
+def _tok1(t: torch.Tensor) -> torch.Tensor:
+    """View a one-token tensor [L,B,H,w] (or [B,H,w], [B,w]) as [L,B,1,H,w]."""
+    if t.dim() == 4:
+        return t.unsqueeze(2)
+    if t.dim() == 3:
+        return t.unsqueeze(0).unsqueeze(2)
+    if t.dim() == 2:
+        return t.unsqueeze(0).unsqueeze(2).unsqueeze(3)
+    raise ValueError(f"one-token tensors are 2- to 4-D, got {t.dim()}-D")
+
+
+def _delta(delta: torch.Tensor, L, B, H, rows, cols) -> torch.Tensor:
+    if delta.dtype != torch.float32 or not delta.is_contiguous():
+        raise TypeError("delta must be a contiguous float32 tensor")
+    if delta.numel() != L * B * H * rows * cols:
+        raise ValueError(f"delta must be [L,B,H,d_out,d_in] = {(L, B, H, rows, cols)}")
+    return delta
+
+
+def _per_unit(v, L, B, H, device):
+    if isinstance(v, torch.Tensor):
+        return v.to(device=device, dtype=torch.float32).expand(L, B, H).contiguous()
+    return torch.full((L, B, H), float(v), dtype=torch.float32, device=device)
+
+
+def decode_read(x, W0, delta, act=None, want_act_out=False, y=None, act_out=None):
+    """Deployment read for one token per unit: y = (W0 + delta) x (Sec. 3).
+
+    x [L,B,H,d_in] (or [B,H,d_in], [B,d_in]); W0 fp32 [L,H,d_out,d_in]; delta fp32
+    [L,B,H,d_out,d_in], the fast weights minus W0.  Returns y [.., d_out], or
+    (y, sigma(y)) with want_act_out.
+    """
+    lib = load_library()
+    x5 = _tok1(x)
+    if not x5.is_cuda:
+        raise ValueError("tensors must be on a CUDA device")
+    L, B, _, H, d_in = x5.shape
+    d_out = W0.shape[-2]
+    W = _w0(W0, L, H, d_out, d_in)
+    D = _delta(delta, L, B, H, d_out, d_in)
+    code = _act_code(act)
+    if y is None:
+        y = torch.empty(tuple(x.shape[:-1]) + (d_out,), dtype=x5.dtype, device=x5.device)
+    y5 = _tok1(y)
+    _check_same(x5, y5)
+    if want_act_out and act_out is None:
+        act_out = torch.empty_like(y)
+    a5 = _tok1(act_out) if act_out is not None else None
+    desc = _desc(x5, d_out, _dtype_code(x5))
+    tx, ty = _tensor(x5), _tensor(y5)
+    ta = _tensor(a5) if a5 is not None else None
+    stream = torch.cuda.current_stream(x5.device).cuda_stream
+    with torch.cuda.device(x5.device):
+        rc = lib.gradlev_decode_read(ctypes.byref(desc), ctypes.byref(tx), ctypes.c_void_p(W.data_ptr()),
+                                     ctypes.c_void_p(D.data_ptr()), code, ctypes.byref(ty),
+                                     ctypes.byref(ta) if ta is not None else None,
+                                     ctypes.c_void_p(stream))
+    _call(rc, "gradlev_decode_read")
+    if act_out is not None:
+        return y, act_out
+    return y
+
+
+def decode_workspace_bytes(L, B, H, d_in, d_out, dtype=GRADLEV_BF16) -> int:
+    d = _Desc(L, B, 1, H, d_in, d_out, dtype, 0)
+    return int(load_library().gradlev_decode_workspace_bytes(ctypes.byref(d)))
+
+
+def decode_write(x, g, W0, delta, eta, alpha=None, want_g_in=True, act=None, z=None, g_in=None,
+                 workspace=None):
+    """Deployment write for one token per unit, after its target was scored (Sec. 3).
+
+    With want_g_in, first g_in = (W0 + delta)^T g with the weights before the write
+    (times sigma'(z) when z is given); then delta <- alpha delta - eta g x^T in place
+    (Eq. 2).  x [L,B,H,d_in], g [L,B,H,d_out] (the true costate dl/dy), eta and alpha
+    scalars or per-unit [L,B,H].  Returns g_in, or None.
+    """
+    lib = load_library()
+    x5, g5 = _tok1(x), _tok1(g)
+    _check_same(x5, g5)
+    if not x5.is_cuda:
+        raise ValueError("tensors must be on a CUDA device")
+    L, B, _, H, d_in = x5.shape
+    d_out = g5.shape[4]
+    D = _delta(delta, L, B, H, d_out, d_in)
+    W = _w0(W0, L, H, d_out, d_in) if want_g_in else None
+    et = _per_unit(eta, L, B, H, x5.device)
+    al = _per_unit(alpha, L, B, H, x5.device) if alpha is not None else None
+    code = _act_code(act)
+    z5 = _tok1(z) if z is not None else None
+    if want_g_in and g_in is None:
+        g_in = torch.empty(tuple(x.shape), dtype=x5.dtype, device=x5.device)
+    gi5 = _tok1(g_in) if want_g_in else None
+    desc = _desc(x5, d_out, _dtype_code(x5))
+    ws = None
+    if want_g_in:
+        nbytes = int(lib.gradlev_decode_workspace_bytes(ctypes.byref(desc)))
+        if nbytes:
+            ws = workspace if workspace is not None else _workspace(nbytes, x5.device)
+    tx, tg = _tensor(x5), _tensor(g5)
+    tz = _tensor(z5) if z5 is not None else None
+    tgi = _tensor(gi5) if gi5 is not None else None
+    stream = torch.cuda.current_stream(x5.device).cuda_stream
+    with torch.cuda.device(x5.device):
+        rc = lib.gradlev_decode_write(
+            ctypes.byref(desc), ctypes.byref(tx), ctypes.byref(tg),
+            ctypes.c_void_p(W.data_ptr()) if W is not None else None, ctypes.c_void_p(D.data_ptr()),
+            ctypes.c_void_p(et.data_ptr()), ctypes.c_void_p(al.data_ptr()) if al is not None else None,
+            code, ctypes.byref(tz) if tz is not None else None,
+            ctypes.byref(tgi) if tgi is not None else None,
+            ctypes.c_void_p(ws.data_ptr()) if ws is not None else None,
+            ws.numel() if ws is not None else 0, ctypes.c_void_p(stream))
+    _call(rc, "gradlev_decode_write")
+    return g_in

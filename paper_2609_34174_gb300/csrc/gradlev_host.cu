@@ -27,6 +27,8 @@ size_t gated_serial_smem(int din, int dout, bool costate);
 cudaError_t launch_gated_serial(const GatedParams& p, bool costate, bool bf16, cudaStream_t stream);
 cudaError_t launch_gated_prescale(const void* g, const TokStr& gs, const float* eta, void* out, int L,
                                   int B, int T, int H, int w, bool bf16, cudaStream_t stream);
+cudaError_t launch_decode_read(const DecodeParams& p, bool bf16, cudaStream_t stream);
+cudaError_t launch_decode_write(const DecodeParams& p, bool bf16, bool gin, cudaStream_t stream);
 }  // namespace gl
 
 namespace {
@@ -568,6 +570,156 @@ int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
     return GRADLEV_OK;
 }
 
+// Deployment (decode) calls: one token per unit, Delta = W - W0 held by the caller.
+constexpr long long kDecodeTileBytes = 64 << 10;  // bytes of Delta per CTA tile
+
+struct DecodePlan {
+    int lanes = 32, rows_read = 0, n_rt_read = 0, rows_write = 0, n_rt_write = 0, n_strips = 0;
+    size_t off_cnt = 0, ws_bytes = 0;  // workspace of a write that returns g_in
+};
+
+// Tiles of about 64 KB of Delta: enough bytes in flight per CTA, and thousands of
+// CTAs for the large maps.  Depends on the shape only, so the workspace size does too.
+DecodePlan decode_plan(const gradlev_desc& d) {
+    DecodePlan pl;
+    const int cpr = d.d_in / 4;
+    if (cpr < 32) {
+        pl.lanes = 1;
+        while (pl.lanes < cpr) pl.lanes <<= 1;
+    }
+    const int pass_rows = 8 * (32 / pl.lanes);  // rows the eight warps of a CTA cover at once
+    const long long all_rows = (long long)(d.d_out + pass_rows - 1) / pass_rows * pass_rows;
+    auto tile_rows = [&](long long row_bytes) {
+        long long r = kDecodeTileBytes / row_bytes / pass_rows * pass_rows;
+        if (r < pass_rows) r = pass_rows;
+        return (int)(r < all_rows ? r : all_rows);
+    };
+    pl.rows_read = tile_rows(4ll * d.d_in);
+    pl.n_rt_read = (d.d_out + pl.rows_read - 1) / pl.rows_read;
+    pl.n_strips = (cpr + 31) / 32;
+    pl.rows_write = tile_rows(cpr < 32 ? 4ll * d.d_in : 512ll);
+    pl.n_rt_write = (d.d_out + pl.rows_write - 1) / pl.rows_write;
+    if (pl.n_rt_write > 1) {
+        const size_t units = (size_t)d.L * d.B * d.H;
+        pl.off_cnt = round_up(units * pl.n_rt_write * (size_t)d.d_in * sizeof(float), 256);
+        pl.ws_bytes = pl.off_cnt + round_up(units * pl.n_strips * sizeof(unsigned int), 256);
+    }
+    return pl;
+}
+
+// Checks shared by both decode calls.  The arguments the read or the write does
+// not use are passed as NULL.
+int decode_check(const gradlev_desc* desc, const float* delta, int act, DevInfo* dev) {
+    if (!desc_ok(desc)) return GRADLEV_ERR_INVALID_ARG;
+    const gradlev_desc& d = *desc;
+    if (d.T != 1 || !delta) return GRADLEV_ERR_INVALID_ARG;
+    if (act < GRADLEV_ACT_NONE || act > GRADLEV_ACT_TANH) return GRADLEV_ERR_INVALID_ARG;
+    if (d.d_in % 4 != 0 || (long long)d.L * d.H > 65535 || !aligned16(delta))
+        return GRADLEV_ERR_UNSUPPORTED;
+    if (!device_info(dev)) return GRADLEV_ERR_CUDA;
+    if (!(dev->major == 10 && dev->minor == 3)) return GRADLEV_ERR_UNSUPPORTED;
+    return GRADLEV_OK;
+}
+
+void decode_common(gl::DecodeParams* p, const gradlev_desc& d, const DecodePlan& pl,
+                   const float* W0, float* delta, const Tok& tx) {
+    memset(p, 0, sizeof(*p));
+    p->L = d.L;
+    p->B = d.B;
+    p->H = d.H;
+    p->din = d.d_in;
+    p->dout = d.d_out;
+    p->cpr = d.d_in / 4;
+    p->lanes = pl.lanes;
+    p->n_strips = pl.n_strips;
+    p->W0 = W0;
+    p->delta = delta;
+    p->x = tx.data;
+    for (int i = 0; i < 4; ++i) p->x_s[i] = tx.s[i];
+}
+
+bool tok_elem_aligned(const Tok& t, int elem) {
+    return !t.data || (reinterpret_cast<uintptr_t>(t.data) % elem) == 0;
+}
+
+int run_decode_read(const gradlev_desc* desc, const gradlev_tensor* x, const float* W0,
+                    const float* delta, int act, const gradlev_tensor* y,
+                    const gradlev_tensor* act_out, cudaStream_t stream) {
+    DevInfo dev;
+    const int rc = decode_check(desc, delta, act, &dev);
+    if (rc != GRADLEV_OK) return rc;
+    const gradlev_desc& d = *desc;
+    if (!W0) return GRADLEV_ERR_INVALID_ARG;
+    if (!aligned16(W0)) return GRADLEV_ERR_UNSUPPORTED;
+    Tok tx, ty, ta, tz;
+    if (!resolve(d, x, d.d_in, &tx, true) || !resolve(d, y, d.d_out, &ty, true) ||
+        !resolve(d, act_out, d.d_out, &ta, false))
+        return GRADLEV_ERR_INVALID_ARG;
+    if (ta.data && act == GRADLEV_ACT_NONE) return GRADLEV_ERR_INVALID_ARG;
+    const int elem = d.dtype == GRADLEV_BF16 ? 2 : 4;
+    if (!tok_elem_aligned(tx, 4 * elem) || !tok_elem_aligned(ty, elem) ||
+        !tok_elem_aligned(ta, elem))
+        return GRADLEV_ERR_UNSUPPORTED;
+    for (int i = 0; i < 4; ++i)  // x is read four elements at a time
+        if (tx.s[i] % 4 != 0) return GRADLEV_ERR_UNSUPPORTED;
+    const DecodePlan pl = decode_plan(d);
+    gl::DecodeParams p;
+    decode_common(&p, d, pl, W0, const_cast<float*>(delta), tx);
+    p.rows = pl.rows_read;
+    p.n_rt = pl.n_rt_read;
+    fill_epi(&p.epi, ty, ta, tz, act);
+    if (gl::launch_decode_read(p, d.dtype == GRADLEV_BF16, stream) != cudaSuccess)
+        return GRADLEV_ERR_CUDA;
+    return GRADLEV_OK;
+}
+
+int run_decode_write(const gradlev_desc* desc, const gradlev_tensor* x, const gradlev_tensor* g,
+                     const float* W0, float* delta, const float* eta, const float* alpha, int act,
+                     const gradlev_tensor* z, const gradlev_tensor* g_in, void* ws, size_t ws_bytes,
+                     cudaStream_t stream) {
+    DevInfo dev;
+    const int rc = decode_check(desc, delta, act, &dev);
+    if (rc != GRADLEV_OK) return rc;
+    const gradlev_desc& d = *desc;
+    if (!eta || (reinterpret_cast<uintptr_t>(eta) & 3u) ||
+        (alpha && (reinterpret_cast<uintptr_t>(alpha) & 3u)))
+        return GRADLEV_ERR_INVALID_ARG;
+    Tok tx, tg, tgi, tz, none;
+    if (!resolve(d, x, d.d_in, &tx, true) || !resolve(d, g, d.d_out, &tg, true) ||
+        !resolve(d, g_in, d.d_in, &tgi, false) || !resolve(d, z, d.d_in, &tz, false))
+        return GRADLEV_ERR_INVALID_ARG;
+    const bool gin = tgi.data != nullptr;
+    if (tz.data && (!gin || act == GRADLEV_ACT_NONE)) return GRADLEV_ERR_INVALID_ARG;
+    if (gin && !W0) return GRADLEV_ERR_INVALID_ARG;
+    if (gin && !aligned16(W0)) return GRADLEV_ERR_UNSUPPORTED;
+    const int elem = d.dtype == GRADLEV_BF16 ? 2 : 4;
+    if (!tok_elem_aligned(tx, elem) || !tok_elem_aligned(tg, elem) ||
+        !tok_elem_aligned(tgi, elem) || !tok_elem_aligned(tz, elem))
+        return GRADLEV_ERR_UNSUPPORTED;
+    const DecodePlan pl = decode_plan(d);
+    gl::DecodeParams p;
+    decode_common(&p, d, pl, gin ? W0 : nullptr, delta, tx);
+    p.rows = pl.rows_write;
+    p.n_rt = pl.n_rt_write;
+    p.g = tg.data;
+    for (int i = 0; i < 4; ++i) p.g_s[i] = tg.s[i];
+    p.eta = eta;
+    p.alpha = alpha;
+    fill_epi(&p.epi, tgi, none, tz, act);
+    if (gin && pl.ws_bytes) {
+        if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < pl.ws_bytes)
+            return GRADLEV_ERR_WORKSPACE;
+        uint8_t* wsb = static_cast<uint8_t*>(ws);
+        p.part = reinterpret_cast<float*>(wsb);
+        p.cnt = reinterpret_cast<unsigned int*>(wsb + pl.off_cnt);
+        if (cudaMemsetAsync(p.cnt, 0, pl.ws_bytes - pl.off_cnt, stream) != cudaSuccess)
+            return GRADLEV_ERR_CUDA;
+    }
+    if (gl::launch_decode_write(p, d.dtype == GRADLEV_BF16, gin, stream) != cudaSuccess)
+        return GRADLEV_ERR_CUDA;
+    return GRADLEV_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -612,6 +764,27 @@ size_t gradlev_workspace_bytes_gated(const gradlev_desc* desc) {
     DevInfo dev;
     int sms = device_info(&dev) ? dev.sms : 160;
     return gated_ws_bytes(*desc, sms);
+}
+
+int gradlev_decode_read(const gradlev_desc* desc, const gradlev_tensor* x, const float* W0,
+                        const float* delta, int act, const gradlev_tensor* y,
+                        const gradlev_tensor* act_out, gradlev_stream_t stream) {
+    return run_decode_read(desc, x, W0, delta, act, y, act_out,
+                           reinterpret_cast<cudaStream_t>(stream));
+}
+
+int gradlev_decode_write(const gradlev_desc* desc, const gradlev_tensor* x,
+                         const gradlev_tensor* g, const float* W0, float* delta, const float* eta,
+                         const float* alpha, int act, const gradlev_tensor* z,
+                         const gradlev_tensor* g_in, void* workspace, size_t workspace_bytes,
+                         gradlev_stream_t stream) {
+    return run_decode_write(desc, x, g, W0, delta, eta, alpha, act, z, g_in, workspace,
+                            workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t gradlev_decode_workspace_bytes(const gradlev_desc* desc) {
+    if (!desc_ok(desc) || desc->T != 1 || desc->d_in % 4 != 0) return 0;
+    return decode_plan(*desc).ws_bytes;
 }
 
 size_t gradlev_workspace_bytes(const gradlev_desc* desc) {

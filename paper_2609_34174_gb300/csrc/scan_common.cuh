@@ -140,6 +140,27 @@ struct GatedParams {
     EpiParams epi;
 };
 
+// Parameters of the deployment kernels (decode.cu): one token per unit, fast
+// weights held as Delta = W - W0 in fp32 between calls (Sec. 3, deployment).
+struct DecodeParams {
+    int L, B, H;
+    int din, dout;         // columns (d_in) and rows (d_out) of every matrix
+    int cpr;               // din / 4: 16-byte pieces per matrix row
+    int lanes;             // lanes sharing one row: 32, or the power of two >= cpr below 32
+    int rows;              // matrix rows per CTA tile
+    int n_rt;              // row tiles per unit
+    int n_strips;          // column strips of 32 pieces (write kernel)
+    const float* W0;       // [L][H][dout][din]
+    float* delta;          // [L][B][H][dout][din]
+    const void* x; long long x_s[4];   // [L][B][1][H][din]
+    const void* g; long long g_s[4];   // [L][B][1][H][dout] (write: the true costate)
+    const float* eta;      // [L][B][H] (write)
+    const float* alpha;    // [L][B][H] or null (write)
+    EpiParams epi;         // read: out = y, out2 = sigma(y); write: out = g_in, zin = z
+    float* part;           // write with g_in over several row tiles: [U][n_rt][din]
+    unsigned int* cnt;     // ... and its arrival counters [U][n_strips], zero on entry
+};
+
 // Error bits written to ctrl[1].
 constexpr unsigned int kErrWaitTimeout = 1u;
 constexpr unsigned int kErrLookbackTimeout = 2u;

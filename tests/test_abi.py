@@ -139,3 +139,33 @@ def test_workspace_bytes_cover_the_segment_carry(lib):
     assert wl > 1 << 20
     assert 256 <= wm < 1 << 20
     assert wl % 256 == 0 or wl > 0
+
+
+def test_decode_arguments_rejected_before_launch(lib):
+    d = _desc(T=1)
+    x, g, y = _t(), _t(), _t()
+    delta, W0, eta = ctypes.c_void_p(0x4000), ctypes.c_void_p(0x8000), ctypes.c_void_p(0x9000)
+    # a decode call covers exactly one token per unit
+    d2 = _desc(T=2)
+    assert lib.gradlev_decode_read(ctypes.byref(d2), ctypes.byref(x), W0, delta, 0,
+                                   ctypes.byref(y), None, None) == -1
+    # missing Delta
+    assert lib.gradlev_decode_read(ctypes.byref(d), ctypes.byref(x), W0, None, 0,
+                                   ctypes.byref(y), None, None) == -1
+    # d_in not a multiple of 4
+    d3 = _desc(T=1, d_in=6)
+    assert lib.gradlev_decode_write(ctypes.byref(d3), ctypes.byref(x), ctypes.byref(g), W0, delta,
+                                    eta, None, 0, None, None, None, 0, None) == -2
+    # activation out of range
+    assert lib.gradlev_decode_write(ctypes.byref(d), ctypes.byref(x), ctypes.byref(g), W0, delta,
+                                    eta, None, 9, None, None, None, 0, None) == -1
+
+
+def test_decode_workspace_sizes(lib):
+    # one row tile per unit: no workspace
+    assert lib.gradlev_decode_workspace_bytes(ctypes.byref(_desc(L=12, B=8, H=12, T=1))) == 0
+    # 1024 -> 4096 for two sequences: 32 tiles of 128 rows x 1024 fp32 partial sums per
+    # sequence, plus one counter per (sequence, strip of 128 columns), each 256-aligned
+    d = _desc(B=2, T=1, d_in=1024, d_out=4096)
+    assert lib.gradlev_decode_workspace_bytes(ctypes.byref(d)) == 2 * 32 * 1024 * 4 + 256
+    assert lib.gradlev_decode_workspace_bytes(ctypes.byref(_desc(T=3))) == 0
