@@ -60,6 +60,8 @@ def _load():
     lib.oracle_act.restype = ctypes.c_double
     lib.oracle_act_deriv.argtypes = [I, ctypes.c_double]
     lib.oracle_act_deriv.restype = ctypes.c_double
+    lib.oracle_suffix_batch.argtypes = [I, I, I, I, P, P, P, P, I]
+    lib.oracle_suffix_batch.restype = I
     lib.oracle_max_threads.argtypes = []
     lib.oracle_max_threads.restype = I
     _lib = lib
@@ -173,6 +175,21 @@ def mlp_deploy(x, W10, W20, eta1, eta2, gout, act=ACT_GELU_TANH, alpha=None, nth
     Same shapes and outputs as mlp_scan."""
     return mlp_scan(x, None, None, W10, W20, eta1, eta2, act=act, alpha=alpha, gout=gout,
                     nthreads=nthreads)
+
+
+def suffix_scan(q, k, v, nthreads=0):
+    """Anti-causal read r_s = sum_{t>s} (k_t . q_s) v_t for U independent units
+    (outer gradients through the reads).  q, k [U,T,dq], v [U,T,dv] -> r [U,T,dv]."""
+    lib = _load()
+    q, k, v = _f64(q), _f64(k), _f64(v)
+    U, T, dq = q.shape
+    dv = v.shape[2]
+    if k.shape != (U, T, dq) or v.shape[:2] != (U, T):
+        raise ValueError("suffix_scan shape mismatch")
+    r = np.empty((U, T, dv))
+    if lib.oracle_suffix_batch(U, T, dq, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(r), int(nthreads)):
+        raise MemoryError("oracle_suffix_batch could not allocate scratch")
+    return r
 
 
 def act(code, z):

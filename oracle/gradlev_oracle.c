@@ -268,6 +268,60 @@ int oracle_mlp_batch(int U, int T, int d, int m, int k, int act, const double* x
     return err;
 }
 
+/*
+ * oracle_suffix -- the anti-causal read of the writes, for outer gradients
+ * through the reads (Sec. 3, practical architecture and training: the gates
+ * are learned and their derivatives kept, the writes are detached):
+ *     r_s = sum_{t > s} (k_t . q_s) v_t
+ * walked backwards in time with R = sum_{t > s} v_t k_t^T (dv x dq), read before
+ * its own write, the mirror image of the forward learner.
+ *   q, k [T][dq], v [T][dv], r [T][dv]; R [dv][dq] is scratch.
+ * For the forward read y_t = W_t x_t with per-token step sizes, the derivative
+ * of sum_t u_t . y_t with respect to eta_s is -ghat_s . r_s (q = k = x, v = u).
+ */
+void oracle_suffix(int T, int dq, int dv, const double* q, const double* k, const double* v,
+                   double* r, double* R) {
+    memset(R, 0, sizeof(double) * (size_t)dv * dq);
+    for (int s = T - 1; s >= 0; --s) {
+        const double* qs = q + (size_t)s * dq;
+        for (int i = 0; i < dv; ++i) {
+            double acc = 0.0;
+            for (int j = 0; j < dq; ++j) acc += R[(size_t)i * dq + j] * qs[j];
+            r[(size_t)s * dv + i] = acc;
+        }
+        const double* ks = k + (size_t)s * dq;
+        const double* vs = v + (size_t)s * dv;
+        for (int i = 0; i < dv; ++i)
+            for (int j = 0; j < dq; ++j) R[(size_t)i * dq + j] += vs[i] * ks[j];
+    }
+}
+
+/* oracle_suffix over U independent units ([U][...] contiguous), in parallel. */
+int oracle_suffix_batch(int U, int T, int dq, int dv, const double* q, const double* k,
+                        const double* v, double* r, int nthreads) {
+    int err = 0;
+#ifdef _OPENMP
+    if (nthreads > 0) omp_set_num_threads(nthreads);
+#else
+    (void)nthreads;
+#endif
+#pragma omp parallel
+    {
+        double* R = (double*)malloc(sizeof(double) * (size_t)dv * dq);
+        if (!R) {
+#pragma omp atomic write
+            err = -1;
+        } else {
+#pragma omp for schedule(dynamic, 1)
+            for (int u = 0; u < U; ++u)
+                oracle_suffix(T, dq, dv, q + (size_t)u * T * dq, k + (size_t)u * T * dq,
+                              v + (size_t)u * T * dv, r + (size_t)u * T * dv, R);
+            free(R);
+        }
+    }
+    return err;
+}
+
 /* Threads the OpenMP runtime would use (for reporting the CPU baseline). */
 int oracle_max_threads(void) {
 #ifdef _OPENMP

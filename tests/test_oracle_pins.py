@@ -373,3 +373,61 @@ def test_mlp_deploy_is_the_fixed_point_of_proposals():
             assert np.abs(ghz[:, n:] - dep["gz"][:, n:]).max() > 1e-9
     for key in ("z", "h", "y", "gh", "gx"):
         assert np.abs(o[key] - dep[key]).max() < 1e-12, key
+
+
+# ------------------------------------------------------ suffix read (gradients)
+def test_suffix_scan_brute_force():
+    """r_s = sum_{t>s} (k_t . q_s) v_t written as the double sum; r_{T-1} = 0."""
+    U, T, dq, dv = 2, 9, 3, 4
+    r = _rng(401)
+    q, k, v = r.standard_normal((U, T, dq)), r.standard_normal((U, T, dq)), r.standard_normal((U, T, dv))
+    out = oracle.suffix_scan(q, k, v)
+    ref = np.zeros((U, T, dv))
+    for u in range(U):
+        for s in range(T):
+            for t in range(s + 1, T):
+                ref[u, s] += np.dot(k[u, t], q[u, s]) * v[u, t]
+    assert np.abs(out - ref).max() < 1e-13
+    assert np.abs(out[:, -1]).max() == 0.0
+
+
+def _fd_eta(loss, eta, h=1e-3):
+    g = np.empty_like(eta)
+    for s in range(eta.shape[0]):
+        e1, e2 = eta.copy(), eta.copy()
+        e1[s] += h
+        e2[s] -= h
+        g[s] = (loss(e1) - loss(e2)) / (2 * h)
+    return g
+
+
+def test_eta_gradient_of_forward_read_is_a_suffix_read():
+    """y_t is linear in every eta_s (unit retention), so central differences of
+    the sequential learner give dL/deta_s exactly (up to rounding); with
+    L = sum_t u_t . y_t they equal -ghat_s . r_s, r the suffix read with q = k = x, v = u."""
+    T, d, m = 24, 5, 7
+    r = _rng(402)
+    x, gh, u = r.standard_normal((1, T, d)), r.standard_normal((1, T, m)), r.standard_normal((1, T, m))
+    W0 = r.standard_normal((m, d)) * 0.3
+    eta = r.uniform(0.01, 0.2, T)
+    loss = lambda e: float(np.sum(u * oracle.linear_scan(x, gh, W0, e)[0]))
+    fd = _fd_eta(loss, eta)
+    rs = oracle.suffix_scan(x, x, u)[0]
+    an = -np.sum(gh[0] * rs, axis=1)
+    assert np.abs(fd - an).max() < 1e-7 * max(1.0, np.abs(an).max())
+
+
+def test_eta_gradient_of_costate_read_is_a_suffix_read():
+    """gin_t = W_t^T g_t: with L = sum_t w_t . gin_t, dL/deta_s = -x_s . r_s where r is
+    the suffix read with q = ghat, k = g_out, v = w."""
+    T, d, m = 20, 6, 4
+    r = _rng(403)
+    x, gh, go = r.standard_normal((1, T, d)), r.standard_normal((1, T, m)), r.standard_normal((1, T, m))
+    w = r.standard_normal((1, T, d))
+    W0 = r.standard_normal((m, d)) * 0.3
+    eta = r.uniform(0.01, 0.2, T)
+    loss = lambda e: float(np.sum(w * oracle.linear_scan(x, gh, W0, e, gout=go, want_y=False)[1]))
+    fd = _fd_eta(loss, eta)
+    rs = oracle.suffix_scan(gh, go, w)[0]
+    an = -np.sum(x[0] * rs, axis=1)
+    assert np.abs(fd - an).max() < 1e-7 * max(1.0, np.abs(an).max())
