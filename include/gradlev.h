@@ -229,6 +229,46 @@ int gradlev_decode_write(const gradlev_desc* desc, const gradlev_tensor* x,
  * an invalid descriptor). */
 size_t gradlev_decode_workspace_bytes(const gradlev_desc* desc);
 
+/*
+ * Outer gradients through the reads -- Sec. 3, practical architecture and
+ * training: the gates are learned and their derivatives kept, while the writes
+ * are detached.  The reads are then linear in every step size, and the derivative
+ * with respect to eta_s is a read of the same writes in the other direction of time.
+ *
+ * gradlev_suffix_scan -- the anti-causal read
+ *     r_s = sum_{t>s} (k_t . q_s) v_t          (r_{T-1} = 0)
+ *   desc     d_in = width of q and k, d_out = width of v and r; T, strides and dtype
+ *            as for the scans
+ *   q, k     [L][B][T][H][d_in] (read);  v [L][B][T][H][d_out] (read)
+ *   r        [L][B][T][H][d_out] (out)
+ *   workspace/workspace_bytes  at least gradlev_suffix_workspace_bytes(desc) bytes
+ *            (NULL if that is 0)
+ * d_in at most 256 (GRADLEV_ERR_UNSUPPORTED otherwise).
+ */
+int gradlev_suffix_scan(const gradlev_desc* desc, const gradlev_tensor* q,
+                        const gradlev_tensor* k, const gradlev_tensor* v, const gradlev_tensor* r,
+                        void* workspace, size_t workspace_bytes, gradlev_stream_t stream);
+size_t gradlev_suffix_workspace_bytes(const gradlev_desc* desc);
+
+/*
+ * gradlev_eta_grad -- dL/deta_s of one adapted map's read, for per-token step sizes
+ * (unit retention):
+ *   read 0 (forward, y_t = W_t x_t):        deta_s = -ghat_s . sum_{t>s} (x_t . x_s) u_t,
+ *            u = dL/dy [L][B][T][H][d_out]
+ *   read 1 (costate, gin_t = W_t^T g_out_t): deta_s = -x_s . sum_{t>s} (g_out_t . ghat_s) u_t,
+ *            u = dL/dgin [L][B][T][H][d_in]; g_out required
+ *   x, g_hat, g_out  the map's tensors as for the scans (read)
+ *   deta     fp32 [L][B][T][H], contiguous (out)
+ *   workspace/workspace_bytes  at least gradlev_eta_grad_workspace_bytes(desc, read)
+ *            bytes, 256-byte aligned (it holds the suffix read)
+ * The same value for every eta_t: the reads are linear in the step sizes.
+ */
+int gradlev_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x,
+                     const gradlev_tensor* g_hat, const gradlev_tensor* g_out,
+                     const gradlev_tensor* upstream, float* deta, void* workspace,
+                     size_t workspace_bytes, gradlev_stream_t stream);
+size_t gradlev_eta_grad_workspace_bytes(const gradlev_desc* desc, int read);
+
 /* Size of the fixed device array used by gradlev_forward_scan_noalloc (4 MiB). */
 #define GRADLEV_NOALLOC_SCRATCH_BYTES (4u << 20)
 

@@ -89,6 +89,14 @@ def load_library():
         lib.gradlev_decode_write.restype = ctypes.c_int
         lib.gradlev_decode_workspace_bytes.argtypes = [D]
         lib.gradlev_decode_workspace_bytes.restype = ctypes.c_size_t
+        lib.gradlev_suffix_scan.argtypes = [D, Tp, Tp, Tp, Tp, P, ctypes.c_size_t, P]
+        lib.gradlev_suffix_scan.restype = ctypes.c_int
+        lib.gradlev_suffix_workspace_bytes.argtypes = [D]
+        lib.gradlev_suffix_workspace_bytes.restype = ctypes.c_size_t
+        lib.gradlev_eta_grad.argtypes = [D, ctypes.c_int, Tp, Tp, Tp, Tp, P, P, ctypes.c_size_t, P]
+        lib.gradlev_eta_grad.restype = ctypes.c_int
+        lib.gradlev_eta_grad_workspace_bytes.argtypes = [D, ctypes.c_int]
+        lib.gradlev_eta_grad_workspace_bytes.restype = ctypes.c_size_t
         lib.gradlev_workspace_bytes.argtypes = [D]
         lib.gradlev_workspace_bytes.restype = ctypes.c_size_t
         lib.gradlev_workspace_status.argtypes = [P, P]
@@ -487,3 +495,69 @@ def decode_write(x, g, W0, delta, eta, alpha=None, want_g_in=True, act=None, z=N
             ws.numel() if ws is not None else 0, ctypes.c_void_p(stream))
     _call(rc, "gradlev_decode_write")
     return g_in
+
+
+# ------------------------------------------------------------- outer gradients
+def suffix_scan(q, k, v, r=None, workspace=None):
+    """Anti-causal read r_s = sum_{t>s} (k_t . q_s) v_t (outer gradients through the
+    reads).  q, k [L,B,T,H,dq] (or fewer leading dims), v [.., dv].  Returns r [.., dv]."""
+    lib = load_library()
+    q5, k5, v5 = _as5(q), _as5(k), _as5(v)
+    _check_same(q5, k5, v5)
+    if not q5.is_cuda:
+        raise ValueError("tensors must be on a CUDA device")
+    if tuple(k5.shape) != tuple(q5.shape) or tuple(v5.shape[:4]) != tuple(q5.shape[:4]):
+        raise ValueError("q, k and v token shapes differ")
+    dv = v5.shape[4]
+    if r is None:
+        r = torch.empty(tuple(v.shape), dtype=v5.dtype, device=v5.device)
+    r5 = _as5(r)
+    _check_same(q5, r5)
+    desc = _desc(q5, dv, _dtype_code(q5))
+    nbytes = int(lib.gradlev_suffix_workspace_bytes(ctypes.byref(desc)))
+    ws = workspace if workspace is not None else (_workspace(nbytes, q5.device) if nbytes else None)
+    tq, tk, tv, tr = _tensor(q5), _tensor(k5), _tensor(v5), _tensor(r5)
+    stream = torch.cuda.current_stream(q5.device).cuda_stream
+    with torch.cuda.device(q5.device):
+        rc = lib.gradlev_suffix_scan(ctypes.byref(desc), ctypes.byref(tq), ctypes.byref(tk),
+                                     ctypes.byref(tv), ctypes.byref(tr),
+                                     ctypes.c_void_p(ws.data_ptr()) if ws is not None else None,
+                                     ws.numel() if ws is not None else 0, ctypes.c_void_p(stream))
+    _call(rc, "gradlev_suffix_scan")
+    return r
+
+
+def eta_grad(x, g_hat, upstream, read="forward", g_out=None, deta=None, workspace=None):
+    """dL/deta_t of one map's read for per-token step sizes (writes detached).
+
+    read="forward": upstream = dL/dy ([.., d_out]); read="costate": upstream = dL/dg_in
+    ([.., d_in]) and g_out is required.  Returns fp32 [L,B,T,H] (the token shape of x).
+    """
+    lib = load_library()
+    x5, g5, u5 = _as5(x), _as5(g_hat), _as5(upstream)
+    go5 = _as5(g_out) if g_out is not None else None
+    _check_same(x5, g5, u5, go5)
+    if not x5.is_cuda:
+        raise ValueError("tensors must be on a CUDA device")
+    rd = {"forward": 0, "costate": 1}[read]
+    if rd == 1 and go5 is None:
+        raise ValueError("the costate read needs g_out")
+    L, B, T, H, d_in = x5.shape
+    d_out = g5.shape[4]
+    desc = _desc(x5, d_out, _dtype_code(x5))
+    if deta is None:
+        deta = torch.empty((L, B, T, H), dtype=torch.float32, device=x5.device)
+    if deta.dtype != torch.float32 or not deta.is_contiguous() or deta.numel() != L * B * T * H:
+        raise ValueError("deta must be a contiguous float32 [L,B,T,H] tensor")
+    nbytes = int(lib.gradlev_eta_grad_workspace_bytes(ctypes.byref(desc), rd))
+    ws = workspace if workspace is not None else _workspace(nbytes, x5.device)
+    tx, tg, tu = _tensor(x5), _tensor(g5), _tensor(u5)
+    tgo = _tensor(go5) if go5 is not None else None
+    stream = torch.cuda.current_stream(x5.device).cuda_stream
+    with torch.cuda.device(x5.device):
+        rc = lib.gradlev_eta_grad(ctypes.byref(desc), rd, ctypes.byref(tx), ctypes.byref(tg),
+                                  ctypes.byref(tgo) if tgo is not None else None, ctypes.byref(tu),
+                                  ctypes.c_void_p(deta.data_ptr()), ctypes.c_void_p(ws.data_ptr()),
+                                  ws.numel(), ctypes.c_void_p(stream))
+    _call(rc, "gradlev_eta_grad")
+    return deta

@@ -18,7 +18,10 @@ namespace gl {
 cudaError_t launch_tc_scan(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
                            const CUtensorMap& o, const TcScanParams& p, bool costate, int grid,
                            cudaStream_t stream);
-cudaError_t launch_simt_scan(const SimtScanParams& p, bool bf16, cudaStream_t stream);
+cudaError_t launch_simt_scan(const SimtScanParams& p, bool bf16, bool rev, cudaStream_t stream);
+cudaError_t launch_rowdot(const void* a, const TokStr& as, const void* r, const TokStr& rs,
+                          float* out, int L, int B, int T, int H, int w, float scale, bool bf16,
+                          cudaStream_t stream);
 cudaError_t launch_seg_gemm(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b,
                             const CUtensorMap& a2, const CUtensorMap& b2, const SegGemmParams& p,
                             int grid, cudaStream_t stream);
@@ -457,7 +460,7 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
             p.v_str[i] = tv.s[i];
         }
         fill_epi(&p.epi, to, to2, tz, act);
-        if (gl::launch_simt_scan(p, d.dtype == GRADLEV_BF16, stream) != cudaSuccess)
+        if (gl::launch_simt_scan(p, d.dtype == GRADLEV_BF16, false, stream) != cudaSuccess)
             return GRADLEV_ERR_CUDA;
         return GRADLEV_OK;
     }
@@ -567,6 +570,117 @@ int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
     }
     fill_epi(&p.epi, to, to2, tz, act);
     if (gl::launch_gated_serial(p, costate, bf16, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
+    return GRADLEV_OK;
+}
+
+// Suffix (anti-causal) read r_s = sum_{t>s} (k_t . q_s) v_t: d_in is the width of q
+// and k, d_out the width of v and r.  Runs the CUDA-core scan in reverse with no
+// base matrix and eta = -1.
+size_t suffix_ws_bytes(const gradlev_desc& d) {
+    (void)d;
+    return 0;
+}
+
+int run_suffix_scan(const gradlev_desc* desc, const gradlev_tensor* q, const gradlev_tensor* k,
+                    const gradlev_tensor* v, const gradlev_tensor* r, void* ws, size_t ws_bytes,
+                    cudaStream_t stream) {
+    if (!desc_ok(desc)) return GRADLEV_ERR_INVALID_ARG;
+    const gradlev_desc& d = *desc;
+    Tok tq, tk, tv, tr;
+    if (!resolve(d, q, d.d_in, &tq, true) || !resolve(d, k, d.d_in, &tk, true) ||
+        !resolve(d, v, d.d_out, &tv, true) || !resolve(d, r, d.d_out, &tr, true))
+        return GRADLEV_ERR_INVALID_ARG;
+    DevInfo dev;
+    if (!device_info(&dev)) return GRADLEV_ERR_CUDA;
+    if (!(dev.major == 10 && dev.minor == 3)) return GRADLEV_ERR_UNSUPPORTED;
+    if (ws_bytes < suffix_ws_bytes(d)) return GRADLEV_ERR_WORKSPACE;
+    (void)ws;
+    if (d.T == 0) return GRADLEV_OK;
+    const int elem = d.dtype == GRADLEV_BF16 ? 2 : 4;
+    const Tok* all[4] = {&tq, &tk, &tv, &tr};
+    for (const Tok* t : all)
+        if ((reinterpret_cast<uintptr_t>(t->data) % elem) != 0) return GRADLEV_ERR_UNSUPPORTED;
+    if (!simt_shape_ok(d, d.d_in)) return GRADLEV_ERR_UNSUPPORTED;
+    gl::SimtScanParams p;
+    memset(&p, 0, sizeof(p));
+    p.L = d.L;
+    p.B = d.B;
+    p.T = d.T;
+    p.H = d.H;
+    p.dq = d.d_in;
+    p.dv = d.d_out;
+    p.eta = -1.0f;
+    p.W0 = nullptr;
+    p.q = tq.data;
+    p.k = tk.data;
+    p.v = tv.data;
+    for (int i = 0; i < 4; ++i) {
+        p.q_str[i] = tq.s[i];
+        p.k_str[i] = tk.s[i];
+        p.v_str[i] = tv.s[i];
+    }
+    Tok none;
+    fill_epi(&p.epi, tr, none, none, GRADLEV_ACT_NONE);
+    if (gl::launch_simt_scan(p, d.dtype == GRADLEV_BF16, true, stream) != cudaSuccess)
+        return GRADLEV_ERR_CUDA;
+    return GRADLEV_OK;
+}
+
+// Step-size gradients of one map's read (read 0: forward y = W x; read 1: costate
+// gin = W^T g_out): deta_s = -a_s . r_s, r the suffix read of the upstream gradient.
+gradlev_desc suffix_desc(const gradlev_desc& d, int read) {
+    gradlev_desc s = d;
+    if (read == 1) {
+        s.d_in = d.d_out;
+        s.d_out = d.d_in;
+    }
+    return s;
+}
+
+size_t eta_grad_ws_bytes(const gradlev_desc& d, int read) {
+    const gradlev_desc s = suffix_desc(d, read);
+    const size_t elem = d.dtype == GRADLEV_BF16 ? 2 : 4;
+    return round_up(suffix_ws_bytes(s), 256) +
+           round_up((size_t)d.L * d.B * d.T * d.H * s.d_out * elem, 256);
+}
+
+int run_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x,
+                 const gradlev_tensor* g_hat, const gradlev_tensor* g_out,
+                 const gradlev_tensor* upstream, float* deta, void* ws, size_t ws_bytes,
+                 cudaStream_t stream) {
+    if (!desc_ok(desc) || (read != 0 && read != 1) || !deta ||
+        (reinterpret_cast<uintptr_t>(deta) & 3u))
+        return GRADLEV_ERR_INVALID_ARG;
+    const gradlev_desc& d = *desc;
+    const gradlev_desc sd = suffix_desc(d, read);
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < eta_grad_ws_bytes(d, read))
+        return GRADLEV_ERR_WORKSPACE;
+    Tok tx, tg, tu;
+    if (!resolve(d, x, d.d_in, &tx, true) || !resolve(d, g_hat, d.d_out, &tg, true) ||
+        !resolve(d, upstream, read == 0 ? d.d_out : d.d_in, &tu, true))
+        return GRADLEV_ERR_INVALID_ARG;
+    if (read == 1 && (!g_out || !g_out->data)) return GRADLEV_ERR_INVALID_ARG;
+    if (d.T == 0) return GRADLEV_OK;
+    const size_t base = round_up(suffix_ws_bytes(sd), 256);
+    gradlev_tensor rt;
+    rt.data = static_cast<uint8_t*>(ws) + base;
+    for (int i = 0; i < 4; ++i) rt.stride[i] = 0;
+    // forward read: q = k = x, v = dL/dy;  costate read: q = ghat, k = g_out, v = dL/dgin
+    const int rc = read == 0
+                       ? run_suffix_scan(&sd, x, x, upstream, &rt, ws, base, stream)
+                       : run_suffix_scan(&sd, g_hat, g_out, upstream, &rt, ws, base, stream);
+    if (rc != GRADLEV_OK) return rc;
+    Tok trr;
+    resolve(sd, &rt, sd.d_out, &trr, true);
+    const Tok& ta = read == 0 ? tg : tx;
+    gl::TokStr as, rs;
+    for (int i = 0; i < 4; ++i) {
+        as.s[i] = ta.s[i];
+        rs.s[i] = trr.s[i];
+    }
+    if (gl::launch_rowdot(ta.data, as, trr.data, rs, deta, d.L, d.B, d.T, d.H, sd.d_out, -1.0f,
+                          d.dtype == GRADLEV_BF16, stream) != cudaSuccess)
+        return GRADLEV_ERR_CUDA;
     return GRADLEV_OK;
 }
 
@@ -764,6 +878,31 @@ size_t gradlev_workspace_bytes_gated(const gradlev_desc* desc) {
     DevInfo dev;
     int sms = device_info(&dev) ? dev.sms : 160;
     return gated_ws_bytes(*desc, sms);
+}
+
+int gradlev_suffix_scan(const gradlev_desc* desc, const gradlev_tensor* q,
+                        const gradlev_tensor* k, const gradlev_tensor* v, const gradlev_tensor* r,
+                        void* workspace, size_t workspace_bytes, gradlev_stream_t stream) {
+    return run_suffix_scan(desc, q, k, v, r, workspace, workspace_bytes,
+                           reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t gradlev_suffix_workspace_bytes(const gradlev_desc* desc) {
+    if (!desc_ok(desc)) return 0;
+    return suffix_ws_bytes(*desc);
+}
+
+int gradlev_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x,
+                     const gradlev_tensor* g_hat, const gradlev_tensor* g_out,
+                     const gradlev_tensor* upstream, float* deta, void* workspace,
+                     size_t workspace_bytes, gradlev_stream_t stream) {
+    return run_eta_grad(desc, read, x, g_hat, g_out, upstream, deta, workspace, workspace_bytes,
+                        reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t gradlev_eta_grad_workspace_bytes(const gradlev_desc* desc, int read) {
+    if (!desc_ok(desc) || (read != 0 && read != 1)) return 0;
+    return eta_grad_ws_bytes(*desc, read);
 }
 
 int gradlev_decode_read(const gradlev_desc* desc, const gradlev_tensor* x, const float* W0,

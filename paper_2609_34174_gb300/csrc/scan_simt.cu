@@ -35,7 +35,10 @@ __device__ __forceinline__ void st_from_f32<__nv_bfloat16>(__nv_bfloat16* p, flo
 }
 
 // Shared memory: Q, K [32][dq], V [32][32], scores [32][33], S^T [dq][32].
-template <typename T>
+// REV walks the chunks from the last to the first and mixes in the strictly LATER
+// tokens of each chunk: the anti-causal read sum_{s>t} (k_s . q_t) v_s of the same
+// writes (outer gradients through the reads).  W0 may be null (no base matrix).
+template <typename T, bool REV>
 __global__ void __launch_bounds__(kSimtThreads) simt_scan_kernel(const SimtScanParams p) {
     extern __shared__ float sm[];
     const int dq = p.dq;
@@ -62,12 +65,14 @@ __global__ void __launch_bounds__(kSimtThreads) simt_scan_kernel(const SimtScanP
     for (int i = tid; i < dq * kSimtNv; i += kSimtThreads) {
         const int qi = i / kSimtNv, c = i % kSimtNv;
         float w = 0.0f;
-        if (v0 + c < p.dv)
+        if (p.W0 && v0 + c < p.dv)
             w = p.w0_transposed ? w0[(size_t)qi * p.dv + v0 + c] : w0[(size_t)(v0 + c) * dq + qi];
         ST[i] = w;
     }
 
-    for (int t0 = 0; t0 < p.T; t0 += kSimtChunk) {
+    const int n_ch = (p.T + kSimtChunk - 1) / kSimtChunk;
+    for (int ci = 0; ci < n_ch; ++ci) {
+        const int t0 = (REV ? n_ch - 1 - ci : ci) * kSimtChunk;
         __syncthreads();
         for (int i = tid; i < kSimtChunk * dq; i += kSimtThreads) {
             const int r = i / dq, c = i % dq, t = t0 + r;
@@ -86,11 +91,11 @@ __global__ void __launch_bounds__(kSimtThreads) simt_scan_kernel(const SimtScanP
             Vs[i] = a;
         }
         __syncthreads();
-        // scores of the strictly earlier tokens of this chunk, scaled by -eta
+        // scores of the strictly earlier (REV: later) tokens of this chunk, scaled by -eta
         for (int i = tid; i < kSimtChunk * kSimtChunk; i += kSimtThreads) {
             const int r = i / kSimtChunk, s = i % kSimtChunk;
             float acc = 0.0f;
-            if (s < r)
+            if (REV ? s > r : s < r)
                 for (int c = 0; c < dq; ++c) acc = fmaf(Qs[r * dq + c], Ks[s * dq + c], acc);
             Sc[r * (kSimtChunk + 1) + s] = -p.eta * acc;
         }
@@ -100,7 +105,8 @@ __global__ void __launch_bounds__(kSimtThreads) simt_scan_kernel(const SimtScanP
             const int r = i / kSimtNv, c = i % kSimtNv, t = t0 + r;
             float acc = 0.0f;
             for (int qi = 0; qi < dq; ++qi) acc = fmaf(Qs[r * dq + qi], ST[qi * kSimtNv + c], acc);
-            for (int s = 0; s < r; ++s) acc = fmaf(Sc[r * (kSimtChunk + 1) + s], Vs[s * kSimtNv + c], acc);
+            for (int s = REV ? r + 1 : 0; s < (REV ? kSimtChunk : r); ++s)
+                acc = fmaf(Sc[r * (kSimtChunk + 1) + s], Vs[s * kSimtNv + c], acc);
             if (t < p.T && v0 + c < p.dv) {
                 const EpiParams& e = p.epi;
                 float o = acc;
@@ -129,24 +135,25 @@ size_t simt_smem_bytes(int dq) {
                             kSimtChunk * (kSimtChunk + 1) + (size_t)dq * kSimtNv);
 }
 
-cudaError_t launch_simt_scan(const SimtScanParams& p, bool bf16, cudaStream_t stream) {
+template <typename T, bool REV>
+static cudaError_t launch_simt_t(const SimtScanParams& p, int grid, size_t smem, cudaStream_t stream) {
+    const cudaError_t e = cudaFuncSetAttribute(simt_scan_kernel<T, REV>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    simt_scan_kernel<T, REV><<<grid, kSimtThreads, smem, stream>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_simt_scan(const SimtScanParams& p, bool bf16, bool rev, cudaStream_t stream) {
     const int n_tiles = (p.dv + kSimtNv - 1) / kSimtNv;
     const long long grid = (long long)p.L * p.B * p.H * n_tiles;
     if (grid <= 0 || grid > 0x7FFFFFFF) return cudaErrorInvalidValue;
     const size_t smem = simt_smem_bytes(p.dq);
-    cudaError_t e;
-    if (bf16) {
-        e = cudaFuncSetAttribute(simt_scan_kernel<__nv_bfloat16>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        simt_scan_kernel<__nv_bfloat16><<<(int)grid, kSimtThreads, smem, stream>>>(p);
-    } else {
-        e = cudaFuncSetAttribute(simt_scan_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)smem);
-        if (e != cudaSuccess) return e;
-        simt_scan_kernel<float><<<(int)grid, kSimtThreads, smem, stream>>>(p);
-    }
-    return cudaGetLastError();
+    if (bf16)
+        return rev ? launch_simt_t<__nv_bfloat16, true>(p, (int)grid, smem, stream)
+                   : launch_simt_t<__nv_bfloat16, false>(p, (int)grid, smem, stream);
+    return rev ? launch_simt_t<float, true>(p, (int)grid, smem, stream)
+               : launch_simt_t<float, false>(p, (int)grid, smem, stream);
 }
 
 }  // namespace gl
