@@ -19,6 +19,9 @@ cudaError_t launch_tc_scan(const CUtensorMap& q, const CUtensorMap& k, const CUt
                            const CUtensorMap& o, const TcScanParams& p, bool costate, int grid,
                            cudaStream_t stream);
 cudaError_t launch_simt_scan(const SimtScanParams& p, bool bf16, bool rev, cudaStream_t stream);
+cudaError_t launch_tc_suffix(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
+                             const CUtensorMap& o, const TcScanParams& p, bool shared_qk, int grid,
+                             cudaStream_t stream);
 cudaError_t launch_rowdot(const void* a, const TokStr& as, const void* r, const TokStr& rs,
                           float* out, int L, int B, int T, int H, int w, float scale, bool bf16,
                           cudaStream_t stream);
@@ -574,33 +577,108 @@ int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
 }
 
 // Suffix (anti-causal) read r_s = sum_{t>s} (k_t . q_s) v_t: d_in is the width of q
-// and k, d_out the width of v and r.  Runs the CUDA-core scan in reverse with no
-// base matrix and eta = -1.
-size_t suffix_ws_bytes(const gradlev_desc& d) {
-    (void)d;
-    return 0;
+// and k, d_out the width of v and r.  The scan kernels run in reverse with no base
+// matrix and eta = -1: the tensor-core kernel for bf16 with 64-wide q and k, the
+// CUDA-core kernel otherwise.
+bool suffix_tc_shape(const gradlev_desc& d) {
+    return d.dtype == GRADLEV_BF16 && d.d_in == 64 && d.d_out % 64 == 0;
 }
 
-int run_suffix_scan(const gradlev_desc* desc, const gradlev_tensor* q, const gradlev_tensor* k,
-                    const gradlev_tensor* v, const gradlev_tensor* r, void* ws, size_t ws_bytes,
+int dev_sms_or_default() {
+    DevInfo dev;
+    return device_info(&dev) ? dev.sms : 160;
+}
+
+size_t suffix_ws_bytes(const gradlev_desc& d, int sms) {
+    return suffix_tc_shape(d) ? plan_tc(d, 64, d.d_out, sms).ws_bytes : 0;
+}
+
+bool same_tensor(const Tok& a, const Tok& b) {
+    if (a.data != b.data) return false;
+    for (int i = 0; i < 4; ++i)
+        if (a.s[i] != b.s[i]) return false;
+    return true;
+}
+
+// With dot_out, the tensor-core path reduces every result row to the per-token
+// dot_out[t] = dot_scale * (r_t . a_t) in its epilogue and stores no r (r may then be
+// null); *fused tells whether it did (else r holds the read and no dot was formed).
+int run_suffix_impl(const gradlev_desc* desc, const gradlev_tensor* q, const gradlev_tensor* k,
+                    const gradlev_tensor* v, const gradlev_tensor* r, const Tok* dot_a,
+                    float* dot_out, float dot_scale, bool* fused, void* ws, size_t ws_bytes,
                     cudaStream_t stream) {
+    if (fused) *fused = false;
     if (!desc_ok(desc)) return GRADLEV_ERR_INVALID_ARG;
     const gradlev_desc& d = *desc;
     Tok tq, tk, tv, tr;
     if (!resolve(d, q, d.d_in, &tq, true) || !resolve(d, k, d.d_in, &tk, true) ||
-        !resolve(d, v, d.d_out, &tv, true) || !resolve(d, r, d.d_out, &tr, true))
+        !resolve(d, v, d.d_out, &tv, true) || !resolve(d, r, d.d_out, &tr, dot_out == nullptr))
         return GRADLEV_ERR_INVALID_ARG;
     DevInfo dev;
     if (!device_info(&dev)) return GRADLEV_ERR_CUDA;
     if (!(dev.major == 10 && dev.minor == 3)) return GRADLEV_ERR_UNSUPPORTED;
-    if (ws_bytes < suffix_ws_bytes(d)) return GRADLEV_ERR_WORKSPACE;
-    (void)ws;
+    const size_t need = suffix_ws_bytes(d, dev.sms);
+    if (ws_bytes < need || (need && (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)))
+        return GRADLEV_ERR_WORKSPACE;
     if (d.T == 0) return GRADLEV_OK;
     const int elem = d.dtype == GRADLEV_BF16 ? 2 : 4;
     const Tok* all[4] = {&tq, &tk, &tv, &tr};
     for (const Tok* t : all)
         if ((reinterpret_cast<uintptr_t>(t->data) % elem) != 0) return GRADLEV_ERR_UNSUPPORTED;
-    if (!simt_shape_ok(d, d.d_in)) return GRADLEV_ERR_UNSUPPORTED;
+    const bool dot_ok = dot_out && dot_a && tc_layout_ok(*dot_a, 2);
+    if (suffix_tc_shape(d) && tc_layout_ok(tq, 2) && tc_layout_ok(tk, 2) && tc_layout_ok(tv, 2) &&
+        tc_layout_ok(tr, 2) && (dot_out == nullptr || dot_ok) && (tr.data || dot_ok)) {
+        const Plan pl = plan_tc(d, 64, d.d_out, dev.sms);
+        CUtensorMap mq, mk, mv, mo;
+        if (!make_tmap(&mq, d, tq, 64) || !make_tmap(&mk, d, tk, 64) ||
+            !make_tmap(&mv, d, tv, d.d_out) || !make_tmap(&mo, d, tr.data ? tr : tv, d.d_out))
+            return GRADLEV_ERR_UNSUPPORTED;
+        TcScanParams p;
+        memset(&p, 0, sizeof(p));
+        p.L = d.L;
+        p.B = d.B;
+        p.T = d.T;
+        p.H = d.H;
+        p.dq = 64;
+        p.dv = d.d_out;
+        p.n_tiles = pl.n_tiles;
+        p.seg_len = pl.seg_len;
+        p.n_seg = pl.n_seg;
+        p.n_items = pl.n_items;
+        p.n_ut = pl.n_items / pl.n_seg;
+        p.lookback_limit_ns = 4000000000ull;
+        p.test_skip_publish = -1;
+        p.eta = -1.0f;  // + sum over the later tokens
+        p.lam = 1.0f;
+        p.inv_lam = 1.0f;
+        p.mu = 1.0f;
+        p.W0 = nullptr;  // the suffix read has no base matrix
+        Tok none;
+        fill_epi(&p.epi, tr, none, none, GRADLEV_ACT_NONE);
+        if (dot_out) {
+            p.epi.dot_a = dot_a->data;
+            for (int i = 0; i < 4; ++i) p.epi.dot_a_str[i] = dot_a->s[i];
+            p.epi.dot_out = dot_out;
+            p.epi.dot_scale = dot_scale;
+            // several 64-wide tiles add their partial dots
+            if (pl.n_tiles > 1 &&
+                cudaMemsetAsync(dot_out, 0, sizeof(float) * (size_t)d.L * d.B * d.T * d.H, stream) !=
+                    cudaSuccess)
+                return GRADLEV_ERR_CUDA;
+            if (fused) *fused = true;
+        }
+        uint8_t* wsb = static_cast<uint8_t*>(ws);
+        p.ctrl = reinterpret_cast<unsigned int*>(wsb);
+        p.flags = reinterpret_cast<unsigned int*>(wsb + pl.off_flags);
+        p.agg = reinterpret_cast<float*>(wsb + pl.off_agg);
+        p.incl = reinterpret_cast<float*>(wsb + pl.off_incl);
+        if (cudaMemsetAsync(ws, 0, pl.zero_bytes, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
+        const int grid = pl.n_items < dev.sms ? pl.n_items : dev.sms;
+        if (gl::launch_tc_suffix(mq, mk, mv, mo, p, same_tensor(tq, tk), grid, stream) != cudaSuccess)
+            return GRADLEV_ERR_CUDA;
+        return GRADLEV_OK;
+    }
+    if (!simt_shape_ok(d, d.d_in) || !tr.data) return GRADLEV_ERR_UNSUPPORTED;
     gl::SimtScanParams p;
     memset(&p, 0, sizeof(p));
     p.L = d.L;
@@ -637,10 +715,10 @@ gradlev_desc suffix_desc(const gradlev_desc& d, int read) {
     return s;
 }
 
-size_t eta_grad_ws_bytes(const gradlev_desc& d, int read) {
+size_t eta_grad_ws_bytes(const gradlev_desc& d, int read, int sms) {
     const gradlev_desc s = suffix_desc(d, read);
     const size_t elem = d.dtype == GRADLEV_BF16 ? 2 : 4;
-    return round_up(suffix_ws_bytes(s), 256) +
+    return round_up(suffix_ws_bytes(s, sms), 256) +
            round_up((size_t)d.L * d.B * d.T * d.H * s.d_out * elem, 256);
 }
 
@@ -653,7 +731,9 @@ int run_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x,
         return GRADLEV_ERR_INVALID_ARG;
     const gradlev_desc& d = *desc;
     const gradlev_desc sd = suffix_desc(d, read);
-    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < eta_grad_ws_bytes(d, read))
+    const int sms = dev_sms_or_default();
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 ||
+        ws_bytes < eta_grad_ws_bytes(d, read, sms))
         return GRADLEV_ERR_WORKSPACE;
     Tok tx, tg, tu;
     if (!resolve(d, x, d.d_in, &tx, true) || !resolve(d, g_hat, d.d_out, &tg, true) ||
@@ -661,18 +741,29 @@ int run_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x,
         return GRADLEV_ERR_INVALID_ARG;
     if (read == 1 && (!g_out || !g_out->data)) return GRADLEV_ERR_INVALID_ARG;
     if (d.T == 0) return GRADLEV_OK;
-    const size_t base = round_up(suffix_ws_bytes(sd), 256);
+    const size_t base = round_up(suffix_ws_bytes(sd, sms), 256);
     gradlev_tensor rt;
     rt.data = static_cast<uint8_t*>(ws) + base;
     for (int i = 0; i < 4; ++i) rt.stride[i] = 0;
-    // forward read: q = k = x, v = dL/dy;  costate read: q = ghat, k = g_out, v = dL/dgin
-    const int rc = read == 0
-                       ? run_suffix_scan(&sd, x, x, upstream, &rt, ws, base, stream)
-                       : run_suffix_scan(&sd, g_hat, g_out, upstream, &rt, ws, base, stream);
-    if (rc != GRADLEV_OK) return rc;
+    const Tok& ta = read == 0 ? tg : tx;
+    // forward read: q = k = x, v = dL/dy;  costate read: q = ghat, k = g_out, v = dL/dgin.
+    // The tensor-core path forms the dot in its epilogue; otherwise r goes through the
+    // workspace and a row-dot kernel.
+    bool fused = false;
+    const int rc = read == 0 ? run_suffix_impl(&sd, x, x, upstream, nullptr, &ta, deta, -1.0f,
+                                               &fused, ws, base, stream)
+                             : run_suffix_impl(&sd, g_hat, g_out, upstream, nullptr, &ta, deta,
+                                               -1.0f, &fused, ws, base, stream);
+    if (rc == GRADLEV_OK && fused) return GRADLEV_OK;
+    if (rc != GRADLEV_OK && rc != GRADLEV_ERR_UNSUPPORTED) return rc;
+    const int rc2 = read == 0
+                        ? run_suffix_impl(&sd, x, x, upstream, &rt, nullptr, nullptr, 0.f, nullptr,
+                                          ws, base, stream)
+                        : run_suffix_impl(&sd, g_hat, g_out, upstream, &rt, nullptr, nullptr, 0.f,
+                                          nullptr, ws, base, stream);
+    if (rc2 != GRADLEV_OK) return rc2;
     Tok trr;
     resolve(sd, &rt, sd.d_out, &trr, true);
-    const Tok& ta = read == 0 ? tg : tx;
     gl::TokStr as, rs;
     for (int i = 0; i < 4; ++i) {
         as.s[i] = ta.s[i];
@@ -883,13 +974,13 @@ size_t gradlev_workspace_bytes_gated(const gradlev_desc* desc) {
 int gradlev_suffix_scan(const gradlev_desc* desc, const gradlev_tensor* q,
                         const gradlev_tensor* k, const gradlev_tensor* v, const gradlev_tensor* r,
                         void* workspace, size_t workspace_bytes, gradlev_stream_t stream) {
-    return run_suffix_scan(desc, q, k, v, r, workspace, workspace_bytes,
-                           reinterpret_cast<cudaStream_t>(stream));
+    return run_suffix_impl(desc, q, k, v, r, nullptr, nullptr, 0.f, nullptr, workspace,
+                           workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
 }
 
 size_t gradlev_suffix_workspace_bytes(const gradlev_desc* desc) {
     if (!desc_ok(desc)) return 0;
-    return suffix_ws_bytes(*desc);
+    return suffix_ws_bytes(*desc, dev_sms_or_default());
 }
 
 int gradlev_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x,
@@ -902,7 +993,7 @@ int gradlev_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x
 
 size_t gradlev_eta_grad_workspace_bytes(const gradlev_desc* desc, int read) {
     if (!desc_ok(desc) || (read != 0 && read != 1)) return 0;
-    return eta_grad_ws_bytes(*desc, read);
+    return eta_grad_ws_bytes(*desc, read, dev_sms_or_default());
 }
 
 int gradlev_decode_read(const gradlev_desc* desc, const gradlev_tensor* x, const float* W0,

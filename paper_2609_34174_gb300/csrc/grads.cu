@@ -25,16 +25,39 @@ __device__ __forceinline__ float ld(const void* p, long long i) {
         return static_cast<const float*>(p)[i];
 }
 
-// out[l][b][t][h] = scale * sum_j a[l,b,t,h,j] * r[l,b,t,h,j]; one warp per token row.
+// 8 bf16 or 4 fp32 values of one 16-byte piece, as floats; returns the count.
+template <bool BF16>
+__device__ __forceinline__ int ld16(const void* p, long long i, float* f) {
+    const uint4 v = *reinterpret_cast<const uint4*>(static_cast<const char*>(p) + i * (BF16 ? 2 : 4));
+    if constexpr (BF16) {
+        const __nv_bfloat16* h = reinterpret_cast<const __nv_bfloat16*>(&v);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) f[k] = __bfloat162float(h[k]);
+        return 8;
+    } else {
+        f[0] = __uint_as_float(v.x);
+        f[1] = __uint_as_float(v.y);
+        f[2] = __uint_as_float(v.z);
+        f[3] = __uint_as_float(v.w);
+        return 4;
+    }
+}
+
+// out[l][b][t][h] = scale * sum_j a[l,b,t,h,j] * r[l,b,t,h,j].  A group of `lanes`
+// lanes (a power of two up to 32) takes one token row in 16-byte pieces when
+// `vec`, else element by element with a whole warp per row.
 template <bool BF16>
 __global__ void __launch_bounds__(kThreads)
     rowdot_kernel(const void* __restrict__ a, TokStr as, const void* __restrict__ r, TokStr rs,
-                  float* __restrict__ out, int L, int B, int T, int H, int w, float scale) {
+                  float* __restrict__ out, int L, int B, int T, int H, int w, float scale, int vec,
+                  int lanes) {
     const long long rows = (long long)L * B * T * H;
-    const long long row = (long long)blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
-    if (row >= rows) return;  // warp-uniform
-    long long t = row;
+    const int LR = vec ? lanes : 32;
+    const int sub = lane / LR, cl = lane - sub * LR;
+    const long long row = ((long long)blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5)) * (32 / LR) + sub;
+    const bool live = row < rows;
+    long long t = live ? row : 0;
     const int h = (int)(t % H);
     t /= H;
     const int tt = (int)(t % T);
@@ -43,9 +66,22 @@ __global__ void __launch_bounds__(kThreads)
     const int l = (int)(t / B);
     const long long ao = tok_off(as.s, l, b, tt, h), ro = tok_off(rs.s, l, b, tt, h);
     float acc = 0.f;
-    for (int j = lane; j < w; j += 32) acc = fmaf(ld<BF16>(a, ao + j), ld<BF16>(r, ro + j), acc);
-    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) out[row] = scale * acc;
+    if (live) {
+        if (vec) {
+            constexpr int kPer = BF16 ? 8 : 4;
+            for (int j = cl * kPer; j < w; j += LR * kPer) {
+                float fa[8], fr[8];
+                ld16<BF16>(a, ao + j, fa);
+                ld16<BF16>(r, ro + j, fr);
+#pragma unroll
+                for (int k = 0; k < kPer; ++k) acc = fmaf(fa[k], fr[k], acc);
+            }
+        } else {
+            for (int j = cl; j < w; j += 32) acc = fmaf(ld<BF16>(a, ao + j), ld<BF16>(r, ro + j), acc);
+        }
+    }
+    for (int o = LR >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (live && cl == 0) out[row] = scale * acc;
 }
 
 }  // namespace grads
@@ -54,14 +90,26 @@ cudaError_t launch_rowdot(const void* a, const TokStr& as, const void* r, const 
                           float* out, int L, int B, int T, int H, int w, float scale, bool bf16,
                           cudaStream_t stream) {
     const long long rows = (long long)L * B * T * H;
-    const long long grid = (rows + grads::kThreads / 32 - 1) / (grads::kThreads / 32);
+    // 16-byte pieces when every row starts on a 16-byte boundary
+    const int per = bf16 ? 8 : 4, elem = bf16 ? 2 : 4;
+    bool vec = w % per == 0 && (reinterpret_cast<uintptr_t>(a) & 15u) == 0 &&
+               (reinterpret_cast<uintptr_t>(r) & 15u) == 0;
+    for (int i = 0; i < 4; ++i) vec = vec && (as.s[i] * elem) % 16 == 0 && (rs.s[i] * elem) % 16 == 0;
+    int lanes = 32;
+    if (vec) {
+        const int pieces = w / per;
+        lanes = 1;
+        while (lanes < pieces && lanes < 32) lanes <<= 1;
+    }
+    const long long rows_per_cta = (long long)(grads::kThreads / 32) * (vec ? 32 / lanes : 1);
+    const long long grid = (rows + rows_per_cta - 1) / rows_per_cta;
     if (grid <= 0 || grid > 0x7FFFFFFF) return cudaErrorInvalidValue;
     if (bf16)
-        grads::rowdot_kernel<true><<<(int)grid, grads::kThreads, 0, stream>>>(a, as, r, rs, out, L, B,
-                                                                               T, H, w, scale);
+        grads::rowdot_kernel<true><<<(int)grid, grads::kThreads, 0, stream>>>(
+            a, as, r, rs, out, L, B, T, H, w, scale, vec ? 1 : 0, lanes);
     else
-        grads::rowdot_kernel<false><<<(int)grid, grads::kThreads, 0, stream>>>(a, as, r, rs, out, L,
-                                                                                B, T, H, w, scale);
+        grads::rowdot_kernel<false><<<(int)grid, grads::kThreads, 0, stream>>>(
+            a, as, r, rs, out, L, B, T, H, w, scale, vec ? 1 : 0, lanes);
     return cudaGetLastError();
 }
 

@@ -67,6 +67,12 @@ struct EpiParams {
     const void* zin;      // optional preactivation: out = sigma'(z) (.) result (costate)
     long long z_str[4];
     int act;
+    // optional per-token dot (suffix read only): dot_out[l][b][t][h] +=
+    // dot_scale * (result row . dot_a row), fp32 [L][B][T][H] contiguous
+    const void* dot_a;
+    long long dot_a_str[4];
+    float* dot_out;
+    float dot_scale;
 };
 
 // Parameters of the tensor-core scan kernel (bf16, dq in {64, 128}, dv % 64 == 0).

@@ -102,6 +102,9 @@ struct Item {
 // Items are numbered segment-major: every (unit, tile) pair's segment k comes
 // before any segment k+1, so segment k's predecessor is item - n_ut and a
 // look-back mostly finds inclusive prefixes published by earlier waves.
+// REV (the anti-causal suffix read) numbers segments from the end of the sequence:
+// segment k covers [T - (k+1) seg_len, T - k seg_len), clipped at token 0.
+template <bool REV>
 __device__ __forceinline__ Item decode_item(int item, const TcScanParams& p) {
     Item I;
     I.k = item / p.n_ut;
@@ -112,11 +115,39 @@ __device__ __forceinline__ Item decode_item(int item, const TcScanParams& p) {
     int lb = u / p.H;
     I.b = lb % p.B;
     I.l = lb / p.B;
-    I.t_begin = I.k * p.seg_len;
-    I.t_end = min(p.T, I.t_begin + p.seg_len);
+    if constexpr (REV) {
+        I.t_end = p.T - I.k * p.seg_len;
+        I.t_begin = max(0, I.t_end - p.seg_len);
+    } else {
+        I.t_begin = I.k * p.seg_len;
+        I.t_end = min(p.T, I.t_begin + p.seg_len);
+    }
     I.nch = (I.t_end - I.t_begin + kChunk - 1) / kChunk;
     I.phase1 = (p.n_seg > 1) && (I.k < p.n_seg - 1);
     return I;
+}
+
+// First token of chunk c of an item: chunks run forward from the segment start, or
+// (REV) backward from its end, so that a reverse item's lowest chunk may start
+// before token 0 (its missing rows load as zeros and are not stored).
+template <bool REV>
+__device__ __forceinline__ int chunk_t0(const Item& I, int c) {
+    return REV ? I.t_end - (c + 1) * kChunk : I.t_begin + c * kChunk;
+}
+
+// One 64-wide bf16 output row written straight to global memory: a TMA store may
+// not start at a negative coordinate, so a reverse chunk that begins before token 0
+// is stored row by row.
+__device__ __noinline__ void epi_store_row(const EpiParams& e, long long o_off, const float* v) {
+    __nv_bfloat16* op = static_cast<__nv_bfloat16*>(e.out) + o_off;
+    for (int q = 0; q < 8; ++q) {
+        uint4 w;
+        w.x = pack_bf16x2(v[8 * q + 0], v[8 * q + 1]);
+        w.y = pack_bf16x2(v[8 * q + 2], v[8 * q + 3]);
+        w.z = pack_bf16x2(v[8 * q + 4], v[8 * q + 5]);
+        w.w = pack_bf16x2(v[8 * q + 6], v[8 * q + 7]);
+        *reinterpret_cast<uint4*>(op + 8 * q) = w;
+    }
 }
 
 __device__ __forceinline__ void raise_error(const TcScanParams& p, unsigned int bits,
@@ -177,7 +208,7 @@ __host__ __device__ constexpr uint32_t kmaj_step(int kk) {
 // MN-major operand: step kk starts 16 rows (two 8-row groups of 1024 B) further.
 __host__ __device__ constexpr uint32_t mnmaj_step(int kk) { return (uint32_t)((kk * 2048) >> 4); }
 
-template <int DQ, bool COSTATE>
+template <int DQ, bool COSTATE, bool REV>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_scan_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
@@ -281,7 +312,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         break;
                     }
                     uint8_t* st = smem + s * Lay::kStageBytes;
-                    const int t0 = I.t_begin + c * kChunk;
+                    const int t0 = chunk_t0<REV>(I, c);
                     mbar_arrive_expect_tx(&full[s], pass == 1 ? Lay::kTxPass1 : Lay::kTxPass2);
                     if (COSTATE && pass == 2) {
 #pragma unroll
@@ -310,10 +341,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 item_slot[slot] = item;
                 mbar_arrive(&item_full[slot]);
                 if (item >= 0) {
-                    const Item I = decode_item(item, p);
+                    const Item I = decode_item<REV>(item, p);
                     if (I.phase1) load_pass(I, 1);
                 }
-                if (pending >= 0) load_pass(decode_item(pending, p), 2);
+                if (pending >= 0) load_pass(decode_item<REV>(pending, p), 2);
                 pending = item;
                 if (item < 0) break;
             }
@@ -359,7 +390,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_arrive(&item_empty[slot]);
                 // phase 1 of the new item: its segment aggregate sum K^T V
                 if (item >= 0) {
-                    const Item I = decode_item(item, p);
+                    const Item I = decode_item<REV>(item, p);
                     if (I.phase1) {
                         const uint32_t b = dzc & 1;
                         if (!(ok = wait_or_fail(&dz_free[b], ((dzc >> 1) & 1) ^ 1))) break;
@@ -380,7 +411,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // phase 2 of the previous item: score and dZ of every chunk (dZ of the
                 // last chunk is not needed)
                 if (pending >= 0) {
-                    const Item I = decode_item(pending, p);
+                    const Item I = decode_item<REV>(pending, p);
                     for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
                         const int s = n % NS;
                         if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
@@ -434,11 +465,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // the new item's phase-1 stages precede the previous item's phase 2 and
                 // are released by the front issuer
                 if (item >= 0) {
-                    const Item In = decode_item(item, p);
+                    const Item In = decode_item<REV>(item, p);
                     if (In.phase1) n += In.nch;
                 }
                 if (pending >= 0) {
-                    const Item I = decode_item(pending, p);
+                    const Item I = decode_item<REV>(pending, p);
                     for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
                         const int s = n % NS;
                         const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
@@ -495,7 +526,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(&item_empty[slot]);
             if (item < 0) break;
-            const Item I = decode_item(item, p);
+            const Item I = decode_item<REV>(item, p);
             bool ok = true;
             for (int c = 0; c < I.nch; ++c, ++c2) {
                 const uint32_t sb = c2 & 1;
@@ -515,9 +546,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t base = tmem + col_sc(sb) + lane_off;
 #pragma unroll 1
                 for (int half = 0; half < 2; ++half) {
-                    const bool mine = half == 0 ? !helper : (q4 < 2 ? !helper : (helper || kPHelpers == 0));
+                    // REV keeps tokens s > t: rows >= 64 have an all-zero first half, and
+                    // rows < 64 (whose lanes no helper warp can reach) build both halves
+                    const bool mine =
+                        REV ? (q4 < 2 ? !helper : (half == 0 ? !helper : (helper || kPHelpers == 0)))
+                            : (half == 0 ? !helper : (q4 < 2 ? !helper : (helper || kPHelpers == 0)));
                     if (!mine) continue;
-                    if ((half == 1 && q4 < 2) || p.mu == 0.0f) {
+                    if ((REV ? (half == 0 && q4 >= 2) : (half == 1 && q4 < 2)) || p.mu == 0.0f) {
                         // rows < 64: tokens >= 64 all masked; eta = 0: no P at all
                         tmem_zero32_async(base + half * 64);
                         continue;
@@ -530,8 +565,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
                             const int s0 = half * 64 + sub * 32 + 2 * i;
-                            w[i] = pack_bf16x2(s0 < row ? v[2 * i] : 0.0f,
-                                               s0 + 1 < row ? v[2 * i + 1] : 0.0f);
+                            if constexpr (REV)
+                                w[i] = pack_bf16x2(s0 > row ? v[2 * i] : 0.0f,
+                                                   s0 + 1 > row ? v[2 * i + 1] : 0.0f);
+                            else
+                                w[i] = pack_bf16x2(s0 < row ? v[2 * i] : 0.0f,
+                                                   s0 + 1 < row ? v[2 * i + 1] : 0.0f);
                         }
                         tmem_st16_async(base + half * 64 + sub * 16, w);
                     }
@@ -561,7 +600,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(&item_empty[slot]);
             if (item < 0) break;
-            const Item I = decode_item(item, p);
+            const Item I = decode_item<REV>(item, p);
             bool ok = true;
             for (int c = 0; c < I.nch; ++c, ++c2) {
                 const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
@@ -578,12 +617,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (lane == 0) mbar_arrive(&o_free[ob]);
 #pragma unroll
                 for (int i = 0; i < 64; ++i) v[i] *= p.lam;  // O = lam * (Q S'^T + L(Q K^T) V)
-                const int t0 = I.t_begin + c * kChunk;
+                const int t0 = chunk_t0<REV>(I, c);
                 const int t = t0 + row;
                 const int col0 = I.j * 64;
+                const bool valid = REV ? (t >= I.t_begin && t < I.t_end) : t < I.t_end;
                 // The activation paths (MLP layers only) run out of line, so the hot
                 // loop of the plain scans stays small in the instruction cache.
-                if (e.zin && t < I.t_end) {
+                if (e.zin && valid) {
                     float tmp[64];
 #pragma unroll
                     for (int i = 0; i < 64; ++i) tmp[i] = v[i];
@@ -591,7 +631,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int i = 0; i < 64; ++i) v[i] = tmp[i];
                 }
-                if (e.out2 && t < I.t_end) {
+                if (e.out2 && valid) {
                     float tmp[64];
 #pragma unroll
                     for (int i = 0; i < 64; ++i) tmp[i] = v[i];
@@ -605,12 +645,67 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 const uint32_t otile = sbase + Lay::kOOff + ob * kTile;
+                // (REV only) a chunk starting before token 0 is stored row by row, and a
+                // suffix read reduced to a per-token dot stores no rows at all
+                const bool direct = REV && (t0 < 0 || e.out == nullptr);
+                if constexpr (REV) {
+                    if (e.dot_out) {
+                        // dot_out[t] (+)= dot_scale * (row . a row) over this 64-wide tile.
+                        // The warp's 32 rows of a arrive coalesced (cp.async, one chunk
+                        // ahead) in its 4 KB slice of the staging tiles, which are free
+                        // because no rows are stored; the 128B swizzle lets each lane read
+                        // its own row without bank conflicts.
+                        const __nv_bfloat16* ab = static_cast<const __nv_bfloat16*>(e.dot_a);
+                        auto fetch = [&](uint32_t dst, int tc0) {
+#pragma unroll
+                            for (int it = 0; it < 8; ++it) {
+                                const int pc = it * 32 + lane, pr = pc >> 3, pq = pc & 7;
+                                const int tr = tc0 + q4 * 32 + pr;
+                                const bool ok = tr >= I.t_begin && tr < I.t_end;
+                                cp_async16(dst + sw128_off(pr, pq),
+                                           ok ? ab + tok_off(e.dot_a_str, I.l, I.b, tr, I.h) + col0 + pq * 8 : ab,
+                                           ok);
+                            }
+                            cp_async_commit();
+                        };
+                        const uint32_t slice = otile + (uint32_t)q4 * 4096u;
+                        if (c == 0) fetch(slice, t0);
+                        if (c + 1 < I.nch) {
+                            fetch(sbase + Lay::kOOff + (ob ^ 1) * kTile + (uint32_t)q4 * 4096u,
+                                  chunk_t0<REV>(I, c + 1));
+                            cp_async_wait<1>();
+                        } else {
+                            cp_async_wait<0>();
+                        }
+                        __syncwarp();
+                        float acc = 0.f;
+#pragma unroll
+                        for (int q = 0; q < 8; ++q) {
+                            const uint4 a4 = ld_shared_v4(slice + sw128_off(lane, q));
+                            const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&a4);
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) acc = fmaf(v[8 * q + i], __bfloat162float(hb[i]), acc);
+                        }
+                        __syncwarp();
+                        if (valid) {
+                            float* dst = e.dot_out + (((long long)I.l * p.B + I.b) * p.T + t) * p.H + I.h;
+                            if (p.n_tiles > 1)
+                                atomicAdd(dst, e.dot_scale * acc);
+                            else
+                                *dst = e.dot_scale * acc;
+                        }
+                    }
+                }
+                if (direct) {
+                    if (valid && e.out) epi_store_row(e, tok_off(e.out_str, I.l, I.b, t, I.h) + col0, v);
+                } else {
 #pragma unroll
                 for (int q = 0; q < 8; ++q)
                     st_shared_v4(otile + sw128_off(row, q), pack_bf16x2(v[8 * q], v[8 * q + 1]),
                                  pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
                                  pack_bf16x2(v[8 * q + 4], v[8 * q + 5]),
                                  pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+                }
                 fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&o_staged[ob]);
@@ -619,7 +714,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         raise_error(p, kErrWaitTimeout, abort_flag);
                         ok = false;
                     } else {
-                        tma_store_5d(&tm_o, smem + Lay::kOOff + ob * kTile, col0, I.h, t0, I.b, I.l);
+                        if (!direct)
+                            tma_store_5d(&tm_o, smem + Lay::kOOff + ob * kTile, col0, I.h, t0, I.b, I.l);
                         bulk_commit_group();
                         // the previous chunk's store (other tile) has finished reading
                         bulk_wait_group_read<1>();
@@ -679,7 +775,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // ---- phase 1 of the newly taken item (before phase 2 of the previous one)
             if (new_item >= 0) {
                 const int item = new_item;
-                const Item I = decode_item(item, p);
+                const Item I = decode_item<REV>(item, p);
                 // ---- phase 1: this segment's aggregate sum_{s in seg} k_s v_s^T.  The
                 // first segment's aggregate is already its inclusive prefix (flag 2);
                 // later segments publish the aggregate (flag 1) and look back.
@@ -712,7 +808,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // ---- look-back and phase 2 of the previous item
             if (pending >= 0) {
                 const int item = pending;
-                const Item I = decode_item(item, p);
+                const Item I = decode_item<REV>(item, p);
                 const int n_ut = p.n_ut;
                 const int r_ut = item - I.k * n_ut;
                 // ---- look-back: E = sum of the earlier segments' aggregates, stopping at
@@ -807,8 +903,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     if (!publish(item, 2u)) break;
                 }
-                // ---- starting state S'^T row = (B0^T row - eta * E) / lam
-                if (active) {
+                // ---- starting state S'^T row = (B0^T row - eta * E) / lam (REV: no base)
+                if (REV && active) {
+    #pragma unroll
+                    for (int i = 0; i < 64; ++i) st[i] *= p.mu;
+                } else if (active) {
                     const float* w0 = p.W0 + (size_t)(I.l * p.H + I.h) * p.dq * p.dv;
                     const int v0 = I.j * 64;
                     if (p.w0_transposed) {
@@ -887,12 +986,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ------------------------------------------------------------------ host side
-template <int DQ, bool COSTATE>
+template <int DQ, bool COSTATE, bool REV>
 static cudaError_t launch_one(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
                               const CUtensorMap& o, const TcScanParams& p, int grid,
                               cudaStream_t stream) {
     using Lay = TcLayout<DQ, COSTATE>;
-    auto kern = tc_scan_kernel<DQ, COSTATE>;
+    auto kern = tc_scan_kernel<DQ, COSTATE, REV>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          Lay::kSmemBytes);
     if (e != cudaSuccess) return e;
@@ -904,12 +1003,22 @@ cudaError_t launch_tc_scan(const CUtensorMap& q, const CUtensorMap& k, const CUt
                            const CUtensorMap& o, const TcScanParams& p, bool costate, int grid,
                            cudaStream_t stream) {
     if (p.dq == 64)
-        return costate ? launch_one<64, true>(q, k, v, o, p, grid, stream)
-                       : launch_one<64, false>(q, k, v, o, p, grid, stream);
+        return costate ? launch_one<64, true, false>(q, k, v, o, p, grid, stream)
+                       : launch_one<64, false, false>(q, k, v, o, p, grid, stream);
     if (p.dq == 128)
-        return costate ? launch_one<128, true>(q, k, v, o, p, grid, stream)
-                       : launch_one<128, false>(q, k, v, o, p, grid, stream);
+        return costate ? launch_one<128, true, false>(q, k, v, o, p, grid, stream)
+                       : launch_one<128, false, false>(q, k, v, o, p, grid, stream);
     return cudaErrorInvalidValue;
+}
+
+// The anti-causal suffix read r_t = sum_{s>t} (k_s . q_t) v_s (no base matrix) on the
+// 64-wide kernels: shared_qk when q and k are one tensor (one tile per chunk).
+cudaError_t launch_tc_suffix(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
+                             const CUtensorMap& o, const TcScanParams& p, bool shared_qk, int grid,
+                             cudaStream_t stream) {
+    if (p.dq != 64) return cudaErrorInvalidValue;
+    return shared_qk ? launch_one<64, false, true>(q, k, v, o, p, grid, stream)
+                     : launch_one<64, true, true>(q, k, v, o, p, grid, stream);
 }
 
 }  // namespace gl

@@ -33,6 +33,9 @@ SUFFIX = {
     "17x33-f32-odd": (2, 1, 65, 3, 17, 33, torch.float32),
     "128x64-bf16": (1, 1, 200, 2, 128, 64, torch.bfloat16),
     "8x8-f32-one-token": (1, 1, 1, 1, 8, 8, torch.float32),
+    # tensor-core reverse kernel (bf16, 64-wide q and k)
+    "64x128-bf16-tc": (1, 1, 1024, 2, 64, 128, torch.bfloat16),
+    "64x64-bf16-tc-segmented-ragged-start": (1, 1, 3000, 2, 64, 64, torch.bfloat16),
 }
 
 
@@ -54,10 +57,23 @@ def test_suffix_scan_matches_oracle(case):
         assert np.abs(out[:, -1]).max() == 0.0  # nothing comes after the last token
 
 
+def test_suffix_scan_shared_q_and_k():
+    """q and k one tensor (the forward read's case): one tile per chunk."""
+    L, B, T, H = 1, 2, 700, 1
+    x = _rand((L, B, T, H, 64), 5, torch.bfloat16, 1 / 8)
+    v = _rand((L, B, T, H, 64), 6, torch.bfloat16)
+    xd = x.cuda()
+    r = gl.suffix_scan(xd, xd, v.cuda())
+    torch.cuda.synchronize()
+    ref = oracle.suffix_scan(_units(x), _units(x), _units(v))
+    assert rel_l2(_units(r.cpu()), ref) <= TOL["bf16"]
+
+
+@pytest.mark.parametrize("m", [48, 64], ids=["cuda-core", "tensor-core"])
 @pytest.mark.parametrize("dt", [torch.float32, torch.bfloat16], ids=["f32", "bf16"])
 @pytest.mark.parametrize("read", ["forward", "costate"])
-def test_eta_grad_matches_oracle(read, dt):
-    L, B, T, H, d, m = 1, 2, 333, 2, 64, 48
+def test_eta_grad_matches_oracle(read, dt, m):
+    L, B, T, H, d = 1, 2, 333, 2, 64
     x = _rand((L, B, T, H, d), 11, dt, 1 / np.sqrt(d))
     gh = _rand((L, B, T, H, m), 12, dt, 0.1)
     go = _rand((L, B, T, H, m), 13, dt, 0.1)
@@ -73,3 +89,21 @@ def test_eta_grad_matches_oracle(read, dt):
     out = deta.permute(0, 1, 3, 2).reshape(L * B * H, T).double().cpu().numpy()
     tol = TOL["bf16"] if dt == torch.bfloat16 else TOL["f32"]
     assert rel_l2(out, ref) <= tol, f"rel-L2 {rel_l2(out, ref):.3e}"
+
+
+def test_eta_grad_long_context_sampled_units():
+    """The long-context workload at full size (B2 H16 T32768, 64 x 64): the
+    segmented tensor-core reverse kernel; four units checked against the oracle."""
+    import workloads as W
+    wl = W.workload("c4")
+    inp = W.make_linear(wl, device="cuda")
+    u = _rand((wl.L, wl.B, wl.T, wl.H, wl.d_out), 21, torch.bfloat16).cuda()
+    deta = gl.eta_grad(inp["x"], inp["g_hat"], u)
+    torch.cuda.synchronize()
+    for (b, h) in [(0, 0), (0, 15), (1, 7), (1, 12)]:
+        x = inp["x"][0, b, :, h].double().cpu().numpy()[None]
+        gh = inp["g_hat"][0, b, :, h].double().cpu().numpy()[None]
+        uu = u[0, b, :, h].double().cpu().numpy()[None]
+        ref = -np.sum(gh * oracle.suffix_scan(x, x, uu), axis=2)[0]
+        out = deta[0, b, :, h].double().cpu().numpy()
+        assert rel_l2(out, ref) <= TOL["bf16"], f"unit ({b},{h}): rel-L2 {rel_l2(out, ref):.3e}"
