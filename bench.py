@@ -308,6 +308,104 @@ class LinearJob:
                 f"forward and costate reads in one sequential walk per unit, fp64")
 
 
+class GradsJob(LinearJob):
+    """Step-size gradients of both reads of one linear map per unit, writes
+    detached (Sec. 3, practical architecture and training): dL/deta_t of the
+    forward read for an upstream u = dL/dy, and of the costate read for
+    w = dL/dg_in.  Each is the anti-causal suffix read of the same writes,
+    reduced per token by a dot in the reverse kernel's epilogue."""
+
+    kind = "grads"
+
+    def __init__(self, gl, wl, device, rank):
+        super().__init__(gl, wl, device, rank)
+        gen = torch.Generator(device=device)
+        gen.manual_seed(wl.seed * 1000 + 29)
+        dt = self.inp["x"].dtype
+        self.inp["u"] = torch.randn(self.inp["g_hat"].shape, generator=gen, device=device).to(dt)
+        self.inp["w"] = torch.randn(self.inp["x"].shape, generator=gen, device=device).to(dt)
+        shape = (wl.L, wl.B, wl.T, wl.H)
+        self.outs = {"deta_f": torch.empty(shape, device=device),
+                     "deta_c": torch.empty(shape, device=device)}
+        from paper_2609_34174_gb300 import _binding as _B
+        code = 1 if wl.dtype == "bf16" else 0
+        d = _B._Desc(wl.L, wl.B, wl.T, wl.H, wl.d_in, wl.d_out, code, 0)
+        lib = _B.load_library()
+        nb = max(lib.gradlev_eta_grad_workspace_bytes(ctypes.byref(d), 0),
+                 lib.gradlev_eta_grad_workspace_bytes(ctypes.byref(d), 1))
+        self.ws = torch.empty(max(256, int(nb)), dtype=torch.uint8, device=device)
+        self.in_keys = ("x", "g_hat", "g_out", "u", "w")
+        self.out_keys = ("deta_f", "deta_c")
+        self.kernel = {"fwd": "tc_scan_kernel<64, false, REV> (suffix read, q = k = x, dot with ghat)",
+                       "costate": "tc_scan_kernel<64, true, REV> (suffix read, q = ghat, k = g_out, dot with x)"}
+
+    def input_bytes(self):
+        return _bytes(*(self.inp[k] for k in self.in_keys))
+
+    def _run(self, src, cut, ws):
+        gl = self.gl
+        gl.eta_grad(cut(src["x"]), cut(src["g_hat"]), cut(src["u"]), deta=cut(self.outs["deta_f"]),
+                    workspace=ws)
+        yield
+        gl.eta_grad(cut(src["x"]), cut(src["g_hat"]), cut(src["w"]), read="costate",
+                    g_out=cut(src["g_out"]), deta=cut(self.outs["deta_c"]), workspace=ws)
+        yield
+
+    def step(self, inp=None, events=None):
+        inp = inp or self.inp
+        if events is not None:
+            events[0].record()
+        for i, _ in enumerate(self._run(inp, lambda t: t, self.ws)):
+            if events is not None:
+                events[i + 1].record()
+
+    def e2e_inputs(self, host, dev, sl, first):
+        return [(k, self._cut(host[k], sl), self._cut(dev[k], sl)) for k in self.in_keys]
+
+    def e2e_step(self, dev, sl, ws):
+        for _ in self._run(dev, lambda t: self._cut(t, sl), ws):
+            pass
+
+    def e2e_workspace_bytes(self):
+        return self.ws.numel()
+
+    def counts(self, scan):
+        """Per token and unit: the suffix read's flops 4*d*m + C*(d+m) (C = 64) plus
+        the dot; compulsory bytes e*(2d + m) + 4 for the forward read's gradient
+        (x, u, ghat in; deta out) and e*(2m + 2d) + 4 for the costate read's
+        (ghat, g_out, w, x in; deta out)."""
+        wl = self.wl
+        e = 2 if wl.dtype == "bf16" else 4
+        d, m = wl.d_in, wl.d_out
+        tu = wl.L * wl.B * wl.T * wl.H
+        if scan == "fwd":
+            return tu * (4 * d * m + COUNT_CHUNK * (d + m) + 2 * m), tu * (e * (d + 2 * m) + 4)
+        return tu * (4 * d * m + COUNT_CHUNK * (d + m) + 2 * d), tu * (e * (2 * d + 2 * m) + 4)
+
+    def config(self):
+        c = super().config()
+        c["computes"] = "dL/deta_t of the forward and costate reads (suffix read + dot)"
+        return c
+
+    def oracle_run(self, inp, n_units, cores, t_tokens=None):
+        """The fp64 oracle's suffix reads and dots for the first n_units units."""
+        import numpy as np
+        import oracle
+        wl = self.wl
+        units = [(l, b, h) for l in range(wl.L) for b in range(wl.B) for h in range(wl.H)]
+        units = units[:n_units]
+        f = lambda k: W.units_fp64(inp[k], units)
+        x, g, go, u, w = f("x"), f("g_hat"), f("g_out"), f("u"), f("w")
+        t = time.perf_counter()
+        np.sum(g * oracle.suffix_scan(x, x, u, nthreads=cores), axis=2)
+        np.sum(x * oracle.suffix_scan(g, go, w, nthreads=cores), axis=2)
+        return time.perf_counter() - t, len(units) * wl.T / wl.H
+
+    def sample_text(self, n):
+        return (f"{n} of {self.n_units()} (layer, batch, head) units at full T={self.wl.T}, "
+                f"suffix reads and dots of both reads, fp64")
+
+
 class MLPJob:
     """The two-layer fast-weight MLP of Appendix A: forward through both layers
     (sigma fused in the layer-1 epilogue), then costates back through both
@@ -427,7 +525,11 @@ class MLPJob:
                 f"tokens, both layers forward and costate in one sequential walk, fp64")
 
 
-def make_job(gl, wl, device, rank, gates=None):
+def make_job(gl, wl, device, rank, gates=None, grads=False):
+    if grads:
+        if isinstance(wl, W.MLPWorkload) or gates:
+            raise SystemExit("--grads applies to the ungated linear workloads")
+        return GradsJob(gl, wl, device, rank)
     if isinstance(wl, W.MLPWorkload):
         if gates:
             raise SystemExit("--gates applies to the linear workloads")
@@ -637,6 +739,8 @@ def run_reference(args, wl, rank, world):
                     "d2h_bytes_per_step": 0}}
 
 
+GRADS_METRIC = ("tokens/s of dL/deta_t per read (forward read, costate read) at 1 GB300; "
+                "% of roofline")
 DECODE_METRIC = "deployment tokens/s (one token per sequence per step) at 1 GB300; % of HBM roofline"
 
 
@@ -863,7 +967,7 @@ def run_gradlev(args, wl, rank, world, local_rank):
     device = torch.device("cuda", local_rank)
     torch.cuda.set_device(device)
     gl.load_library()
-    job = make_job(gl, wl, device, rank, args.gates)
+    job = make_job(gl, wl, device, rank, args.gates, args.grads)
     flush = None
     if job.input_bytes() < 2 * L2_BYTES:
         flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
@@ -918,11 +1022,13 @@ def run_gradlev(args, wl, rank, world, local_rank):
     dominant = "costate" if cos_ms >= fwd_ms else "fwd"
     rl = dict(scans[dominant]["roofline"])
     rl["kernel"] = job.kernel[dominant]
-    rl["traffic"] = None if (args.resize or args.gates) else recorded_traffic(args.workload, dominant)
+    rl["traffic"] = (None if (args.resize or args.gates or args.grads)
+                     else recorded_traffic(args.workload, dominant))
     cfg = {"workload": f"{args.workload}: {wl.name}", **job.config(),
            "tokens_per_step": job.tokens, "parallelism": f"replicas x{world}",
            "l2": "inputs larger than L2" if flush is None else "L2 flushed between steps"}
-    line = {"metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+    line = {"metric": GRADS_METRIC if args.grads else METRIC, "value": round(value, 1),
+            "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms, 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
             "data": "synthetic", "config": cfg, "scans": scans, "roofline": rl,
@@ -950,6 +1056,8 @@ def main(argv=None):
                          "for small profiling captures; the headline uses the full workload")
     ap.add_argument("--gates", default=None, choices=["eta", "alpha"],
                     help="time the gated scans of Eq. 2: per-token eta_t, or eta_t with retention")
+    ap.add_argument("--grads", action="store_true",
+                    help="time the step-size gradients of both reads (suffix reads) instead")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args(argv)
