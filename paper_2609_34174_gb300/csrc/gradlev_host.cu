@@ -20,7 +20,7 @@ cudaError_t launch_tc_scan(const CUtensorMap& q, const CUtensorMap& k, const CUt
                            cudaStream_t stream);
 cudaError_t launch_simt_scan(const SimtScanParams& p, bool bf16, bool rev, cudaStream_t stream);
 cudaError_t launch_tc_suffix(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
-                             const CUtensorMap& o, const TcScanParams& p, bool shared_qk, int grid,
+                             const CUtensorMap& o, const TcScanParams& p, int grid,
                              cudaStream_t stream);
 cudaError_t launch_rowdot(const void* a, const TokStr& as, const void* r, const TokStr& rs,
                           float* out, int L, int B, int T, int H, int w, float scale, bool bf16,
@@ -593,13 +593,6 @@ size_t suffix_ws_bytes(const gradlev_desc& d, int sms) {
     return suffix_tc_shape(d) ? plan_tc(d, 64, d.d_out, sms).ws_bytes : 0;
 }
 
-bool same_tensor(const Tok& a, const Tok& b) {
-    if (a.data != b.data) return false;
-    for (int i = 0; i < 4; ++i)
-        if (a.s[i] != b.s[i]) return false;
-    return true;
-}
-
 // With dot_out, the tensor-core path reduces every result row to the per-token
 // dot_out[t] = dot_scale * (r_t . a_t) in its epilogue and stores no r (r may then be
 // null); *fused tells whether it did (else r holds the read and no dot was formed).
@@ -625,13 +618,14 @@ int run_suffix_impl(const gradlev_desc* desc, const gradlev_tensor* q, const gra
     const Tok* all[4] = {&tq, &tk, &tv, &tr};
     for (const Tok* t : all)
         if ((reinterpret_cast<uintptr_t>(t->data) % elem) != 0) return GRADLEV_ERR_UNSUPPORTED;
-    const bool dot_ok = dot_out && dot_a && tc_layout_ok(*dot_a, 2);
+    // the dotted rows arrive through the output tensor map: no r is stored then
+    const bool dot_ok = dot_out && dot_a && !tr.data && tc_layout_ok(*dot_a, 2);
     if (suffix_tc_shape(d) && tc_layout_ok(tq, 2) && tc_layout_ok(tk, 2) && tc_layout_ok(tv, 2) &&
         tc_layout_ok(tr, 2) && (dot_out == nullptr || dot_ok) && (tr.data || dot_ok)) {
         const Plan pl = plan_tc(d, 64, d.d_out, dev.sms);
         CUtensorMap mq, mk, mv, mo;
         if (!make_tmap(&mq, d, tq, 64) || !make_tmap(&mk, d, tk, 64) ||
-            !make_tmap(&mv, d, tv, d.d_out) || !make_tmap(&mo, d, tr.data ? tr : tv, d.d_out))
+            !make_tmap(&mv, d, tv, d.d_out) || !make_tmap(&mo, d, dot_ok ? *dot_a : tr, d.d_out))
             return GRADLEV_ERR_UNSUPPORTED;
         TcScanParams p;
         memset(&p, 0, sizeof(p));
@@ -674,7 +668,7 @@ int run_suffix_impl(const gradlev_desc* desc, const gradlev_tensor* q, const gra
         p.incl = reinterpret_cast<float*>(wsb + pl.off_incl);
         if (cudaMemsetAsync(ws, 0, pl.zero_bytes, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
         const int grid = pl.n_items < dev.sms ? pl.n_items : dev.sms;
-        if (gl::launch_tc_suffix(mq, mk, mv, mo, p, same_tensor(tq, tk), grid, stream) != cudaSuccess)
+        if (gl::launch_tc_suffix(mq, mk, mv, mo, p, grid, stream) != cudaSuccess)
             return GRADLEV_ERR_CUDA;
         return GRADLEV_OK;
     }

@@ -236,6 +236,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* p_ready = bars + 36;         // [2] P written over the score buffer (P warps)
     uint64_t* o_staged = bars + 44;        // [2] output tile staged by all 4 epilogue warps
     uint64_t* o_buf_free = bars + 46;      // [2] output staging tile read by its TMA store
+    uint64_t* a_full = bars + 32;          // [2] (REV, dot) tile of the dotted tensor landed
     uint64_t* z_pub = bars + 40;           // state warps: all rows written before a flag
     uint64_t* z_lb = bars + 41;            // state warps: look-back result broadcast
     uint64_t* z_ack = bars + 42;           // state warps: broadcast consumed
@@ -251,6 +252,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int lane = threadIdx.x & 31;
     constexpr int kZActiveWarps = DQ / 32;          // state warps holding rows
     constexpr int kPHelpers = 4 - kZActiveWarps;    // state-slot warps building P half 1
+    // REV (64-wide, separate q and k tiles) keeps the state rows in TMEM lanes 64..127,
+    // so that the spare state-slot warps reach lanes 0..63, the rows whose P needs both
+    // halves once the mask is reversed.
+    static_assert(!REV || (DQ == 64 && COSTATE), "the reverse read uses the 64-wide q|k|v layout");
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < NS; ++i) {
@@ -279,6 +284,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(z_ack, kZActiveWarps);
         mbar_init(drain, 1);
         mbar_init(drain2, 1);
+        if constexpr (REV) {
+            mbar_init(&a_full[0], 1);
+            mbar_init(&a_full[1], 1);
+        }
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -374,7 +383,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             // 16 KB apart; for DQ = 64 the second M block is the V tile, whose rows
             // land in TMEM lanes 64..127 that nobody reads.
             auto issue_dz = [&](uint32_t st, uint32_t dcol, bool first) {
-                const uint32_t a_lo = sdesc_lo(st + Lay::kKOff, kTile);
+                // REV: A starts one block early (the q tile), so K^T lands in lanes 64..127
+                const uint32_t a_lo = sdesc_lo(st + (REV ? Lay::kQOff : Lay::kKOff), kTile);
                 const uint32_t b_lo = sdesc_lo(st + Lay::kVOff, kTile);
 #pragma unroll
                 for (int kk = 0; kk < kChunk / 16; ++kk)
@@ -507,7 +517,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_commit(drain2);
             mbar_drain(drain2, 0);
         }
-    } else if (warp < kWarpO0 || (warp >= kWarpZ0 && (warp & 3) >= kZActiveWarps)) {
+    } else if (warp < kWarpO0 ||
+               (warp >= kWarpZ0 && (REV ? (warp & 3) < 2 : (warp & 3) >= kZActiveWarps))) {
         // ------------------------------------------------------ score -> P
         // Warps 2-5 build P; with 64-wide keys the two state-slot warps whose
         // lanes (64..127) hold no state rows build the second half of P for them.
@@ -549,7 +560,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // REV keeps tokens s > t: rows >= 64 have an all-zero first half, and
                     // rows < 64 (whose lanes no helper warp can reach) build both halves
                     const bool mine =
-                        REV ? (q4 < 2 ? !helper : (half == 0 ? !helper : (helper || kPHelpers == 0)))
+                        REV ? (q4 < 2 ? (half == 0 ? !helper : helper) : !helper)
                             : (half == 0 ? !helper : (q4 < 2 ? !helper : (helper || kPHelpers == 0)));
                     if (!mine) continue;
                     if ((REV ? (half == 0 && q4 >= 2) : (half == 1 && q4 < 2)) || p.mu == 0.0f) {
@@ -590,6 +601,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool storer = (warp == kWarpO0) && (lane == 0);  // issues the TMA stores
         const EpiParams& e = p.epi;
         uint32_t c2 = 0;
+        // (REV, dot) the storer loads each chunk's tile of the dotted tensor by TMA into
+        // the staging tile of that chunk (no rows are stored), two chunks ahead
+        const bool dot = REV && e.dot_out != nullptr;
+        uint32_t a_n[2] = {0u, 0u};
         for (int it = 0;; ++it) {
             const int slot = it % kRing;
             if (!warp_wait(&item_full[slot], (it / kRing) & 1, abort_flag)) {
@@ -602,6 +617,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (item < 0) break;
             const Item I = decode_item<REV>(item, p);
             bool ok = true;
+            auto load_a = [&](uint32_t b, int cc) {
+                mbar_arrive_expect_tx(&a_full[b], kTile);
+                tma_load_5d(smem + Lay::kOOff + b * kTile, &tm_o, &a_full[b], I.j * 64, I.h,
+                            chunk_t0<REV>(I, cc), I.b, I.l);
+                ++a_n[b];
+            };
+            if (dot && storer) {
+                // both staging tiles are free: every earlier chunk's dot has been formed
+                load_a(c2 & 1, 0);
+                if (I.nch > 1) load_a((c2 + 1) & 1, 1);
+            }
             for (int c = 0; c < I.nch; ++c, ++c2) {
                 const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
                 if (!warp_wait(&o_full[ob], oph, abort_flag)) {
@@ -651,37 +677,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if constexpr (REV) {
                     if (e.dot_out) {
                         // dot_out[t] (+)= dot_scale * (row . a row) over this 64-wide tile.
-                        // The warp's 32 rows of a arrive coalesced (cp.async, one chunk
-                        // ahead) in its 4 KB slice of the staging tiles, which are free
-                        // because no rows are stored; the 128B swizzle lets each lane read
-                        // its own row without bank conflicts.
-                        const __nv_bfloat16* ab = static_cast<const __nv_bfloat16*>(e.dot_a);
-                        auto fetch = [&](uint32_t dst, int tc0) {
-#pragma unroll
-                            for (int it = 0; it < 8; ++it) {
-                                const int pc = it * 32 + lane, pr = pc >> 3, pq = pc & 7;
-                                const int tr = tc0 + q4 * 32 + pr;
-                                const bool ok = tr >= I.t_begin && tr < I.t_end;
-                                cp_async16(dst + sw128_off(pr, pq),
-                                           ok ? ab + tok_off(e.dot_a_str, I.l, I.b, tr, I.h) + col0 + pq * 8 : ab,
-                                           ok);
-                            }
-                            cp_async_commit();
-                        };
-                        const uint32_t slice = otile + (uint32_t)q4 * 4096u;
-                        if (c == 0) fetch(slice, t0);
-                        if (c + 1 < I.nch) {
-                            fetch(sbase + Lay::kOOff + (ob ^ 1) * kTile + (uint32_t)q4 * 4096u,
-                                  chunk_t0<REV>(I, c + 1));
-                            cp_async_wait<1>();
-                        } else {
-                            cp_async_wait<0>();
+                        // The tile of a (TMA, 128B-swizzled like an output tile) lets each
+                        // lane read its own row without bank conflicts.
+                        if (!warp_wait(&a_full[ob], oph, abort_flag)) {
+                            raise_error(p, kErrWaitTimeout, abort_flag);
+                            ok = false;
+                            break;
                         }
-                        __syncwarp();
                         float acc = 0.f;
 #pragma unroll
                         for (int q = 0; q < 8; ++q) {
-                            const uint4 a4 = ld_shared_v4(slice + sw128_off(lane, q));
+                            const uint4 a4 = ld_shared_v4(otile + sw128_off(row, q));
                             const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&a4);
 #pragma unroll
                             for (int i = 0; i < 8; ++i) acc = fmaf(v[8 * q + i], __bfloat162float(hb[i]), acc);
@@ -697,7 +703,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
                 if (direct) {
-                    if (valid && e.out) epi_store_row(e, tok_off(e.out_str, I.l, I.b, t, I.h) + col0, v);
+                    if (valid && e.out) {
+                        float tmp[64];  // a copy, so that v itself stays in registers
+#pragma unroll
+                        for (int i = 0; i < 64; ++i) tmp[i] = v[i];
+                        epi_store_row(e, tok_off(e.out_str, I.l, I.b, t, I.h) + col0, tmp);
+                    }
                 } else {
 #pragma unroll
                 for (int q = 0; q < 8; ++q)
@@ -720,6 +731,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         // the previous chunk's store (other tile) has finished reading
                         bulk_wait_group_read<1>();
                         if (c2 > 0) mbar_arrive(&o_buf_free[ob ^ 1]);
+                        // this chunk's dots are formed: its tile takes chunk c + 2
+                        if (dot && c + 2 < I.nch) load_a(ob, c + 2);
                     }
                 }
                 if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
@@ -730,13 +743,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) break;
         }
         if (storer) bulk_wait_group_all();
+        if (dot && storer) {  // every load issued has landed before the CTA exits
+            for (int b = 0; b < 2; ++b)
+                if (a_n[b] > 0) mbar_drain(&a_full[b], (a_n[b] - 1) & 1);
+        }
     } else {
         const int q4 = warp & 3;
         {
         // ------------------------------------------------------------ state
-        const int row = q4 * 32 + lane;         // contraction index q of this thread's state row
-        const bool active = row < DQ;           // warp-uniform
-        const bool leader = (q4 == 0) && (lane == 0);
+        const int row = q4 * 32 + lane;         // TMEM lane of this thread's state row
+        const int srow = REV ? row - 64 : row;  // contraction index q of that row
+        const bool active = REV ? row >= 64 : row < DQ;  // warp-uniform
+        constexpr int kLeadQ4 = REV ? 2 : 0;    // lane quarter of the lead state warp
+        const bool leader = (q4 == kLeadQ4) && (lane == 0);
         const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
         // The state is kept in units of lam = -eta (1 when eta = 0): the rows hold
         // S' = S / lam, so the S^T tile carries the -eta of P and the update is
@@ -787,7 +806,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     tc_fence_after();
                     if (active) {
-                        float* dst = (I.k == 0 ? p.incl : p.agg) + (size_t)item * blk + (size_t)row * 64;
+                        float* dst = (I.k == 0 ? p.incl : p.agg) + (size_t)item * blk + (size_t)srow * 64;
                         float a[32];
     #pragma unroll
                         for (int h = 0; h < 2; ++h) {
@@ -819,7 +838,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int i = 0; i < 64; ++i) st[i] = 0.0f;
                 if (active && I.k > 0) {
-                    if (q4 == 0) {
+                    if (q4 == kLeadQ4) {
                         // predecessor segment sk of this (unit, tile) is item sk * n_ut + r_ut
                         int total = 0, base_pred = I.k - 1, remaining = I.k;
                         bool found = false, timed_out = false;
@@ -879,7 +898,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int i = 0; i < cnt; ++i) {
                             const int pred = (I.k - 1 - i) * n_ut + r_ut;
                             const float* src = ((i == cnt - 1 && ends_incl) ? p.incl : p.agg) +
-                                               (size_t)pred * blk + (size_t)row * 64;
+                                               (size_t)pred * blk + (size_t)srow * 64;
     #pragma unroll
                             for (int e4 = 0; e4 < 64; e4 += 4) {
                                 float4 a = __ldcg(reinterpret_cast<const float4*>(src + e4));
@@ -893,8 +912,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 // ---- publish the inclusive prefix E + aggregate (flag 2)
                 if (active && I.phase1 && I.k > 0) {
-                    const float* own = p.agg + (size_t)item * blk + (size_t)row * 64;
-                    float* dst = p.incl + (size_t)item * blk + (size_t)row * 64;
+                    const float* own = p.agg + (size_t)item * blk + (size_t)srow * 64;
+                    float* dst = p.incl + (size_t)item * blk + (size_t)srow * 64;
     #pragma unroll
                     for (int i = 0; i < 64; i += 4) {
                         float4 a = __ldcg(reinterpret_cast<const float4*>(own + i));
@@ -938,7 +957,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t tile = sbase + Lay::kStOff + sb * Lay::kStBytes;
     #pragma unroll
                         for (int q = 0; q < 8; ++q)
-                            st_shared_v4(tile + sw128_off(row, q), pack_bf16x2(st[8 * q], st[8 * q + 1]),
+                            st_shared_v4(tile + sw128_off(srow, q), pack_bf16x2(st[8 * q], st[8 * q + 1]),
                                          pack_bf16x2(st[8 * q + 2], st[8 * q + 3]),
                                          pack_bf16x2(st[8 * q + 4], st[8 * q + 5]),
                                          pack_bf16x2(st[8 * q + 6], st[8 * q + 7]));
@@ -1012,13 +1031,13 @@ cudaError_t launch_tc_scan(const CUtensorMap& q, const CUtensorMap& k, const CUt
 }
 
 // The anti-causal suffix read r_t = sum_{s>t} (k_s . q_t) v_s (no base matrix) on the
-// 64-wide kernels: shared_qk when q and k are one tensor (one tile per chunk).
+// 64-wide kernel with separate q, k and v tiles (q and k may be one tensor: its
+// second load of a chunk then comes from L2).
 cudaError_t launch_tc_suffix(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
-                             const CUtensorMap& o, const TcScanParams& p, bool shared_qk, int grid,
+                             const CUtensorMap& o, const TcScanParams& p, int grid,
                              cudaStream_t stream) {
     if (p.dq != 64) return cudaErrorInvalidValue;
-    return shared_qk ? launch_one<64, false, true>(q, k, v, o, p, grid, stream)
-                     : launch_one<64, true, true>(q, k, v, o, p, grid, stream);
+    return launch_one<64, true, true>(q, k, v, o, p, grid, stream);
 }
 
 }  // namespace gl
