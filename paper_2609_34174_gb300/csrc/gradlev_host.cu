@@ -20,7 +20,7 @@ cudaError_t launch_tc_scan(const CUtensorMap& q, const CUtensorMap& k, const CUt
                            cudaStream_t stream);
 cudaError_t launch_simt_scan(const SimtScanParams& p, bool bf16, bool rev, cudaStream_t stream);
 cudaError_t launch_tc_suffix(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
-                             const CUtensorMap& o, const TcScanParams& p, int grid,
+                             const CUtensorMap& o, const TcScanParams& p, bool shared_qk, int grid,
                              cudaStream_t stream);
 cudaError_t launch_rowdot(const void* a, const TokStr& as, const void* r, const TokStr& rs,
                           float* out, int L, int B, int T, int H, int w, float scale, bool bf16,
@@ -589,6 +589,13 @@ int dev_sms_or_default() {
     return device_info(&dev) ? dev.sms : 160;
 }
 
+bool same_tensor(const Tok& a, const Tok& b) {
+    if (a.data != b.data) return false;
+    for (int i = 0; i < 4; ++i)
+        if (a.s[i] != b.s[i]) return false;
+    return true;
+}
+
 size_t suffix_ws_bytes(const gradlev_desc& d, int sms) {
     return suffix_tc_shape(d) ? plan_tc(d, 64, d.d_out, sms).ws_bytes : 0;
 }
@@ -668,7 +675,7 @@ int run_suffix_impl(const gradlev_desc* desc, const gradlev_tensor* q, const gra
         p.incl = reinterpret_cast<float*>(wsb + pl.off_incl);
         if (cudaMemsetAsync(ws, 0, pl.zero_bytes, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
         const int grid = pl.n_items < dev.sms ? pl.n_items : dev.sms;
-        if (gl::launch_tc_suffix(mq, mk, mv, mo, p, grid, stream) != cudaSuccess)
+        if (gl::launch_tc_suffix(mq, mk, mv, mo, p, same_tensor(tq, tk), grid, stream) != cudaSuccess)
             return GRADLEV_ERR_CUDA;
         return GRADLEV_OK;
     }

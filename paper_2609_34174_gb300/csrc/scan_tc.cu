@@ -67,13 +67,17 @@ __host__ __device__ constexpr uint32_t col_sc(uint32_t i) { return i * 128u; }
 __host__ __device__ constexpr uint32_t col_o(uint32_t i) { return 256u + i * 64u; }
 __host__ __device__ constexpr uint32_t col_dz(uint32_t i) { return 384u + i * 64u; }
 
-template <int DQ, bool COSTATE>
+// Stage layout [q | k | v] (costate), [qk | v] (forward).  The reverse read with one
+// q/k tile puts v first, [v | qk]: the dZ product's A operand then starts one block
+// before k in both reverse layouts, which places K^T in TMEM lanes 64..127.
+template <int DQ, bool COSTATE, bool REV = false>
 struct TcLayout {
     static constexpr int kQkBlocks = DQ / 64;
-    static constexpr int kQOff = 0;
-    static constexpr int kKOff = COSTATE ? kQkBlocks * kTile : 0;
-    static constexpr int kVOff = kKOff + kQkBlocks * kTile;
-    static constexpr int kStageBytes = kVOff + kTile;
+    static constexpr bool kVFirst = REV && !COSTATE;
+    static constexpr int kQOff = kVFirst ? kTile : 0;
+    static constexpr int kKOff = COSTATE ? kQkBlocks * kTile : kQOff;
+    static constexpr int kVOff = kVFirst ? 0 : kKOff + kQkBlocks * kTile;
+    static constexpr int kStageBytes = ((COSTATE ? 2 : 1) * kQkBlocks + 1) * kTile;
     // Stage ring: what is left of the 227 KB opt-in budget after the two S^T
     // tiles, the two output staging tiles, the barrier block and the alignment
     // slack (at most 6 stages).
@@ -213,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_scan_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
                    const TcScanParams p) {
-    using Lay = TcLayout<DQ, COSTATE>;
+    using Lay = TcLayout<DQ, COSTATE, REV>;
     constexpr int NS = Lay::kStages;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -255,7 +259,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // REV (64-wide, separate q and k tiles) keeps the state rows in TMEM lanes 64..127,
     // so that the spare state-slot warps reach lanes 0..63, the rows whose P needs both
     // halves once the mask is reversed.
-    static_assert(!REV || (DQ == 64 && COSTATE), "the reverse read uses the 64-wide q|k|v layout");
+    static_assert(!REV || DQ == 64, "the reverse read is built for 64-wide q and k");
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < NS; ++i) {
@@ -383,8 +387,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             // 16 KB apart; for DQ = 64 the second M block is the V tile, whose rows
             // land in TMEM lanes 64..127 that nobody reads.
             auto issue_dz = [&](uint32_t st, uint32_t dcol, bool first) {
-                // REV: A starts one block early (the q tile), so K^T lands in lanes 64..127
-                const uint32_t a_lo = sdesc_lo(st + (REV ? Lay::kQOff : Lay::kKOff), kTile);
+                // REV: A starts one block before k, so K^T lands in lanes 64..127
+                const uint32_t a_lo = sdesc_lo(st + (REV ? Lay::kKOff - kTile : Lay::kKOff), kTile);
                 const uint32_t b_lo = sdesc_lo(st + Lay::kVOff, kTile);
 #pragma unroll
                 for (int kk = 0; kk < kChunk / 16; ++kk)
@@ -1009,7 +1013,7 @@ template <int DQ, bool COSTATE, bool REV>
 static cudaError_t launch_one(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
                               const CUtensorMap& o, const TcScanParams& p, int grid,
                               cudaStream_t stream) {
-    using Lay = TcLayout<DQ, COSTATE>;
+    using Lay = TcLayout<DQ, COSTATE, REV>;
     auto kern = tc_scan_kernel<DQ, COSTATE, REV>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          Lay::kSmemBytes);
@@ -1031,13 +1035,13 @@ cudaError_t launch_tc_scan(const CUtensorMap& q, const CUtensorMap& k, const CUt
 }
 
 // The anti-causal suffix read r_t = sum_{s>t} (k_s . q_t) v_s (no base matrix) on the
-// 64-wide kernel with separate q, k and v tiles (q and k may be one tensor: its
-// second load of a chunk then comes from L2).
+// 64-wide kernel: shared_qk when q and k are one tensor (one tile per chunk).
 cudaError_t launch_tc_suffix(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
-                             const CUtensorMap& o, const TcScanParams& p, int grid,
+                             const CUtensorMap& o, const TcScanParams& p, bool shared_qk, int grid,
                              cudaStream_t stream) {
     if (p.dq != 64) return cudaErrorInvalidValue;
-    return launch_one<64, true, true>(q, k, v, o, p, grid, stream);
+    return shared_qk ? launch_one<64, false, true>(q, k, v, o, p, grid, stream)
+                     : launch_one<64, true, true>(q, k, v, o, p, grid, stream);
 }
 
 }  // namespace gl
