@@ -703,6 +703,20 @@ def run_reference(args, wl, rank, world):
 
         sample = f"{wl.B} sequences x {t_tok} tokens of the deployed MLP per step, fp64"
         metric = DECODE_METRIC
+    elif args.grads:
+        job = GradsJob.__new__(GradsJob)
+        job.wl = wl
+        inp = W.make_linear(wl, device="cpu")
+        gen = torch.Generator()
+        gen.manual_seed(wl.seed * 1000 + 29)
+        dt = inp["x"].dtype
+        inp["u"] = torch.randn(inp["g_hat"].shape, generator=gen).to(dt)
+        inp["w"] = torch.randn(inp["x"].shape, generator=gen).to(dt)
+        n = min(job.n_units(), max(cores, 2 * cores))
+        run = lambda: job.oracle_run(inp, n, cores)
+        sample = (f"{n} of {job.n_units()} (layer, batch, head) units at full T={wl.T} per step, "
+                  f"suffix reads and dots of both reads, fp64")
+        metric = GRADS_METRIC
     elif isinstance(wl, W.MLPWorkload):
         inp = W.make_mlp(wl, device="cpu")
         job = MLPJob.__new__(MLPJob)

@@ -107,3 +107,23 @@ def test_eta_grad_long_context_sampled_units():
         ref = -np.sum(gh * oracle.suffix_scan(x, x, uu), axis=2)[0]
         out = deta[0, b, :, h].double().cpu().numpy()
         assert rel_l2(out, ref) <= TOL["bf16"], f"unit ({b},{h}): rel-L2 {rel_l2(out, ref):.3e}"
+
+
+def test_suffix_scan_and_eta_grad_strided_views():
+    """Token tensors that are feature slices of wider buffers (non-default token
+    strides) on the tensor-core reverse kernel."""
+    L, B, T, H = 1, 2, 640, 2
+    big = _rand((L, B, T, H, 192), 31, torch.bfloat16, 1 / 8).cuda()
+    q, k, v = big[..., :64], big[..., 64:128], big[..., 128:]
+    r = gl.suffix_scan(q, k, v)
+    torch.cuda.synchronize()
+    ref = oracle.suffix_scan(_units(q.cpu()), _units(k.cpu()), _units(v.cpu()))
+    assert rel_l2(_units(r.cpu()), ref) <= TOL["bf16"]
+    # eta gradient of the forward read with x, ghat and u all strided views
+    x, gh, u = big[..., :64], big[..., 64:128] * 1, big[..., 128:]
+    deta = gl.eta_grad(x, big[..., 64:128], u)
+    torch.cuda.synchronize()
+    xu, gu, uu = _units(x.cpu()), _units(gh.cpu()), _units(u.cpu())
+    want = -np.sum(gu * oracle.suffix_scan(xu, xu, uu), axis=2)
+    got = deta.permute(0, 1, 3, 2).reshape(L * B * H, T).double().cpu().numpy()
+    assert rel_l2(got, want) <= TOL["bf16"]
