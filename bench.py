@@ -45,6 +45,12 @@ COUNT_CHUNK = 64  # chunk size fixed for counting flops (scan roofline conventio
 L2_BYTES = 129 * 1024 * 1024
 
 
+def nvtx(name):
+    """An NVTX range around one library call of the timed step (for ncu --nvtx and
+    timeline tools); host-side markers only."""
+    return torch.cuda.nvtx.range(name)
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -196,12 +202,14 @@ class LinearJob:
             events[0].record()
         eta = inp["eta_t"] if self.gates else wl.eta
         alpha = inp.get("alpha_t")
-        gl.forward_scan(inp["x"], inp["g_hat"], inp["W0"], eta, y=o["y"], workspace=self.ws,
-                        alpha=alpha)
+        with nvtx("gradlev forward scan"):
+            gl.forward_scan(inp["x"], inp["g_hat"], inp["W0"], eta, y=o["y"], workspace=self.ws,
+                            alpha=alpha)
         if events is not None:
             events[1].record()
-        gl.costate_scan(inp["x"], inp["g_hat"], inp["W0"], eta, inp["g_out"], g_in=o["g_in"],
-                        workspace=self.ws, alpha=alpha)
+        with nvtx("gradlev costate scan"):
+            gl.costate_scan(inp["x"], inp["g_hat"], inp["W0"], eta, inp["g_out"], g_in=o["g_in"],
+                            workspace=self.ws, alpha=alpha)
         if events is not None:
             events[2].record()
 
@@ -344,11 +352,13 @@ class GradsJob(LinearJob):
 
     def _run(self, src, cut, ws):
         gl = self.gl
-        gl.eta_grad(cut(src["x"]), cut(src["g_hat"]), cut(src["u"]), deta=cut(self.outs["deta_f"]),
-                    workspace=ws)
+        with nvtx("gradlev eta_grad forward read"):
+            gl.eta_grad(cut(src["x"]), cut(src["g_hat"]), cut(src["u"]),
+                        deta=cut(self.outs["deta_f"]), workspace=ws)
         yield
-        gl.eta_grad(cut(src["x"]), cut(src["g_hat"]), cut(src["w"]), read="costate",
-                    g_out=cut(src["g_out"]), deta=cut(self.outs["deta_c"]), workspace=ws)
+        with nvtx("gradlev eta_grad costate read"):
+            gl.eta_grad(cut(src["x"]), cut(src["g_hat"]), cut(src["w"]), read="costate",
+                        g_out=cut(src["g_out"]), deta=cut(self.outs["deta_c"]), workspace=ws)
         yield
 
     def step(self, inp=None, events=None):
@@ -439,15 +449,18 @@ class MLPJob:
         inp = inp or self.inp
         if events is not None:
             events[0].record()
-        gl.forward_scan(inp["x"], inp["g_hat_z"], inp["W1"], wl.eta1, act=wl.act, y=o["z"],
-                        act_out=o["h"], workspace=self.ws)
-        gl.forward_scan(o["h"], inp["g_hat_y"], inp["W2"], wl.eta2, y=o["y"], workspace=self.ws)
+        with nvtx("gradlev MLP forward"):
+            gl.forward_scan(inp["x"], inp["g_hat_z"], inp["W1"], wl.eta1, act=wl.act, y=o["z"],
+                            act_out=o["h"], workspace=self.ws)
+            gl.forward_scan(o["h"], inp["g_hat_y"], inp["W2"], wl.eta2, y=o["y"],
+                            workspace=self.ws)
         if events is not None:
             events[1].record()
-        gl.costate_scan(o["h"], inp["g_hat_y"], inp["W2"], wl.eta2, inp["g_out"], act=wl.act,
-                        z=o["z"], g_in=o["gz"], workspace=self.ws)
-        gl.costate_scan(inp["x"], inp["g_hat_z"], inp["W1"], wl.eta1, o["gz"], g_in=o["gx"],
-                        workspace=self.ws)
+        with nvtx("gradlev MLP costate"):
+            gl.costate_scan(o["h"], inp["g_hat_y"], inp["W2"], wl.eta2, inp["g_out"], act=wl.act,
+                            z=o["z"], g_in=o["gz"], workspace=self.ws)
+            gl.costate_scan(inp["x"], inp["g_hat_z"], inp["W1"], wl.eta1, o["gz"], g_in=o["gx"],
+                            workspace=self.ws)
         if events is not None:
             events[2].record()
 
