@@ -43,6 +43,52 @@ __device__ __forceinline__ void st(void* p, long long i, float v) {
         static_cast<float*>(p)[i] = v;
 }
 
+constexpr int kFlatThreads = 256;
+
+// The same scaling for a contiguous input: piece v (16 bytes) belongs to token
+// v / vpr at the same offset in and out.  Each thread keeps four pieces in flight.
+template <bool BF16>
+__global__ void __launch_bounds__(kFlatThreads)
+    prescale_flat_kernel(const void* __restrict__ g, const float* __restrict__ eta,
+                         void* __restrict__ out, int n, int vpr) {
+    const uint4* in = static_cast<const uint4*>(g);
+    uint4* o = static_cast<uint4*>(out);
+    const int stride = gridDim.x * kFlatThreads;
+    for (int v0 = blockIdx.x * kFlatThreads + threadIdx.x; v0 < n; v0 += 4 * stride) {
+        uint4 x[4];
+        float e[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int v = v0 + k * stride;
+            if (v < n) {
+                x[k] = __ldcs(in + v);
+                e[k] = __ldg(eta + v / vpr);
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int v = v0 + k * stride;
+            if (v >= n) continue;
+            uint4 y;
+            if constexpr (BF16) {
+                const __nv_bfloat162* pi = reinterpret_cast<const __nv_bfloat162*>(&x[k]);
+                __nv_bfloat162* po = reinterpret_cast<__nv_bfloat162*>(&y);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const float2 f = __bfloat1622float2(pi[i]);
+                    po[i] = __floats2bfloat162_rn(e[k] * f.x, e[k] * f.y);
+                }
+            } else {
+                y = make_uint4(__float_as_uint(e[k] * __uint_as_float(x[k].x)),
+                               __float_as_uint(e[k] * __uint_as_float(x[k].y)),
+                               __float_as_uint(e[k] * __uint_as_float(x[k].z)),
+                               __float_as_uint(e[k] * __uint_as_float(x[k].w)));
+            }
+            o[v] = y;
+        }
+    }
+}
+
 // ghat'[l,b,t,h,:] = eta_t[l,b,t,h] * ghat[l,b,t,h,:], written contiguous.  One
 // thread per 16-byte piece of a token row (w a multiple of 16 bytes / element).
 template <bool BF16>
@@ -248,6 +294,20 @@ cudaError_t launch_gated_prescale(const void* g, const TokStr& gs, const float* 
                                   int B, int T, int H, int w, bool bf16, cudaStream_t stream) {
     const long long n = (long long)L * B * T * H * (w / (bf16 ? 8 : 4));
     if (n <= 0) return cudaSuccess;
+    // contiguous rows (the output's own layout) and 32-bit piece indices: the flat
+    // kernel, four independent 16-byte pieces per thread and pass
+    const bool contig = gs.s[3] == w && gs.s[2] == (long long)H * w &&
+                        gs.s[1] == (long long)T * H * w && gs.s[0] == (long long)B * T * H * w;
+    if (contig && n < (1ll << 31) - 4 * (long long)gated::kFlatThreads * 152 * 8) {
+        const int grid = 152 * 8;
+        if (bf16)
+            gated::prescale_flat_kernel<true><<<grid, gated::kFlatThreads, 0, stream>>>(
+                g, eta, out, (int)n, w / 8);
+        else
+            gated::prescale_flat_kernel<false><<<grid, gated::kFlatThreads, 0, stream>>>(
+                g, eta, out, (int)n, w / 4);
+        return cudaGetLastError();
+    }
     long long blocks = (n + 255) / 256;
     if (blocks > 152 * 16) blocks = 152 * 16;
     if (bf16)
