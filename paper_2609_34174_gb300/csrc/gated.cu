@@ -261,6 +261,157 @@ __global__ void __launch_bounds__(kThreads)
     }
 }
 
+// The same recurrence for bf16 reads of at most kRegJ inputs, with the state in
+// registers: thread 4i+p owns the entries (i, j) of output i for the contiguous
+// inputs j in [16p, 16p + 16) and holds W0 and D for them in registers.  The
+// per-token vectors (q, b, the tile's a, eta_t, alpha_t) arrive by cp.async in
+// blocks of kBlk tokens, one block ahead, so the CTA synchronises once per block
+// instead of once per token, and no state ever goes through shared memory.
+constexpr int kRegJ = 64;
+constexpr int kBlk = 16;
+constexpr int kTokBytes = 3 * 128 + 16;  // q, b, a (64 bf16 each), eta and alpha (+ pad)
+
+__device__ __forceinline__ void cpa16(uint32_t dst, const void* src, bool valid) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+                 "r"(valid ? 16 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cpa4(uint32_t dst, const void* src, bool valid) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src),
+                 "r"(valid ? 4 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cpa_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cpa_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+template <bool COSTATE>
+__global__ void __launch_bounds__(kThreads)
+    serial_reg_kernel(GatedParams p) {
+    __shared__ __align__(16) unsigned char buf[2][kBlk * kTokBytes];
+    constexpr int JP = kRegJ / 4;            // entries per thread
+    const int J = COSTATE ? p.dout : p.din;  // a multiple of 16, at most kRegJ
+    const int NO = COSTATE ? p.din : p.dout;
+    const int tiles = (NO + kTile - 1) / kTile;
+    const int tile = blockIdx.x % tiles;
+    const int unit = blockIdx.x / tiles;
+    const int h = unit % p.H;
+    const int l = unit / (p.H * p.B);
+    const int b = (unit / p.H) % p.B;
+    const int o0 = tile * kTile;
+    const float* w0 = p.W0 + (size_t)(l * p.H + h) * p.din * p.dout;  // [dout][din]
+    const int tid = threadIdx.x;
+    const int i_own = tid >> 2, part = tid & 3;
+    const int o = o0 + i_own;
+    const int j0 = part * JP;
+    float w[JP], d[JP];
+#pragma unroll
+    for (int k = 0; k < JP; ++k) {
+        const int j = j0 + k;
+        w[k] = (o < NO && j < J) ? (COSTATE ? w0[(size_t)j * p.din + o] : w0[(size_t)o * p.din + j])
+                                 : 0.0f;
+        d[k] = 0.0f;
+    }
+    // token-0 positions of the vectors and their steps per token
+    const __nv_bfloat16* X = static_cast<const __nv_bfloat16*>(p.x) + tok_off(p.x_s, l, b, 0, h);
+    const __nv_bfloat16* G = static_cast<const __nv_bfloat16*>(p.g) + tok_off(p.g_s, l, b, 0, h);
+    const __nv_bfloat16* Qb = static_cast<const __nv_bfloat16*>(p.q) + tok_off(p.q_s, l, b, 0, h);
+    const __nv_bfloat16* Bb = COSTATE ? G : X;
+    const __nv_bfloat16* Ab = (COSTATE ? X : G) + o0;
+    const long long qst = p.q_s[2], bst = COSTATE ? p.g_s[2] : p.x_s[2],
+                    ast = COSTATE ? p.x_s[2] : p.g_s[2];
+    const long long gate0 = ((long long)l * p.B + b) * p.T * p.H + h;
+    // stage tokens [kBlk k, kBlk k + kBlk) into buffer k & 1: 24 pieces of 16 bytes per
+    // token (q, b, a: 8 each) plus the two gates; zeros past T, J or the tile
+    auto stage = [&](int k) {
+        const uint32_t base = (uint32_t)__cvta_generic_to_shared(buf[k & 1]);
+        for (int pc = tid; pc < kBlk * 24; pc += kThreads) {
+            const int u = pc / 24, kind = pc - u * 24, t = k * kBlk + u;
+            const int sub = kind & 7;
+            const uint32_t dst = base + u * kTokBytes + kind * 16;
+            // a zero-filled piece reads nothing; it is given a valid address all the same
+            if (kind < 8) {
+                const bool ok = t < p.T && sub * 8 < J;
+                cpa16(dst, ok ? Qb + (long long)t * qst + sub * 8 : Qb, ok);
+            } else if (kind < 16) {
+                const bool ok = t < p.T && sub * 8 < J;
+                cpa16(dst, ok ? Bb + (long long)t * bst + sub * 8 : Qb, ok);
+            } else {
+                const bool ok = t < p.T && o0 + sub * 8 < NO;
+                cpa16(dst, ok ? Ab + (long long)t * ast + sub * 8 : Qb, ok);
+            }
+        }
+        if (tid < 2 * kBlk) {
+            const int u = tid >> 1, t = k * kBlk + u;
+            const float* src = (tid & 1) ? p.alpha : p.eta;
+            const bool ok = t < p.T && src != nullptr;
+            cpa4(base + u * kTokBytes + 384 + (tid & 1) * 4, ok ? src + gate0 + (long long)t * p.H : p.eta,
+                 ok);
+        }
+        cpa_commit();
+    };
+    const int n_blk = (p.T + kBlk - 1) / kBlk;
+    if (n_blk > 0) stage(0);
+    for (int k = 0; k < n_blk; ++k) {
+        if (k + 1 < n_blk) {
+            stage(k + 1);
+            cpa_wait<1>();
+        } else {
+            cpa_wait<0>();
+        }
+        __syncthreads();  // block k staged by every thread
+        const unsigned char* bk = buf[k & 1];
+        const int nt = min(kBlk, p.T - k * kBlk);
+        for (int u = 0; u < nt; ++u) {
+            const int t = k * kBlk + u;
+            const unsigned char* tk = bk + u * kTokBytes;
+            const uint4 q0 = *reinterpret_cast<const uint4*>(tk + j0 * 2);
+            const uint4 q1 = *reinterpret_cast<const uint4*>(tk + j0 * 2 + 16);
+            const uint4 b0 = *reinterpret_cast<const uint4*>(tk + 128 + j0 * 2);
+            const uint4 b1 = *reinterpret_cast<const uint4*>(tk + 128 + j0 * 2 + 16);
+            const float a_i = __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(tk + 256)[i_own]);
+            const float eta = *reinterpret_cast<const float*>(tk + 384);
+            const float alpha = p.alpha ? *reinterpret_cast<const float*>(tk + 388) : 1.0f;
+            const float ea = eta * a_i;
+            const uint32_t qw[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
+            const uint32_t bw[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+            // read before write: out_i = sum_j (W0 + D)[i][j] q_j, then
+            // D[i][j] = alpha D[i][j] - eta a_i b_j on the same entries
+            float ac[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+            for (int k2 = 0; k2 < JP / 2; ++k2) {
+                const float2 qf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qw[k2]));
+                const float2 bf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&bw[k2]));
+                const int kk = 2 * k2;
+                ac[kk & 3] = fmaf(w[kk] + d[kk], qf.x, ac[kk & 3]);
+                ac[(kk + 1) & 3] = fmaf(w[kk + 1] + d[kk + 1], qf.y, ac[(kk + 1) & 3]);
+                d[kk] = fmaf(alpha, d[kk], -ea * bf.x);
+                d[kk + 1] = fmaf(alpha, d[kk + 1], -ea * bf.y);
+            }
+            float acc = (ac[0] + ac[1]) + (ac[2] + ac[3]);
+            acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+            acc += __shfl_xor_sync(0xffffffffu, acc, 2);
+            if (part == 0 && o < NO) {
+                const EpiParams& e = p.epi;
+                const long long oo = tok_off(e.out_str, l, b, t, h) + o;
+                float v = acc;
+                if (e.zin) v *= act_df(e.act, ld<true>(e.zin, tok_off(e.z_str, l, b, t, h) + o));
+                st<true>(e.out, oo, v);
+                if (e.out2) st<true>(e.out2, tok_off(e.out2_str, l, b, t, h) + o, act_f(e.act, acc));
+            }
+        }
+        __syncthreads();  // block k read: its buffer may take block k + 2
+    }
+}
+
+template <bool COSTATE>
+cudaError_t launch_serial_reg(const GatedParams& p, int blocks, cudaStream_t stream) {
+    serial_reg_kernel<COSTATE><<<blocks, kThreads, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
 template <bool COSTATE, bool BF16>
 cudaError_t launch_serial(const GatedParams& p, int blocks, size_t smem, cudaStream_t stream) {
     auto kern = serial_kernel<COSTATE, BF16>;
@@ -277,12 +428,30 @@ size_t gated_serial_smem(int din, int dout, bool costate) {
     return sizeof(float) * ((size_t)2 * gated::kTile * (J + 4) + 2 * (2 * (size_t)J + gated::kTile + 2));
 }
 
+// The register kernel reads 16-byte pieces of bf16 rows: widths a multiple of 16,
+// the read at most kRegJ wide, every token row 16-byte aligned.
+static bool serial_reg_ok(const GatedParams& p, bool costate, bool bf16) {
+    const int J = costate ? p.dout : p.din;
+    if (!bf16 || J > gated::kRegJ || J % 16 != 0) return false;
+    const void* ptrs[3] = {p.x, p.g, p.q};
+    const long long* strs[3] = {p.x_s, p.g_s, p.q_s};
+    for (int k = 0; k < 3; ++k) {
+        if ((reinterpret_cast<uintptr_t>(ptrs[k]) & 15u) != 0) return false;
+        for (int i = 0; i < 4; ++i)
+            if (strs[k][i] % 8 != 0) return false;
+    }
+    return true;
+}
+
 cudaError_t launch_gated_serial(const GatedParams& p, bool costate, bool bf16, cudaStream_t stream) {
     const int NO = costate ? p.din : p.dout;
     const int tiles = (NO + gated::kTile - 1) / gated::kTile;
     const long long blocks = (long long)p.L * p.B * p.H * tiles;
     const size_t smem = gated_serial_smem(p.din, p.dout, costate);
     if (blocks <= 0) return cudaSuccess;
+    if (serial_reg_ok(p, costate, bf16))  // the state fits in registers
+        return costate ? gated::launch_serial_reg<true>(p, (int)blocks, stream)
+                       : gated::launch_serial_reg<false>(p, (int)blocks, stream);
     if (costate)
         return bf16 ? gated::launch_serial<true, true>(p, (int)blocks, smem, stream)
                     : gated::launch_serial<true, false>(p, (int)blocks, smem, stream);
