@@ -262,6 +262,10 @@ size_t gradlev_suffix_workspace_bytes(const gradlev_desc* desc);
  *   workspace/workspace_bytes  at least gradlev_eta_grad_workspace_bytes(desc, read)
  *            bytes, 256-byte aligned (it holds the suffix read)
  * The same value for every eta_t: the reads are linear in the step sizes.
+ * With bf16 tensors and 64-wide q and k (d_in for read 0, d_out for read 1) the dot
+ * is formed inside the tensor-core kernel; when the dotted width exceeds 128, its
+ * 64-wide tiles add their dots atomically and the last bit may differ between runs.
+ * Other shapes and fp32 go through the workspace and a row-dot kernel.
  */
 int gradlev_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x,
                      const gradlev_tensor* g_hat, const gradlev_tensor* g_out,
