@@ -464,9 +464,12 @@ class MLPJob:
         if events is not None:
             events[2].record()
 
-    # --- pipelined end-to-end step: chunks along the batch rows
+    # --- pipelined end-to-end step: two chunks of batch rows (a single row leaves the
+    # wide passes too few tiles to fill the GPU)
     def e2e_chunks(self):
-        return [(b, b + 1) for b in range(self.wl.B)]
+        B = self.wl.B
+        half = (B + 1) // 2
+        return [(0, half), (half, B)] if B > 1 else [(0, 1)]
 
     def e2e_inputs(self, host, dev, sl, first):
         out = []
@@ -583,7 +586,12 @@ def e2e_measure(job, steps, stream):
     c.  Every input byte is copied in and every result byte out on every step."""
     dev_id = job.ws.device
     host = {k: job.inp[k].cpu().pin_memory() for k in job.in_keys}
-    dev = {k: torch.empty_like(job.inp[k]) for k in job.in_keys}
+    # two sets of device inputs and outputs, used by alternate steps: a step's copies
+    # in do not wait for the previous step's scans of the same chunk, nor its scans
+    # for the previous step's copies out
+    devs = [{k: torch.empty_like(job.inp[k]) for k in job.in_keys} for _ in range(2)]
+    outs = [job.outs, {k: torch.empty_like(v) for k, v in job.outs.items()}]
+    dev = devs[0]
     hout = {k: torch.empty(job.outs[k].shape, dtype=job.outs[k].dtype, pin_memory=True)
             for k in job.out_keys}
     bi = _bytes(*host.values())
@@ -595,32 +603,38 @@ def e2e_measure(job, steps, stream):
     s_run = torch.cuda.Stream(dev_id)
     s_out = torch.cuda.Stream(dev_id)
     n = len(chunks)
-    ev_in = [torch.cuda.Event() for _ in range(n)]
-    ev_run = [torch.cuda.Event() for _ in range(n)]
-    ev_out = [torch.cuda.Event() for _ in range(n)]
-    started = [False] * n
+    ev_in = [[torch.cuda.Event() for _ in range(n)] for _ in range(2)]
+    ev_run = [[torch.cuda.Event() for _ in range(n)] for _ in range(2)]
+    ev_out = [[torch.cuda.Event() for _ in range(n)] for _ in range(2)]
+    started = [[False] * n for _ in range(2)]
+    par = [0]
 
     def one():
+        b = par[0]
+        dv_set = devs[b]
+        job.outs = outs[b]
         for c, sl in enumerate(chunks):
             with torch.cuda.stream(s_in):
-                if started[c]:
-                    s_in.wait_event(ev_run[c])  # the previous step's scans of chunk c are done
-                for k, hv, dv in job.e2e_inputs(host, dev, sl, c == 0):
+                if started[b][c]:
+                    s_in.wait_event(ev_run[b][c])  # this set's last scans of chunk c are done
+                for k, hv, dv in job.e2e_inputs(host, dv_set, sl, c == 0):
                     dv.copy_(hv, non_blocking=True)
-                ev_in[c].record(s_in)
+                ev_in[b][c].record(s_in)
             with torch.cuda.stream(s_run):
-                s_run.wait_event(ev_in[c])
-                if started[c]:
-                    s_run.wait_event(ev_out[c])  # its previous results have been read out
-                job.e2e_step(dev, sl, ws)
-                ev_run[c].record(s_run)
+                s_run.wait_event(ev_in[b][c])
+                if started[b][c]:
+                    s_run.wait_event(ev_out[b][c])  # this set's last results have been read out
+                job.e2e_step(dv_set, sl, ws)
+                ev_run[b][c].record(s_run)
             with torch.cuda.stream(s_out):
-                s_out.wait_event(ev_run[c])
+                s_out.wait_event(ev_run[b][c])
                 for dv, hv in job.e2e_outputs(hout, sl):
                     hv.copy_(dv, non_blocking=True)
-                ev_out[c].record(s_out)
-            started[c] = True
+                ev_out[b][c].record(s_out)
+            started[b][c] = True
+        par[0] = b ^ 1
 
+    one()
     one()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -633,6 +647,7 @@ def e2e_measure(job, steps, stream):
     torch.cuda.synchronize()
     sec = e0.elapsed_time(e1) / 1e3
     # the results that came back agree with the whole-step call on resident inputs
+    job.outs = outs[0]
     job.step()
     torch.cuda.synchronize()
     worst = 0.0
@@ -642,9 +657,11 @@ def e2e_measure(job, steps, stream):
         worst = max(worst, float((got - ref).norm() / max(float(ref.norm()), 1e-30)))
     if not worst <= 2e-2:
         raise RuntimeError(f"pipelined end-to-end results differ from the resident step: {worst:.3e}")
+    ms = sec / steps * 1e3
     return {"value": round(job.tokens * steps / sec, 1), "unit": UNIT, "h2d_bytes_per_step": bi,
-            "d2h_bytes_per_step": bo, "steps": steps, "ms_per_step": round(sec / steps * 1e3, 3),
-            "pipeline": f"{n} chunks, copies overlapped with the scans on three streams",
+            "d2h_bytes_per_step": bo, "steps": steps, "ms_per_step": round(ms, 3),
+            "pipeline": (f"{n} chunks, copies overlapped with the scans on three streams, "
+                         "two sets of device buffers"),
             "rel_l2_vs_resident_step": worst}
 
 
