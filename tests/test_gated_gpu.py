@@ -65,6 +65,9 @@ CASES = {
     "alpha-serial-64": ("c5", dict(L=1, B=2, H=2, T=700), True),
     "alpha-serial-128x64": ("c2", dict(B=1, H=2, T=500, d_in=128, d_out=64), True),
     "alpha-serial-fp32": ("c1", dict(T=300), True),
+    # forward read 48 wide (register kernel, one quarter of each row's inputs empty,
+    # a 40-row output tile); costate read 40 wide (shared-memory kernel)
+    "alpha-serial-48x40": ("c2", dict(B=1, H=2, T=333, d_in=48, d_out=40, w_std=1 / 7), True),
 }
 
 
