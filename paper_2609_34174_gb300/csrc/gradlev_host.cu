@@ -94,7 +94,10 @@ struct Tok {
 };
 
 bool resolve(const gradlev_desc& d, const gradlev_tensor* t, int width, Tok* out, bool required) {
-    if (!t || !t->data) return !required;
+    if (!t) return !required;
+    // an empty sequence (T = 0) has no storage: a null pointer is then accepted, and
+    // every caller returns before it launches anything
+    if (!t->data) return !required || d.T == 0;
     out->data = t->data;
     bool zero = true;
     for (int i = 0; i < 4; ++i) zero = zero && t->stride[i] == 0;
@@ -500,7 +503,7 @@ int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
               cudaStream_t stream) {
     if (!desc_ok(desc)) return GRADLEV_ERR_INVALID_ARG;
     const gradlev_desc& d = *desc;
-    if (!W0 || !eta_t || (reinterpret_cast<uintptr_t>(eta_t) & 3u) ||
+    if (!W0 || (!eta_t && d.T > 0) || (reinterpret_cast<uintptr_t>(eta_t) & 3u) ||
         (alpha_t && (reinterpret_cast<uintptr_t>(alpha_t) & 3u)))
         return GRADLEV_ERR_INVALID_ARG;
     if (act < GRADLEV_ACT_NONE || act > GRADLEV_ACT_TANH) return GRADLEV_ERR_INVALID_ARG;
@@ -727,7 +730,7 @@ int run_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x,
                  const gradlev_tensor* g_hat, const gradlev_tensor* g_out,
                  const gradlev_tensor* upstream, float* deta, void* ws, size_t ws_bytes,
                  cudaStream_t stream) {
-    if (!desc_ok(desc) || (read != 0 && read != 1) || !deta ||
+    if (!desc_ok(desc) || (read != 0 && read != 1) || (!deta && desc->T > 0) ||
         (reinterpret_cast<uintptr_t>(deta) & 3u))
         return GRADLEV_ERR_INVALID_ARG;
     const gradlev_desc& d = *desc;
@@ -740,7 +743,7 @@ int run_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x,
     if (!resolve(d, x, d.d_in, &tx, true) || !resolve(d, g_hat, d.d_out, &tg, true) ||
         !resolve(d, upstream, read == 0 ? d.d_out : d.d_in, &tu, true))
         return GRADLEV_ERR_INVALID_ARG;
-    if (read == 1 && (!g_out || !g_out->data)) return GRADLEV_ERR_INVALID_ARG;
+    if (read == 1 && (!g_out || (!g_out->data && d.T > 0))) return GRADLEV_ERR_INVALID_ARG;
     if (d.T == 0) return GRADLEV_OK;
     const size_t base = round_up(suffix_ws_bytes(sd, sms), 256);
     gradlev_tensor rt;

@@ -127,3 +127,14 @@ def test_suffix_scan_and_eta_grad_strided_views():
     want = -np.sum(gu * oracle.suffix_scan(xu, xu, uu), axis=2)
     got = deta.permute(0, 1, 3, 2).reshape(L * B * H, T).double().cpu().numpy()
     assert rel_l2(got, want) <= TOL["bf16"]
+
+
+def test_empty_sequences():
+    """T = 0: nothing to read, no error."""
+    x = torch.zeros((1, 2, 0, 2, 64), dtype=torch.bfloat16, device="cuda")
+    g = torch.zeros((1, 2, 0, 2, 64), dtype=torch.bfloat16, device="cuda")
+    r = gl.suffix_scan(x, x, g)
+    deta = gl.eta_grad(x, g, g)
+    deta_c = gl.eta_grad(x, g, x, read="costate", g_out=g)
+    torch.cuda.synchronize()
+    assert r.shape == g.shape and deta.shape == (1, 2, 0, 2) and deta_c.shape == (1, 2, 0, 2)

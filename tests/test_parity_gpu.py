@@ -249,3 +249,22 @@ def test_length_sweep_one_to_three_chunks(dq):
         y, g, yr, gr = _run_linear(wl, inputs)
         _assert_close(f"T={T} forward", y, yr, TOL["bf16"])
         _assert_close(f"T={T} costate", g, gr, TOL["bf16"])
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32], ids=["bf16", "f32"])
+def test_empty_sequences_every_entry_point(dtype):
+    """T = 0 (the header allows it): every token entry point returns without error."""
+    L, B, H, d, m = 1, 2, 2, 64, 64
+    z = lambda w: torch.zeros((L, B, 0, H, w), dtype=dtype, device="cuda")
+    x, g = z(d), z(m)
+    W0 = torch.zeros((L, H, m, d), device="cuda")
+    eta_t = torch.zeros((L, B, 0, H), device="cuda")
+    y = gl.forward_scan(x, g, W0, 0.1)
+    gi = gl.costate_scan(x, g, W0, 0.1, g)
+    yg = gl.forward_scan(x, g, W0, eta_t, alpha=eta_t)
+    gg = gl.costate_scan(x, g, W0, eta_t, g)
+    r = gl.suffix_scan(x, x, g)
+    de = gl.eta_grad(x, g, g)
+    torch.cuda.synchronize()
+    assert y.shape == g.shape and gi.shape == x.shape and yg.shape == g.shape
+    assert gg.shape == x.shape and r.shape == g.shape and de.shape == (L, B, 0, H)
