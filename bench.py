@@ -182,7 +182,8 @@ class LinearJob:
             nb = int(_B.load_library().gradlev_workspace_bytes_gated(ctypes.byref(d)))
         self.ws = torch.empty(max(256, nb), dtype=torch.uint8, device=device)
         self.tokens = wl.tokens
-        self.launches_per_step = 2
+        # one chunk-kernel launch per scan; eta_t adds the prescale launch to each
+        self.launches_per_step = 4 if gates == "eta" else 2
         self.in_keys = ("x", "g_hat", "g_out", "W0") + (
             ("eta_t",) if gates else ()) + (("alpha_t",) if gates == "alpha" else ())
         self.out_keys = ("y", "g_in")
