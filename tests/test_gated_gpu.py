@@ -3,7 +3,8 @@ sizes eta_t and retention alpha_t, decay centred at W0) against the fp64 oracle,
 which runs the same recurrence token by token.
 
 Per-token eta_t alone takes the chunked kernels on eta-scaled proposals;
-with alpha_t the token-serial kernel runs.  alpha_t = 0 marks resets (the fast
+with alpha_t, bf16 64 x 64 maps run the chunked retention kernel and every
+other shape the token-serial kernels.  alpha_t = 0 marks resets (the fast
 weights return to W0, as at a document boundary).
 """
 import numpy as np
@@ -121,3 +122,81 @@ def test_constant_gates_match_plain_scan():
     torch.cuda.synchronize()
     err = rel_l2(y_serial.double().cpu().numpy(), y_plain.double().cpu().numpy())
     assert err <= TOL["bf16"], f"serial vs chunked rel-L2 {err:.3e}"
+
+
+# The retention path for bf16 64 x 64 maps runs in chunks of 64 tokens.  These
+# cases put the chunk boundaries, resets and odd gates where a chunked form of
+# Eq. 2 could go wrong: T below, at and just past one chunk; resets on the last
+# and first token of a chunk and two in a row; a negative alpha; many units.
+CHUNK_T = [1, 37, 64, 65, 128, 191, 1000]
+
+
+def _chunk_gates(shape, T, seed):
+    g = torch.Generator().manual_seed(seed)
+    eta = torch.rand(shape, generator=g, dtype=torch.float64) * 0.04
+    alpha = 0.85 + 0.15 * torch.rand(shape, generator=g, dtype=torch.float64)
+    for t in (63, 64, 127, 130, 131, 500):
+        if t < T:
+            alpha[:, :, t, :] = 0.0
+    if T > 20:
+        alpha[:, :, 20, :] = -0.5
+    return eta.float(), alpha.float()
+
+
+@pytest.mark.parametrize("T", CHUNK_T)
+def test_retention_chunk_boundaries(T):
+    wl = W.workload("c5").resized(L=2, B=1, H=3, T=T)
+    inputs = W.make_linear(wl)
+    eta, alpha = _chunk_gates((wl.L, wl.B, wl.T, wl.H), T, 900 + T)
+    dev = {k: (v.cuda() if isinstance(v, torch.Tensor) else v) for k, v in inputs.items()}
+    y = gl.forward_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), alpha=alpha.cuda())
+    gin = gl.costate_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), dev["g_out"],
+                          alpha=alpha.cuda())
+    torch.cuda.synchronize()
+    yr, gr = _oracle(inputs, eta, alpha, wl)
+    _check(f"T={T} forward", y, yr, TOL["bf16"])
+    _check(f"T={T} costate", gin, gr, TOL["bf16"])
+
+
+def test_retention_fused_activation_epilogues():
+    """sigma(y) from the forward read and sigma'(z) (.) g_in from the costate read
+    (the MLP's fused epilogues) on the retention path."""
+    wl = W.workload("c5").resized(L=1, B=2, H=2, T=300)
+    inputs = W.make_linear(wl)
+    eta, alpha = _chunk_gates((wl.L, wl.B, wl.T, wl.H), wl.T, 77)
+    dev = {k: (v.cuda() if isinstance(v, torch.Tensor) else v) for k, v in inputs.items()}
+    gz = torch.Generator().manual_seed(78)
+    z = torch.randn(dev["x"].shape, generator=gz).to(torch.bfloat16)
+    y, hy = gl.forward_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), act="gelu_tanh",
+                            want_act_out=True, alpha=alpha.cuda())
+    gin = gl.costate_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), dev["g_out"],
+                          act="gelu_tanh", z=z.cuda(), alpha=alpha.cuda())
+    torch.cuda.synchronize()
+    yr, gr = _oracle(inputs, eta, alpha, wl)
+    _check("y", y, yr, TOL["bf16"])
+    _check("sigma(y)", hy, oracle.act(oracle.ACT_GELU_TANH, y.double().cpu().numpy()), TOL["bf16"])
+    want = oracle.act_deriv(oracle.ACT_GELU_TANH, z.double().numpy()) * gr
+    _check("sigma'(z) g_in", gin, want, TOL["bf16"])
+
+
+@pytest.mark.parametrize("offset", [0, 4], ids=["aligned-rows", "8-byte-rows"])
+def test_retention_strided_views(offset):
+    """Token rows taken from wider buffers: 16-byte aligned rows (the chunked
+    kernel) and rows that start 8 bytes off (the token-serial kernel)."""
+    wl = W.workload("c5").resized(L=1, B=2, H=2, T=200)
+    inputs = W.make_linear(wl)
+    eta, alpha = _chunk_gates((wl.L, wl.B, wl.T, wl.H), wl.T, 55)
+    wide = {}
+    for k in ("x", "g_hat", "g_out"):
+        t = inputs[k]
+        buf = torch.zeros(t.shape[:-1] + (96,), dtype=t.dtype)
+        buf[..., offset:offset + 64] = t
+        wide[k] = buf.cuda()[..., offset:offset + 64]
+    W0 = inputs["W0"].cuda()
+    y = gl.forward_scan(wide["x"], wide["g_hat"], W0, eta.cuda(), alpha=alpha.cuda())
+    gin = gl.costate_scan(wide["x"], wide["g_hat"], W0, eta.cuda(), wide["g_out"],
+                          alpha=alpha.cuda())
+    torch.cuda.synchronize()
+    yr, gr = _oracle(inputs, eta, alpha, wl)
+    _check("forward", y, yr, TOL["bf16"])
+    _check("costate", gin, gr, TOL["bf16"])
