@@ -190,8 +190,8 @@ class LinearJob:
         self.kernel = {"fwd": "tc_scan_kernel<64, false> (forward scan)",
                        "costate": "tc_scan_kernel<64, true> (costate scan)"}
         if gates == "alpha":
-            self.kernel = {"fwd": "gated serial_kernel (forward scan)",
-                           "costate": "gated serial_kernel (costate scan)"}
+            self.kernel = {"fwd": "chunk_decay_kernel<false> (forward scan, retention)",
+                           "costate": "chunk_decay_kernel<true> (costate scan, retention)"}
 
     def input_bytes(self):
         return _bytes(self.inp["x"], self.inp["g_hat"], self.inp["g_out"])
@@ -290,7 +290,7 @@ class LinearJob:
              "eta": wl.eta}
         if self.gates:
             c["gates"] = ("per-token eta_t" if self.gates == "eta"
-                          else "per-token eta_t and retention alpha_t (token-serial kernel)")
+                          else "per-token eta_t and retention alpha_t (chunked retention kernel)")
         return c
 
     def oracle_run(self, inp, n_units, cores, t_tokens=None):

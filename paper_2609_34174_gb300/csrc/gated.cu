@@ -449,22 +449,24 @@ __host__ __device__ constexpr size_t smem_bytes() {        // B0, S copy, two ch
 __device__ __forceinline__ uint32_t swz(int row, int piece) {
     return (uint32_t)(row * 128 + ((piece ^ (row & 7)) << 4));
 }
+// The fragment loads read shared memory (memory clobber: they stay between the
+// barriers and stores around them); the MMAs are pure register operations, free
+// to be scheduled between the loads.
 __device__ __forceinline__ void ldsm4(uint32_t a, uint32_t (&r)[4]) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+    asm("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
                  : "r"(a)
                  : "memory");
 }
 __device__ __forceinline__ void ldsm4t(uint32_t a, uint32_t (&r)[4]) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+    asm("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
                  : "r"(a)
                  : "memory");
 }
 // d += a b: a 16 x 16 (row), b 16 x 8 (col), bf16 in, fp32 accumulate
 __device__ __forceinline__ void mma(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
         "{%8,%9}, {%0,%1,%2,%3};"
         : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
@@ -580,9 +582,8 @@ __global__ void __launch_bounds__(kThr, 3) chunk_decay_kernel(GatedParams p) {
             tpr[j] = tp;
         }
 
-        uint32_t qa[4][4];
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) ldsm4(sQ + swz(16 * warp + (lane & 15), 2 * kk + (lane >> 4)), qa[kk]);
+        // this warp's Q fragments, reloaded where used (fewer live registers)
+        auto ldq = [&](int kk, uint32_t (&q)[4]) { ldsm4(sQ + swz(16 * warp + (lane & 15), 2 * kk + (lane >> 4)), q); };
         // P = Q K^T over the column tiles at or before this warp's tokens
         float pacc[8][4];
 #pragma unroll
@@ -592,10 +593,11 @@ __global__ void __launch_bounds__(kThr, 3) chunk_decay_kernel(GatedParams p) {
             if (jp <= warp) {
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
-                    uint32_t r[4];
+                    uint32_t r[4], q[4];
+                    ldq(kk, q);
                     ld_b_nk(sK, 16 * jp, 16 * kk, lane, r);
-                    mma(pacc[2 * jp], qa[kk], r[0], r[1]);
-                    mma(pacc[2 * jp + 1], qa[kk], r[2], r[3]);
+                    mma(pacc[2 * jp], q, r[0], r[1]);
+                    mma(pacc[2 * jp + 1], q, r[2], r[3]);
                 }
             }
         }
@@ -607,38 +609,47 @@ __global__ void __launch_bounds__(kThr, 3) chunk_decay_kernel(GatedParams p) {
         for (int jp = 0; jp < 4; ++jp)
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
-                uint32_t r[4];
+                uint32_t r[4], q[4];
+                ldq(kk, q);
                 ld_b_nk(sS, 16 * jp, 16 * kk, lane, r);
-                mma(oacc[2 * jp], qa[kk], r[0], r[1]);
-                mma(oacc[2 * jp + 1], qa[kk], r[2], r[3]);
+                mma(oacc[2 * jp], q, r[0], r[1]);
+                mma(oacc[2 * jp + 1], q, r[2], r[3]);
             }
         __syncthreads();  // decay pieces ready; every read of the S copy done
 
         float tp[8];
 #pragma unroll
         for (int j = 0; j < 8; ++j) tp[j] = tpr[j];
+        // eta_s sig_s for this thread's columns s = 8j + 2cq + e (reads and write)
+        float se[8][2];
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) se[j][e] = et[8 * j + 2 * cq + e] * sig[8 * j + 2 * cq + e];
         // P'_ts = -E_ts P_ts (zero for s >= t); a_t for this thread's two tokens
         float a_row[2];
 #pragma unroll
         for (int hr = 0; hr < 2; ++hr) {
             const int t = 16 * warp + g + 8 * hr;
             const int jt = t >> 3;
+            float dd[2];  // columns in t's own piece: the alphas strictly between s and t
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const int s = 8 * jt + 2 * cq + e;
+                float d = s < t ? et[s] : 0.0f;
+                for (int r = s + 1; r < t; ++r) d *= al[r];
+                dd[e] = d;
+            }
             float tau = pim[t];  // alphas in [8j + 8, t) for the piece j being scaled
 #pragma unroll
             for (int j = 7; j >= 0; --j) {
+                const bool below = j < jt;
 #pragma unroll
                 for (int e = 0; e < 2; ++e) {
-                    const int s = 8 * j + 2 * cq + e;
-                    float dec = 0.0f;
-                    if (j < jt) {
-                        dec = sig[s] * tau;
-                    } else if (j == jt && s < t) {
-                        dec = 1.0f;
-                        for (int r = s + 1; r < t; ++r) dec *= al[r];
-                    }
-                    pacc[j][2 * hr + e] *= -dec * et[s];
+                    const float dec = below ? se[j][e] * tau : (j == jt ? dd[e] : 0.0f);
+                    pacc[j][2 * hr + e] *= -dec;
                 }
-                if (j < jt) tau *= tp[j];
+                tau = below ? tau * tp[j] : tau;
             }
             a_row[hr] = tau;
         }
@@ -654,10 +665,11 @@ __global__ void __launch_bounds__(kThr, 3) chunk_decay_kernel(GatedParams p) {
         for (int jp = 0; jp < 4; ++jp)
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
-                uint32_t r[4];
+                uint32_t r[4], q[4];
+                ldq(kk, q);
                 ld_b_nk(sB0, 16 * jp, 16 * kk, lane, r);
-                mma(oacc[2 * jp], qa[kk], r[0], r[1]);
-                mma(oacc[2 * jp + 1], qa[kk], r[2], r[3]);
+                mma(oacc[2 * jp], q, r[0], r[1]);
+                mma(oacc[2 * jp + 1], q, r[2], r[3]);
             }
         // + P' V (P' carries the minus sign)
 #pragma unroll
@@ -678,6 +690,18 @@ __global__ void __launch_bounds__(kThr, 3) chunk_decay_kernel(GatedParams p) {
         }
         // epilogue: rows of this thread's two tokens, two adjacent columns per tile
         const EpiParams& ep = p.epi;
+        if (!ep.out2 && !ep.zin) {
+#pragma unroll
+            for (int hr = 0; hr < 2; ++hr) {
+                const int t = c * kC + 16 * warp + g + 8 * hr;
+                if (t < p.T) {
+                    bf* orow = static_cast<bf*>(ep.out) + tok_off(ep.out_str, l, b, t, h) + 2 * cq;
+#pragma unroll
+                    for (int n = 0; n < 8; ++n)
+                        *reinterpret_cast<uint32_t*>(orow + 8 * n) = pack(oacc[n][2 * hr], oacc[n][2 * hr + 1]);
+                }
+            }
+        } else {
 #pragma unroll
         for (int hr = 0; hr < 2; ++hr) {
             const int t = c * kC + 16 * warp + g + 8 * hr;
@@ -701,6 +725,7 @@ __global__ void __launch_bounds__(kThr, 3) chunk_decay_kernel(GatedParams p) {
                 }
             }
         }
+        }
         // the write: S <- a_end S - sum_s w_s v_s k_s^T, w_s = eta_s sig_s prod_{pieces after s} tp
         float sfx[8];
         sfx[7] = 1.0f;
@@ -719,10 +744,8 @@ __global__ void __launch_bounds__(kThr, 3) chunk_decay_kernel(GatedParams p) {
             // A = (w o V)^T rows [16 warp, +16), tokens [16 kk, +16), from V stored [s][v]
             uint32_t va[4];
             ldsm4t(sV + swz(16 * kk + (lane & 7) + ((lane >> 4) << 3), 2 * warp + ((lane >> 3) & 1)), va);
-            const int s0 = 16 * kk + 2 * cq, s1 = s0 + 8;
-            const float w00 = -et[s0] * sig[s0] * sfx[2 * kk], w01 = -et[s0 + 1] * sig[s0 + 1] * sfx[2 * kk];
-            const float w10 = -et[s1] * sig[s1] * sfx[2 * kk + 1],
-                        w11 = -et[s1 + 1] * sig[s1 + 1] * sfx[2 * kk + 1];
+            const float w00 = -se[2 * kk][0] * sfx[2 * kk], w01 = -se[2 * kk][1] * sfx[2 * kk];
+            const float w10 = -se[2 * kk + 1][0] * sfx[2 * kk + 1], w11 = -se[2 * kk + 1][1] * sfx[2 * kk + 1];
             va[0] = scale2(va[0], w00, w01);
             va[1] = scale2(va[1], w00, w01);
             va[2] = scale2(va[2], w10, w11);
@@ -750,6 +773,8 @@ cudaError_t launch(const GatedParams& p, int blocks, cudaStream_t stream) {
     auto kern = chunk_decay_kernel<COSTATE>;
     const size_t smem = smem_bytes<COSTATE>();
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e == cudaSuccess)  // room for the CTAs the registers allow
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     if (e != cudaSuccess) return e;
     kern<<<blocks, kThr, smem, stream>>>(p);
     return cudaGetLastError();
