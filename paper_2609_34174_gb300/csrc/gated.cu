@@ -588,13 +588,16 @@ __global__ void __launch_bounds__(kThr, 3) chunk_decay_kernel(GatedParams p) {
         float pacc[8][4];
 #pragma unroll
         for (int n = 0; n < 8; ++n) pacc[n][0] = pacc[n][1] = pacc[n][2] = pacc[n][3] = 0.0f;
+        // (k-steps outside, column tiles inside: consecutive MMAs use different
+        // accumulators)
 #pragma unroll
-        for (int jp = 0; jp < 4; ++jp) {
-            if (jp <= warp) {
+        for (int kk = 0; kk < 4; ++kk) {
+            uint32_t q[4];
+            ldq(kk, q);
 #pragma unroll
-                for (int kk = 0; kk < 4; ++kk) {
-                    uint32_t r[4], q[4];
-                    ldq(kk, q);
+            for (int jp = 0; jp < 4; ++jp) {
+                if (jp <= warp) {
+                    uint32_t r[4];
                     ld_b_nk(sK, 16 * jp, 16 * kk, lane, r);
                     mma(pacc[2 * jp], q, r[0], r[1]);
                     mma(pacc[2 * jp + 1], q, r[2], r[3]);
@@ -606,15 +609,17 @@ __global__ void __launch_bounds__(kThr, 3) chunk_decay_kernel(GatedParams p) {
 #pragma unroll
         for (int n = 0; n < 8; ++n) oacc[n][0] = oacc[n][1] = oacc[n][2] = oacc[n][3] = 0.0f;
 #pragma unroll
-        for (int jp = 0; jp < 4; ++jp)
+        for (int kk = 0; kk < 4; ++kk) {
+            uint32_t q[4];
+            ldq(kk, q);
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk) {
-                uint32_t r[4], q[4];
-                ldq(kk, q);
+            for (int jp = 0; jp < 4; ++jp) {
+                uint32_t r[4];
                 ld_b_nk(sS, 16 * jp, 16 * kk, lane, r);
                 mma(oacc[2 * jp], q, r[0], r[1]);
                 mma(oacc[2 * jp + 1], q, r[2], r[3]);
             }
+        }
         __syncthreads();  // decay pieces ready; every read of the S copy done
 
         float tp[8];
@@ -662,15 +667,17 @@ __global__ void __launch_bounds__(kThr, 3) chunk_decay_kernel(GatedParams p) {
         }
         // + B0 q_t
 #pragma unroll
-        for (int jp = 0; jp < 4; ++jp)
+        for (int kk = 0; kk < 4; ++kk) {
+            uint32_t q[4];
+            ldq(kk, q);
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk) {
-                uint32_t r[4], q[4];
-                ldq(kk, q);
+            for (int jp = 0; jp < 4; ++jp) {
+                uint32_t r[4];
                 ld_b_nk(sB0, 16 * jp, 16 * kk, lane, r);
                 mma(oacc[2 * jp], q, r[0], r[1]);
                 mma(oacc[2 * jp + 1], q, r[2], r[3]);
             }
+        }
         // + P' V (P' carries the minus sign)
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk) {
