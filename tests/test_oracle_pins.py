@@ -56,6 +56,41 @@ def test_closed_form_eq2_with_gates(T, d, m):
         np.testing.assert_allclose(gin[0, t], W_t.T @ gout[0, t], rtol=0, atol=1e-14)
 
 
+@pytest.mark.parametrize("T", [6, 11])
+def test_closed_form_eq2_resets_and_negative_retention(T):
+    """alpha_t = 0 (resets, also two in a row) and alpha_t < 0 still follow Eq. 2."""
+    x, ghat, W0, gout = _rand_problem(300 + T, 1, T, 5, 4)
+    r = _rng(8 + T)
+    eta = r.uniform(0.05, 0.5, T)
+    alpha = r.uniform(0.5, 1.0, T)
+    alpha[[1, 3, 4]] = 0.0
+    alpha[T - 2] = -0.7
+    y, gin = oracle.linear_scan(x, ghat, W0, eta, alpha=alpha, gout=gout)
+    for t in range(T):
+        W_t = W0[0] + _closed_form_delta(t, x[0], ghat[0], eta, alpha)
+        np.testing.assert_allclose(y[0, t], W_t @ x[0, t], rtol=0, atol=1e-14)
+        np.testing.assert_allclose(gin[0, t], W_t.T @ gout[0, t], rtol=0, atol=1e-14)
+
+
+def test_reset_restarts_a_fresh_learner():
+    """After alpha_r = 0 the map is W0 minus the writes from token r on, so every read
+    after r equals the read of a learner started at token r from W0 (whatever alpha_r)."""
+    T, rr = 40, 17
+    x, ghat, W0, gout = _rand_problem(77, 1, T, 8, 6)
+    r = _rng(78)
+    eta = r.uniform(0.05, 0.3, T)
+    alpha = r.uniform(0.6, 1.0, T)
+    alpha[rr] = 0.0
+    y, gin = oracle.linear_scan(x, ghat, W0, eta, alpha=alpha, gout=gout)
+    a2 = alpha[rr:].copy()
+    a2[0] = 0.37  # scales the fresh learner's zero fast weights: no effect
+    y2, g2 = oracle.linear_scan(x[:, rr:], ghat[:, rr:], W0, eta[rr:], alpha=a2, gout=gout[:, rr:])
+    # the read at r itself comes before r's write and still sees the history
+    np.testing.assert_allclose(y[0, rr + 1:], y2[0, 1:], rtol=0, atol=1e-13)
+    np.testing.assert_allclose(gin[0, rr + 1:], g2[0, 1:], rtol=0, atol=1e-13)
+    assert np.abs(y[0, rr] - y2[0, 0]).max() > 1e-3
+
+
 def test_first_read_is_slow_weights():
     """W_hat_0 = W_0 (Delta_0 = 0; read before write): row t=0 is a plain GEMV."""
     x, ghat, W0, gout = _rand_problem(3, 4, 6, 16, 8)
