@@ -152,9 +152,14 @@ int gradlev_costate_scan(const gradlev_desc* desc, const gradlev_tensor* x,
  *   eta is replaced by eta_t).
  * Without alpha_t the proposals are scaled by eta_t into the workspace (one
  * elementwise pass, rounded to the input dtype) and the chunked scan runs with
- * eta = 1.  With alpha_t a token-serial kernel runs the recurrence as written
- * (state W - W0 in fp32 shared memory; the read width, d_in forward and d_out
- * costate, must be at most 256, else GRADLEV_ERR_UNSUPPORTED).
+ * eta = 1.  With alpha_t:
+ *   - bf16 64 x 64 maps whose token rows are 16-byte aligned (the outputs 4-byte
+ *     aligned with even strides) run in chunks of 64 tokens on the tensor cores,
+ *     with the decays formed as products of the alphas (exact zeros at resets;
+ *     any real alpha_t is accepted);
+ *   - every other shape runs the recurrence token by token, the state W - W0 in
+ *     fp32.  The read width (d_in forward, d_out costate) must be at most 256,
+ *     else GRADLEV_ERR_UNSUPPORTED.
  * Workspace: at least gradlev_workspace_bytes_gated(desc) bytes, 256-byte aligned.
  */
 int gradlev_forward_scan_gated(const gradlev_desc* desc, const gradlev_tensor* x,
