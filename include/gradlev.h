@@ -173,6 +173,31 @@ int gradlev_costate_scan_gated(const gradlev_desc* desc, const gradlev_tensor* x
                                const gradlev_tensor* z, const gradlev_tensor* g_in, void* workspace,
                                size_t workspace_bytes, gradlev_stream_t stream);
 
+/*
+ * gradlev_document_gates -- gate arrays for sequences packed from several
+ * documents.  A read excludes every write made before the most recent document
+ * start (Appendix C, scan reads; Appendix E, packed rows).  In the gates of Eq. 2
+ * a document starting at token s > 0 is alpha = 0 and eta = 0 at token s - 1:
+ * the fast weights return to W0 and the previous document's last write (seen by
+ * none of its reads) is dropped, so the read at s sees W0.  The outputs feed
+ * gradlev_forward_scan_gated / gradlev_costate_scan_gated.
+ *   desc       only L, B, T, H (and reserved = 0) are read
+ *   doc_start  uint8 [B][T], contiguous device array, nonzero where a document
+ *              begins; entry t = 0 is ignored (every row begins one).  The same
+ *              documents hold for every layer and head.
+ *   eta        step size of every write where eta_t is NULL (finite)
+ *   eta_t      fp32 [L][B][T][H] contiguous per-token step sizes, or NULL
+ *   alpha_t    fp32 [L][B][T][H] contiguous retention, or NULL for alpha = 1
+ *   eta_out, alpha_out  fp32 [L][B][T][H] contiguous device outputs (written);
+ *              eta_out may be eta_t and alpha_out may be alpha_t (in place)
+ * Returns GRADLEV_OK (nothing to do when L*B*T*H = 0), GRADLEV_ERR_INVALID_ARG
+ * for a null pointer, a non-finite eta or an fp32 array not 4-byte aligned, and
+ * GRADLEV_ERR_CUDA if the launch fails.  Asynchronous on `stream`.
+ */
+int gradlev_document_gates(const gradlev_desc* desc, const uint8_t* doc_start, float eta,
+                           const float* eta_t, const float* alpha_t, float* eta_out,
+                           float* alpha_out, gradlev_stream_t stream);
+
 /* Bytes of workspace the gated scans need for this shape (0 for an invalid
  * descriptor). */
 size_t gradlev_workspace_bytes_gated(const gradlev_desc* desc);

@@ -124,6 +124,40 @@ def linear_scan(x, ghat, W0, eta, alpha=None, gout=None, want_y=True, nthreads=0
     return y, gin
 
 
+def linear_scan_docs(x, ghat, W0, eta, doc_start, alpha=None, gout=None):
+    """Document resets (Appendix C, scan reads; Appendix E, packed documents): every
+    read excludes the writes made before the most recent document start, so each
+    document is its own sequential learner starting from W0.
+
+    doc_start [U,T] booleans, True where a document begins (token 0 always begins
+    one); eta and alpha as in linear_scan (scalar or [T], shared by the units), each
+    document taking its own slice.  Returns (y [U,T,m], gin [U,T,d] or None).
+    """
+    x = _f64(x)
+    ghat = _f64(ghat)
+    U, T, d = x.shape
+    m = ghat.shape[2]
+    W0 = _f64(W0)
+    starts = np.asarray(doc_start, dtype=bool)
+    if starts.shape != (U, T):
+        raise ValueError(f"doc_start must be [{U},{T}]")
+    eta_a = _steps(eta, T)
+    alpha_a = _steps(alpha, T) if alpha is not None else None
+    y = np.empty((U, T, m))
+    gin = np.empty((U, T, d)) if gout is not None else None
+    for u in range(U):
+        cuts = [0] + [t for t in range(1, T) if starts[u, t]] + [T]
+        for a, b in zip(cuts[:-1], cuts[1:]):
+            w0 = W0 if W0.ndim == 2 else W0[u]
+            yy, gg = linear_scan(x[u:u + 1, a:b], ghat[u:u + 1, a:b], w0, eta_a[a:b],
+                                 alpha=None if alpha_a is None else alpha_a[a:b],
+                                 gout=None if gout is None else _f64(gout)[u:u + 1, a:b])
+            y[u, a:b] = yy[0]
+            if gin is not None:
+                gin[u, a:b] = gg[0]
+    return y, gin
+
+
 def mlp_scan(x, ghz, ghy, W10, W20, eta1, eta2, act=ACT_GELU_TANH, alpha=None, gout=None,
              nthreads=0):
     """Sequential online MLP (Appendix A) for U independent sequences.

@@ -82,6 +82,8 @@ def load_library():
         lib.gradlev_costate_scan_gated.restype = ctypes.c_int
         lib.gradlev_workspace_bytes_gated.argtypes = [D]
         lib.gradlev_workspace_bytes_gated.restype = ctypes.c_size_t
+        lib.gradlev_document_gates.argtypes = [D, P, ctypes.c_float, P, P, P, P, P]
+        lib.gradlev_document_gates.restype = ctypes.c_int
         lib.gradlev_decode_read.argtypes = [D, Tp, P, P, ctypes.c_int, Tp, Tp, P]
         lib.gradlev_decode_read.restype = ctypes.c_int
         lib.gradlev_decode_write.argtypes = [D, Tp, Tp, P, P, P, P, ctypes.c_int, Tp, Tp, P,
@@ -229,13 +231,65 @@ def _gates(eta, alpha, x5):
     return norm(eta), (norm(alpha) if alpha is not None else None)
 
 
+def _document_gates(doc_start, x5, eta, alpha):
+    """Fold document starts into fp32 [L,B,T,H] (eta_t, alpha_t) on x5's device."""
+    lib = load_library()
+    L, B, T, H = (int(v) for v in x5.shape[:4])
+    ds = doc_start if isinstance(doc_start, torch.Tensor) else torch.as_tensor(doc_start)
+    ds = ds.to(device=x5.device)
+    if ds.dim() == 1 and B == 1:
+        ds = ds.unsqueeze(0)
+    if tuple(ds.shape) != (B, T):
+        raise ValueError(f"doc_start must be [B, T] = {(B, T)}, got {tuple(ds.shape)}")
+    ds = (ds != 0).to(torch.uint8).contiguous()
+    shape = (L, B, T, H)
+
+    def per_token(v):
+        if not isinstance(v, torch.Tensor):
+            return None
+        return v.to(device=x5.device, dtype=torch.float32).reshape(shape).contiguous()
+
+    et, at = per_token(eta), per_token(alpha)
+    if alpha is not None and at is None:
+        at = torch.full(shape, float(alpha), dtype=torch.float32, device=x5.device)
+    eo = torch.empty(shape, dtype=torch.float32, device=x5.device)
+    ao = torch.empty(shape, dtype=torch.float32, device=x5.device)
+    desc = _Desc(L, B, T, H, 0, 0, 0, 0)
+    stream = torch.cuda.current_stream(x5.device).cuda_stream
+    ptr = lambda t: ctypes.c_void_p(t.data_ptr()) if t is not None else None
+    with torch.cuda.device(x5.device):
+        rc = lib.gradlev_document_gates(ctypes.byref(desc), ptr(ds),
+                                        0.0 if et is not None else float(eta), ptr(et), ptr(at),
+                                        ptr(eo), ptr(ao), ctypes.c_void_p(stream))
+    _call(rc, "gradlev_document_gates")
+    return eo, ao
+
+
+def document_gates(doc_start, x, eta, alpha=None):
+    """Per-token gates for sequences packed from several documents (Appendix C:
+    a read excludes every write before the most recent document start; Appendix E).
+
+    doc_start: bool / integer [B, T] (or [T] when B = 1), nonzero where a document
+    begins, the same for every layer and head.  eta: scalar or per-token tensor;
+    alpha: None, scalar or per-token tensor.  Returns fp32 (eta_t, alpha_t) with the
+    token shape of x, with eta = alpha = 0 on the last token of every document that
+    another follows.  forward_scan / costate_scan take doc_start= and do this
+    themselves.
+    """
+    x5 = _as5(x)
+    if not x5.is_cuda:
+        raise ValueError("tensors must be on a CUDA device")
+    eo, ao = _document_gates(doc_start, x5, eta, alpha)
+    return eo.reshape(x.shape[:-1]), ao.reshape(x.shape[:-1])
+
+
 def _call(rc: int, what: str):
     if rc != 0:
         raise GradLevError(rc, what)
 
 
 def forward_scan(x, g_hat, W0, eta, act=None, y=None, act_out=None, want_act_out=False,
-                 workspace=None, alpha=None):
+                 workspace=None, alpha=None, doc_start=None):
     """y_t = (W0 - eta sum_{s<t} ghat_s x_s^T) x_t for every token (Sec. 3 step 2, Eq. 3).
 
     x [L,B,T,H,d_in] (or [B,T,H,d_in], [B,T,d_in], [T,d_in]), g_hat with d_out features,
@@ -244,7 +298,8 @@ def forward_scan(x, g_hat, W0, eta, act=None, y=None, act_out=None, want_act_out
 
     Gates (Eq. 2): `eta` may be a tensor of per-token step sizes with the token
     shape of x, and `alpha` an optional per-token retention (decay centred at W0;
-    alpha = 0 resets to W0).
+    alpha = 0 resets to W0).  `doc_start` ([B, T], nonzero where a document begins)
+    resets the fast weights at document starts (see document_gates).
     """
     lib = load_library()
     x5, g5 = _as5(x), _as5(g_hat)
@@ -269,6 +324,8 @@ def forward_scan(x, g_hat, W0, eta, act=None, y=None, act_out=None, want_act_out
         act_out = torch.empty_like(y)
     a5 = _as5(act_out) if act_out is not None else None
     desc = _desc(x5, d_out, _dtype_code(x5))
+    if doc_start is not None:
+        eta, alpha = _document_gates(doc_start, x5, eta, alpha)
     gates = _gates(eta, alpha, x5)
     if gates is not None:
         nbytes = int(lib.gradlev_workspace_bytes_gated(ctypes.byref(desc)))
@@ -303,12 +360,12 @@ def forward_scan(x, g_hat, W0, eta, act=None, y=None, act_out=None, want_act_out
 
 
 def costate_scan(x, g_hat, W0, eta, g_out, act=None, z=None, g_in=None, workspace=None,
-                 alpha=None):
+                 alpha=None, doc_start=None):
     """g_in_t = (W0 - eta sum_{s<t} ghat_s x_s^T)^T g_out_t (Sec. 3 step 3, Eq. 4).
 
     With z (the preactivation that fed this map's input through sigma = act) the
     result is sigma'(z_t) * (What_t^T g_out_t).  Returns g_in [.., d_in].
-    Gates as for forward_scan.
+    Gates and doc_start as for forward_scan.
     """
     lib = load_library()
     x5, g5, go5 = _as5(x), _as5(g_hat), _as5(g_out)
@@ -331,6 +388,8 @@ def costate_scan(x, g_hat, W0, eta, g_out, act=None, z=None, g_in=None, workspac
     gi5 = _as5(g_in)
     _check_same(x5, gi5)
     desc = _desc(x5, d_out, _dtype_code(x5))
+    if doc_start is not None:
+        eta, alpha = _document_gates(doc_start, x5, eta, alpha)
     gates = _gates(eta, alpha, x5)
     if gates is not None:
         nbytes = int(lib.gradlev_workspace_bytes_gated(ctypes.byref(desc)))

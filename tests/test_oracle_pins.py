@@ -91,6 +91,60 @@ def test_reset_restarts_a_fresh_learner():
     assert np.abs(y[0, rr] - y2[0, 0]).max() > 1e-3
 
 
+# ---------------------------------------------------- document resets (App. C, E)
+def _doc_starts(T, cuts):
+    ds = np.zeros((1, T), dtype=bool)
+    ds[0, list(cuts)] = True
+    return ds
+
+
+@pytest.mark.parametrize("gated", [False, True])
+def test_documents_closed_form(gated):
+    """Each read sees W0 plus the writes of its own document only (Appendix C: a read
+    excludes all writes before the most recent document start), checked against the
+    closed form of Eq. 2 over that document's tokens."""
+    T, cuts = 13, (1, 5, 6, 10)
+    x, ghat, W0, gout = _rand_problem(400 + gated, 1, T, 4, 3)
+    r = _rng(401)
+    eta = r.uniform(0.05, 0.5, T)
+    alpha = r.uniform(0.4, 1.0, T) if gated else np.ones(T)
+    y, gin = oracle.linear_scan_docs(x, ghat, W0, eta, _doc_starts(T, cuts),
+                                     alpha=alpha if gated else None, gout=gout)
+    bounds = [0, *cuts, T]
+    for a, b in zip(bounds[:-1], bounds[1:]):
+        for t in range(a, b):
+            W_t = W0[0] + _closed_form_delta(t - a, x[0, a:b], ghat[0, a:b], eta[a:b], alpha[a:b])
+            np.testing.assert_allclose(y[0, t], W_t @ x[0, t], rtol=0, atol=1e-14)
+            np.testing.assert_allclose(gin[0, t], W_t.T @ gout[0, t], rtol=0, atol=1e-14)
+
+
+def test_documents_are_eq2_gates_zeroed_before_each_start():
+    """The reading the GPU path takes: a document starting at s is alpha = eta = 0 at
+    token s - 1 in the one-sequence recurrence of Eq. 2."""
+    T, cuts = 90, (1, 2, 30, 64, 65, 89)
+    x, ghat, W0, gout = _rand_problem(402, 1, T, 6, 5)
+    r = _rng(403)
+    eta = r.uniform(0.02, 0.3, T)
+    alpha = r.uniform(0.8, 1.0, T)
+    yd, gd = oracle.linear_scan_docs(x, ghat, W0, eta, _doc_starts(T, cuts), alpha=alpha, gout=gout)
+    e2, a2 = eta.copy(), alpha.copy()
+    for c in cuts:
+        e2[c - 1] = 0.0
+        a2[c - 1] = 0.0
+    y, g = oracle.linear_scan(x, ghat, W0, e2, alpha=a2, gout=gout)
+    np.testing.assert_allclose(y, yd, rtol=0, atol=1e-13)
+    np.testing.assert_allclose(g, gd, rtol=0, atol=1e-13)
+
+
+def test_documents_of_one_token_read_slow_weights():
+    """Every token its own document: no read sees any write, y_t = W0 x_t."""
+    T = 9
+    x, ghat, W0, gout = _rand_problem(404, 1, T, 5, 4)
+    y, gin = oracle.linear_scan_docs(x, ghat, W0, 0.4, np.ones((1, T), dtype=bool), gout=gout)
+    np.testing.assert_allclose(y[0], x[0] @ W0[0].T, rtol=0, atol=1e-14)
+    np.testing.assert_allclose(gin[0], gout[0] @ W0[0], rtol=0, atol=1e-14)
+
+
 def test_first_read_is_slow_weights():
     """W_hat_0 = W_0 (Delta_0 = 0; read before write): row t=0 is a plain GEMV."""
     x, ghat, W0, gout = _rand_problem(3, 4, 6, 16, 8)
