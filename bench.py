@@ -163,12 +163,24 @@ class LinearJob:
         self.outs = {"y": torch.empty_like(self.inp["g_hat"]),
                      "g_in": torch.empty_like(self.inp["x"])}
         # Gated scans (Eq. 2): per-token eta_t in [0, 2 eta] and, for "alpha",
-        # retention alpha_t in [0.9, 1]; tensors [L, B, T, H] drawn once.
+        # retention alpha_t in [0.9, 1]; tensors [L, B, T, H] drawn once.  "docs":
+        # the scalar eta with document starts per batch row (packed documents of
+        # 512 to 1535 tokens), folded into the gates by the library every call.
         self.gates = gates
         self.eta_t = self.alpha_t = None
         code = 1 if wl.dtype == "bf16" else 0
         nb = gl.workspace_bytes(wl.L, wl.B, wl.T, wl.H, wl.d_in, wl.d_out, code)
-        if gates:
+        if gates == "docs":
+            gen = torch.Generator()
+            gen.manual_seed(wl.seed * 1000 + 19)
+            ds = torch.zeros(wl.B, wl.T, dtype=torch.uint8)
+            for b in range(wl.B):
+                t = int(torch.randint(512, 1536, (1,), generator=gen))
+                while t < wl.T:
+                    ds[b, t] = 1
+                    t += int(torch.randint(512, 1536, (1,), generator=gen))
+            self.inp["doc_start"] = ds.to(device)
+        elif gates:
             gen = torch.Generator(device=device)
             gen.manual_seed(wl.seed * 1000 + 17)
             shape = (wl.L, wl.B, wl.T, wl.H)
@@ -177,19 +189,22 @@ class LinearJob:
                 self.alpha_t = 0.9 + 0.1 * torch.rand(shape, generator=gen, device=device)
                 self.inp["alpha_t"] = self.alpha_t
             self.inp["eta_t"] = self.eta_t
+        if gates:
             from paper_2609_34174_gb300 import _binding as _B
             d = _B._Desc(wl.L, wl.B, wl.T, wl.H, wl.d_in, wl.d_out, code, 0)
             nb = int(_B.load_library().gradlev_workspace_bytes_gated(ctypes.byref(d)))
         self.ws = torch.empty(max(256, nb), dtype=torch.uint8, device=device)
         self.tokens = wl.tokens
-        # one chunk-kernel launch per scan; eta_t adds the prescale launch to each
-        self.launches_per_step = 4 if gates == "eta" else 2
+        # one chunk-kernel launch per scan; eta_t adds the prescale launch to each,
+        # documents the gate-folding launch
+        self.launches_per_step = 4 if gates in ("eta", "docs") else 2
         self.in_keys = ("x", "g_hat", "g_out", "W0") + (
-            ("eta_t",) if gates else ()) + (("alpha_t",) if gates == "alpha" else ())
+            ("eta_t",) if gates in ("eta", "alpha") else ()) + (
+            ("alpha_t",) if gates == "alpha" else ()) + (("doc_start",) if gates == "docs" else ())
         self.out_keys = ("y", "g_in")
         self.kernel = {"fwd": "tc_scan_kernel<64, false> (forward scan)",
                        "costate": "tc_scan_kernel<64, true> (costate scan)"}
-        if gates == "alpha":
+        if gates in ("alpha", "docs"):
             self.kernel = {"fwd": "chunk_decay_kernel<false> (forward scan, retention)",
                            "costate": "chunk_decay_kernel<true> (costate scan, retention)"}
 
@@ -201,16 +216,17 @@ class LinearJob:
         inp = inp or self.inp
         if events is not None:
             events[0].record()
-        eta = inp["eta_t"] if self.gates else wl.eta
+        eta = inp["eta_t"] if self.gates in ("eta", "alpha") else wl.eta
         alpha = inp.get("alpha_t")
+        ds = inp.get("doc_start")
         with nvtx("gradlev forward scan"):
             gl.forward_scan(inp["x"], inp["g_hat"], inp["W0"], eta, y=o["y"], workspace=self.ws,
-                            alpha=alpha)
+                            alpha=alpha, doc_start=ds)
         if events is not None:
             events[1].record()
         with nvtx("gradlev costate scan"):
             gl.costate_scan(inp["x"], inp["g_hat"], inp["W0"], eta, inp["g_out"], g_in=o["g_in"],
-                            workspace=self.ws, alpha=alpha)
+                            workspace=self.ws, alpha=alpha, doc_start=ds)
         if events is not None:
             events[2].record()
 
@@ -233,7 +249,12 @@ class LinearJob:
     def e2e_inputs(self, host, dev, sl, first):
         out = []
         for k in self.in_keys:
-            if k == "W0":
+            if k == "doc_start":  # [B, T]: whole with layer chunks, rows with batch chunks
+                if sl[0] == "B":
+                    out.append((k, host[k][sl[1]:sl[2]], dev[k][sl[1]:sl[2]]))
+                elif first:
+                    out.append((k, host[k], dev[k]))
+            elif k == "W0":
                 if sl[0] == "L":
                     out.append((k, host[k][sl[1]:sl[2]], dev[k][sl[1]:sl[2]]))
                 elif first:
@@ -249,12 +270,15 @@ class LinearJob:
         gl, wl = self.gl, self.wl
         cut = lambda t: self._cut(t, sl)
         w0 = dev["W0"][sl[1]:sl[2]] if sl[0] == "L" else dev["W0"]
-        eta = cut(dev["eta_t"]) if self.gates else wl.eta
+        eta = cut(dev["eta_t"]) if self.gates in ("eta", "alpha") else wl.eta
         alpha = cut(dev["alpha_t"]) if self.gates == "alpha" else None
+        ds = None
+        if self.gates == "docs":
+            ds = dev["doc_start"][sl[1]:sl[2]] if sl[0] == "B" else dev["doc_start"]
         gl.forward_scan(cut(dev["x"]), cut(dev["g_hat"]), w0, eta, y=cut(self.outs["y"]),
-                        workspace=ws, alpha=alpha)
+                        workspace=ws, alpha=alpha, doc_start=ds)
         gl.costate_scan(cut(dev["x"]), cut(dev["g_hat"]), w0, eta, cut(dev["g_out"]),
-                        g_in=cut(self.outs["g_in"]), workspace=ws, alpha=alpha)
+                        g_in=cut(self.outs["g_in"]), workspace=ws, alpha=alpha, doc_start=ds)
 
     def e2e_workspace_bytes(self):
         wl = self.wl
@@ -289,8 +313,10 @@ class LinearJob:
         c = {"L": wl.L, "B": wl.B, "T": wl.T, "H": wl.H, "d_in": wl.d_in, "d_out": wl.d_out,
              "eta": wl.eta}
         if self.gates:
-            c["gates"] = ("per-token eta_t" if self.gates == "eta"
-                          else "per-token eta_t and retention alpha_t (chunked retention kernel)")
+            c["gates"] = {"eta": "per-token eta_t",
+                          "alpha": "per-token eta_t and retention alpha_t (chunked retention kernel)",
+                          "docs": "document resets, documents of 512-1535 tokens, scalar eta "
+                                  "(gate folding + chunked retention kernel)"}[self.gates]
         return c
 
     def oracle_run(self, inp, n_units, cores, t_tokens=None):
@@ -1099,8 +1125,9 @@ def main(argv=None):
     ap.add_argument("--resize", default="",
                     help="comma-separated K=V overrides of the workload's sizes (e.g. L=2), "
                          "for small profiling captures; the headline uses the full workload")
-    ap.add_argument("--gates", default=None, choices=["eta", "alpha"],
-                    help="time the gated scans of Eq. 2: per-token eta_t, or eta_t with retention")
+    ap.add_argument("--gates", default=None, choices=["eta", "alpha", "docs"],
+                    help="time the gated scans of Eq. 2: per-token eta_t, eta_t with retention, "
+                         "or document resets of packed sequences")
     ap.add_argument("--grads", action="store_true",
                     help="time the step-size gradients of both reads (suffix reads) instead")
     ap.add_argument("--no-e2e", action="store_true")

@@ -241,7 +241,9 @@ def _document_gates(doc_start, x5, eta, alpha):
         ds = ds.unsqueeze(0)
     if tuple(ds.shape) != (B, T):
         raise ValueError(f"doc_start must be [B, T] = {(B, T)}, got {tuple(ds.shape)}")
-    ds = (ds != 0).to(torch.uint8).contiguous()
+    if ds.dtype != torch.uint8:
+        ds = (ds != 0).to(torch.uint8)
+    ds = ds.contiguous()
     shape = (L, B, T, H)
 
     def per_token(v):
