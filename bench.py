@@ -151,6 +151,30 @@ def _bytes(*ts):
     return sum(t.numel() * t.element_size() for t in ts)
 
 
+def make_gates(wl, gates, device):
+    """Synthetic gates of the gated modes, drawn once: per-token eta_t in [0, 2 eta]
+    and, for "alpha", retention alpha_t in [0.9, 1] (fp32 [L, B, T, H]); for "docs",
+    document starts per batch row (uint8 [B, T]) with documents of 512 to 1535 tokens
+    and the scalar eta."""
+    gen = torch.Generator()
+    gen.manual_seed(wl.seed * 1000 + 17)
+    out = {}
+    shape = (wl.L, wl.B, wl.T, wl.H)
+    if gates in ("eta", "alpha"):
+        out["eta_t"] = (torch.rand(shape, generator=gen) * (2 * wl.eta)).to(device)
+        if gates == "alpha":
+            out["alpha_t"] = (0.9 + 0.1 * torch.rand(shape, generator=gen)).to(device)
+    elif gates == "docs":
+        ds = torch.zeros(wl.B, wl.T, dtype=torch.uint8)
+        for b in range(wl.B):
+            t = int(torch.randint(512, 1536, (1,), generator=gen))
+            while t < wl.T:
+                ds[b, t] = 1
+                t += int(torch.randint(512, 1536, (1,), generator=gen))
+        out["doc_start"] = ds.to(device)
+    return out
+
+
 class LinearJob:
     """One fast-weight linear map per (layer, batch, head) unit: the forward scan
     (Eq. 3) and the costate scan (Eq. 4), one library call each."""
@@ -162,33 +186,13 @@ class LinearJob:
         self.inp = W.make_linear(wl.resized(seed=wl.seed + 1000 * rank), device=device)
         self.outs = {"y": torch.empty_like(self.inp["g_hat"]),
                      "g_in": torch.empty_like(self.inp["x"])}
-        # Gated scans (Eq. 2): per-token eta_t in [0, 2 eta] and, for "alpha",
-        # retention alpha_t in [0.9, 1]; tensors [L, B, T, H] drawn once.  "docs":
-        # the scalar eta with document starts per batch row (packed documents of
-        # 512 to 1535 tokens), folded into the gates by the library every call.
+        # Gated scans (Eq. 2) and document resets, inputs from make_gates; the
+        # library folds document starts into the gates on every call.
         self.gates = gates
-        self.eta_t = self.alpha_t = None
         code = 1 if wl.dtype == "bf16" else 0
         nb = gl.workspace_bytes(wl.L, wl.B, wl.T, wl.H, wl.d_in, wl.d_out, code)
-        if gates == "docs":
-            gen = torch.Generator()
-            gen.manual_seed(wl.seed * 1000 + 19)
-            ds = torch.zeros(wl.B, wl.T, dtype=torch.uint8)
-            for b in range(wl.B):
-                t = int(torch.randint(512, 1536, (1,), generator=gen))
-                while t < wl.T:
-                    ds[b, t] = 1
-                    t += int(torch.randint(512, 1536, (1,), generator=gen))
-            self.inp["doc_start"] = ds.to(device)
-        elif gates:
-            gen = torch.Generator(device=device)
-            gen.manual_seed(wl.seed * 1000 + 17)
-            shape = (wl.L, wl.B, wl.T, wl.H)
-            self.eta_t = torch.rand(shape, generator=gen, device=device) * (2 * wl.eta)
-            if gates == "alpha":
-                self.alpha_t = 0.9 + 0.1 * torch.rand(shape, generator=gen, device=device)
-                self.inp["alpha_t"] = self.alpha_t
-            self.inp["eta_t"] = self.eta_t
+        self.inp.update(make_gates(wl, gates, device))
+        self.eta_t, self.alpha_t = self.inp.get("eta_t"), self.inp.get("alpha_t")
         if gates:
             from paper_2609_34174_gb300 import _binding as _B
             d = _B._Desc(wl.L, wl.B, wl.T, wl.H, wl.d_in, wl.d_out, code, 0)
@@ -330,8 +334,30 @@ class LinearJob:
         g = W.units_fp64(inp["g_hat"], units)
         w0 = W.w0_fp64(inp["W0"], units)
         go = W.units_fp64(inp["g_out"], units)
-        t = time.perf_counter()
-        oracle.linear_scan(x, g, w0, wl.eta, gout=go, nthreads=cores)
+        gates = getattr(self, "gates", None)
+        if not gates:
+            t = time.perf_counter()
+            oracle.linear_scan(x, g, w0, wl.eta, gout=go, nthreads=cores)
+        else:
+            # every unit with its own gate sequences: one oracle call per unit, the
+            # calls spread over the cores (the C oracle releases the interpreter)
+            import concurrent.futures as cf
+            f64 = lambda t_: t_.detach().to("cpu", torch.float64).numpy()
+            if gates == "docs":
+                ds = inp["doc_start"].cpu().numpy() != 0
+                calls = [(oracle.linear_scan_docs, (x[i:i + 1], g[i:i + 1], w0[i], wl.eta,
+                                                    ds[b][None]), {"gout": go[i:i + 1]})
+                         for i, (l, b, h) in enumerate(units)]
+            else:
+                calls = [(oracle.linear_scan,
+                          (x[i:i + 1], g[i:i + 1], w0[i], f64(inp["eta_t"][l, b, :, h])),
+                          {"gout": go[i:i + 1], "nthreads": 1,
+                           "alpha": (f64(inp["alpha_t"][l, b, :, h]) if "alpha_t" in inp
+                                     else None)})
+                         for i, (l, b, h) in enumerate(units)]
+            t = time.perf_counter()
+            with cf.ThreadPoolExecutor(max_workers=cores) as ex:
+                list(ex.map(lambda c: c[0](*c[1], **c[2]), calls))
         # one metric token spans all H heads of a layer
         return time.perf_counter() - t, len(units) * wl.T / wl.H
 
@@ -339,8 +365,11 @@ class LinearJob:
         return self.wl.L * self.wl.B * self.wl.H
 
     def sample_text(self, n):
+        gates = getattr(self, "gates", None)
+        with_gates = {None: "", "eta": ", with their eta_t", "alpha": ", with their eta_t and alpha_t",
+                      "docs": ", one learner per document"}[gates]
         return (f"{n} of {self.n_units()} (layer, batch, head) units at full T={self.wl.T}, "
-                f"forward and costate reads in one sequential walk per unit, fp64")
+                f"forward and costate reads in one sequential walk per unit{with_gates}, fp64")
 
 
 class GradsJob(LinearJob):
@@ -745,6 +774,7 @@ def run_reference(args, wl, rank, world):
     oracle.build()
     cores = len(os.sched_getaffinity(0))
     metric = METRIC
+    job_cfg = {}
     if args.workload == "decode_mlp":
         inp = W.make_mlp(wl, device="cpu")
         f = lambda t, T: t[:, :T].to(torch.float64).numpy()
@@ -786,10 +816,12 @@ def run_reference(args, wl, rank, world):
         inp = W.make_linear(wl, device="cpu")
         job = LinearJob.__new__(LinearJob)
         job.wl = wl
+        job.gates = args.gates
+        inp.update(make_gates(wl, args.gates, "cpu"))
         n = min(job.n_units(), max(cores, 2 * cores))
         run = lambda: job.oracle_run(inp, n, cores)
-        sample = (f"{n} of {job.n_units()} (layer, batch, head) units at full T={wl.T} per step, "
-                  f"fp64 sequential walk")
+        sample = job.sample_text(n) + " per step"
+        job_cfg = job.config()
     for _ in range(args.warmup):
         run()
     sec = 0.0
@@ -803,7 +835,7 @@ def run_reference(args, wl, rank, world):
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(sec / args.steps * 1e3, 3), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": f"{args.workload}: {wl.name}", "sample": sample},
+            "config": {"workload": f"{args.workload}: {wl.name}", **job_cfg, "sample": sample},
             "cpu_baseline": {"value": round(value, 1), "unit": UNIT, "cores": cores,
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0,

@@ -37,6 +37,19 @@ def test_reference_line_small_workload(extra, metric):
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
 
 
+@pytest.mark.parametrize("extra,words", [
+    (["--gates", "alpha"], "eta_t and alpha_t"),
+    (["--gates", "docs", "--resize", "T=3000"], "one learner per document"),
+], ids=["retention", "documents"])
+def test_reference_line_gated(extra, words):
+    """The gated modes time the oracle on the gated workload itself: each unit with
+    its own gate sequences, or one learner per document."""
+    d = _line(["--impl", "reference", "--workload", "c1", "--steps", "1", "--warmup", "3"] + extra)
+    assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["value"] > 0
+    assert words in d["cpu_baseline"]["sample"]
+    assert d["config"]["gates"]
+
+
 def test_reference_line_deployment():
     d = _line(["--impl", "reference", "--workload", "decode_mlp", "--steps", "1", "--warmup", "3"])
     assert d["impl"] == "reference" and d["metric"] == bench.DECODE_METRIC
