@@ -167,9 +167,10 @@ int oracle_linear_batch(int U, int T, int d, int m, const double* x, const doubl
  *   writes (online-update, with the proposals as the written costates):
  *     W1 <- W10 + alpha (W1 - W10) - eta1_t ghz_t x_t^T
  *     W2 <- W20 + alpha (W2 - W20) - eta2_t ghy_t h_t^T
- * Deployment (Sec. 3, training objective paragraph; Appendix A: after each scored
- * target the learner writes true costates): with ghz NULL layer 1 writes its
- * reconstructed gz_t, and with ghy NULL layer 2 writes gout_t.  Either needs gout.
+ * Deployment (Sec. 3, training objective paragraph; Appendix A: once a target is
+ * scored, the maps are written with actual costates, not proposals): with ghz
+ * NULL layer 1 writes its reconstructed gz_t, and with ghy NULL layer 2 writes
+ * gout_t.  Either needs gout.
  * Widths: input d, hidden m, output k (Appendix A has k = d; Sec. 4.1 uses 4->7->3).
  * Shapes: x [T][d], ghz [T][m], ghy [T][k], W10 [m][d], W20 [k][m], gout [T][k].
  * Outputs (each nullable): z, h [T][m]; y [T][k]; gh, gz [T][m]; gx [T][d].

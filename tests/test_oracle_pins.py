@@ -430,8 +430,8 @@ def test_activation_values():
 # -------------------------------------------------------------- deployment
 @pytest.mark.parametrize("seed", [17, 42])
 def test_mlp_deploy_matches_serial_learner(seed):
-    """Deployment writes true costates (Sec. 3; Appendix A): layer 2 writes the
-    supplied gout_t and layer 1 its own reconstructed gz_t.  The hand-written serial
+    """Deployment (Sec. 3; Appendix A) writes actual costates, not proposals: layer 2
+    writes the supplied gout_t and layer 1 its own reconstructed gz_t.  The hand-written serial
     learner of Sec. 4.1 does exactly that, so the deployed oracle reproduces it."""
     p = _e1_serial(seed)
     o = oracle.mlp_deploy(p["x"][None], p["W10"], p["W20"], p["eta1"], p["eta2"],
