@@ -175,9 +175,10 @@ int gradlev_costate_scan_gated(const gradlev_desc* desc, const gradlev_tensor* x
 
 /*
  * gradlev_document_gates -- gate arrays for sequences packed from several
- * documents.  A read excludes every write made before the most recent document
- * start (Appendix C, scan reads; Appendix E, packed rows).  In the gates of Eq. 2
- * a document starting at token s > 0 is alpha = 0 and eta = 0 at token s - 1:
+ * documents.  A read sees only the writes of its own document, those since the
+ * latest document start (Appendix C, scan reads; Appendix E, packed rows).  In
+ * the gates of Eq. 2 a document starting at token s > 0 is alpha = 0 and eta = 0
+ * at token s - 1:
  * the fast weights return to W0 and the previous document's last write (seen by
  * none of its reads) is dropped, so the read at s sees W0.  The outputs feed
  * gradlev_forward_scan_gated / gradlev_costate_scan_gated.

@@ -126,7 +126,7 @@ def linear_scan(x, ghat, W0, eta, alpha=None, gout=None, want_y=True, nthreads=0
 
 def linear_scan_docs(x, ghat, W0, eta, doc_start, alpha=None, gout=None):
     """Document resets (Appendix C, scan reads; Appendix E, packed documents): every
-    read excludes the writes made before the most recent document start, so each
+    read sees only the writes of its own document (since the latest start), so each
     document is its own sequential learner starting from W0.
 
     doc_start [U,T] booleans, True where a document begins (token 0 always begins

@@ -269,7 +269,7 @@ def _document_gates(doc_start, x5, eta, alpha):
 
 def document_gates(doc_start, x, eta, alpha=None):
     """Per-token gates for sequences packed from several documents (Appendix C:
-    a read excludes every write before the most recent document start; Appendix E).
+    a read sees only the writes of its own document; Appendix E).
 
     doc_start: bool / integer [B, T] (or [T] when B = 1), nonzero where a document
     begins, the same for every layer and head.  eta: scalar or per-token tensor;

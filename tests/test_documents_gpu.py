@@ -1,7 +1,7 @@
 """GPU parity of document resets for packed sequences against the fp64 oracle's
 per-document learners.
 
-A read excludes every write made before the most recent document start
+A read sees only the writes of its own document, those since the latest start
 (Appendix C, scan reads; Appendix E, resets at document boundaries).  On the GPU
 the starts are folded into the gates of Eq. 2 (alpha = eta = 0 on the token
 before each start) and the gated scans run; the oracle instead runs one

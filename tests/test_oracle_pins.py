@@ -100,9 +100,8 @@ def _doc_starts(T, cuts):
 
 @pytest.mark.parametrize("gated", [False, True])
 def test_documents_closed_form(gated):
-    """Each read sees W0 plus the writes of its own document only (Appendix C: a read
-    excludes all writes before the most recent document start), checked against the
-    closed form of Eq. 2 over that document's tokens."""
+    """Each read sees W0 plus the writes of its own document only (Appendix C, scan
+    reads), checked against the closed form of Eq. 2 over that document's tokens."""
     T, cuts = 13, (1, 5, 6, 10)
     x, ghat, W0, gout = _rand_problem(400 + gated, 1, T, 4, 3)
     r = _rng(401)
