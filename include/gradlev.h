@@ -3,8 +3,8 @@
  *
  * GradLev (Token-Parallel Test-Time Training via Costate Prediction) turns
  * token-by-token online gradient descent on a fast-weight matrix into two
- * associative scans once the per-token costates are supplied (Sec. 3,
- * "Observation: known costates expose exact scans").  With slow weights W0
+ * associative scans once the per-token costates are supplied (Sec. 3, the
+ * "Observation" paragraph).  With slow weights W0
  * (d_out x d_in), a step size eta and proposals ghat_t, the adapted weights
  * before token t are (Eq. 2 with unit retention, Eq. 3)
  *
