@@ -50,3 +50,24 @@ def test_mlp_shapes():
     assert t["g_hat_y"].shape == (1, 16, 512) and t["g_out"].shape == (1, 16, 512)
     assert t["W1"].shape == (2048, 512) and t["W2"].shape == (512, 2048)
     assert abs(t["W1"].std().item() - math.sqrt(2 / 2560)) < 1e-3
+
+
+def test_bench_gate_recipe():
+    """The gated bench modes' synthetic gates: eta_t in [0, 2 eta], alpha_t in
+    [0.9, 1], document starts with every document 512 to 1535 tokens long (the last
+    one cut by T), the same on every call."""
+    import bench
+    wl = W.workload("c5").resized(L=2, B=3, H=2, T=5000)
+    g = bench.make_gates(wl, "alpha", "cpu")
+    assert g["eta_t"].shape == (2, 3, 5000, 2) and g["alpha_t"].shape == (2, 3, 5000, 2)
+    assert float(g["eta_t"].min()) >= 0 and float(g["eta_t"].max()) <= 2 * wl.eta
+    assert float(g["alpha_t"].min()) >= 0.9 and float(g["alpha_t"].max()) <= 1.0
+    d = bench.make_gates(wl, "docs", "cpu")["doc_start"]
+    assert d.shape == (3, 5000) and d.dtype == torch.uint8
+    for b in range(3):
+        starts = [0] + torch.nonzero(d[b]).flatten().tolist()
+        assert d[b, 0] == 0 and len(starts) >= 4
+        lengths = [b2 - a for a, b2 in zip(starts[:-1], starts[1:])]
+        assert all(512 <= n <= 1535 for n in lengths)
+    assert torch.equal(d, bench.make_gates(wl, "docs", "cpu")["doc_start"])
+    assert bench.make_gates(wl, None, "cpu") == {}
