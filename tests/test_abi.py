@@ -169,3 +169,26 @@ def test_decode_workspace_sizes(lib):
     d = _desc(B=2, T=1, d_in=1024, d_out=4096)
     assert lib.gradlev_decode_workspace_bytes(ctypes.byref(d)) == 2 * 32 * 1024 * 4 + 256
     assert lib.gradlev_decode_workspace_bytes(ctypes.byref(_desc(T=3))) == 0
+
+
+def test_document_gates_arguments_rejected_before_launch(lib):
+    """gradlev_document_gates validates everything before it launches: these calls
+    return without touching a device."""
+    P = ctypes.c_void_p
+    ok_ptr = P(0x10000)
+    d = _desc(L=1, B=2, T=8, H=3)
+    call = lambda desc, ds, eta, et, at, eo, ao: lib.gradlev_document_gates(
+        desc, ds, eta, et, at, eo, ao, None)
+    assert call(None, ok_ptr, 0.1, None, None, ok_ptr, ok_ptr) == -1           # no descriptor
+    assert call(ctypes.byref(_desc(reserved=1)), ok_ptr, 0.1, None, None, ok_ptr, ok_ptr) == -1
+    assert call(ctypes.byref(_desc(T=-1)), ok_ptr, 0.1, None, None, ok_ptr, ok_ptr) == -1
+    assert call(ctypes.byref(d), None, 0.1, None, None, ok_ptr, ok_ptr) == -1  # no starts
+    assert call(ctypes.byref(d), ok_ptr, 0.1, None, None, None, ok_ptr) == -1  # no eta_out
+    assert call(ctypes.byref(d), ok_ptr, 0.1, None, None, ok_ptr, None) == -1  # no alpha_out
+    assert call(ctypes.byref(d), ok_ptr, float("nan"), None, None, ok_ptr, ok_ptr) == -1
+    assert call(ctypes.byref(d), ok_ptr, float("inf"), None, None, ok_ptr, ok_ptr) == -1
+    assert call(ctypes.byref(d), ok_ptr, 0.1, P(0x10002), None, ok_ptr, ok_ptr) == -1  # misaligned
+    assert call(ctypes.byref(d), ok_ptr, 0.1, None, None, ok_ptr, P(0x10001)) == -1
+    # nothing to do: OK with no pointers at all
+    assert call(ctypes.byref(_desc(T=0)), None, float("nan"), None, None, None, None) == 0
+    assert call(ctypes.byref(_desc(H=0)), None, 0.1, None, None, None, None) == 0
