@@ -519,3 +519,32 @@ def test_eta_gradient_of_costate_read_is_a_suffix_read():
     rs = oracle.suffix_scan(gh, go, w)[0]
     an = -np.sum(x[0] * rs, axis=1)
     assert np.abs(fd - an).max() < 1e-7 * max(1.0, np.abs(an).max())
+
+
+def test_gated_learner_property_sweep():
+    """Random shapes and gates (zeros, negative retention, document cuts) against the
+    closed form of Eq. 2, restricted to each document."""
+    hyp = pytest.importorskip("hypothesis")
+    st = pytest.importorskip("hypothesis.strategies")
+
+    @hyp.settings(max_examples=60, deadline=None, derandomize=True)
+    @hyp.given(T=st.integers(1, 12), d=st.integers(1, 5), m=st.integers(1, 5),
+               seed=st.integers(0, 10_000), n_cuts=st.integers(0, 3))
+    def check(T, d, m, seed, n_cuts):
+        r = _rng(seed)
+        x, ghat, W0, gout = _rand_problem(seed, 1, T, d, m)
+        eta = r.uniform(0.0, 0.6, T)
+        alpha = r.uniform(-1.0, 1.0, T)
+        alpha[r.random(T) < 0.25] = 0.0
+        cuts = sorted(set(int(c) for c in r.integers(1, max(T, 2), n_cuts) if 0 < c < T))
+        y, gin = oracle.linear_scan_docs(x, ghat, W0, eta, _doc_starts(T, cuts), alpha=alpha,
+                                         gout=gout)
+        bounds = [0, *cuts, T]
+        for a, b in zip(bounds[:-1], bounds[1:]):
+            for t in range(a, b):
+                W_t = W0[0] + _closed_form_delta(t - a, x[0, a:b], ghat[0, a:b], eta[a:b],
+                                                 alpha[a:b])
+                np.testing.assert_allclose(y[0, t], W_t @ x[0, t], rtol=0, atol=1e-13)
+                np.testing.assert_allclose(gin[0, t], W_t.T @ gout[0, t], rtol=0, atol=1e-13)
+
+    check()
