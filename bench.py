@@ -1064,6 +1064,32 @@ def decode_cpu_baseline(wl, inp, target_s=12.0):
             "sample": f"{wl.B} sequences x first {T} tokens of the deployed MLP, fp64"}
 
 
+def side_scans(gl, key, device, steps=20, warmup=3):
+    """Per-scan times and rooflines of another linear workload at its full size,
+    timed like the headline (CUDA events on the launching stream, inputs larger
+    than L2), so that one default run also records it."""
+    job = make_job(gl, W.workload(key), device, 0)
+    for _ in range(warmup):
+        job.step()
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for i in range(steps):
+        job.step(events=ev[i])
+    torch.cuda.synchronize()
+    if gl.workspace_status(job.ws) != 0:
+        raise RuntimeError("device-side timeout reported by the scan kernels")
+    pk = peaks()
+    out = {"workload": f"{key}: {job.wl.name}", "steps": steps}
+    for name, a, b in (("fwd", 0, 1), ("costate", 1, 2)):
+        ms = sum(e[a].elapsed_time(e[b]) for e in ev) / steps
+        fl, nb = job.counts(name)
+        out[name] = {"ms": round(ms, 4), "tokens_per_s": round(job.tokens / (ms / 1e3), 1),
+                     "roofline": roofline_entry(fl, nb, ms / 1e3, pk)}
+    del job
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_gradlev(args, wl, rank, world, local_rank):
     import paper_2609_34174_gb300 as gl
 
@@ -1138,6 +1164,10 @@ def run_gradlev(args, wl, rank, world, local_rank):
             "clocks": sampler.summary(), "gpu_launches": job.launches_per_step * args.steps}
     if rank == 0 and world == 1 and not args.no_e2e:
         line["e2e"] = e2e_measure(job, max(3, min(args.steps, 20)), stream)
+    if (rank == 0 and world == 1 and args.workload == "c5" and not
+            (args.gates or args.grads or args.no_side)):
+        # the long-context workload, the other one with a roofline target
+        line["also"] = {"c4": side_scans(gl, "c4", device)}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
 
@@ -1163,6 +1193,8 @@ def main(argv=None):
     ap.add_argument("--grads", action="store_true",
                     help="time the step-size gradients of both reads (suffix reads) instead")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-side", action="store_true",
+                    help="skip the long-context (c4) scans added to the default line")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args(argv)
     if args.warmup < 3:

@@ -111,7 +111,10 @@ typedef struct {
  *   x        [L][B][T][H][d_in]   layer inputs x_t (read)
  *   g_hat    [L][B][T][H][d_out]  costate proposals ghat_t: the writes (read)
  *   W0       [L][H][d_out][d_in]  fp32 slow weights (read)
- *   eta      step size of every write (finite; 0 gives y = W0 x)
+ *   eta      step size of every write (finite; 0 gives y = W0 x).  On the tensor
+ *            cores the running state is kept in units of -eta, so |eta| must lie
+ *            in [2^-64, 2^64] there; any other finite eta runs on the CUDA-core
+ *            kernel (exact fp32 FMA, slower), with the same results.
  *   act      activation applied for act_out (GRADLEV_ACT_NONE: act_out unused)
  *   y        [L][B][T][H][d_out]  out: y_t = What_t x_t (pre-activation)
  *   act_out  [L][B][T][H][d_out]  optional out (data NULL to skip): sigma(y_t)
@@ -326,12 +329,23 @@ size_t gradlev_eta_grad_workspace_bytes(const gradlev_desc* desc, int read);
  *   - All calls on a device share the array and it keeps the last call's
  *     contents; each call clears what must start at zero on its own stream.
  *     Calls that may overlap on the GPU race on it and must not be issued.
- *   - gradlev_workspace_status does not apply (there is no caller workspace).
+ *   - The size check is against the forward scan's own scratch need.
+ *   - A timed-out device wait is reported by
+ *     gradlev_forward_scan_noalloc_status, not gradlev_workspace_status (there
+ *     is no caller workspace).
+ *   - The looked-up address is cached per device for the life of the process;
+ *     do not use this entry point on a device after cudaDeviceReset.
  */
 int gradlev_forward_scan_noalloc(const gradlev_desc* desc, const gradlev_tensor* x,
                                  const gradlev_tensor* g_hat, const float* W0, float eta, int act,
                                  const gradlev_tensor* y, const gradlev_tensor* act_out,
                                  gradlev_stream_t stream);
+
+/* Waits for `stream`, then reads the status word that the last
+ * gradlev_forward_scan_noalloc on the current device left in the library's
+ * array: GRADLEV_OK, GRADLEV_ERR_TIMEOUT if a bounded device wait expired (that
+ * call's outputs are then undefined), or GRADLEV_ERR_CUDA.  Allocates nothing. */
+int gradlev_forward_scan_noalloc_status(gradlev_stream_t stream);
 
 /* Bytes of workspace either scan needs for this shape (the same bound serves
  * both).  Returns 0 for an invalid descriptor. */

@@ -200,6 +200,16 @@ bool tc_shape_ok(const gradlev_desc& d, int dq, int dv) {
     return d.dtype == GRADLEV_BF16 && (dq == 64 || dq == 128) && dv % 64 == 0 && dv > 0;
 }
 
+// The chunk kernel keeps its running state in units of lambda = -eta (it holds
+// S / lambda, so that the masked score needs no scaling and the output is
+// multiplied by lambda once).  That needs 1 / lambda and W0 / lambda to stay
+// well inside fp32: |eta| within [2^-64, 2^64] (or eta = 0, which keeps lambda = 1).
+// Any other finite eta runs on the CUDA-core kernel, which scales by eta directly.
+bool tc_eta_ok(float eta) {
+    const float a = fabsf(eta);
+    return eta == 0.0f || (a >= 0x1p-64f && a <= 0x1p64f);
+}
+
 constexpr int kSimtMaxDq = 256;
 
 bool simt_shape_ok(const gradlev_desc& d, int dq) {
@@ -332,7 +342,7 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
     const Tok& tv = costate ? tx : tg;
     const int elem = d.dtype == GRADLEV_BF16 ? 2 : 4;
 
-    if (tc_shape_ok(d, dq, dv) && tc_layout_ok(tq, 2) && tc_layout_ok(tk, 2) &&
+    if (tc_shape_ok(d, dq, dv) && tc_eta_ok(eta) && tc_layout_ok(tq, 2) && tc_layout_ok(tk, 2) &&
         tc_layout_ok(tv, 2) && tc_layout_ok(to, 2) && tc_layout_ok(to2, 2) && tc_layout_ok(tz, 2)) {
         Plan pl = plan_tc(d, dq, dv, dev.sms);
         if (!ws || ws_bytes < pl.ws_bytes) return GRADLEV_ERR_WORKSPACE;
@@ -930,6 +940,17 @@ int run_decode_write(const gradlev_desc* desc, const gradlev_tensor* x, const gr
 }
 
 }  // namespace
+
+namespace gl {
+// Workspace bytes of the forward scan alone (gradlev_workspace_bytes covers both
+// directions).  0 for an invalid descriptor.
+size_t forward_workspace_bytes(const gradlev_desc* desc) {
+    if (!desc_ok(desc)) return 0;
+    DevInfo dev;
+    const int sms = device_info(&dev) ? dev.sms : 160;
+    return ws_bytes_for(*desc, desc->d_in, desc->d_out, sms);
+}
+}  // namespace gl
 
 extern "C" {
 

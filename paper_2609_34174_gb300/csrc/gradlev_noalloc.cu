@@ -16,11 +16,19 @@
 // caller's stream.  Calls that could overlap on the GPU (different streams, or
 // different host threads on the same device without ordering) race on the
 // array and must not be issued.
+//
+// A bounded device-side wait that expires leaves its error bit in the array's
+// status word, as it would in a caller workspace; gradlev_forward_scan_noalloc_status
+// reads it back.
 #include <cuda_runtime.h>
 
 #include <mutex>
 
 #include "../../include/gradlev.h"
+
+namespace gl {
+size_t forward_workspace_bytes(const gradlev_desc* desc);
+}
 
 namespace {
 
@@ -31,6 +39,8 @@ constexpr int kMaxDevices = 64;
 // Device address of the array on the current device.  Host code cannot use the
 // symbol itself (on the host it names a stand-in, not device memory), so the
 // address is looked up once per device, with that device current, and cached.
+// The cache outlives a cudaDeviceReset, after which the address is stale: the
+// entry point is not for processes that reset a device they have called it on.
 void* scratch_on_current_device() {
     static void* addr[kMaxDevices] = {};
     static std::mutex mu;
@@ -52,11 +62,25 @@ extern "C" int gradlev_forward_scan_noalloc(const gradlev_desc* desc, const grad
                                             float eta, int act, const gradlev_tensor* y,
                                             const gradlev_tensor* act_out,
                                             gradlev_stream_t stream) {
-    const size_t need = gradlev_workspace_bytes(desc);
+    // the forward scan's own need (gradlev_workspace_bytes is the larger of
+    // both directions, which would reject forward shapes that fit)
+    const size_t need = gl::forward_workspace_bytes(desc);
     if (need == 0) return GRADLEV_ERR_INVALID_ARG;
     if (need > (size_t)GRADLEV_NOALLOC_SCRATCH_BYTES) return GRADLEV_ERR_WORKSPACE;
     void* scratch = scratch_on_current_device();
     if (!scratch) return GRADLEV_ERR_CUDA;
     return gradlev_forward_scan(desc, x, g_hat, W0, eta, act, y, act_out, scratch,
                                 (size_t)GRADLEV_NOALLOC_SCRATCH_BYTES, stream);
+}
+
+extern "C" int gradlev_forward_scan_noalloc_status(gradlev_stream_t stream) {
+    // Word 1 of the scratch is the status word the kernels set when a bounded
+    // wait expires (the same layout as a caller workspace).
+    unsigned int word = 0;
+    if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return GRADLEV_ERR_CUDA;
+    if (cudaMemcpyFromSymbol(&word, g_noalloc_scratch, sizeof(word), sizeof(unsigned int),
+                             cudaMemcpyDeviceToHost) != cudaSuccess)
+        return GRADLEV_ERR_CUDA;
+    return word == 0 ? GRADLEV_OK : GRADLEV_ERR_TIMEOUT;
 }

@@ -15,7 +15,7 @@ import pytest
 import torch
 
 import oracle
-from parity_util import TOL, rel_l2
+from parity_util import TOL, assert_parity, rel_l2
 
 gl = pytest.importorskip("paper_2609_34174_gb300")
 
@@ -87,9 +87,10 @@ def test_decode_linear_matches_oracle(case):
     yr, gr = oracle.linear_scan(xu, gu, wu, eta_t, alpha=alpha_t, gout=gu)
     yg = np.stack([_f64(y[l, b, :, h]) for (l, b, h) in units])
     gg = np.stack([_f64(gin[l, b, :, h]) for (l, b, h) in units])
-    tol = TOL["bf16"] if dtype == torch.bfloat16 else TOL["f32"]
-    assert rel_l2(yg, yr) <= tol, f"y rel-L2 {rel_l2(yg, yr):.3e}"
-    assert rel_l2(gg, gr) <= tol, f"g_in rel-L2 {rel_l2(gg, gr):.3e}"
+    key = "bf16" if dtype == torch.bfloat16 else "f32"
+    tol = TOL[key]
+    assert_parity(f"{case} y", yg, yr, key)
+    assert_parity(f"{case} g_in", gg, gr, key)
     # the fast weights matter: the slow-only reads differ by far more than the tolerance
     y0, _ = oracle.linear_scan(xu, gu, wu, 0.0)
     assert rel_l2(y0, yr) > 5 * tol
@@ -105,8 +106,8 @@ def test_decode_per_unit_step_sizes():
         yr, gr = oracle.linear_scan(_f64(x[l, b, :, h])[None], _f64(g[l, b, :, h])[None],
                                     _f64(W0[l, h]), float(eta_u[l, b, h]),
                                     gout=_f64(g[l, b, :, h])[None])
-        assert rel_l2(_f64(y[l, b, :, h]), yr[0]) <= TOL["f32"]
-        assert rel_l2(_f64(gin[l, b, :, h]), gr[0]) <= TOL["f32"]
+        assert_parity(f"unit {i} y", _f64(y[l, b, :, h])[None], yr, "f32")
+        assert_parity(f"unit {i} g_in", _f64(gin[l, b, :, h])[None], gr, "f32")
 
 
 def test_decode_write_is_reproducible():
@@ -163,5 +164,4 @@ def test_decode_mlp_deployment(shape):
     ref = oracle.mlp_deploy(_f64(x), _f64(W1), _f64(W2), eta1, eta2, gout=_f64(gout),
                             act=oracle.ACT_GELU_TANH)
     for key in ("z", "h", "y", "gz"):
-        err = rel_l2(out[key], ref[key])
-        assert err <= TOL["bf16"], f"{key}: rel-L2 {err:.3e}"
+        assert_parity(key, out[key], ref[key], "bf16")

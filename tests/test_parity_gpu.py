@@ -11,7 +11,8 @@ import torch
 
 import oracle
 import workloads as W
-from parity_util import TOL, all_units, gpu_units, oracle_linear, rel_l2, to_device
+from parity_util import (TOL, all_units, assert_parity, check_all_units_by_layer, gpu_units,
+                         oracle_linear, to_device)
 
 gl = pytest.importorskip("paper_2609_34174_gb300")
 
@@ -29,10 +30,10 @@ def _run_linear(wl, inputs, units=None, check_units=None):
 
 
 def _assert_close(name, out, ref, tol):
-    err = rel_l2(out, ref)
-    assert np.isfinite(out).all(), f"{name}: non-finite output"
-    assert err <= tol, f"{name}: rel-L2 {err:.3e} > {tol:.1e}"
-    return err
+    """Whole-output, per-unit and per-row bounds (parity_util.Parity); out and
+    ref [U, T, w]."""
+    key = "f32" if tol == TOL["f32"] else "bf16"
+    return assert_parity(name, out, ref, key)["rel_l2"]
 
 
 # ---------------------------------------------------------------- fp32 path
@@ -109,6 +110,23 @@ def test_degenerate_plain_gemm(which):
     yr, gr = oracle_linear(inputs, units, eta)
     _assert_close("degenerate forward", gpu_units(y, units), yr, TOL["bf16"])
     _assert_close("degenerate costate", gpu_units(gin, units), gr, TOL["bf16"])
+
+
+@pytest.mark.parametrize("eta", [1e-40, 1e-30, -3e-25, 3e20, 0.01], ids=str)
+def test_step_sizes_outside_the_scaled_state_window(eta):
+    """The chunk kernel holds its state in units of -eta; step sizes whose
+    reciprocal (or W0 / eta) would leave fp32 run on the CUDA-core kernel.  Every
+    finite eta, a subnormal one included, matches the oracle."""
+    wl = W.workload("c5").resized(L=1, B=1, H=2, T=300)
+    inputs = W.make_linear(wl)
+    dev = to_device(inputs)
+    y = gl.forward_scan(dev["x"], dev["g_hat"], dev["W0"], eta)
+    gin = gl.costate_scan(dev["x"], dev["g_hat"], dev["W0"], eta, dev["g_out"])
+    torch.cuda.synchronize()
+    units = all_units(wl)
+    yr, gr = oracle_linear(inputs, units, eta)
+    _assert_close(f"eta={eta} forward", gpu_units(y, units), yr, TOL["bf16"])
+    _assert_close(f"eta={eta} costate", gpu_units(gin, units), gr, TOL["bf16"])
 
 
 def test_strided_inputs_and_outputs():
@@ -207,28 +225,20 @@ def test_fused_activation_small_mlp(act):
     _assert_close("mlp g_x", f64(gx), ref["gx"], TOL["bf16"])
 
 
-# ------------------------------------------------ full sizes, sampled units
-FULL = {
-    "c2": [(0, 0, 0), (0, 3, 7)],
-    "c4": [(0, 0, 0), (0, 1, 15)],
-    "c5": [(0, 0, 0), (11, 7, 11), (5, 3, 6)],
-}
-
-
-@pytest.mark.parametrize("key", sorted(FULL))
-def test_full_size_sampled_units(key):
+# ------------------------------------------------ full sizes, every unit
+@pytest.mark.parametrize("key", ["c2", "c4", "c5"])
+def test_full_size_every_unit(key):
     """The workload at its full size, in the launch configuration the bench times,
-    checked on sampled units the oracle computes one by one."""
+    with every unit checked against the oracle: whole output, each unit and each
+    token row (the oracle walks the units one layer at a time)."""
     wl = W.workload(key)
     inputs = W.make_linear(wl, device="cuda")
     y = gl.forward_scan(inputs["x"], inputs["g_hat"], inputs["W0"], wl.eta)
     gin = gl.costate_scan(inputs["x"], inputs["g_hat"], inputs["W0"], wl.eta, inputs["g_out"])
     torch.cuda.synchronize()
-    assert torch.isfinite(y).all() and torch.isfinite(gin).all()
-    units = FULL[key]
-    yr, gr = oracle_linear(inputs, units, wl.eta)
-    _assert_close(f"{key} full forward", gpu_units(y, units), yr, TOL["bf16"])
-    _assert_close(f"{key} full costate", gpu_units(gin, units), gr, TOL["bf16"])
+    res = check_all_units_by_layer(key, wl, inputs, wl.eta, y=y, gin=gin)
+    print(f"{key} every unit: {res}")
+    assert res["forward"]["units"] == wl.units and res["costate"]["units"] == wl.units
 
 
 # ------------------------------------------------ pipeline phase bookkeeping
