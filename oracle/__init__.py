@@ -2,7 +2,8 @@
 
 A plain fp64 CPU implementation of the sequential online learner
 (GradLev Sec. 3, Eqs. 2-4, and the online MLP of Appendix A), written in C
-(``gradlev_oracle.c``) and loaded through ctypes.  Only ``tests/``,
+(``gradlev_oracle.c``) and loaded through ctypes, plus the per-token consistency
+term of the training objective (Eq. 5) written out in numpy.  Only ``tests/``,
 ``__graft_entry__.smoke()`` and the ``cpu_baseline`` / ``--impl reference``
 legs of ``bench.py`` may import this package.  It shares no code with the CUDA
 library and never calls it.
@@ -224,6 +225,21 @@ def suffix_scan(q, k, v, nthreads=0):
     if lib.oracle_suffix_batch(U, T, dq, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(r), int(nthreads)):
         raise MemoryError("oracle_suffix_batch could not allocate scratch")
     return r
+
+
+def consistency(proposal, target):
+    """Per-token consistency term of the training objective (Sec. 3, Eq. 5; Appendix A,
+    eq. consistency): ||ghat_t - gtilde_t||^2 / w for every token, where ghat is a
+    proposed costate, gtilde the costate reconstructed at the same place and w their
+    width.  The objective averages these terms over tokens (and, for an MLP, adds
+    one such term per adapted map).  proposal, target [U,T,w] -> [U,T] in fp64."""
+    p = _f64(proposal)
+    g = _f64(target)
+    if p.shape != g.shape or p.ndim < 1:
+        raise ValueError("consistency: proposal and target shapes differ")
+    w = p.shape[-1]
+    diff = p - g
+    return (diff * diff).sum(axis=-1) / w
 
 
 def act(code, z):

@@ -463,6 +463,47 @@ def test_mlp_deploy_is_the_fixed_point_of_proposals():
         assert np.abs(o[key] - dep[key]).max() < 1e-12, key
 
 
+# ------------------------------------------------- consistency term (Eq. 5)
+def test_consistency_hand_values():
+    """||ghat - gtilde||^2 / w on vectors small enough to add by hand."""
+    p = np.array([[[1.0, 2.0, 3.0, 4.0], [0.5, -0.5, 0.0, 2.0]]])
+    g = np.array([[[0.0, 2.0, 5.0, 4.0], [0.5, 0.5, 0.0, -1.0]]])
+    c = oracle.consistency(p, g)
+    assert c.shape == (1, 2)
+    assert c[0, 0] == (1.0 + 0.0 + 4.0 + 0.0) / 4.0
+    assert c[0, 1] == (0.0 + 1.0 + 0.0 + 9.0) / 4.0
+    assert np.all(oracle.consistency(g, g) == 0.0)
+
+
+def test_consistency_vanishes_at_the_serial_learner():
+    """Theorem 1: with the deployed learner's own costates as proposals, the costates
+    the scans reconstruct equal the proposals, so both terms of the MLP consistency
+    loss (Appendix A) vanish; a proposal perturbed at one token raises the layer-1
+    term there by exactly ||perturbation||^2 / m and leaves every earlier token at 0."""
+    U, T, d, m, k = 2, 10, 5, 7, 3
+    r = _rng(77)
+    x = r.standard_normal((U, T, d))
+    gout = r.standard_normal((U, T, k)) * 0.5
+    W10 = r.standard_normal((m, d)) / np.sqrt(d)
+    W20 = r.standard_normal((k, m)) / np.sqrt(m)
+    eta1, eta2 = 0.3, 0.2
+    dep = oracle.mlp_deploy(x, W10, W20, eta1, eta2, gout=gout, act=oracle.ACT_GELU_TANH)
+    o = oracle.mlp_scan(x, dep["gz"], gout, W10, W20, eta1, eta2, act=oracle.ACT_GELU_TANH,
+                        gout=gout)
+    assert oracle.consistency(dep["gz"], o["gz"]).max() < 1e-28
+    assert oracle.consistency(gout, gout).max() == 0.0
+    t0 = 4
+    bump = np.zeros((U, T, m))
+    bump[:, t0] = r.standard_normal((U, m))
+    o2 = oracle.mlp_scan(x, dep["gz"] + bump, gout, W10, W20, eta1, eta2,
+                         act=oracle.ACT_GELU_TANH, gout=gout)
+    c2 = oracle.consistency(dep["gz"] + bump, o2["gz"])
+    assert c2[:, :t0].max() < 1e-28
+    # token t0's reconstruction reads only writes before t0, so it is unchanged
+    expect = (bump[:, t0] ** 2).sum(axis=-1) / m
+    assert np.allclose(c2[:, t0], expect, rtol=1e-12, atol=0)
+
+
 # ------------------------------------------------------ suffix read (gradients)
 def test_suffix_scan_brute_force():
     """r_s = sum_{t>s} (k_t . q_s) v_t written as the double sum; r_{T-1} = 0."""
