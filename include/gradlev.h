@@ -144,6 +144,36 @@ int gradlev_costate_scan(const gradlev_desc* desc, const gradlev_tensor* x,
                          gradlev_stream_t stream);
 
 /*
+ * gradlev_fused_scan -- the forward scan and the costate scan of one map in a single
+ * call (Sec. 3, steps 2 and 3: both reads use the same historical writes), with the
+ * optional per-token consistency term of the training objective (Eq. 5; Appendix A,
+ * eq. consistency).
+ *   x, g_hat, W0, eta  the writes and slow weights, as in gradlev_forward_scan
+ *   g_out    [L][B][T][H][d_out]  incoming costates (read)
+ *   y        [L][B][T][H][d_out]  out: What_t x_t          (as gradlev_forward_scan)
+ *   g_in     [L][B][T][H][d_in]   out: What_t^T g_out_t    (as gradlev_costate_scan)
+ *   cons_proposal  [L][B][T][H][d_in], optional (NULL or data NULL): proposals to
+ *            compare with g_in, e.g. the proposals of the map below this one
+ *   cons     fp32 [L][B][T][H] contiguous, 4-byte aligned; out when cons_proposal is
+ *            given (and must then be non-NULL, else NULL):
+ *            cons_t = ||cons_proposal_t - g_in_t||^2 / d_in, with g_in_t taken in fp32
+ *            before its rounding to the output dtype
+ *   workspace/workspace_bytes  at least gradlev_workspace_bytes(desc), 256-byte aligned.
+ * bf16 maps with d_in = d_out = 64 and 16-byte aligned token rows (eta as for the
+ * tensor-core forward scan) run one tensor-core kernel that reads x, g_hat and g_out
+ * once and keeps one running state for both reads.  Every other shape runs the forward
+ * and the costate scan one after the other, then (with cons) one row-reduction kernel;
+ * the results are the same.  All arguments of both passes are checked before anything
+ * is launched.  A timed-out device wait is reported by gradlev_workspace_status.
+ * Returns GRADLEV_OK or an error code; nothing is launched on error.
+ */
+int gradlev_fused_scan(const gradlev_desc* desc, const gradlev_tensor* x,
+                       const gradlev_tensor* g_hat, const float* W0, float eta,
+                       const gradlev_tensor* g_out, const gradlev_tensor* y,
+                       const gradlev_tensor* g_in, const gradlev_tensor* cons_proposal, float* cons,
+                       void* workspace, size_t workspace_bytes, gradlev_stream_t stream);
+
+/*
  * gradlev_forward_scan_gated / gradlev_costate_scan_gated -- the scans with the
  * general gates of Sec. 3 ("Observation", Eq. 2): a step size eta_t >= 0 per token
  * and, optionally, a retention alpha_t in [0, 1] with decay centred at W0,

@@ -74,6 +74,9 @@ def load_library():
         lib.gradlev_costate_scan.argtypes = [D, Tp, Tp, P, ctypes.c_float, Tp, ctypes.c_int, Tp, Tp,
                                              P, ctypes.c_size_t, P]
         lib.gradlev_costate_scan.restype = ctypes.c_int
+        lib.gradlev_fused_scan.argtypes = [D, Tp, Tp, P, ctypes.c_float, Tp, Tp, Tp, Tp, P, P,
+                                           ctypes.c_size_t, P]
+        lib.gradlev_fused_scan.restype = ctypes.c_int
         lib.gradlev_forward_scan_gated.argtypes = [D, Tp, Tp, P, P, P, ctypes.c_int, Tp, Tp, P,
                                                    ctypes.c_size_t, P]
         lib.gradlev_forward_scan_gated.restype = ctypes.c_int
@@ -419,6 +422,63 @@ def costate_scan(x, g_hat, W0, eta, g_out, act=None, z=None, g_in=None, workspac
                                       ctypes.c_void_p(stream))
     _call(rc, "gradlev_costate_scan")
     return g_in
+
+
+def fused_scan(x, g_hat, W0, eta, g_out, y=None, g_in=None, cons_proposal=None, cons=None,
+               workspace=None):
+    """Both reads of one map in one call (Sec. 3 steps 2 and 3, Eqs. 3-4):
+    y_t = What_t x_t and g_in_t = What_t^T g_out_t over the same writes.
+
+    With cons_proposal (shape of x) also the per-token consistency term
+    cons_t = ||cons_proposal_t - g_in_t||^2 / d_in of Eq. 5, fp32 [L,B,T,H] (or the
+    token shape of x).  Returns (y, g_in) or (y, g_in, cons).
+    """
+    lib = load_library()
+    x5, g5, go5 = _as5(x), _as5(g_hat), _as5(g_out)
+    _check_same(x5, g5, go5)
+    if not x5.is_cuda:
+        raise ValueError("tensors must be on a CUDA device")
+    L, B, T, H, d_in = x5.shape
+    d_out = g5.shape[4]
+    if tuple(g5.shape) != tuple(go5.shape) or tuple(g5.shape[:4]) != (L, B, T, H):
+        raise ValueError("g_hat / g_out shapes differ from x")
+    W = _w0(W0, L, H, d_out, d_in)
+    if W.device != x5.device:
+        raise ValueError("W0 must be on the tensors' device")
+    if y is None:
+        y = torch.empty(tuple(x.shape[:-1]) + (d_out,), dtype=x5.dtype, device=x5.device)
+    if g_in is None:
+        g_in = torch.empty(x5.shape, dtype=x5.dtype, device=x5.device).view(x.shape)
+    y5, gi5 = _as5(y), _as5(g_in)
+    _check_same(x5, y5, gi5)
+    if tuple(y5.shape) != (L, B, T, H, d_out) or tuple(gi5.shape) != tuple(x5.shape):
+        raise ValueError("y / g_in have the wrong shape")
+    p5 = None
+    if cons_proposal is not None:
+        p5 = _as5(cons_proposal)
+        _check_same(x5, p5)
+        if tuple(p5.shape) != tuple(x5.shape):
+            raise ValueError("cons_proposal must have the shape of x")
+        if cons is None:
+            cons = torch.empty(tuple(x.shape[:-1]), dtype=torch.float32, device=x5.device)
+        if cons.dtype != torch.float32 or not cons.is_contiguous() or cons.numel() != L * B * T * H:
+            raise ValueError("cons must be a contiguous float32 tensor of L*B*T*H entries")
+    desc = _desc(x5, d_out, _dtype_code(x5))
+    nbytes = int(lib.gradlev_workspace_bytes(ctypes.byref(desc)))
+    ws = workspace if workspace is not None else _workspace(nbytes, x5.device)
+    tx, tg, tgo, ty, tgi = _tensor(x5), _tensor(g5), _tensor(go5), _tensor(y5), _tensor(gi5)
+    tp = _tensor(p5) if p5 is not None else None
+    stream = torch.cuda.current_stream(x5.device).cuda_stream
+    with torch.cuda.device(x5.device):
+        rc = lib.gradlev_fused_scan(ctypes.byref(desc), ctypes.byref(tx), ctypes.byref(tg),
+                                    ctypes.c_void_p(W.data_ptr()), float(eta), ctypes.byref(tgo),
+                                    ctypes.byref(ty), ctypes.byref(tgi),
+                                    ctypes.byref(tp) if tp is not None else None,
+                                    ctypes.c_void_p(cons.data_ptr()) if tp is not None else None,
+                                    ctypes.c_void_p(ws.data_ptr()), ws.numel(),
+                                    ctypes.c_void_p(stream))
+    _call(rc, "gradlev_fused_scan")
+    return (y, g_in, cons) if p5 is not None else (y, g_in)
 
 
 def mlp_forward(x, g_hat_z, g_hat_y, W1, W2, eta1, eta2, act="gelu_tanh"):

@@ -24,7 +24,10 @@ cudaError_t launch_tc_suffix(const CUtensorMap& q, const CUtensorMap& k, const C
                              cudaStream_t stream);
 cudaError_t launch_rowdot(const void* a, const TokStr& as, const void* r, const TokStr& rs,
                           float* out, int L, int B, int T, int H, int w, float scale, bool bf16,
-                          cudaStream_t stream);
+                          cudaStream_t stream, bool sqdist = false);
+cudaError_t launch_tc_fused(const CUtensorMap& x, const CUtensorMap& ghat, const CUtensorMap& gout,
+                            const CUtensorMap& y, const CUtensorMap& gin, const TcScanParams& p,
+                            int grid, cudaStream_t stream);
 cudaError_t launch_seg_gemm(int mode, int bn, const CUtensorMap& a, const CUtensorMap& b,
                             const CUtensorMap& a2, const CUtensorMap& b2, const SegGemmParams& p,
                             int grid, cudaStream_t stream);
@@ -309,10 +312,12 @@ void fill_epi(gl::EpiParams* e, const Tok& out, const Tok& out2, const Tok& z, i
 // Shared driver of both scans.  Roles (Sec. 3, Eqs. 3-4):
 //   forward:  q = k = x, v = g_hat, B0 = W0     (dq = d_in,  dv = d_out)
 //   costate:  q = g_out, k = g_hat, v = x, B0 = W0^T (dq = d_out, dv = d_in)
+// With dry set, every argument check runs and nothing is launched.
 int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
              const gradlev_tensor* g_hat, const float* W0, float eta, const gradlev_tensor* g_out,
              int act, const gradlev_tensor* out, const gradlev_tensor* out2,
-             const gradlev_tensor* z, void* ws, size_t ws_bytes, cudaStream_t stream) {
+             const gradlev_tensor* z, void* ws, size_t ws_bytes, cudaStream_t stream,
+             bool dry = false) {
     if (!desc_ok(desc)) return GRADLEV_ERR_INVALID_ARG;
     const gradlev_desc& d = *desc;
     if (!W0 || !isfinite(eta)) return GRADLEV_ERR_INVALID_ARG;
@@ -385,6 +390,7 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
         p.flags = reinterpret_cast<unsigned int*>(wsb + pl.off_flags);
         p.agg = reinterpret_cast<float*>(wsb + pl.off_agg);
         p.incl = reinterpret_cast<float*>(wsb + pl.off_incl);
+        if (dry) return GRADLEV_OK;
         if (cudaMemsetAsync(ws, 0, pl.zero_bytes, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
         const int grid = pl.n_items < dev.sms ? pl.n_items : dev.sms;
         if (gl::launch_tc_scan(mq, mk, mv, mo, p, costate, grid, stream) != cudaSuccess)
@@ -426,6 +432,7 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
         p.pbuf = reinterpret_cast<__nv_bfloat16*>(wsb + sp.off_pbuf);
         fill_epi(&p.epi, to, to2, tz, act);
         p.ctrl = reinterpret_cast<unsigned int*>(wsb);
+        if (dry) return GRADLEV_OK;
         if (cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
         const long long tiles[3] = {sp.tiles_state, sp.tiles_score, sp.tiles_out};
         for (int mode = 0; mode < 3; ++mode) {
@@ -451,8 +458,9 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
             if (t->data && (reinterpret_cast<uintptr_t>(t->data) % elem) != 0)
                 return GRADLEV_ERR_UNSUPPORTED;
         if ((reinterpret_cast<uintptr_t>(W0) & 3u) != 0) return GRADLEV_ERR_INVALID_ARG;
+        if (ws && (reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return GRADLEV_ERR_WORKSPACE;
+        if (dry) return GRADLEV_OK;
         if (ws) {
-            if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return GRADLEV_ERR_WORKSPACE;
             if (ws_bytes >= 256 && cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess)
                 return GRADLEV_ERR_CUDA;
         }
@@ -481,6 +489,109 @@ int run_scan(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
         return GRADLEV_OK;
     }
     return GRADLEV_ERR_UNSUPPORTED;
+}
+
+// Both reads of a map in one call (Sec. 3, steps 2 and 3): y_t = W_t x_t and
+// g_in_t = W_t^T g_out_t over the same writes, with the optional per-token
+// consistency term cons_t = ||p_t - g_in_t||^2 / d_in against proposals p (Eq. 5).
+// 64 x 64 bf16 maps run the single-pass kernel; other shapes run the forward and
+// the costate scan one after the other (every check of both passes first).
+int run_fused(const gradlev_desc* desc, const gradlev_tensor* x, const gradlev_tensor* g_hat,
+              const float* W0, float eta, const gradlev_tensor* g_out, const gradlev_tensor* y,
+              const gradlev_tensor* g_in, const gradlev_tensor* cons_p, float* cons, void* ws,
+              size_t ws_bytes, cudaStream_t stream) {
+    if (!desc_ok(desc)) return GRADLEV_ERR_INVALID_ARG;
+    const gradlev_desc& d = *desc;
+    if (!W0 || !isfinite(eta)) return GRADLEV_ERR_INVALID_ARG;
+    const int din = d.d_in, dout = d.d_out;
+    Tok tx, tg, tgo, ty, tgi, tp;
+    if (!resolve(d, x, din, &tx, true) || !resolve(d, g_hat, dout, &tg, true) ||
+        !resolve(d, g_out, dout, &tgo, true) || !resolve(d, y, dout, &ty, true) ||
+        !resolve(d, g_in, din, &tgi, true) || !resolve(d, cons_p, din, &tp, false))
+        return GRADLEV_ERR_INVALID_ARG;
+    const bool want_cons = tp.data != nullptr && d.T > 0;
+    if ((cons_p && cons_p->data) != (cons != nullptr)) return GRADLEV_ERR_INVALID_ARG;
+    if (cons && (reinterpret_cast<uintptr_t>(cons) & 3u) != 0) return GRADLEV_ERR_INVALID_ARG;
+    DevInfo dev;
+    if (!device_info(&dev)) return GRADLEV_ERR_CUDA;
+    if (!(dev.major == 10 && dev.minor == 3)) return GRADLEV_ERR_UNSUPPORTED;
+    if (d.T == 0) return GRADLEV_OK;
+    const bool bf16 = d.dtype == GRADLEV_BF16;
+    if (bf16 && din == 64 && dout == 64 && tc_eta_ok(eta) && tc_layout_ok(tx, 2) &&
+        tc_layout_ok(tg, 2) && tc_layout_ok(tgo, 2) && tc_layout_ok(ty, 2) && tc_layout_ok(tgi, 2) &&
+        tc_layout_ok(tp, 2)) {
+        Plan pl = plan_tc(d, 64, 64, dev.sms);
+        if (!ws || ws_bytes < pl.ws_bytes) return GRADLEV_ERR_WORKSPACE;
+        if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return GRADLEV_ERR_WORKSPACE;
+        CUtensorMap mx, mg, mgo, my, mgi;
+        if (!make_tmap(&mx, d, tx, 64) || !make_tmap(&mg, d, tg, 64) || !make_tmap(&mgo, d, tgo, 64) ||
+            !make_tmap(&my, d, ty, 64) || !make_tmap(&mgi, d, tgi, 64))
+            return GRADLEV_ERR_UNSUPPORTED;
+        TcScanParams p;
+        memset(&p, 0, sizeof(p));
+        p.L = d.L;
+        p.B = d.B;
+        p.T = d.T;
+        p.H = d.H;
+        p.dq = 64;
+        p.dv = 64;
+        p.n_tiles = pl.n_tiles;
+        p.seg_len = pl.seg_len;
+        p.n_seg = pl.n_seg;
+        p.n_items = pl.n_items;
+        p.n_ut = pl.n_items / pl.n_seg;
+        p.lookback_limit_ns = 4000000000ull;
+        p.test_skip_publish = -1;
+        if (const char* v = getenv("GRADLEV_TEST_SKIP_PUBLISH")) p.test_skip_publish = atoi(v);
+        if (const char* v = getenv("GRADLEV_TEST_LOOKBACK_LIMIT_MS"))
+            p.lookback_limit_ns = 1000000ull * (unsigned long long)atoi(v);
+        p.eta = eta;
+        p.lam = eta != 0.0f ? -eta : 1.0f;
+        p.inv_lam = 1.0f / p.lam;
+        p.mu = eta != 0.0f ? 1.0f : 0.0f;
+        p.w0_transposed = 0;  // the state in the forward orientation, W0^T rows
+        p.W0 = W0;
+        const Tok none;
+        fill_epi(&p.epi, ty, none, none, GRADLEV_ACT_NONE);
+        if (want_cons) {
+            p.epi.cons_p = tp.data;
+            for (int i = 0; i < 4; ++i) p.epi.cons_str[i] = tp.s[i];
+            p.epi.cons_out = cons;
+            p.epi.cons_scale = 1.0f / (float)din;
+        }
+        uint8_t* wsb = static_cast<uint8_t*>(ws);
+        p.ctrl = reinterpret_cast<unsigned int*>(wsb);
+        p.flags = reinterpret_cast<unsigned int*>(wsb + pl.off_flags);
+        p.agg = reinterpret_cast<float*>(wsb + pl.off_agg);
+        p.incl = reinterpret_cast<float*>(wsb + pl.off_incl);
+        if (cudaMemsetAsync(ws, 0, pl.zero_bytes, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
+        const int grid = pl.n_items < dev.sms ? pl.n_items : dev.sms;
+        if (gl::launch_tc_fused(mx, mg, mgo, my, mgi, p, grid, stream) != cudaSuccess)
+            return GRADLEV_ERR_CUDA;
+        return GRADLEV_OK;
+    }
+    // Other shapes: check both passes before launching either.
+    int rc = run_scan(desc, false, x, g_hat, W0, eta, nullptr, GRADLEV_ACT_NONE, y, nullptr, nullptr,
+                      ws, ws_bytes, stream, true);
+    if (rc == GRADLEV_OK)
+        rc = run_scan(desc, true, x, g_hat, W0, eta, g_out, GRADLEV_ACT_NONE, g_in, nullptr, nullptr,
+                      ws, ws_bytes, stream, true);
+    if (rc != GRADLEV_OK) return rc;
+    rc = run_scan(desc, false, x, g_hat, W0, eta, nullptr, GRADLEV_ACT_NONE, y, nullptr, nullptr, ws,
+                  ws_bytes, stream);
+    if (rc == GRADLEV_OK)
+        rc = run_scan(desc, true, x, g_hat, W0, eta, g_out, GRADLEV_ACT_NONE, g_in, nullptr, nullptr,
+                      ws, ws_bytes, stream);
+    if (rc != GRADLEV_OK || !want_cons) return rc;
+    gl::TokStr ps, gs;
+    for (int i = 0; i < 4; ++i) {
+        ps.s[i] = tp.s[i];
+        gs.s[i] = tgi.s[i];
+    }
+    if (gl::launch_rowdot(tp.data, ps, tgi.data, gs, cons, d.L, d.B, d.T, d.H, din, 1.0f / (float)din,
+                          bf16, stream, true) != cudaSuccess)
+        return GRADLEV_ERR_CUDA;
+    return GRADLEV_OK;
 }
 
 size_t ws_bytes_for(const gradlev_desc& d, int dq, int dv, int sms) {
@@ -969,6 +1080,15 @@ int gradlev_costate_scan(const gradlev_desc* desc, const gradlev_tensor* x,
                          gradlev_stream_t stream) {
     return run_scan(desc, true, x, g_hat, W0, eta, g_out, act, g_in, nullptr, z, workspace,
                     workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int gradlev_fused_scan(const gradlev_desc* desc, const gradlev_tensor* x, const gradlev_tensor* g_hat,
+                       const float* W0, float eta, const gradlev_tensor* g_out,
+                       const gradlev_tensor* y, const gradlev_tensor* g_in,
+                       const gradlev_tensor* cons_proposal, float* cons, void* workspace,
+                       size_t workspace_bytes, gradlev_stream_t stream) {
+    return run_fused(desc, x, g_hat, W0, eta, g_out, y, g_in, cons_proposal, cons, workspace,
+                     workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
 }
 
 int gradlev_forward_scan_gated(const gradlev_desc* desc, const gradlev_tensor* x,

@@ -43,10 +43,11 @@ __device__ __forceinline__ int ld16(const void* p, long long i, float* f) {
     }
 }
 
-// out[l][b][t][h] = scale * sum_j a[l,b,t,h,j] * r[l,b,t,h,j].  A group of `lanes`
-// lanes (a power of two up to 32) takes one token row in 16-byte pieces when
+// out[l][b][t][h] = scale * sum_j a[l,b,t,h,j] * r[l,b,t,h,j], or with SQ the squared
+// distance scale * sum_j (a - r)^2 (the consistency term of Eq. 5).  A group of
+// `lanes` lanes (a power of two up to 32) takes one token row in 16-byte pieces when
 // `vec`, else element by element with a whole warp per row.
-template <bool BF16>
+template <bool BF16, bool SQ>
 __global__ void __launch_bounds__(kThreads)
     rowdot_kernel(const void* __restrict__ a, TokStr as, const void* __restrict__ r, TokStr rs,
                   float* __restrict__ out, int L, int B, int T, int H, int w, float scale, int vec,
@@ -74,10 +75,24 @@ __global__ void __launch_bounds__(kThreads)
                 ld16<BF16>(a, ao + j, fa);
                 ld16<BF16>(r, ro + j, fr);
 #pragma unroll
-                for (int k = 0; k < kPer; ++k) acc = fmaf(fa[k], fr[k], acc);
+                for (int k = 0; k < kPer; ++k) {
+                    if constexpr (SQ) {
+                        const float dlt = fa[k] - fr[k];
+                        acc = fmaf(dlt, dlt, acc);
+                    } else {
+                        acc = fmaf(fa[k], fr[k], acc);
+                    }
+                }
             }
         } else {
-            for (int j = cl; j < w; j += 32) acc = fmaf(ld<BF16>(a, ao + j), ld<BF16>(r, ro + j), acc);
+            for (int j = cl; j < w; j += 32) {
+                if constexpr (SQ) {
+                    const float dlt = ld<BF16>(a, ao + j) - ld<BF16>(r, ro + j);
+                    acc = fmaf(dlt, dlt, acc);
+                } else {
+                    acc = fmaf(ld<BF16>(a, ao + j), ld<BF16>(r, ro + j), acc);
+                }
+            }
         }
     }
     for (int o = LR >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
@@ -88,7 +103,7 @@ __global__ void __launch_bounds__(kThreads)
 
 cudaError_t launch_rowdot(const void* a, const TokStr& as, const void* r, const TokStr& rs,
                           float* out, int L, int B, int T, int H, int w, float scale, bool bf16,
-                          cudaStream_t stream) {
+                          cudaStream_t stream, bool sqdist) {
     const long long rows = (long long)L * B * T * H;
     // 16-byte pieces when every row starts on a 16-byte boundary
     const int per = bf16 ? 8 : 4, elem = bf16 ? 2 : 4;
@@ -104,12 +119,10 @@ cudaError_t launch_rowdot(const void* a, const TokStr& as, const void* r, const 
     const long long rows_per_cta = (long long)(grads::kThreads / 32) * (vec ? 32 / lanes : 1);
     const long long grid = (rows + rows_per_cta - 1) / rows_per_cta;
     if (grid <= 0 || grid > 0x7FFFFFFF) return cudaErrorInvalidValue;
-    if (bf16)
-        grads::rowdot_kernel<true><<<(int)grid, grads::kThreads, 0, stream>>>(
-            a, as, r, rs, out, L, B, T, H, w, scale, vec ? 1 : 0, lanes);
-    else
-        grads::rowdot_kernel<false><<<(int)grid, grads::kThreads, 0, stream>>>(
-            a, as, r, rs, out, L, B, T, H, w, scale, vec ? 1 : 0, lanes);
+    auto kern = bf16 ? (sqdist ? grads::rowdot_kernel<true, true> : grads::rowdot_kernel<true, false>)
+                     : (sqdist ? grads::rowdot_kernel<false, true> : grads::rowdot_kernel<false, false>);
+    kern<<<(int)grid, grads::kThreads, 0, stream>>>(a, as, r, rs, out, L, B, T, H, w, scale,
+                                                    vec ? 1 : 0, lanes);
     return cudaGetLastError();
 }
 

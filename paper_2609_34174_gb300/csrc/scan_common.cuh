@@ -73,6 +73,12 @@ struct EpiParams {
     long long dot_a_str[4];
     float* dot_out;
     float dot_scale;
+    // optional consistency term (fused pass, costate read): cons_out[l][b][t][h] =
+    // cons_scale * ||cons_p row - result row||^2, fp32 [L][B][T][H] contiguous
+    const void* cons_p;
+    long long cons_str[4];
+    float* cons_out;
+    float cons_scale;
 };
 
 // Parameters of the tensor-core scan kernel (bf16, dq in {64, 128}, dv % 64 == 0).

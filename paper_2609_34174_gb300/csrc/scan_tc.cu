@@ -70,14 +70,19 @@ __host__ __device__ constexpr uint32_t col_dz(uint32_t i) { return 384u + i * 64
 // Stage layout [q | k | v] (costate), [qk | v] (forward).  The reverse read with one
 // q/k tile puts v first, [v | qk]: the dZ product's A operand then starts one block
 // before k in both reverse layouts, which places K^T in TMEM lanes 64..127.
-template <int DQ, bool COSTATE, bool REV = false>
+// FUSED (both reads in one pass, 64-wide maps): [x | ghat | g_out].  The forward read
+// takes q = k = x, v = ghat; the costate read q = g_out, k = ghat, v = x; the
+// writes (state increment) are those of the forward orientation, x^T ghat.
+template <int DQ, bool COSTATE, bool REV = false, bool FUSED = false>
 struct TcLayout {
     static constexpr int kQkBlocks = DQ / 64;
     static constexpr bool kVFirst = REV && !COSTATE;
-    static constexpr int kQOff = kVFirst ? kTile : 0;
-    static constexpr int kKOff = COSTATE ? kQkBlocks * kTile : kQOff;
-    static constexpr int kVOff = kVFirst ? 0 : kKOff + kQkBlocks * kTile;
-    static constexpr int kStageBytes = ((COSTATE ? 2 : 1) * kQkBlocks + 1) * kTile;
+    static constexpr int kQOff = FUSED ? 0 : (kVFirst ? kTile : 0);
+    static constexpr int kKOff = FUSED ? 0 : (COSTATE ? kQkBlocks * kTile : kQOff);
+    static constexpr int kVOff = FUSED ? kTile : (kVFirst ? 0 : kKOff + kQkBlocks * kTile);
+    static constexpr int kGOff = 2 * kTile;  // FUSED: the g_out tile
+    static constexpr int kStageBytes =
+        FUSED ? 3 * kTile : ((COSTATE ? 2 : 1) * kQkBlocks + 1) * kTile;
     // Stage ring: what is left of the 227 KB opt-in budget after the two S^T
     // tiles, the two output staging tiles, the barrier block and the alignment
     // slack (at most 6 stages).
@@ -92,7 +97,7 @@ struct TcLayout {
     static constexpr int kSmemBytes = kBarOff + kBarBytes + 1024;  // + alignment slack
     // Bytes one stage receives in each pass.
     static constexpr uint32_t kTxPass1 = (kQkBlocks + 1) * kTile;
-    static constexpr uint32_t kTxPass2 = ((COSTATE ? 2 : 1) * kQkBlocks + 1) * kTile;
+    static constexpr uint32_t kTxPass2 = kStageBytes;
     static_assert(kStages >= 2, "not enough shared memory for two stages");
     static_assert(kSmemBytes <= 232448, "shared memory budget exceeded");
 };
@@ -203,6 +208,25 @@ __device__ __noinline__ void epi_store_act(const EpiParams& e, long long o_off, 
     }
 }
 
+// e.cons_out[idx] = e.cons_scale * ||p row - v||^2 for one 64-wide output row piece:
+// the per-token consistency term between a proposal and the reconstructed costate
+// (Sec. 3, Eq. 5; Appendix A).
+__device__ __noinline__ void epi_consistency(const EpiParams& e, long long p_off, const float* v,
+                                             long long idx) {
+    const __nv_bfloat16* pp = static_cast<const __nv_bfloat16*>(e.cons_p) + p_off;
+    float acc = 0.f;
+    for (int q = 0; q < 8; ++q) {
+        const uint4 pv = *reinterpret_cast<const uint4*>(pp + 8 * q);
+        const __nv_bfloat16* pb = reinterpret_cast<const __nv_bfloat16*>(&pv);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const float dlt = __bfloat162float(pb[i]) - v[8 * q + i];
+            acc = fmaf(dlt, dlt, acc);
+        }
+    }
+    e.cons_out[idx] = e.cons_scale * acc;
+}
+
 // K-step offsets (in the 16-byte units of a descriptor's low word).
 // K-major operand, 64-wide K blocks 16 KB apart: step kk starts 32 B further in
 // its 128-byte swizzled row, and every 4 steps moves to the next block.
@@ -212,12 +236,19 @@ __host__ __device__ constexpr uint32_t kmaj_step(int kk) {
 // MN-major operand: step kk starts 16 rows (two 8-row groups of 1024 B) further.
 __host__ __device__ constexpr uint32_t mnmaj_step(int kk) { return (uint32_t)((kk * 2048) >> 4); }
 
-template <int DQ, bool COSTATE, bool REV>
+// FUSED runs the forward and the costate read of one 64-wide map in a single pass
+// over the shared writes (Sec. 3, steps 2 and 3): per chunk two jobs, the forward
+// read (score, P and O buffers 0, stored through tm_o) and the costate read (buffers
+// 1, stored through tm_o2), one S'^T tile and one state update.  Maps: tm_q = x,
+// tm_k = ghat, tm_v = g_out.
+template <int DQ, bool COSTATE, bool REV, bool FUSED>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_scan_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
-                   const TcScanParams p) {
-    using Lay = TcLayout<DQ, COSTATE, REV>;
+                   const __grid_constant__ CUtensorMap tm_o2, const TcScanParams p) {
+    using Lay = TcLayout<DQ, COSTATE, REV, FUSED>;
+    static_assert(!FUSED || (DQ == 64 && !COSTATE && !REV), "the fused pass is built for 64-wide maps");
+    constexpr int kJobs = FUSED ? 2 : 1;  // reads per chunk
     constexpr int NS = Lay::kStages;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -305,6 +336,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         prefetch_tmap(&tm_k);
         prefetch_tmap(&tm_v);
         prefetch_tmap(&tm_o);
+        if constexpr (FUSED) prefetch_tmap(&tm_o2);
     }
     __syncthreads();
     tc_fence_after();
@@ -327,6 +359,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     uint8_t* st = smem + s * Lay::kStageBytes;
                     const int t0 = chunk_t0<REV>(I, c);
                     mbar_arrive_expect_tx(&full[s], pass == 1 ? Lay::kTxPass1 : Lay::kTxPass2);
+                    if constexpr (FUSED) {
+                        tma_load_5d(st + Lay::kQOff, &tm_q, &full[s], 0, I.h, t0, I.b, I.l);
+                        tma_load_5d(st + Lay::kVOff, &tm_k, &full[s], 0, I.h, t0, I.b, I.l);
+                        if (pass == 2)
+                            tma_load_5d(st + Lay::kGOff, &tm_v, &full[s], 0, I.h, t0, I.b, I.l);
+                        continue;
+                    }
                     if (COSTATE && pass == 2) {
 #pragma unroll
                         for (int kb = 0; kb < Lay::kQkBlocks; ++kb)
@@ -441,6 +480,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                             mma_bf16_ss(tmem + col_sc(sb), sdesc_from_lo(q_lo + kmaj_step(kk)),
                                         sdesc_from_lo(k_lo + kmaj_step(kk)), ID_SC, kk > 0 ? 1u : 0u);
                         mma_commit(&sc_full[sb]);
+                        if constexpr (FUSED) {
+                            // the costate read of the same chunk: score G Ghat^T into buffer 1
+                            ++c2;
+                            const uint32_t sb2 = c2 & 1;
+                            if (!(ok = wait_or_fail(&sc_free[sb2], ((c2 >> 1) & 1) ^ 1))) break;
+                            tc_fence_after();
+                            const uint32_t g_lo = sdesc_lo(st + Lay::kGOff, 16);
+                            const uint32_t h_lo = sdesc_lo(st + Lay::kVOff, 16);
+#pragma unroll
+                            for (int kk = 0; kk < DQ / 16; ++kk)
+                                mma_bf16_ss(tmem + col_sc(sb2), sdesc_from_lo(g_lo + kmaj_step(kk)),
+                                            sdesc_from_lo(h_lo + kmaj_step(kk)), ID_SC, kk > 0 ? 1u : 0u);
+                            mma_commit(&sc_full[sb2]);
+                        }
                         if (c < I.nch - 1) {
                             const uint32_t b = dzc & 1;
                             if (!(ok = wait_or_fail(&dz_free[b], ((dzc >> 1) & 1) ^ 1))) break;
@@ -482,7 +535,55 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const Item In = decode_item<REV>(item, p);
                     if (In.phase1) n += In.nch;
                 }
-                if (pending >= 0) {
+                if (FUSED && pending >= 0) {
+                    // Both reads of a chunk: O_y = X S'^T and O_g = G S' from one S'^T tile
+                    // (read MN-major for the forward, K-major for the costate), then the
+                    // two P V products.  Each direction owns one O and one score buffer,
+                    // used once per chunk; the S'^T tiles alternate by chunk.
+                    constexpr uint32_t ID_OK = idesc_bf16(128, 64, false, false);  // G S'
+                    const Item I = decode_item<REV>(pending, p);
+                    for (int c = 0; c < I.nch; ++c, ++n, c2 += 2) {
+                        const int s = n % NS;
+                        const uint32_t cc = c2 >> 1;  // chunks of this CTA so far
+                        const uint32_t sbb = cc & 1, sph = (cc >> 1) & 1, oph = cc & 1;
+                        if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
+                        if (!(ok = wait_or_fail(&st_ready[sbb], sph))) break;
+                        if (!(ok = wait_or_fail(&o_free[0], oph ^ 1))) break;
+                        if (!(ok = wait_or_fail(&o_free[1], oph ^ 1))) break;
+                        tc_fence_after();
+                        const uint32_t st = sbase + s * Lay::kStageBytes;
+                        const uint32_t tile = sbase + Lay::kStOff + sbb * Lay::kStBytes;
+                        const uint32_t x_lo = sdesc_lo(st + Lay::kQOff, 16);
+                        const uint32_t g_lo = sdesc_lo(st + Lay::kGOff, 16);
+                        const uint32_t s_mn = sdesc_lo(tile, kTile);
+                        const uint32_t s_k = sdesc_lo(tile, 16);
+#pragma unroll
+                        for (int kk = 0; kk < DQ / 16; ++kk)
+                            mma_bf16_ss(tmem + col_o(0), sdesc_from_lo(x_lo + kmaj_step(kk)),
+                                        sdesc_from_lo(s_mn + mnmaj_step(kk)), ID_O, kk > 0 ? 1u : 0u);
+#pragma unroll
+                        for (int kk = 0; kk < DQ / 16; ++kk)
+                            mma_bf16_ss(tmem + col_o(1), sdesc_from_lo(g_lo + kmaj_step(kk)),
+                                        sdesc_from_lo(s_k + kmaj_step(kk)), ID_OK, kk > 0 ? 1u : 0u);
+                        mma_commit(&st_free[sbb]);
+#pragma unroll 1
+                        for (int dir = 0; dir < 2; ++dir) {
+                            if (!(ok = wait_or_fail(&p_ready[dir], oph))) break;
+                            tc_fence_after();
+                            // forward: V = ghat; costate: V = x (both MN-major [128 t][64])
+                            const uint32_t v_lo = sdesc_lo(st + (dir == 0 ? Lay::kVOff : Lay::kQOff), kTile);
+#pragma unroll
+                            for (int kk = 0; kk < kChunk / 16; ++kk)
+                                mma_bf16_ts(tmem + col_o(dir),
+                                            tmem + col_sc(dir) + (kk < 4 ? kk * 8 : 64 + (kk - 4) * 8),
+                                            sdesc_from_lo(v_lo + mnmaj_step(kk)), ID_O, 1u);
+                            mma_commit(&o_full[dir]);
+                            mma_commit(&sc_free[dir]);
+                        }
+                        if (!ok) break;
+                        mma_commit(&empty[s]);
+                    }
+                } else if (pending >= 0) {
                     const Item I = decode_item<REV>(pending, p);
                     for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
                         const int s = n % NS;
@@ -543,7 +644,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (item < 0) break;
             const Item I = decode_item<REV>(item, p);
             bool ok = true;
-            for (int c = 0; c < I.nch; ++c, ++c2) {
+            for (int c = 0; c < kJobs * I.nch; ++c, ++c2) {
                 const uint32_t sb = c2 & 1;
                 if (!warp_wait(&sc_full[sb], (c2 >> 1) & 1, abort_flag)) {
                     raise_error(p, kErrWaitTimeout, abort_flag);
@@ -632,7 +733,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 load_a(c2 & 1, 0);
                 if (I.nch > 1) load_a((c2 + 1) & 1, 1);
             }
-            for (int c = 0; c < I.nch; ++c, ++c2) {
+            for (int jb = 0; jb < kJobs * I.nch; ++jb, ++c2) {
+                // FUSED: job 2c is chunk c's forward read (y), job 2c+1 its costate read
+                const int c = FUSED ? (jb >> 1) : jb;
+                const int dir = FUSED ? (jb & 1) : 0;
                 const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
                 if (!warp_wait(&o_full[ob], oph, abort_flag)) {
                     raise_error(p, kErrWaitTimeout, abort_flag);
@@ -666,6 +770,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int i = 0; i < 64; ++i) tmp[i] = v[i];
                     epi_store_act(e, tok_off(e.out2_str, I.l, I.b, t, I.h) + col0, tmp);
+                }
+                if constexpr (FUSED) {
+                    // consistency term of the costate read against the given proposals
+                    if (dir == 1 && e.cons_out && valid) {
+                        float tmp[64];
+#pragma unroll
+                        for (int i = 0; i < 64; ++i) tmp[i] = v[i];
+                        epi_consistency(e, tok_off(e.cons_str, I.l, I.b, t, I.h) + col0, tmp,
+                                        (((long long)I.l * p.B + I.b) * p.T + t) * p.H + I.h);
+                    }
                 }
                 // Stage the bf16 row in the 128B-swizzled output tile (the TMA store
                 // clips rows past the end of the sequence).
@@ -730,7 +844,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         ok = false;
                     } else {
                         if (!direct)
-                            tma_store_5d(&tm_o, smem + Lay::kOOff + ob * kTile, col0, I.h, t0, I.b, I.l);
+                            tma_store_5d(dir ? &tm_o2 : &tm_o, smem + Lay::kOOff + ob * kTile, col0,
+                                         I.h, t0, I.b, I.l);
                         bulk_commit_group();
                         // the previous chunk's store (other tile) has finished reading
                         bulk_wait_group_read<1>();
@@ -1009,16 +1124,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ------------------------------------------------------------------ host side
-template <int DQ, bool COSTATE, bool REV>
+template <int DQ, bool COSTATE, bool REV, bool FUSED = false>
 static cudaError_t launch_one(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
                               const CUtensorMap& o, const TcScanParams& p, int grid,
-                              cudaStream_t stream) {
-    using Lay = TcLayout<DQ, COSTATE, REV>;
-    auto kern = tc_scan_kernel<DQ, COSTATE, REV>;
+                              cudaStream_t stream, const CUtensorMap* o2 = nullptr) {
+    using Lay = TcLayout<DQ, COSTATE, REV, FUSED>;
+    auto kern = tc_scan_kernel<DQ, COSTATE, REV, FUSED>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          Lay::kSmemBytes);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kThreads, Lay::kSmemBytes, stream>>>(q, k, v, o, p);
+    kern<<<grid, kThreads, Lay::kSmemBytes, stream>>>(q, k, v, o, o2 ? *o2 : o, p);
     return cudaGetLastError();
 }
 
@@ -1032,6 +1147,14 @@ cudaError_t launch_tc_scan(const CUtensorMap& q, const CUtensorMap& k, const CUt
         return costate ? launch_one<128, true, false>(q, k, v, o, p, grid, stream)
                        : launch_one<128, false, false>(q, k, v, o, p, grid, stream);
     return cudaErrorInvalidValue;
+}
+
+// Both reads of 64-wide maps in one pass: q = x, k = ghat, v = g_out; o = y, o2 = g_in.
+cudaError_t launch_tc_fused(const CUtensorMap& x, const CUtensorMap& ghat, const CUtensorMap& gout,
+                            const CUtensorMap& y, const CUtensorMap& gin, const TcScanParams& p,
+                            int grid, cudaStream_t stream) {
+    if (p.dq != 64 || p.dv != 64) return cudaErrorInvalidValue;
+    return launch_one<64, false, false, true>(x, ghat, gout, y, p, grid, stream, &gin);
 }
 
 // The anti-causal suffix read r_t = sum_{s>t} (k_s . q_t) v_s (no base matrix) on the

@@ -192,3 +192,27 @@ def test_document_gates_arguments_rejected_before_launch(lib):
     # nothing to do: OK with no pointers at all
     assert call(ctypes.byref(_desc(T=0)), None, float("nan"), None, None, None, None) == 0
     assert call(ctypes.byref(_desc(H=0)), None, 0.1, None, None, None, None) == 0
+
+
+def test_fused_scan_rejects_bad_arguments(lib):
+    """gradlev_fused_scan checks its arguments on the host before any CUDA call."""
+    d = _desc()
+    x, g, go, y, gi, pr = _t(), _t(), _t(), _t(), _t(), _t()
+    null = _t(0)
+    W = ctypes.c_void_p(0x2000)
+    cons = ctypes.c_void_p(0x3000)
+
+    def call(desc=ctypes.byref(d), eta=0.1, g_out=ctypes.byref(go), prop=None, c=None, w0=W):
+        return lib.gradlev_fused_scan(desc, ctypes.byref(x), ctypes.byref(g), w0, eta, g_out,
+                                      ctypes.byref(y), ctypes.byref(gi), prop, c, None, 0, None)
+
+    assert call(desc=None) == -1
+    assert call(w0=None) == -1
+    assert call(eta=float("inf")) == -1
+    assert call(g_out=ctypes.byref(null)) == -1
+    assert call(g_out=None) == -1
+    # a proposal without the output array, and the output array without a proposal
+    assert call(prop=ctypes.byref(pr)) == -1
+    assert call(c=cons) == -1
+    # the consistency output must be 4-byte aligned
+    assert call(prop=ctypes.byref(pr), c=ctypes.c_void_p(0x3002)) == -1
