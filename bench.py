@@ -372,6 +372,51 @@ class LinearJob:
                 f"forward and costate reads in one sequential walk per unit{with_gates}, fp64")
 
 
+class FusedJob(LinearJob):
+    """Both reads of one linear map per unit in one pass (gradlev_fused_scan, Sec. 3
+    steps 2 and 3): x, ghat and g_out are read once and one running state serves the
+    forward and the costate read.  The step computes what LinearJob's two scans do."""
+
+    kind = "fused"
+
+    def __init__(self, gl, wl, device, rank):
+        super().__init__(gl, wl, device, rank)
+        self.launches_per_step = 1
+        self.kernel = {"fused": "tc_scan_kernel<64, fused> (forward and costate reads, one pass)"}
+
+    def step(self, inp=None, events=None):
+        gl, wl, o = self.gl, self.wl, self.outs
+        inp = inp or self.inp
+        if events is not None:
+            events[0].record()
+        with nvtx("gradlev fused scan"):
+            gl.fused_scan(inp["x"], inp["g_hat"], inp["W0"], wl.eta, inp["g_out"], y=o["y"],
+                          g_in=o["g_in"], workspace=self.ws)
+        if events is not None:
+            events[1].record()
+            events[2].record()
+
+    def e2e_step(self, dev, sl, ws):
+        cut = lambda t: self._cut(t, sl)
+        w0 = dev["W0"][sl[1]:sl[2]] if sl[0] == "L" else dev["W0"]
+        self.gl.fused_scan(cut(dev["x"]), cut(dev["g_hat"]), w0, self.wl.eta, cut(dev["g_out"]),
+                           y=cut(self.outs["y"]), g_in=cut(self.outs["g_in"]), workspace=ws)
+
+    def counts(self, scan):
+        """Algorithmic flops and compulsory bytes of one fused call.
+
+        Per token and unit: flops 6*d*m + 2*C*(d+m) (two state reads, one state
+        update, the causal halves of both reads' CxC products, C = 64); bytes
+        e*(2d + 3m): x, ghat, g_out in, y and g_in out; plus 4*d*m per W0.
+        """
+        wl = self.wl
+        e = 2 if wl.dtype == "bf16" else 4
+        d, m = wl.d_in, wl.d_out
+        tu = wl.L * wl.B * wl.T * wl.H
+        flops = tu * (6 * d * m + 2 * COUNT_CHUNK * (d + m))
+        return flops, tu * e * (2 * d + 3 * m) + 4 * d * m * wl.L * wl.H
+
+
 class GradsJob(LinearJob):
     """Step-size gradients of both reads of one linear map per unit, writes
     detached (Sec. 3, practical architecture and training): dL/deta_t of the
@@ -597,7 +642,11 @@ class MLPJob:
                 f"tokens, both layers forward and costate in one sequential walk, fp64")
 
 
-def make_job(gl, wl, device, rank, gates=None, grads=False):
+def make_job(gl, wl, device, rank, gates=None, grads=False, fused=False):
+    if fused:
+        if isinstance(wl, W.MLPWorkload) or gates or grads:
+            raise SystemExit("--fused applies to the ungated linear workloads")
+        return FusedJob(gl, wl, device, rank)
     if grads:
         if isinstance(wl, W.MLPWorkload) or gates:
             raise SystemExit("--grads applies to the ungated linear workloads")
@@ -1090,13 +1139,36 @@ def side_scans(gl, key, device, steps=20, warmup=3):
     return out
 
 
+def side_fused(gl, key, device, steps=20, warmup=3):
+    """The fused pass (both reads in one call) on a linear workload at full size, timed
+    like the headline; its roofline counts its own compulsory bytes."""
+    job = FusedJob(gl, W.workload(key), device, 0)
+    for _ in range(warmup):
+        job.step()
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for i in range(steps):
+        job.step(events=ev[i])
+    torch.cuda.synchronize()
+    if gl.workspace_status(job.ws) != 0:
+        raise RuntimeError("device-side timeout reported by the fused kernel")
+    ms = sum(e[0].elapsed_time(e[1]) for e in ev) / steps
+    fl, nb = job.counts("fused")
+    out = {"workload": f"{key}: {job.wl.name}", "steps": steps, "ms": round(ms, 4),
+           "tokens_per_s": round(job.tokens / (ms / 1e3), 1),
+           "roofline": roofline_entry(fl, nb, ms / 1e3, peaks())}
+    del job
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_gradlev(args, wl, rank, world, local_rank):
     import paper_2609_34174_gb300 as gl
 
     device = torch.device("cuda", local_rank)
     torch.cuda.set_device(device)
     gl.load_library()
-    job = make_job(gl, wl, device, rank, args.gates, args.grads)
+    job = make_job(gl, wl, device, rank, args.gates, args.grads, args.fused)
     flush = None
     if job.input_bytes() < 2 * L2_BYTES:
         flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
@@ -1144,11 +1216,12 @@ def run_gradlev(args, wl, rank, world, local_rank):
     step_ms, value = combine_ranks(step_ms, job.tokens, world, device)
     pk = peaks()
     scans = {}
-    for name, ms in (("fwd", fwd_ms), ("costate", cos_ms)):
+    reads = (("fused", fwd_ms),) if job.kind == "fused" else (("fwd", fwd_ms), ("costate", cos_ms))
+    for name, ms in reads:
         fl, nb = job.counts(name)
         scans[name] = {"ms": round(ms, 4), "tokens_per_s": round(job.tokens / (ms / 1e3), 1),
                        "roofline": roofline_entry(fl, nb, ms / 1e3, pk)}
-    dominant = "costate" if cos_ms >= fwd_ms else "fwd"
+    dominant = "fused" if job.kind == "fused" else ("costate" if cos_ms >= fwd_ms else "fwd")
     rl = dict(scans[dominant]["roofline"])
     rl["kernel"] = job.kernel[dominant]
     rl["traffic"] = (None if (args.resize or args.gates or args.grads)
@@ -1156,6 +1229,8 @@ def run_gradlev(args, wl, rank, world, local_rank):
     cfg = {"workload": f"{args.workload}: {wl.name}", **job.config(),
            "tokens_per_step": job.tokens, "parallelism": f"replicas x{world}",
            "l2": "inputs larger than L2" if flush is None else "L2 flushed between steps"}
+    if job.kind == "fused":
+        cfg["step"] = "forward and costate reads in one pass (gradlev_fused_scan)"
     line = {"metric": GRADS_METRIC if args.grads else METRIC, "value": round(value, 1),
             "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms, 4),
@@ -1165,9 +1240,11 @@ def run_gradlev(args, wl, rank, world, local_rank):
     if rank == 0 and world == 1 and not args.no_e2e:
         line["e2e"] = e2e_measure(job, max(3, min(args.steps, 20)), stream)
     if (rank == 0 and world == 1 and args.workload == "c5" and not
-            (args.gates or args.grads or args.no_side)):
-        # the long-context workload, the other one with a roofline target
-        line["also"] = {"c4": side_scans(gl, "c4", device)}
+            (args.gates or args.grads or args.fused or args.no_side)):
+        # the long-context workload, the other one with a roofline target, and both
+        # workloads' reads in one fused pass
+        line["also"] = {"c4": side_scans(gl, "c4", device),
+                        "fused": {k: side_fused(gl, k, device) for k in ("c5", "c4")}}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
 
@@ -1192,6 +1269,8 @@ def main(argv=None):
                          "or document resets of packed sequences")
     ap.add_argument("--grads", action="store_true",
                     help="time the step-size gradients of both reads (suffix reads) instead")
+    ap.add_argument("--fused", action="store_true",
+                    help="time both reads of each map in one pass (gradlev_fused_scan) as the step")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-side", action="store_true",
                     help="skip the long-context (c4) scans added to the default line")

@@ -537,9 +537,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (FUSED && pending >= 0) {
                     // Both reads of a chunk: O_y = X S'^T and O_g = G S' from one S'^T tile
-                    // (read MN-major for the forward, K-major for the costate), then the
-                    // two P V products.  Each direction owns one O and one score buffer,
-                    // used once per chunk; the S'^T tiles alternate by chunk.
+                    // (read MN-major for the forward, K-major for the costate), each
+                    // followed by its P V product.  Each direction owns one O and one score
+                    // buffer, used once per chunk; the S'^T tiles alternate by chunk.
                     constexpr uint32_t ID_OK = idesc_bf16(128, 64, false, false);  // G S'
                     const Item I = decode_item<REV>(pending, p);
                     for (int c = 0; c < I.nch; ++c, ++n, c2 += 2) {
@@ -548,26 +548,33 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t sbb = cc & 1, sph = (cc >> 1) & 1, oph = cc & 1;
                         if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
                         if (!(ok = wait_or_fail(&st_ready[sbb], sph))) break;
-                        if (!(ok = wait_or_fail(&o_free[0], oph ^ 1))) break;
-                        if (!(ok = wait_or_fail(&o_free[1], oph ^ 1))) break;
-                        tc_fence_after();
                         const uint32_t st = sbase + s * Lay::kStageBytes;
                         const uint32_t tile = sbase + Lay::kStOff + sbb * Lay::kStBytes;
-                        const uint32_t x_lo = sdesc_lo(st + Lay::kQOff, 16);
-                        const uint32_t g_lo = sdesc_lo(st + Lay::kGOff, 16);
-                        const uint32_t s_mn = sdesc_lo(tile, kTile);
-                        const uint32_t s_k = sdesc_lo(tile, 16);
-#pragma unroll
-                        for (int kk = 0; kk < DQ / 16; ++kk)
-                            mma_bf16_ss(tmem + col_o(0), sdesc_from_lo(x_lo + kmaj_step(kk)),
-                                        sdesc_from_lo(s_mn + mnmaj_step(kk)), ID_O, kk > 0 ? 1u : 0u);
-#pragma unroll
-                        for (int kk = 0; kk < DQ / 16; ++kk)
-                            mma_bf16_ss(tmem + col_o(1), sdesc_from_lo(g_lo + kmaj_step(kk)),
-                                        sdesc_from_lo(s_k + kmaj_step(kk)), ID_OK, kk > 0 ? 1u : 0u);
-                        mma_commit(&st_free[sbb]);
+                        // direction 0 (forward) completes before direction 1 waits for its
+                        // O buffer, so the forward P V is never held up by the costate
+                        // epilogue of the previous chunk
 #pragma unroll 1
                         for (int dir = 0; dir < 2; ++dir) {
+                            if (!(ok = wait_or_fail(&o_free[dir], oph ^ 1))) break;
+                            tc_fence_after();
+                            if (dir == 0) {
+                                const uint32_t x_lo = sdesc_lo(st + Lay::kQOff, 16);
+                                const uint32_t s_mn = sdesc_lo(tile, kTile);
+#pragma unroll
+                                for (int kk = 0; kk < DQ / 16; ++kk)
+                                    mma_bf16_ss(tmem + col_o(0), sdesc_from_lo(x_lo + kmaj_step(kk)),
+                                                sdesc_from_lo(s_mn + mnmaj_step(kk)), ID_O,
+                                                kk > 0 ? 1u : 0u);
+                            } else {
+                                const uint32_t g_lo = sdesc_lo(st + Lay::kGOff, 16);
+                                const uint32_t s_k = sdesc_lo(tile, 16);
+#pragma unroll
+                                for (int kk = 0; kk < DQ / 16; ++kk)
+                                    mma_bf16_ss(tmem + col_o(1), sdesc_from_lo(g_lo + kmaj_step(kk)),
+                                                sdesc_from_lo(s_k + kmaj_step(kk)), ID_OK,
+                                                kk > 0 ? 1u : 0u);
+                                mma_commit(&st_free[sbb]);  // both reads of the tile issued
+                            }
                             if (!(ok = wait_or_fail(&p_ready[dir], oph))) break;
                             tc_fence_after();
                             // forward: V = ghat; costate: V = x (both MN-major [128 t][64])
