@@ -277,6 +277,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* z_ack = bars + 42;           // state warps: broadcast consumed
     uint64_t* drain = bars + 38;
     uint64_t* drain2 = bars + 39;
+    uint64_t* p1_seen = bars + 34;         // every phase-1 stage of an item consumed
     int* misc = reinterpret_cast<int*>(bars + 56);
     volatile int* abort_flag = misc + 0;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(misc + 1);
@@ -319,6 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(z_ack, kZActiveWarps);
         mbar_init(drain, 1);
         mbar_init(drain2, 1);
+        mbar_init(p1_seen, 1);
         if constexpr (REV) {
             mbar_init(&a_full[0], 1);
             mbar_init(&a_full[1], 1);
@@ -459,6 +461,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         if (!ok) break;
                         mma_commit(&dz_full[b]);
                         ++dzc;
+                        // every phase-1 stage of this item has been consumed: the back
+                        // issuer, which skips them, may now wait on the full barriers
+                        // after them (see there)
+                        mma_commit(p1_seen);
                     }
                 }
                 // phase 2 of the previous item: score and dZ of every chunk (dZ of the
@@ -516,7 +522,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // -------------------------------------------------- back MMA issuer
         if (lane == 0) {
             constexpr uint32_t ID_O = idesc_bf16(128, 64, false, true);  // Q S^T, P V
-            uint32_t n = 0, c2 = 0;
+            uint32_t n = 0, c2 = 0, p1c = 0;
             bool ok = true;
             auto wait_or_fail = [&](uint64_t* bar, uint32_t par) -> bool {
                 if (mbar_wait(bar, par, abort_flag)) return true;
@@ -529,11 +535,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!wait_or_fail(&item_full[slot], (it / kRing) & 1)) break;
                 const int item = item_slot[slot];
                 mbar_arrive(&item_empty[slot]);
-                // the new item's phase-1 stages precede the previous item's phase 2 and
-                // are released by the front issuer
+                // The new item's phase-1 stages precede the previous item's phase 2 and
+                // are consumed and released by the front issuer alone.  A ring slot whose
+                // phase-1 load this issuer never waited for can still be a phase behind,
+                // and a parity wait on it would then pass for the wrong round (and read
+                // the slot before its phase-2 tile lands); so the front issuer's p1_seen
+                // (its phase-1 products complete) comes first.  p1_seen cannot run two
+                // phases ahead of this wait: between two phase-1 passes the ring holds the
+                // phase-2 stages of a full segment (512 tokens or more; the shorter last
+                // segments take the highest tickets, after every phase-1 item), and the
+                // front issuer needs one of their slots, freed only by this issuer.
                 if (item >= 0) {
                     const Item In = decode_item<REV>(item, p);
-                    if (In.phase1) n += In.nch;
+                    if (In.phase1) {
+                        if (!(ok = wait_or_fail(p1_seen, p1c & 1))) break;
+                        ++p1c;
+                        n += In.nch;
+                    }
                 }
                 if (FUSED && pending >= 0) {
                     // Both reads of a chunk: O_y = X S'^T and O_g = G S' from one S'^T tile
