@@ -86,13 +86,16 @@ struct TcLayout {
     // Stage ring: what is left of the 227 KB opt-in budget after the two S^T
     // tiles, the two output staging tiles, the barrier block and the alignment
     // slack (at most 6 stages).
-    static constexpr int kAvail = 232448 - 2 * DQ * 128 - 2 * kTile - 1024 - 1024;
+    // REV: one more tile for the ring of dotted tiles (with the two idle staging tiles)
+    static constexpr int kExtraA = REV ? kTile : 0;
+    static constexpr int kAvail = 232448 - 2 * DQ * 128 - 2 * kTile - kExtraA - 1024 - 1024;
     static constexpr int kStages0 = kAvail / kStageBytes;
     static constexpr int kStages = kStages0 > 6 ? 6 : kStages0;
     static constexpr int kOOff = kStages * kStageBytes;  // two [128 t][64] output tiles
     static constexpr int kStOff = kOOff + 2 * kTile;
     static constexpr int kStBytes = DQ * 128;
-    static constexpr int kBarOff = kStOff + 2 * kStBytes;
+    static constexpr int kAOff = kStOff + 2 * kStBytes;
+    static constexpr int kBarOff = kAOff + kExtraA;
     static constexpr int kBarBytes = 1024;
     static constexpr int kSmemBytes = kBarOff + kBarBytes + 1024;  // + alignment slack
     // Bytes one stage receives in each pass.
@@ -271,7 +274,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* p_ready = bars + 36;         // [2] P written over the score buffer (P warps)
     uint64_t* o_staged = bars + 44;        // [2] output tile staged by all 4 epilogue warps
     uint64_t* o_buf_free = bars + 46;      // [2] output staging tile read by its TMA store
-    uint64_t* a_full = bars + 32;          // [2] (REV, dot) tile of the dotted tensor landed
+    uint64_t* a_full = bars + 60;          // [3] (REV, dot) tile of the dotted tensor landed
+    uint64_t* a_empty = bars + 63;         // [3] (REV, dot) its dot formed
     uint64_t* z_pub = bars + 40;           // state warps: all rows written before a flag
     uint64_t* z_lb = bars + 41;            // state warps: look-back result broadcast
     uint64_t* z_ack = bars + 42;           // state warps: broadcast consumed
@@ -286,6 +290,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
+    // (REV, dot) the ring of dotted tiles: the two output staging tiles, which a dot
+    // read leaves idle, and one more
+    auto a_tile = [&](uint32_t k) -> uint8_t* {
+        return smem + (k < 2 ? Lay::kOOff + k * kTile : Lay::kAOff);
+    };
     constexpr int kZActiveWarps = DQ / 32;          // state warps holding rows
     constexpr int kPHelpers = 4 - kZActiveWarps;    // state-slot warps building P half 1
     // REV (64-wide, separate q and k tiles) keeps the state rows in TMEM lanes 64..127,
@@ -322,8 +331,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(drain2, 1);
         mbar_init(p1_seen, 1);
         if constexpr (REV) {
-            mbar_init(&a_full[0], 1);
-            mbar_init(&a_full[1], 1);
+            for (int i = 0; i < 3; ++i) {
+                mbar_init(&a_full[i], 1);
+                mbar_init(&a_empty[i], 4);  // the four epilogue warps
+            }
         }
         *abort_flag = 0;
         fence_mbar_init();
@@ -347,8 +358,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
-            uint32_t n = 0;
+            uint32_t n = 0, an = 0;
             bool ok = true;
+            const bool dot = REV && p.epi.dot_out != nullptr;
             // Stream the stages of one pass of an item into the ring.
             auto load_pass = [&](const Item& I, int pass) {
                 for (int c = 0; c < I.nch && ok; ++c, ++n) {
@@ -379,6 +391,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tma_load_5d(st + Lay::kKOff + kb * kTile, &tm_k, &full[s], kb * 64, I.h, t0,
                                     I.b, I.l);
                     tma_load_5d(st + Lay::kVOff, &tm_v, &full[s], I.j * 64, I.h, t0, I.b, I.l);
+                    if (dot && pass == 2) {
+                        // the dotted tensor's tile, through its own three-deep ring
+                        const uint32_t k = an % 3;
+                        if (!mbar_wait(&a_empty[k], ((an / 3) & 1) ^ 1, abort_flag)) {
+                            raise_error(p, kErrWaitTimeout, abort_flag);
+                            ok = false;
+                            break;
+                        }
+                        mbar_arrive_expect_tx(&a_full[k], kTile);
+                        tma_load_5d(a_tile(k), &tm_o, &a_full[k], I.j * 64, I.h, t0, I.b, I.l);
+                        ++an;
+                    }
                 }
             };
             // Stage order: P1(i0), P1(i1), P2(i0), P1(i2), P2(i1), ...: phase 1 of a new
@@ -408,6 +432,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (n > (uint32_t)s) {
                         uint32_t last = ((n - 1 - s) / NS) * NS + s;
                         mbar_drain(&full[s], (last / NS) & 1);
+                    }
+                }
+                for (uint32_t k = 0; k < 3; ++k) {
+                    if (an > k) {
+                        const uint32_t last = ((an - 1 - k) / 3) * 3 + k;
+                        mbar_drain(&a_full[k], (last / 3) & 1);
                     }
                 }
             }
@@ -731,10 +761,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool storer = (warp == kWarpO0) && (lane == 0);  // issues the TMA stores
         const EpiParams& e = p.epi;
         uint32_t c2 = 0;
-        // (REV, dot) the storer loads each chunk's tile of the dotted tensor by TMA into
-        // the staging tile of that chunk (no rows are stored), two chunks ahead
-        const bool dot = REV && e.dot_out != nullptr;
-        uint32_t a_n[2] = {0u, 0u};
+        // (REV, dot) each chunk's tile of the dotted tensor arrives through the producer's
+        // three-deep ring (no rows are stored)
+        uint32_t ae = 0;
         for (int it = 0;; ++it) {
             const int slot = it % kRing;
             if (!warp_wait(&item_full[slot], (it / kRing) & 1, abort_flag)) {
@@ -747,17 +776,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (item < 0) break;
             const Item I = decode_item<REV>(item, p);
             bool ok = true;
-            auto load_a = [&](uint32_t b, int cc) {
-                mbar_arrive_expect_tx(&a_full[b], kTile);
-                tma_load_5d(smem + Lay::kOOff + b * kTile, &tm_o, &a_full[b], I.j * 64, I.h,
-                            chunk_t0<REV>(I, cc), I.b, I.l);
-                ++a_n[b];
-            };
-            if (dot && storer) {
-                // both staging tiles are free: every earlier chunk's dot has been formed
-                load_a(c2 & 1, 0);
-                if (I.nch > 1) load_a((c2 + 1) & 1, 1);
-            }
             for (int jb = 0; jb < kJobs * I.nch; ++jb, ++c2) {
                 // FUSED: job 2c is chunk c's forward read (y), job 2c+1 its costate read
                 const int c = FUSED ? (jb >> 1) : jb;
@@ -822,20 +840,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                         // dot_out[t] (+)= dot_scale * (row . a row) over this 64-wide tile.
                         // The tile of a (TMA, 128B-swizzled like an output tile) lets each
                         // lane read its own row without bank conflicts.
-                        if (!warp_wait(&a_full[ob], oph, abort_flag)) {
+                        const uint32_t ak = ae % 3;
+                        if (!warp_wait(&a_full[ak], (ae / 3) & 1, abort_flag)) {
                             raise_error(p, kErrWaitTimeout, abort_flag);
                             ok = false;
                             break;
                         }
+                        const uint32_t atile = smem_u32(a_tile(ak));
                         float acc = 0.f;
 #pragma unroll
                         for (int q = 0; q < 8; ++q) {
-                            const uint4 a4 = ld_shared_v4(otile + sw128_off(row, q));
+                            const uint4 a4 = ld_shared_v4(atile + sw128_off(row, q));
                             const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&a4);
 #pragma unroll
                             for (int i = 0; i < 8; ++i) acc = fmaf(v[8 * q + i], __bfloat162float(hb[i]), acc);
                         }
                         __syncwarp();
+                        if (lane == 0) mbar_arrive(&a_empty[ak]);
+                        ++ae;
                         if (valid) {
                             float* dst = e.dot_out + (((long long)I.l * p.B + I.b) * p.T + t) * p.H + I.h;
                             if (p.n_tiles > 1)
@@ -875,8 +897,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                         // the previous chunk's store (other tile) has finished reading
                         bulk_wait_group_read<1>();
                         if (c2 > 0) mbar_arrive(&o_buf_free[ob ^ 1]);
-                        // this chunk's dots are formed: its tile takes chunk c + 2
-                        if (dot && c + 2 < I.nch) load_a(ob, c + 2);
                     }
                 }
                 if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
@@ -887,10 +907,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) break;
         }
         if (storer) bulk_wait_group_all();
-        if (dot && storer) {  // every load issued has landed before the CTA exits
-            for (int b = 0; b < 2; ++b)
-                if (a_n[b] > 0) mbar_drain(&a_full[b], (a_n[b] - 1) & 1);
-        }
     } else {
         const int q4 = warp & 3;
         {
