@@ -25,6 +25,9 @@ cudaError_t launch_tc_suffix(const CUtensorMap& q, const CUtensorMap& k, const C
 cudaError_t launch_rowdot(const void* a, const TokStr& as, const void* r, const TokStr& rs,
                           float* out, int L, int B, int T, int H, int w, float scale, bool bf16,
                           cudaStream_t stream, bool sqdist = false);
+cudaError_t launch_tc_decay(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
+                            const CUtensorMap& o, const TcScanParams& p, bool costate, int grid,
+                            cudaStream_t stream);
 cudaError_t launch_tc_fused(const CUtensorMap& x, const CUtensorMap& ghat, const CUtensorMap& gout,
                             const CUtensorMap& y, const CUtensorMap& gin, const TcScanParams& p,
                             int grid, cudaStream_t stream);
@@ -657,7 +660,8 @@ int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
         for (int i = 0; i < 4; ++i) gpt.stride[i] = 0;
         return run_scan(desc, costate, x, &gpt, W0, 1.0f, g_out, act, out, out2, z, ws, base, stream);
     }
-    // with retention: the token-serial kernel
+    // with retention: the tensor-core chunked kernel for 64 x 64 bf16 maps whose
+    // tensors a TMA map can describe, else the kernels of gated.cu
     const int J = costate ? d.d_out : d.d_in;
     if (J > kGatedSerialMaxWidth) return GRADLEV_ERR_UNSUPPORTED;
     Tok tgo, to, to2, tz;
@@ -675,6 +679,47 @@ int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
     for (const Tok* t : all)
         if (t->data && (reinterpret_cast<uintptr_t>(t->data) % elem) != 0) return GRADLEV_ERR_UNSUPPORTED;
     if ((reinterpret_cast<uintptr_t>(W0) & 3u) != 0) return GRADLEV_ERR_INVALID_ARG;
+    if (bf16 && d.d_in == 64 && d.d_out == 64 && tc_layout_ok(tx, 2) && tc_layout_ok(tg, 2) &&
+        (!costate || tc_layout_ok(tgo, 2)) && tc_layout_ok(to, 2) && tc_layout_ok(to2, 2) &&
+        tc_layout_ok(tz, 2)) {
+        // 64 x 64 bf16 maps: the chunked retention scan on the tensor cores, one work
+        // item per unit (scan_decay_tc.cu)
+        const Tok& tq = costate ? tgo : tx;
+        const Tok& tk = costate ? tg : tx;
+        const Tok& tv = costate ? tx : tg;
+        CUtensorMap mq, mk, mv, mo;
+        if (!make_tmap(&mq, d, tq, 64) || !make_tmap(&mk, d, tk, 64) || !make_tmap(&mv, d, tv, 64) ||
+            !make_tmap(&mo, d, to, 64))
+            return GRADLEV_ERR_UNSUPPORTED;
+        const long long units = (long long)d.L * d.B * d.H;
+        gl::TcScanParams p;
+        memset(&p, 0, sizeof(p));
+        p.L = d.L;
+        p.B = d.B;
+        p.T = d.T;
+        p.H = d.H;
+        p.dq = 64;
+        p.dv = 64;
+        p.n_tiles = 1;
+        p.seg_len = d.T;
+        p.n_seg = 1;
+        p.n_items = (int)units;
+        p.n_ut = (int)units;
+        p.lam = 1.0f;
+        p.inv_lam = 1.0f;
+        p.mu = 1.0f;
+        p.w0_transposed = costate ? 1 : 0;
+        p.W0 = W0;
+        p.g_eta = eta_t;
+        p.g_alpha = alpha_t;
+        fill_epi(&p.epi, to, to2, tz, act);
+        p.ctrl = static_cast<unsigned int*>(ws);
+        if (cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
+        const int grid = units < dev.sms ? (int)units : dev.sms;
+        if (gl::launch_tc_decay(mq, mk, mv, mo, p, costate, grid, stream) != cudaSuccess)
+            return GRADLEV_ERR_CUDA;
+        return GRADLEV_OK;
+    }
     if (cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
     gl::GatedParams p;
     memset(&p, 0, sizeof(p));

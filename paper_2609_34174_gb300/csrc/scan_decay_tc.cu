@@ -1,0 +1,942 @@
+// scan_decay_tc.cu -- tensor-core (tcgen05) chunked scan with retention, for bf16
+// maps of 64 x 64: Eq. 2 with per-token step sizes eta_t and retention alpha_t and
+// the decay centred at the slow weights,
+//
+//     W_{t+1} = W0 + alpha_t (W_t - W0) - eta_t ghat_t x_t^T,     W_0 = W0,
+//
+// read before each write (Sec. 3, "Observation"; Eqs. 3-4; Appendix C).  In the
+// orientation shared by both reads, with S the fast weights minus W0 (transposed so
+// that rows are the read's contraction index q):
+//   forward  q = k = x, v = ghat, B0 = W0,   S^T = (W - W0)^T   [d][m]
+//   costate  q = g_out, k = ghat, v = x, B0 = W0^T, S^T = (W - W0) [m][d]
+// and over a chunk of C = 128 tokens from the state S at its first token,
+//
+//   o_t = B0 q_t + a_t S q_t - sum_{s<t} E_ts (k_s . q_t) v_s
+//   S'  = a_end S - sum_s w_s v_s k_s^T
+//
+// with a_t = prod_{r<t} alpha_r, E_ts = eta_s prod_{s<r<t} alpha_r,
+// w_s = eta_s prod_{r>s} alpha_r and a_end the product of the chunk's alphas
+// (indices local to the chunk; tokens past T carry alpha = 1, eta = 0).  The decays
+// are plain products of alphas, never ratios or logarithms, so a reset (alpha = 0)
+// and underflow give exact zeros and any real alpha is valid.  They are assembled
+// from 8-token pieces: sig_s (alphas after s to the end of its piece), pim_t (alphas
+// from the start of t's piece up to t) and the piece products tp_j, so that for s in
+// an earlier piece than t, E_ts = (eta_s sig_s) * pim_t * prod_{js<i<jt} tp_i.
+//
+// All three terms of o land in one TMEM accumulator:
+//   O  = Q B0^T                 (B0^T tile in shared memory, per unit)
+//   O += P' V                   P'_ts = -E_ts (q_t . k_s), built over the score
+//   O += Q' S^T                 Q' = diag(a) Q, written by the P warps into the
+//                               free columns of the score buffer (TS product)
+// and the state update is dZ = K^T (W V), with the rows of V scaled by -w_s into a
+// shared-memory tile, then S' = a_end S + dZ in the state warps (fp32 rows).
+//
+// Warp roles (16 warps), with the rings and bounded waits of the chunk kernel of
+// scan_tc.cu:
+//   warp 0      TMA producer (stage = [q | k | v], or [qk | v] forward)
+//   warp 1      front MMA issuer: the score Q K^T of chunk c, then the state update
+//               dZ of chunk c - 1 (one chunk behind, so that the score never waits
+//               for the W V tile)
+//   warp 14     back MMA issuer: Q B0^T, then (P' ready) P' V, then (S ready) Q' S^T
+//   warp 15     gate factors of each chunk from alpha_t and eta_t, in registers and
+//               shuffles, into a ring of three blocks one or two chunks ahead
+//   warps 2-5   P' over score columns 0..63 and Q' (rows 0..63 also zero 64..127)
+//   warps 10-11 P' over columns 64..127 of rows 64..127
+//   (warps 2-3 and 10-11 then write the chunk's W V rows, 0..63 and 64..127)
+//   warps 6-9   epilogue (TMEM -> bf16 staging -> TMA store), as in scan_tc.cu
+//   warps 12-13 state rows, B0^T and S^T tiles, S' = a_end S + dZ
+// One work item is one unit (the chunks of a unit run in order in one CTA).
+#include <cuda.h>
+
+#include "scan_common.cuh"
+#include "sm103_ptx.cuh"
+
+namespace gl {
+namespace dec {
+
+constexpr int kChunk = 128;
+constexpr int kTile = 16384;   // [128 rows][64 bf16], 128-byte swizzle
+constexpr int kStTile = 8192;  // [64 rows][64 bf16]
+constexpr int kWarps = 16;
+constexpr int kThreads = kWarps * 32;
+constexpr int kWarpO0 = 6, kWarpZ0 = 10, kWarpBack = 14, kWarpGate = 15;
+constexpr int kRing = 4;
+constexpr int kItemConsumers = 2 + 4 + 4 + 2 + 2 + 1;
+constexpr uint32_t kTmemCols = 512;
+__host__ __device__ constexpr uint32_t col_sc(uint32_t i) { return i * 128u; }
+__host__ __device__ constexpr uint32_t col_o(uint32_t i) { return 256u + i * 64u; }
+__host__ __device__ constexpr uint32_t col_dz(uint32_t i) { return 384u + i * 64u; }
+constexpr uint32_t kQpCol = 32;  // Q' in columns 32..63 of the score buffer
+
+// Gate block of one chunk (floats), written by the gate warp: per token alpha, eta,
+// -eta_s sig_s, pim_t, a_t and w_t; the products between pieces
+// tpm[j][jt] = prod_{j<i<jt} tp_i (0 for j >= jt) and a_end.
+constexpr int kGbAl = 0, kGbEt = 128, kGbNse = 256, kGbPim = 384, kGbA = 512, kGbW = 640;
+constexpr int kGbTpm = 768, kGbEnd = 1024;
+constexpr int kGbFloats = 1032;  // a multiple of 8 floats: every block 32-byte aligned
+constexpr int kGbBytes = kGbFloats * 4;
+constexpr int kGbRing = 3;
+
+template <bool COSTATE>
+struct DLayout {
+    static constexpr int kQOff = 0;
+    static constexpr int kKOff = COSTATE ? kTile : 0;
+    static constexpr int kVOff = COSTATE ? 2 * kTile : kTile;
+    static constexpr int kStageBytes = (COSTATE ? 3 : 2) * kTile;
+    // fixed regions: the output staging tile, two S^T tiles, the B0^T tile, the W V
+    // tile, the ring of gate blocks, barriers
+    static constexpr int kFixed = kTile + 2 * kStTile + kStTile + kTile + kGbRing * kGbBytes;
+    static constexpr int kAvail = 232448 - kFixed - 1024 - 1024;
+    static constexpr int kStages0 = kAvail / kStageBytes;
+    static constexpr int kStages = kStages0 > 6 ? 6 : kStages0;
+    static constexpr int kOOff = kStages * kStageBytes;
+    static constexpr int kStOff = kOOff + kTile;
+    static constexpr int kB0Off = kStOff + 2 * kStTile;
+    static constexpr int kWvOff = kB0Off + kStTile;
+    static constexpr int kGfOff = kWvOff + kTile;
+    static constexpr int kBarOff = kGfOff + kGbRing * kGbBytes;
+    static constexpr int kSmemBytes = kBarOff + 1024 + 1024;
+    static_assert(kStages >= 3, "the lagged state update holds two stages");
+    static_assert(kSmemBytes <= 232448, "shared memory budget exceeded");
+    static_assert(kGfOff % 32 == 0 && kBarOff % 8 == 0, "alignment");
+};
+
+struct Item {
+    int l, b, h, nch;
+};
+
+__device__ __forceinline__ Item decode_unit(int item, const TcScanParams& p) {
+    Item I;
+    I.h = item % p.H;
+    const int lb = item / p.H;
+    I.b = lb % p.B;
+    I.l = lb / p.B;
+    I.nch = (p.T + kChunk - 1) / kChunk;
+    return I;
+}
+
+__device__ __forceinline__ void raise_error(const TcScanParams& p, unsigned int bits,
+                                            volatile int* abort_flag) {
+    atomicOr(p.ctrl + 1, bits);
+    if (abort_flag) *abort_flag = 1;
+}
+
+__device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
+    uint64_t t0 = globaltimer_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (globaltimer_ns() - t0 > 200000000ull) break;  // 0.2 s
+    }
+}
+
+// The bounded wait out of line, so that the kernel's many wait sites share one copy
+// of the loop (instruction-cache footprint); the first probe stays inline.
+__device__ __noinline__ bool wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+    return mbar_wait(bar, parity, abort_flag);
+}
+__device__ __forceinline__ bool bwait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+    return mbar_try_wait(bar, parity) || wait_slow(bar, parity, abort_flag);
+}
+
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+    const int lane = threadIdx.x & 31;
+    int ok = 1;
+    if (lane == 0) ok = bwait(bar, parity, abort_flag) ? 1 : 0;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    __syncwarp();
+    return ok != 0;
+}
+
+__host__ __device__ constexpr uint32_t kmaj_step(int kk) {
+    return (uint32_t)(((kk >> 2) * kTile + (kk & 3) * 32) >> 4);
+}
+__host__ __device__ constexpr uint32_t mnmaj_step(int kk) { return (uint32_t)((kk * 2048) >> 4); }
+
+__device__ __forceinline__ float4 lds4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+
+// v *= sigma'(z) / out2 = sigma(v) for one 64-wide output row (MLP layer fusion).
+__device__ __noinline__ void epi_apply_dact(const EpiParams& e, long long z_off, float* v) {
+    const __nv_bfloat16* zp = static_cast<const __nv_bfloat16*>(e.zin) + z_off;
+    for (int q = 0; q < 8; ++q) {
+        const uint4 zz = *reinterpret_cast<const uint4*>(zp + 8 * q);
+        const __nv_bfloat16* zb = reinterpret_cast<const __nv_bfloat16*>(&zz);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[8 * q + i] *= act_df(e.act, __bfloat162float(zb[i]));
+    }
+}
+__device__ __noinline__ void epi_store_act(const EpiParams& e, long long o_off, const float* v) {
+    __nv_bfloat16* op2 = static_cast<__nv_bfloat16*>(e.out2) + o_off;
+    for (int q = 0; q < 8; ++q) {
+        uint4 w;
+        w.x = pack_bf16x2(act_f(e.act, v[8 * q + 0]), act_f(e.act, v[8 * q + 1]));
+        w.y = pack_bf16x2(act_f(e.act, v[8 * q + 2]), act_f(e.act, v[8 * q + 3]));
+        w.z = pack_bf16x2(act_f(e.act, v[8 * q + 4]), act_f(e.act, v[8 * q + 5]));
+        w.w = pack_bf16x2(act_f(e.act, v[8 * q + 6]), act_f(e.act, v[8 * q + 7]));
+        *reinterpret_cast<uint4*>(op2 + 8 * q) = w;
+    }
+}
+
+// -E_ts for the tokens s = 8 jt + i of t's own piece: -eta_s prod_{s<r<t} alpha_r for
+// s < t, else 0.
+__device__ __forceinline__ void same_piece_decays(const float* gb, int row, float (&ndd)[8]) {
+    const int jt = row >> 3, it = row & 7;
+    const float4 a0 = lds4(gb + kGbAl + 8 * jt), a1 = lds4(gb + kGbAl + 8 * jt + 4);
+    const float4 e0 = lds4(gb + kGbEt + 8 * jt), e1 = lds4(gb + kGbEt + 8 * jt + 4);
+    const float al[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+    const float et[8] = {e0.x, e0.y, e0.z, e0.w, e1.x, e1.y, e1.z, e1.w};
+    float run = 1.0f;
+#pragma unroll
+    for (int i = 7; i >= 0; --i) {
+        const bool lt = i < it;
+        ndd[i] = lt ? -et[i] * run : 0.0f;
+        run = lt ? run * al[i] : run;
+    }
+}
+
+// Store 4 consecutive 32-bit columns of this thread's TMEM lane without waiting.
+__device__ __forceinline__ void tmem_st4_async(uint32_t taddr, uint32_t a, uint32_t b, uint32_t c,
+                                               uint32_t d) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr), "r"(a),
+                 "r"(b), "r"(c), "r"(d)
+                 : "memory");
+}
+
+// P'_ts = -E_ts (q_t . k_s) over the 64 score columns of pieces PB .. PB+7 of this
+// lane's row: the fp32 scores at TMEM columns taddr .. taddr+63 become 32 packed bf16
+// columns at taddr (stores issued, not waited).  Two pieces per step, in increasing
+// order, so that no packed store reaches a score column still to be read.
+// ALL_BEFORE: every one of these pieces precedes t's own piece.
+template <int PB, bool ALL_BEFORE>
+__device__ __forceinline__ void build_p64(uint32_t taddr, const float* gb, int row, float pim) {
+    const int jt = row >> 3;
+    const int jmax = (row | 31) >> 3;  // the last piece of this warp's rows
+    float ndd[8];
+    if (!ALL_BEFORE) same_piece_decays(gb, row, ndd);
+#pragma unroll 1
+    for (int m = 0; m < 4; ++m) {
+        if (!ALL_BEFORE && PB + 2 * m > jmax) {  // after every row of the warp: masked
+            const uint32_t z[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+            tmem_st8_async(taddr + 8 * m, z);
+            continue;
+        }
+        float v[16];
+        tmem_ld16(taddr + 16 * m, v);
+        uint32_t w[8];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int j = PB + 2 * m + h;
+            const float tau = pim * gb[kGbTpm + 16 * j + jt];  // 0 unless j < jt
+            const float4 s0 = lds4(gb + kGbNse + 8 * j);
+            const float4 s1 = lds4(gb + kGbNse + 8 * j + 4);
+            float e[8] = {s0.x * tau, s0.y * tau, s0.z * tau, s0.w * tau,
+                          s1.x * tau, s1.y * tau, s1.z * tau, s1.w * tau};
+            if (!ALL_BEFORE) {
+                const bool same = j == jt;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) e[i] = same ? ndd[i] : e[i];
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                w[4 * h + i] = pack_bf16x2(e[2 * i] * v[8 * h + 2 * i], e[2 * i + 1] * v[8 * h + 2 * i + 1]);
+        }
+        tmem_st8_async(taddr + 8 * m, w);
+    }
+}
+
+template <bool COSTATE>
+__global__ void __launch_bounds__(kThreads, 1)
+    decay_scan_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                      const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
+                      const TcScanParams p) {
+    using Lay = DLayout<COSTATE>;
+    constexpr int NS = Lay::kStages;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~static_cast<uintptr_t>(1023));
+    const uint32_t sbase = smem_u32(smem);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Lay::kBarOff);
+    uint64_t* full = bars;                 // [NS] stage landed
+    uint64_t* empty = bars + 8;            // [NS] stage read by both MMA issuers
+    uint64_t* sc_full = bars + 16;         // [2] score in TMEM
+    uint64_t* sc_free = bars + 18;         // [2] score/P' buffer reusable
+    uint64_t* o_full = bars + 20;          // [2]
+    uint64_t* o_free = bars + 22;          // [2]
+    uint64_t* dz_full = bars + 24;         // [2]
+    uint64_t* dz_free = bars + 26;         // [2]
+    uint64_t* st_ready = bars + 28;        // [2]
+    uint64_t* st_free = bars + 30;         // [2]
+    uint64_t* gf_full = bars + 32;         // [3] gate block of a chunk written
+    uint64_t* gf_free = bars + 35;         // [3] gate block read by every user
+    uint64_t* p_ready = bars + 38;         // [2] P' (and Q') in TMEM
+    uint64_t* b0_ready = bars + 40;        // B0^T tile of the current unit written
+    uint64_t* b0_free = bars + 41;         // B0^T tile no longer read
+    uint64_t* drain = bars + 42;
+    uint64_t* drain2 = bars + 43;
+    uint64_t* o_staged = bars + 44;        // [2]
+    uint64_t* o_buf_free = bars + 46;      // the staging tile read by its store
+    uint64_t* wv_ready = bars + 47;        // the W V tile written
+    uint64_t* wv_free = bars + 48;         // the W V tile read by the dZ product
+    uint64_t* item_full = bars + 49;       // [kRing]
+    uint64_t* item_empty = bars + 53;      // [kRing]
+    int* misc = reinterpret_cast<int*>(bars + 57);
+    volatile int* abort_flag = misc + 0;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(misc + 1);
+    volatile int* item_slot = misc + 4;    // [kRing]
+    float* gfb = reinterpret_cast<float*>(smem + Lay::kGfOff);  // [kGbRing][kGbFloats]
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < NS; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 2);  // both MMA issuers
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&sc_full[i], 1);
+            mbar_init(&sc_free[i], 1);
+            mbar_init(&p_ready[i], 6);   // warps 2-5 and the two helpers
+            mbar_init(&o_staged[i], 4);
+            mbar_init(&o_full[i], 1);
+            mbar_init(&o_free[i], 4);
+            mbar_init(&dz_full[i], 1);
+            mbar_init(&dz_free[i], 2);   // the two state warps
+            mbar_init(&st_ready[i], 2);
+            mbar_init(&st_free[i], 1);
+        }
+        for (int i = 0; i < kRing; ++i) {
+            mbar_init(&item_full[i], 1);
+            mbar_init(&item_empty[i], kItemConsumers);
+        }
+        for (int i = 0; i < kGbRing; ++i) {
+            mbar_init(&gf_full[i], 1);
+            mbar_init(&gf_free[i], 4 + 2 + 2);  // warps 2-5, the helpers, the state warps
+        }
+        mbar_init(wv_ready, 4);  // warps 2-3 and the two helpers
+        mbar_init(wv_free, 1);
+        mbar_init(o_buf_free, 1);
+        mbar_init(b0_ready, 2);
+        mbar_init(b0_free, 1);
+        mbar_init(drain, 1);
+        mbar_init(drain2, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, kTmemCols);
+        tmem_relinquish();
+        tc_fence_before();
+    }
+    if (warp == 0 && lane == 0) {
+        prefetch_tmap(&tm_q);
+        prefetch_tmap(&tm_k);
+        prefetch_tmap(&tm_v);
+        prefetch_tmap(&tm_o);
+    }
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    // next item from the ring (every role warp reads every slot in order)
+    auto take_item = [&](int it, int& item) -> bool {
+        const int slot = it % kRing;
+        if (!warp_wait(&item_full[slot], (it / kRing) & 1, abort_flag)) {
+            raise_error(p, kErrWaitTimeout, abort_flag);
+            return false;
+        }
+        item = item_slot[slot];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&item_empty[slot]);
+        return true;
+    };
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            uint32_t n = 0;
+            bool ok = true;
+            for (int it = 0; ok; ++it) {
+                const int slot = it % kRing;
+                if (!bwait(&item_empty[slot], ((it / kRing) & 1) ^ 1, abort_flag)) {
+                    raise_error(p, kErrWaitTimeout, abort_flag);
+                    break;
+                }
+                int item = static_cast<int>(atomicAdd(p.ctrl, 1u));
+                if (item >= p.n_items) item = -1;
+                item_slot[slot] = item;
+                mbar_arrive(&item_full[slot]);
+                if (item < 0) break;
+                const Item I = decode_unit(item, p);
+                for (int c = 0; c < I.nch; ++c, ++n) {
+                    const int s = n % NS;
+                    if (!bwait(&empty[s], ((n / NS) & 1) ^ 1, abort_flag)) {
+                        raise_error(p, kErrWaitTimeout, abort_flag);
+                        ok = false;
+                        break;
+                    }
+                    uint8_t* st = smem + s * Lay::kStageBytes;
+                    const int t0 = c * kChunk;
+                    mbar_arrive_expect_tx(&full[s], Lay::kStageBytes);
+                    if (COSTATE) tma_load_5d(st + Lay::kQOff, &tm_q, &full[s], 0, I.h, t0, I.b, I.l);
+                    tma_load_5d(st + Lay::kKOff, &tm_k, &full[s], 0, I.h, t0, I.b, I.l);
+                    tma_load_5d(st + Lay::kVOff, &tm_v, &full[s], 0, I.h, t0, I.b, I.l);
+                }
+            }
+            if (*abort_flag) {  // every issued load has landed before the CTA exits
+                for (int s = 0; s < NS; ++s) {
+                    if (n > (uint32_t)s) {
+                        const uint32_t last = ((n - 1 - s) / NS) * NS + s;
+                        mbar_drain(&full[s], (last / NS) & 1);
+                    }
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------- front MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t ID_SC = idesc_bf16(128, 128, false, false);  // Q K^T
+            constexpr uint32_t ID_DZ = idesc_bf16(128, 64, true, true);     // K^T (W V)
+            const uint32_t wv = sbase + Lay::kWvOff;
+            uint32_t n = 0, c2 = 0, dzc = 0;
+            bool ok = true;
+            auto wait_or_fail = [&](uint64_t* bar, uint32_t par) -> bool {
+                if (bwait(bar, par, abort_flag)) return true;
+                raise_error(p, kErrWaitTimeout, abort_flag);
+                return false;
+            };
+            for (int it = 0; ok; ++it) {
+                const int slot = it % kRing;
+                if (!wait_or_fail(&item_full[slot], (it / kRing) & 1)) break;
+                const int item = item_slot[slot];
+                mbar_arrive(&item_empty[slot]);
+                if (item < 0) break;
+                const Item I = decode_unit(item, p);
+                for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
+                    const int s = n % NS;
+                    const uint32_t sb = c2 & 1;
+                    if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
+                    if (!(ok = wait_or_fail(&sc_free[sb], ((c2 >> 1) & 1) ^ 1))) break;
+                    tc_fence_after();
+                    const uint32_t st = sbase + s * Lay::kStageBytes;
+                    const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
+                    const uint32_t k_lo = sdesc_lo(st + Lay::kKOff, 16);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        mma_bf16_ss(tmem + col_sc(sb), sdesc_from_lo(q_lo + kmaj_step(kk)),
+                                    sdesc_from_lo(k_lo + kmaj_step(kk)), ID_SC, kk > 0 ? 1u : 0u);
+                    mma_commit(&sc_full[sb]);
+                    if (c > 0) {
+                        // dZ of the previous chunk = K^T (W V): A = K^T (MN-major, 64-wide M
+                        // blocks 16 KB apart; the second block's rows land in TMEM lanes
+                        // 64..127, unread)
+                        const int sp = static_cast<int>((n - 1) % NS);
+                        const uint32_t b = dzc & 1;
+                        if (!(ok = wait_or_fail(&dz_free[b], ((dzc >> 1) & 1) ^ 1))) break;
+                        if (!(ok = wait_or_fail(wv_ready, dzc & 1))) break;
+                        tc_fence_after();
+                        const uint32_t a_lo = sdesc_lo(sbase + sp * Lay::kStageBytes + Lay::kKOff, kTile);
+                        const uint32_t b_lo = sdesc_lo(wv, kTile);
+#pragma unroll
+                        for (int kk = 0; kk < kChunk / 16; ++kk)
+                            mma_bf16_ss(tmem + col_dz(b), sdesc_from_lo(a_lo + mnmaj_step(kk)),
+                                        sdesc_from_lo(b_lo + mnmaj_step(kk)), ID_DZ, kk > 0 ? 1u : 0u);
+                        mma_commit(&dz_full[b]);
+                        mma_commit(wv_free);
+                        mma_commit(&empty[sp]);
+                        ++dzc;
+                    }
+                    if (c == I.nch - 1) mma_commit(&empty[s]);  // no state update reads it
+                }
+            }
+            mma_commit(drain);
+            mbar_drain(drain, 0);
+        }
+    } else if (warp == kWarpBack) {
+        // -------------------------------------------------- back MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t ID_O = idesc_bf16(128, 64, false, true);  // [Q|P'|Q'] x [B0^T|V|S^T]
+            uint32_t n = 0, c2 = 0, ucnt = 0;
+            bool ok = true;
+            auto wait_or_fail = [&](uint64_t* bar, uint32_t par) -> bool {
+                if (bwait(bar, par, abort_flag)) return true;
+                raise_error(p, kErrWaitTimeout, abort_flag);
+                return false;
+            };
+            const uint32_t b0_lo = sdesc_lo(sbase + Lay::kB0Off, kTile);
+            for (int it = 0; ok; ++it) {
+                const int slot = it % kRing;
+                if (!wait_or_fail(&item_full[slot], (it / kRing) & 1)) break;
+                const int item = item_slot[slot];
+                mbar_arrive(&item_empty[slot]);
+                if (item < 0) break;
+                const Item I = decode_unit(item, p);
+                if (!(ok = wait_or_fail(b0_ready, ucnt & 1))) break;
+                for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
+                    const int s = n % NS;
+                    const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
+                    if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
+                    if (!(ok = wait_or_fail(&o_free[ob], oph ^ 1))) break;
+                    tc_fence_after();
+                    const uint32_t st = sbase + s * Lay::kStageBytes;
+                    // O = Q B0^T
+                    const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        mma_bf16_ss(tmem + col_o(ob), sdesc_from_lo(q_lo + kmaj_step(kk)),
+                                    sdesc_from_lo(b0_lo + mnmaj_step(kk)), ID_O, kk > 0 ? 1u : 0u);
+                    if (!(ok = wait_or_fail(&p_ready[ob], oph))) break;
+                    tc_fence_after();
+                    // O += P' V  (P' over the score buffer: tokens s < 64 in columns 0..31,
+                    // s >= 64 in columns 64..95)
+                    const uint32_t v_lo = sdesc_lo(st + Lay::kVOff, kTile);
+#pragma unroll
+                    for (int kk = 0; kk < kChunk / 16; ++kk)
+                        mma_bf16_ts(tmem + col_o(ob), tmem + col_sc(ob) + (kk < 4 ? kk * 8 : 64 + (kk - 4) * 8),
+                                    sdesc_from_lo(v_lo + mnmaj_step(kk)), ID_O, 1u);
+                    // O += Q' S^T  (A = a_t q_t from TMEM columns 32..63 of the score buffer)
+                    if (!(ok = wait_or_fail(&st_ready[ob], oph))) break;
+                    tc_fence_after();
+                    const uint32_t s_lo = sdesc_lo(sbase + Lay::kStOff + ob * kStTile, kTile);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        mma_bf16_ts(tmem + col_o(ob), tmem + col_sc(ob) + kQpCol + kk * 8,
+                                    sdesc_from_lo(s_lo + mnmaj_step(kk)), ID_O, 1u);
+                    mma_commit(&st_free[ob]);
+                    mma_commit(&o_full[ob]);
+                    mma_commit(&sc_free[ob]);
+                    mma_commit(&empty[s]);
+                }
+                if (!ok) break;
+                mma_commit(b0_free);  // every product of this unit that reads B0^T issued
+                ++ucnt;
+            }
+            mma_commit(drain2);
+            mbar_drain(drain2, 0);
+        }
+    } else if (warp == kWarpGate) {
+        // ------------------------------------------------------- gate factors
+        // Lane l takes tokens 4l .. 4l+3 of each chunk, so piece j (8 tokens) is lanes
+        // 2j and 2j+1.  Products inside a lane, then across the lane pair, then over the
+        // 16 pieces by shuffles; every factor is a plain product of alphas.
+        uint32_t cc = 0;
+        bool ok = true;
+        for (int it = 0; ok; ++it) {
+            int item;
+            if (!take_item(it, item) || item < 0) break;
+            const Item I = decode_unit(item, p);
+            const long long gbase = ((long long)I.l * p.B + I.b) * p.T * p.H + I.h;
+            // this lane's gates of chunk c (alpha = 1, eta = 0 past T)
+            auto load = [&](int c, float (&al)[4], float (&et)[4]) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int tg = c * kChunk + 4 * lane + i;
+                    const bool in = tg < p.T;
+                    const long long gi = gbase + (long long)(in ? tg : 0) * p.H;
+                    al[i] = in ? (p.g_alpha ? __ldg(p.g_alpha + gi) : 1.0f) : 1.0f;
+                    et[i] = in ? __ldg(p.g_eta + gi) : 0.0f;
+                }
+            };
+            float nal[4], net[4];
+            load(0, nal, net);
+            for (int c = 0; c < I.nch; ++c, ++cc) {
+                float al[4], et[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    al[i] = nal[i];
+                    et[i] = net[i];
+                }
+                if (c + 1 < I.nch) load(c + 1, nal, net);
+                // inside the lane: alphas before / after each token
+                const float pre[4] = {1.0f, al[0], al[0] * al[1], al[0] * al[1] * al[2]};
+                const float suf[4] = {al[1] * al[2] * al[3], al[2] * al[3], al[3], 1.0f};
+                const float prod = pre[3] * al[3];
+                const float other = __shfl_xor_sync(0xffffffffu, prod, 1);
+                const bool hi = lane & 1;  // second half of the piece
+                const float tp = hi ? other * prod : prod * other;
+                // inclusive prefix / suffix of the piece products (pieces are lane pairs)
+                float incl = tp, sincl = tp;
+#pragma unroll
+                for (int o = 2; o < 32; o <<= 1) {
+                    const float u = __shfl_up_sync(0xffffffffu, incl, o);
+                    const float d = __shfl_down_sync(0xffffffffu, sincl, o);
+                    if (lane >= o) incl = u * incl;
+                    if (lane + o < 32) sincl = sincl * d;
+                }
+                float before = __shfl_up_sync(0xffffffffu, incl, 2);   // pieces before j
+                float after = __shfl_down_sync(0xffffffffu, sincl, 2); // pieces after j
+                if (lane < 2) before = 1.0f;
+                if (lane >= 30) after = 1.0f;
+                const float a_end = __shfl_sync(0xffffffffu, incl, 31);
+                const uint32_t k = cc % kGbRing;
+                if (!warp_wait(&gf_free[k], ((cc / kGbRing) & 1) ^ 1, abort_flag)) {
+                    raise_error(p, kErrWaitTimeout, abort_flag);
+                    ok = false;
+                    break;
+                }
+                float* gb = gfb + k * kGbFloats;
+                float pim[4], nse[4], at[4], wt[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    pim[i] = hi ? other * pre[i] : pre[i];  // alphas before t in its piece
+                    const float sig = hi ? suf[i] : suf[i] * other;  // after s in its piece
+                    const float es = et[i] * sig;
+                    nse[i] = -es;
+                    at[i] = before * pim[i];
+                    wt[i] = es * after;
+                }
+                const int t4 = 4 * lane;
+                *reinterpret_cast<float4*>(gb + kGbAl + t4) = make_float4(al[0], al[1], al[2], al[3]);
+                *reinterpret_cast<float4*>(gb + kGbEt + t4) = make_float4(et[0], et[1], et[2], et[3]);
+                *reinterpret_cast<float4*>(gb + kGbNse + t4) = make_float4(nse[0], nse[1], nse[2], nse[3]);
+                *reinterpret_cast<float4*>(gb + kGbPim + t4) = make_float4(pim[0], pim[1], pim[2], pim[3]);
+                *reinterpret_cast<float4*>(gb + kGbA + t4) = make_float4(at[0], at[1], at[2], at[3]);
+                *reinterpret_cast<float4*>(gb + kGbW + t4) = make_float4(wt[0], wt[1], wt[2], wt[3]);
+                // tpm[j][jt] = prod_{j<i<jt} tp_i (0 for j >= jt): lane l fills column
+                // jt = l / 2, rows 8 (l % 2) .. +7
+                {
+                    float tpa[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) tpa[i] = __shfl_sync(0xffffffffu, tp, 2 * i);
+                    const int jc = lane >> 1, j0 = 8 * (lane & 1);
+                    float run = 1.0f;
+#pragma unroll
+                    for (int j = 15; j >= 0; --j) {
+                        const bool lt = j < jc;
+                        const float val = lt ? run : 0.0f;
+                        run = lt ? run * tpa[j] : run;
+                        if (j >= j0 && j < j0 + 8) gb[kGbTpm + 16 * j + jc] = val;
+                    }
+                }
+                if (lane == 0) gb[kGbEnd] = a_end;
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&gf_full[k]);
+            }
+        }
+    } else if (warp < kWarpO0 || warp == kWarpZ0 || warp == kWarpZ0 + 1) {
+        // ------------------------------------------------ P', Q' and the W V rows
+        // Warps 2-5 own token rows row = 32 (warp & 3) + lane of each chunk: P' over
+        // columns 0..63 (rows < 64 also zero columns 64..127) and Q' = a_t q_t.  The
+        // two helpers build P' over columns 64..127 of rows 64..127.  Then warps 2-3
+        // (whose P' has no masked column) and the helpers write the chunk's W V rows
+        // -w_t v_t (rows 0..63 and 64..127), which the front issuer's state update
+        // reads one chunk later.
+        const bool helper = warp >= kWarpZ0;
+        const int q4 = warp & 3;
+        const int row = q4 * 32 + lane;
+        const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
+        const bool wv_writer = helper || q4 >= 2;
+        const int wv_row = helper ? row : row - 64;
+        uint32_t c2 = 0, wvn = 0;
+        bool ok = true;
+        for (int it = 0; ok; ++it) {
+            int item;
+            if (!take_item(it, item) || item < 0) break;
+            const Item I = decode_unit(item, p);
+            for (int c = 0; c < I.nch; ++c, ++c2) {
+                const uint32_t sb = c2 & 1;
+                const int s = static_cast<int>(c2 % NS);  // ring slot: every stage is a chunk
+                const uint32_t st = sbase + s * Lay::kStageBytes;
+                const uint32_t gk = c2 % kGbRing;
+                const float* gb = gfb + gk * kGbFloats;
+                if (!warp_wait(&gf_full[gk], (c2 / kGbRing) & 1, abort_flag) ||
+                    !warp_wait(&full[s], (c2 / NS) & 1, abort_flag) ||
+                    !warp_wait(&sc_full[sb], (c2 >> 1) & 1, abort_flag)) {
+                    raise_error(p, kErrWaitTimeout, abort_flag);
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t base = tmem + col_sc(sb) + lane_off;
+                const float pim_t = gb[kGbPim + row];
+                if (!helper) {
+                    // ---- P'_ts = -E_ts (q_t . k_s) for s < 64
+                    if (q4 >= 2) {
+                        build_p64<0, true>(base, gb, row, pim_t);
+                    } else {
+                        build_p64<0, false>(base, gb, row, pim_t);
+                        tmem_zero32_async(base + 64);  // tokens >= 64 all masked
+                    }
+                    // ---- Q' = a_t q_t into columns 32..63 (read after the score above)
+                    const float a_t = gb[kGbA + row];
+                    const uint32_t qt = st + Lay::kQOff;
+#pragma unroll 1
+                    for (int q = 0; q < 8; ++q) {
+                        const uint4 a = ld_shared_v4(qt + sw128_off(row, q));
+                        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&a);
+                        uint32_t o[4];
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            const float2 f = __bfloat1622float2(h[i]);
+                            o[i] = pack_bf16x2(a_t * f.x, a_t * f.y);
+                        }
+                        tmem_st4_async(base + kQpCol + 4 * q, o[0], o[1], o[2], o[3]);
+                    }
+                } else {
+                    // ---- P'_ts for s >= 64 (rows 64..127)
+                    build_p64<8, false>(base + 64, gb, row, pim_t);
+                }
+                tmem_wait_st();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&p_ready[sb]);
+                if (wv_writer && c < I.nch - 1) {
+                    // ---- the chunk's W V row -w_t v_t (a unit's last chunk needs none)
+                    if (!warp_wait(wv_free, (wvn & 1) ^ 1, abort_flag)) {
+                        raise_error(p, kErrWaitTimeout, abort_flag);
+                        ok = false;
+                        break;
+                    }
+                    const float w = -gb[kGbW + wv_row];
+                    const uint32_t vt = st + Lay::kVOff;
+                    const uint32_t wvt = sbase + Lay::kWvOff;
+#pragma unroll 1
+                    for (int q = 0; q < 8; q += 2) {
+                        const uint4 a0 = ld_shared_v4(vt + sw128_off(wv_row, q));
+                        const uint4 a1 = ld_shared_v4(vt + sw128_off(wv_row, q + 1));
+                        const __nv_bfloat162* h0 = reinterpret_cast<const __nv_bfloat162*>(&a0);
+                        const __nv_bfloat162* h1 = reinterpret_cast<const __nv_bfloat162*>(&a1);
+                        uint32_t o0[4], o1[4];
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            const float2 f0 = __bfloat1622float2(h0[i]);
+                            const float2 f1 = __bfloat1622float2(h1[i]);
+                            o0[i] = pack_bf16x2(w * f0.x, w * f0.y);
+                            o1[i] = pack_bf16x2(w * f1.x, w * f1.y);
+                        }
+                        st_shared_v4(wvt + sw128_off(wv_row, q), o0[0], o0[1], o0[2], o0[3]);
+                        st_shared_v4(wvt + sw128_off(wv_row, q + 1), o1[0], o1[1], o1[2], o1[3]);
+                    }
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(wv_ready);
+                    ++wvn;
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&gf_free[gk]);  // this warp's reads of the block are done
+            }
+        }
+    } else if (warp < kWarpZ0) {
+        // ------------------------------------------------- output epilogue
+        const int q4 = warp & 3;
+        const int row = q4 * 32 + lane;
+        const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
+        const bool storer = (warp == kWarpO0) && (lane == 0);
+        const EpiParams& e = p.epi;
+        uint32_t c2 = 0;
+        bool ok = true;
+        for (int it = 0; ok; ++it) {
+            int item;
+            if (!take_item(it, item) || item < 0) break;
+            const Item I = decode_unit(item, p);
+            for (int c = 0; c < I.nch; ++c, ++c2) {
+                const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
+                if (!warp_wait(&o_full[ob], oph, abort_flag)) {
+                    raise_error(p, kErrWaitTimeout, abort_flag);
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const int t0 = c * kChunk;
+                const int t = t0 + row;
+                const bool valid = t < p.T;
+                const uint32_t otile = sbase + Lay::kOOff;
+                if (!e.zin && !e.out2) {
+                    // plain result: 16 columns at a time from TMEM into the staging tile
+                    if (!warp_wait(o_buf_free, (c2 & 1) ^ 1, abort_flag)) {
+                        raise_error(p, kErrWaitTimeout, abort_flag);
+                        ok = false;
+                        break;
+                    }
+#pragma unroll 1
+                    for (int m = 0; m < 4; ++m) {
+                        float u[16];
+                        tmem_ld16(tmem + col_o(ob) + lane_off + 16 * m, u);
+#pragma unroll
+                        for (int h = 0; h < 2; ++h)
+                            st_shared_v4(otile + sw128_off(row, 2 * m + h), pack_bf16x2(u[8 * h], u[8 * h + 1]),
+                                         pack_bf16x2(u[8 * h + 2], u[8 * h + 3]),
+                                         pack_bf16x2(u[8 * h + 4], u[8 * h + 5]),
+                                         pack_bf16x2(u[8 * h + 6], u[8 * h + 7]));
+                    }
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&o_free[ob]);
+                } else {
+                float v[64];
+                tmem_ld64(tmem + col_o(ob) + lane_off, v);
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&o_free[ob]);
+                if (e.zin && valid) {
+                    float tmp[64];
+#pragma unroll
+                    for (int i = 0; i < 64; ++i) tmp[i] = v[i];
+                    epi_apply_dact(e, tok_off(e.z_str, I.l, I.b, t, I.h), tmp);
+#pragma unroll
+                    for (int i = 0; i < 64; ++i) v[i] = tmp[i];
+                }
+                if (e.out2 && valid) {
+                    float tmp[64];
+#pragma unroll
+                    for (int i = 0; i < 64; ++i) tmp[i] = v[i];
+                    epi_store_act(e, tok_off(e.out2_str, I.l, I.b, t, I.h), tmp);
+                }
+                // one staging tile: the previous chunk's store has read it
+                if (!warp_wait(o_buf_free, (c2 & 1) ^ 1, abort_flag)) {
+                    raise_error(p, kErrWaitTimeout, abort_flag);
+                    ok = false;
+                    break;
+                }
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    st_shared_v4(otile + sw128_off(row, q), pack_bf16x2(v[8 * q], v[8 * q + 1]),
+                                 pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                                 pack_bf16x2(v[8 * q + 4], v[8 * q + 5]),
+                                 pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&o_staged[ob]);
+                if (storer) {
+                    if (!bwait(&o_staged[ob], oph, abort_flag)) {
+                        raise_error(p, kErrWaitTimeout, abort_flag);
+                        ok = false;
+                    } else {
+                        // rows past the end of the sequence are clipped by the store
+                        tma_store_5d(&tm_o, smem + Lay::kOOff, 0, I.h, t0, I.b, I.l);
+                        bulk_commit_group();
+                        bulk_wait_group_read<0>();  // the store has read the tile
+                        mbar_arrive(o_buf_free);
+                    }
+                }
+                if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
+                    ok = false;
+                    break;
+                }
+            }
+        }
+        if (storer) bulk_wait_group_all();
+    } else {
+        // ------------------------------------------------------------ state
+        // Warps 12-13: row q = 32 (warp & 3) + lane of S^T (fp32, registers), the
+        // bf16 B0^T tile once per unit, the bf16 S^T tile per chunk, and the decayed
+        // update S' = a_end S + dZ.
+        const int q4 = warp & 3;
+        const int row = q4 * 32 + lane;
+        const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
+        uint32_t c2 = 0, dzc = 0, ucnt = 0;
+        float st[64];
+        bool ok = true;
+        auto put_row = [&](uint32_t tile) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                st_shared_v4(tile + sw128_off(row, q), pack_bf16x2(st[8 * q], st[8 * q + 1]),
+                             pack_bf16x2(st[8 * q + 2], st[8 * q + 3]),
+                             pack_bf16x2(st[8 * q + 4], st[8 * q + 5]),
+                             pack_bf16x2(st[8 * q + 6], st[8 * q + 7]));
+            fence_proxy_async_smem();
+            __syncwarp();
+        };
+        for (int it = 0; ok; ++it) {
+            int item;
+            if (!take_item(it, item) || item < 0) break;
+            const Item I = decode_unit(item, p);
+            if (!warp_wait(b0_free, (ucnt & 1) ^ 1, abort_flag)) {
+                raise_error(p, kErrWaitTimeout, abort_flag);
+                break;
+            }
+            // B0^T row q: forward B0 = W0 ([m][d], column q), costate B0 = W0^T (row q)
+            const float* w0 = p.W0 + (size_t)(I.l * p.H + I.h) * 64 * 64;
+            if (p.w0_transposed) {
+#pragma unroll
+                for (int i = 0; i < 64; i += 4) {
+                    const float4 a = *reinterpret_cast<const float4*>(w0 + (size_t)row * 64 + i);
+                    st[i] = a.x;
+                    st[i + 1] = a.y;
+                    st[i + 2] = a.z;
+                    st[i + 3] = a.w;
+                }
+            } else {
+#pragma unroll
+                for (int i = 0; i < 64; ++i) st[i] = w0[(size_t)i * 64 + row];
+            }
+            put_row(sbase + Lay::kB0Off);
+            if (lane == 0) mbar_arrive(b0_ready);
+            ++ucnt;
+#pragma unroll
+            for (int i = 0; i < 64; ++i) st[i] = 0.0f;  // the fast weights start at W0
+            for (int c = 0; c < I.nch; ++c, ++c2) {
+                const uint32_t sb = c2 & 1, ph = (c2 >> 1) & 1;
+                if (!warp_wait(&st_free[sb], ph ^ 1, abort_flag)) {
+                    raise_error(p, kErrWaitTimeout, abort_flag);
+                    ok = false;
+                    break;
+                }
+                put_row(sbase + Lay::kStOff + sb * kStTile);
+                if (lane == 0) mbar_arrive(&st_ready[sb]);
+                const uint32_t gk = c2 % kGbRing;
+                if (!warp_wait(&gf_full[gk], (c2 / kGbRing) & 1, abort_flag)) {
+                    raise_error(p, kErrWaitTimeout, abort_flag);
+                    ok = false;
+                    break;
+                }
+                const float a_end = gfb[gk * kGbFloats + kGbEnd];
+                if (c < I.nch - 1) {
+                    const uint32_t b = dzc & 1;
+                    if (!warp_wait(&dz_full[b], (dzc >> 1) & 1, abort_flag)) {
+                        raise_error(p, kErrWaitTimeout, abort_flag);
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    float a[32];
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        tmem_ld32(tmem + col_dz(b) + lane_off + h * 32, a);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) st[h * 32 + i] = fmaf(a_end, st[h * 32 + i], a[i]);
+                    }
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&dz_free[b]);
+                    ++dzc;
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&gf_free[gk]);
+            }
+        }
+    }
+
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+template <bool COSTATE>
+static cudaError_t launch_dec(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
+                              const CUtensorMap& o, const TcScanParams& p, int grid,
+                              cudaStream_t stream) {
+    using Lay = DLayout<COSTATE>;
+    auto kern = decay_scan_kernel<COSTATE>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         Lay::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kThreads, Lay::kSmemBytes, stream>>>(q, k, v, o, p);
+    return cudaGetLastError();
+}
+
+}  // namespace dec
+
+// The retention scan of 64 x 64 bf16 maps on the tensor cores: one work item per
+// unit, gates p.g_eta / p.g_alpha ([L][B][T][H] fp32).
+cudaError_t launch_tc_decay(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
+                            const CUtensorMap& o, const TcScanParams& p, bool costate, int grid,
+                            cudaStream_t stream) {
+    if (p.dq != 64 || p.dv != 64 || !p.g_eta) return cudaErrorInvalidValue;
+    return costate ? dec::launch_dec<true>(q, k, v, o, p, grid, stream)
+                   : dec::launch_dec<false>(q, k, v, o, p, grid, stream);
+}
+
+}  // namespace gl
