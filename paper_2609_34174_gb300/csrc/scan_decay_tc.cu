@@ -128,13 +128,29 @@ __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
     }
 }
 
-// The bounded wait out of line, so that the kernel's many wait sites share one copy
-// of the loop (instruction-cache footprint); the first probe stays inline.
+// One non-blocking probe of a barrier phase.
+__device__ __forceinline__ bool test_probe(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// The bounded wait, out of line so that the kernel's many wait sites share one copy
+// (instruction-cache footprint).  Up to 64 non-blocking probes first: a thread parked
+// by the suspending wait resumes a few thousand cycles after a thread-side arrival,
+// which on the hand-offs between roles here costs more than the spin's issue slots.
 __device__ __noinline__ bool wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+    for (int i = 0; i < 64; ++i)
+        if (test_probe(bar, parity)) return true;
     return mbar_wait(bar, parity, abort_flag);
 }
 __device__ __forceinline__ bool bwait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
-    return mbar_try_wait(bar, parity) || wait_slow(bar, parity, abort_flag);
+    return test_probe(bar, parity) || wait_slow(bar, parity, abort_flag);
 }
 
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
