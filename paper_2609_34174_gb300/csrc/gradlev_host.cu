@@ -701,10 +701,39 @@ int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
         p.dq = 64;
         p.dv = 64;
         p.n_tiles = 1;
-        p.seg_len = d.T;
-        p.n_seg = 1;
-        p.n_items = (int)units;
+        // Few long units: cut each into segments (multiples of 128 tokens, at least
+        // 512) so that about four waves of items fill the SMs; the segments' states
+        // are carried through an aggregate pass (scan_decay_tc.cu).
+        int n_seg = 1;
+        long long seg_len = d.T;
+        if (units < 2ll * dev.sms && d.T > 1024) {
+            const long long want = (4ll * dev.sms + units - 1) / units;
+            seg_len = (((d.T + want - 1) / want) + 127) / 128 * 128;
+            if (seg_len < 512) seg_len = 512;
+            n_seg = (int)((d.T + seg_len - 1) / seg_len);
+            if (n_seg < 2) {
+                n_seg = 1;
+                seg_len = d.T;
+            }
+        }
+        p.seg_len = (int)seg_len;
+        p.n_seg = n_seg;
+        p.n_items = (int)(units * n_seg);
         p.n_ut = (int)units;
+        if (n_seg > 1) {
+            // the segment states go where the eta-only path keeps its scaled proposals
+            // (d_out * elem >= 128 bytes per token-unit, against at most 64 here)
+            const size_t a = ws_bytes_for(d, d.d_in, d.d_out, dev.sms);
+            const size_t bb = ws_bytes_for(d, d.d_out, d.d_in, dev.sms);
+            uint8_t* base = static_cast<uint8_t*>(ws) + round_up(a > bb ? a : bb, 256);
+            const size_t blk = (size_t)p.n_items * 64 * 64 * sizeof(float);
+            p.agg = reinterpret_cast<float*>(base);
+            p.incl = reinterpret_cast<float*>(base + blk);
+            p.seg_a = reinterpret_cast<float*>(base + 2 * blk);
+            if (static_cast<size_t>(base - static_cast<uint8_t*>(ws)) + 2 * blk +
+                    round_up((size_t)p.n_items * sizeof(float), 256) > ws_bytes)
+                return GRADLEV_ERR_WORKSPACE;
+        }
         p.lam = 1.0f;
         p.inv_lam = 1.0f;
         p.mu = 1.0f;
@@ -715,7 +744,7 @@ int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
         fill_epi(&p.epi, to, to2, tz, act);
         p.ctrl = static_cast<unsigned int*>(ws);
         if (cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
-        const int grid = units < dev.sms ? (int)units : dev.sms;
+        const int grid = p.n_items < dev.sms ? p.n_items : dev.sms;
         if (gl::launch_tc_decay(mq, mk, mv, mo, p, costate, grid, stream) != cudaSuccess)
             return GRADLEV_ERR_CUDA;
         return GRADLEV_OK;

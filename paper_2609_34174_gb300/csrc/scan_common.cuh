@@ -103,9 +103,11 @@ struct TcScanParams {
     int test_skip_publish;  // failure tests only: this item never publishes (-1: none)
     float* agg;           // [n_items][dq][64] segment aggregate  sum_s k_s v_s^T
     float* incl;          // [n_items][dq][64] inclusive prefix of the aggregates
-    // retention kernel only: per-token gates, fp32 [L][B][T][H] contiguous
+    // retention kernel only: per-token gates, fp32 [L][B][T][H] contiguous, and the
+    // alpha product of each segment (aggregate pass, [n_items])
     const float* g_eta;
     const float* g_alpha;  // null: alpha = 1
+    float* seg_a;
 };
 
 // Parameters of the wide-layer passes (bf16, dq % 128 == 0, dv % 64 == 0): the

@@ -101,17 +101,23 @@ struct DLayout {
     static_assert(kGfOff % 32 == 0 && kBarOff % 8 == 0, "alignment");
 };
 
+// One work item: segment k (tokens [t_begin, t_end)) of one unit.  Items are
+// segment-major: item = k * n_ut + unit, with n_ut the number of units.
 struct Item {
-    int l, b, h, nch;
+    int l, b, h, k, t_begin, t_end, nch;
 };
 
 __device__ __forceinline__ Item decode_unit(int item, const TcScanParams& p) {
     Item I;
-    I.h = item % p.H;
-    const int lb = item / p.H;
+    const int unit = item % p.n_ut;
+    I.k = item / p.n_ut;
+    I.h = unit % p.H;
+    const int lb = unit / p.H;
     I.b = lb % p.B;
     I.l = lb / p.B;
-    I.nch = (p.T + kChunk - 1) / kChunk;
+    I.t_begin = I.k * p.seg_len;
+    I.t_end = min(p.T, I.t_begin + p.seg_len);
+    I.nch = (I.t_end - I.t_begin + kChunk - 1) / kChunk;
     return I;
 }
 
@@ -258,7 +264,7 @@ __device__ __forceinline__ void build_p64(uint32_t taddr, const float* gb, int r
     }
 }
 
-template <bool COSTATE>
+template <bool COSTATE, bool AGG>
 __global__ void __launch_bounds__(kThreads, 1)
     decay_scan_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                       const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
@@ -305,7 +311,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < NS; ++i) {
             mbar_init(&full[i], 1);
-            mbar_init(&empty[i], 2);  // both MMA issuers
+            mbar_init(&empty[i], AGG ? 1 : 2);  // both MMA issuers (the front one alone in AGG)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&sc_full[i], 1);
@@ -390,9 +396,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         break;
                     }
                     uint8_t* st = smem + s * Lay::kStageBytes;
-                    const int t0 = c * kChunk;
-                    mbar_arrive_expect_tx(&full[s], Lay::kStageBytes);
-                    if (COSTATE) tma_load_5d(st + Lay::kQOff, &tm_q, &full[s], 0, I.h, t0, I.b, I.l);
+                    const int t0 = I.t_begin + c * kChunk;
+                    // the aggregate pass reads no queries
+                    mbar_arrive_expect_tx(&full[s], (COSTATE && AGG) ? Lay::kStageBytes - kTile : Lay::kStageBytes);
+                    if (COSTATE && !AGG) tma_load_5d(st + Lay::kQOff, &tm_q, &full[s], 0, I.h, t0, I.b, I.l);
                     tma_load_5d(st + Lay::kKOff, &tm_k, &full[s], 0, I.h, t0, I.b, I.l);
                     tma_load_5d(st + Lay::kVOff, &tm_v, &full[s], 0, I.h, t0, I.b, I.l);
                 }
@@ -426,10 +433,34 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_arrive(&item_empty[slot]);
                 if (item < 0) break;
                 const Item I = decode_unit(item, p);
+                // dZ = K^T (W V) of the chunk in stage sp: A = K^T (MN-major, 64-wide M
+                // blocks 16 KB apart; the second block's rows land in TMEM lanes 64..127,
+                // unread)
+                auto issue_dz = [&](int sp) -> bool {
+                    const uint32_t b = dzc & 1;
+                    if (!wait_or_fail(&dz_free[b], ((dzc >> 1) & 1) ^ 1)) return false;
+                    if (!wait_or_fail(wv_ready, dzc & 1)) return false;
+                    tc_fence_after();
+                    const uint32_t a_lo = sdesc_lo(sbase + sp * Lay::kStageBytes + Lay::kKOff, kTile);
+                    const uint32_t b_lo = sdesc_lo(wv, kTile);
+#pragma unroll
+                    for (int kk = 0; kk < kChunk / 16; ++kk)
+                        mma_bf16_ss(tmem + col_dz(b), sdesc_from_lo(a_lo + mnmaj_step(kk)),
+                                    sdesc_from_lo(b_lo + mnmaj_step(kk)), ID_DZ, kk > 0 ? 1u : 0u);
+                    mma_commit(&dz_full[b]);
+                    mma_commit(wv_free);
+                    mma_commit(&empty[sp]);
+                    ++dzc;
+                    return true;
+                };
                 for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
                     const int s = n % NS;
                     const uint32_t sb = c2 & 1;
                     if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
+                    if (AGG) {  // the segment's aggregate: the state update of every chunk
+                        if (!(ok = issue_dz(s))) break;
+                        continue;
+                    }
                     if (!(ok = wait_or_fail(&sc_free[sb], ((c2 >> 1) & 1) ^ 1))) break;
                     tc_fence_after();
                     const uint32_t st = sbase + s * Lay::kStageBytes;
@@ -440,26 +471,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         mma_bf16_ss(tmem + col_sc(sb), sdesc_from_lo(q_lo + kmaj_step(kk)),
                                     sdesc_from_lo(k_lo + kmaj_step(kk)), ID_SC, kk > 0 ? 1u : 0u);
                     mma_commit(&sc_full[sb]);
-                    if (c > 0) {
-                        // dZ of the previous chunk = K^T (W V): A = K^T (MN-major, 64-wide M
-                        // blocks 16 KB apart; the second block's rows land in TMEM lanes
-                        // 64..127, unread)
-                        const int sp = static_cast<int>((n - 1) % NS);
-                        const uint32_t b = dzc & 1;
-                        if (!(ok = wait_or_fail(&dz_free[b], ((dzc >> 1) & 1) ^ 1))) break;
-                        if (!(ok = wait_or_fail(wv_ready, dzc & 1))) break;
-                        tc_fence_after();
-                        const uint32_t a_lo = sdesc_lo(sbase + sp * Lay::kStageBytes + Lay::kKOff, kTile);
-                        const uint32_t b_lo = sdesc_lo(wv, kTile);
-#pragma unroll
-                        for (int kk = 0; kk < kChunk / 16; ++kk)
-                            mma_bf16_ss(tmem + col_dz(b), sdesc_from_lo(a_lo + mnmaj_step(kk)),
-                                        sdesc_from_lo(b_lo + mnmaj_step(kk)), ID_DZ, kk > 0 ? 1u : 0u);
-                        mma_commit(&dz_full[b]);
-                        mma_commit(wv_free);
-                        mma_commit(&empty[sp]);
-                        ++dzc;
-                    }
+                    // the previous chunk's state update, one chunk behind its score
+                    if (c > 0 && !(ok = issue_dz(static_cast<int>((n - 1) % NS)))) break;
                     if (c == I.nch - 1) mma_commit(&empty[s]);  // no state update reads it
                 }
             }
@@ -484,6 +497,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int item = item_slot[slot];
                 mbar_arrive(&item_empty[slot]);
                 if (item < 0) break;
+                if (AGG) continue;  // no outputs in the aggregate pass
                 const Item I = decode_unit(item, p);
                 if (!(ok = wait_or_fail(b0_ready, ucnt & 1))) break;
                 for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
@@ -540,12 +554,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!take_item(it, item) || item < 0) break;
             const Item I = decode_unit(item, p);
             const long long gbase = ((long long)I.l * p.B + I.b) * p.T * p.H + I.h;
-            // this lane's gates of chunk c (alpha = 1, eta = 0 past T)
+            // this lane's gates of chunk c (alpha = 1, eta = 0 past the segment)
             auto load = [&](int c, float (&al)[4], float (&et)[4]) {
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
-                    const int tg = c * kChunk + 4 * lane + i;
-                    const bool in = tg < p.T;
+                    const int tg = I.t_begin + c * kChunk + 4 * lane + i;
+                    const bool in = tg < I.t_end;
                     const long long gi = gbase + (long long)(in ? tg : 0) * p.H;
                     al[i] = in ? (p.g_alpha ? __ldg(p.g_alpha + gi) : 1.0f) : 1.0f;
                     et[i] = in ? __ldg(p.g_eta + gi) : 0.0f;
@@ -655,11 +669,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const float* gb = gfb + gk * kGbFloats;
                 if (!warp_wait(&gf_full[gk], (c2 / kGbRing) & 1, abort_flag) ||
                     !warp_wait(&full[s], (c2 / NS) & 1, abort_flag) ||
-                    !warp_wait(&sc_full[sb], (c2 >> 1) & 1, abort_flag)) {
+                    (!AGG && !warp_wait(&sc_full[sb], (c2 >> 1) & 1, abort_flag))) {
                     raise_error(p, kErrWaitTimeout, abort_flag);
                     ok = false;
                     break;
                 }
+                if (!AGG) {  // the aggregate pass forms no outputs
                 tc_fence_after();
                 const uint32_t base = tmem + col_sc(sb) + lane_off;
                 const float pim_t = gb[kGbPim + row];
@@ -694,8 +709,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&p_ready[sb]);
-                if (wv_writer && c < I.nch - 1) {
-                    // ---- the chunk's W V row -w_t v_t (a unit's last chunk needs none)
+                }
+                if (wv_writer && (AGG || c < I.nch - 1)) {
+                    // ---- the chunk's W V row -w_t v_t (an item's last chunk needs none
+                    // unless its state at the segment end is the aggregate)
                     if (!warp_wait(wv_free, (wvn & 1) ^ 1, abort_flag)) {
                         raise_error(p, kErrWaitTimeout, abort_flag);
                         ok = false;
@@ -742,6 +759,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int it = 0; ok; ++it) {
             int item;
             if (!take_item(it, item) || item < 0) break;
+            if (AGG) continue;  // no outputs in the aggregate pass
             const Item I = decode_unit(item, p);
             for (int c = 0; c < I.nch; ++c, ++c2) {
                 const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
@@ -751,7 +769,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 tc_fence_after();
-                const int t0 = c * kChunk;
+                const int t0 = I.t_begin + c * kChunk;
                 const int t = t0 + row;
                 const bool valid = t < p.T;
                 const uint32_t otile = sbase + Lay::kOOff;
@@ -834,8 +852,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
         // ------------------------------------------------------------ state
         // Warps 12-13: row q = 32 (warp & 3) + lane of S^T (fp32, registers), the
-        // bf16 B0^T tile once per unit, the bf16 S^T tile per chunk, and the decayed
-        // update S' = a_end S + dZ.
+        // bf16 B0^T tile once per item, the bf16 S^T tile per chunk, and the decayed
+        // update S' = a_end S + dZ.  A segment after the first starts from the carried
+        // state of the earlier segments; the aggregate pass starts from zero and
+        // writes its end state and alpha product instead of tiles.
         const int q4 = warp & 3;
         const int row = q4 * 32 + lane;
         const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
@@ -852,10 +872,58 @@ __global__ void __launch_bounds__(kThreads, 1)
             fence_proxy_async_smem();
             __syncwarp();
         };
+        // S' = a_end S + dZ with the next product from TMEM
+        auto advance = [&](float a_end) -> bool {
+            const uint32_t b = dzc & 1;
+            if (!warp_wait(&dz_full[b], (dzc >> 1) & 1, abort_flag)) return false;
+            tc_fence_after();
+            float a[32];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                tmem_ld32(tmem + col_dz(b) + lane_off + h * 32, a);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) st[h * 32 + i] = fmaf(a_end, st[h * 32 + i], a[i]);
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&dz_free[b]);
+            ++dzc;
+            return true;
+        };
         for (int it = 0; ok; ++it) {
             int item;
             if (!take_item(it, item) || item < 0) break;
             const Item I = decode_unit(item, p);
+            if (AGG) {
+#pragma unroll
+                for (int i = 0; i < 64; ++i) st[i] = 0.0f;
+                float prod = 1.0f;
+                for (int c = 0; c < I.nch; ++c, ++c2) {
+                    const uint32_t gk = c2 % kGbRing;
+                    if (!warp_wait(&gf_full[gk], (c2 / kGbRing) & 1, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    const float a_end = gfb[gk * kGbFloats + kGbEnd];
+                    if (!advance(a_end)) {
+                        ok = false;
+                        break;
+                    }
+                    prod *= a_end;
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&gf_free[gk]);
+                }
+                if (!ok) {
+                    raise_error(p, kErrWaitTimeout, abort_flag);
+                    break;
+                }
+                float* dst = p.agg + (size_t)item * 64 * 64 + (size_t)row * 64;
+#pragma unroll
+                for (int i = 0; i < 64; i += 4)
+                    *reinterpret_cast<float4*>(dst + i) = make_float4(st[i], st[i + 1], st[i + 2], st[i + 3]);
+                if (row == 0) p.seg_a[item] = prod;
+                continue;
+            }
             if (!warp_wait(b0_free, (ucnt & 1) ^ 1, abort_flag)) {
                 raise_error(p, kErrWaitTimeout, abort_flag);
                 break;
@@ -878,8 +946,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             put_row(sbase + Lay::kB0Off);
             if (lane == 0) mbar_arrive(b0_ready);
             ++ucnt;
+            if (I.k > 0) {  // the carried state at the segment's first token
+                const float* src = p.incl + (size_t)item * 64 * 64 + (size_t)row * 64;
 #pragma unroll
-            for (int i = 0; i < 64; ++i) st[i] = 0.0f;  // the fast weights start at W0
+                for (int i = 0; i < 64; i += 4) {
+                    const float4 a = *reinterpret_cast<const float4*>(src + i);
+                    st[i] = a.x;
+                    st[i + 1] = a.y;
+                    st[i + 2] = a.z;
+                    st[i + 3] = a.w;
+                }
+            } else {
+#pragma unroll
+                for (int i = 0; i < 64; ++i) st[i] = 0.0f;  // the fast weights start at W0
+            }
             for (int c = 0; c < I.nch; ++c, ++c2) {
                 const uint32_t sb = c2 & 1, ph = (c2 >> 1) & 1;
                 if (!warp_wait(&st_free[sb], ph ^ 1, abort_flag)) {
@@ -896,25 +976,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 const float a_end = gfb[gk * kGbFloats + kGbEnd];
-                if (c < I.nch - 1) {
-                    const uint32_t b = dzc & 1;
-                    if (!warp_wait(&dz_full[b], (dzc >> 1) & 1, abort_flag)) {
-                        raise_error(p, kErrWaitTimeout, abort_flag);
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    float a[32];
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        tmem_ld32(tmem + col_dz(b) + lane_off + h * 32, a);
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) st[h * 32 + i] = fmaf(a_end, st[h * 32 + i], a[i]);
-                    }
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&dz_free[b]);
-                    ++dzc;
+                if (c < I.nch - 1 && !advance(a_end)) {
+                    raise_error(p, kErrWaitTimeout, abort_flag);
+                    ok = false;
+                    break;
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&gf_free[gk]);
@@ -930,12 +995,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-template <bool COSTATE>
+template <bool COSTATE, bool AGG>
 static cudaError_t launch_dec(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
                               const CUtensorMap& o, const TcScanParams& p, int grid,
                               cudaStream_t stream) {
     using Lay = DLayout<COSTATE>;
-    auto kern = decay_scan_kernel<COSTATE>;
+    auto kern = decay_scan_kernel<COSTATE, AGG>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          Lay::kSmemBytes);
     if (e != cudaSuccess) return e;
@@ -945,14 +1010,49 @@ static cudaError_t launch_dec(const CUtensorMap& q, const CUtensorMap& k, const 
 
 }  // namespace dec
 
-// The retention scan of 64 x 64 bf16 maps on the tensor cores: one work item per
-// unit, gates p.g_eta / p.g_alpha ([L][B][T][H] fp32).
+// Carried start states of the segments: for each unit and segment k,
+// incl[k] = P_{k-1} with P_{-1} = 0 and P_k = a_k P_{k-1} + agg_k (the affine
+// composition of the segments' transforms S -> a S + U).  One thread per state
+// entry and unit, walking the segments in order.
+__global__ void __launch_bounds__(256)
+    decay_carry_kernel(const float* __restrict__ agg, const float* __restrict__ seg_a,
+                       float* __restrict__ incl, int n_ut, int n_seg) {
+    const long long i = (long long)blockIdx.x * 256 + threadIdx.x;
+    if (i >= (long long)n_ut * 4096) return;
+    const int unit = (int)(i >> 12), e = (int)(i & 4095);
+    float P = 0.0f;
+    for (int k = 0; k < n_seg; ++k) {
+        const size_t item = (size_t)k * n_ut + unit;
+        incl[item * 4096 + e] = P;
+        if (k < n_seg - 1) P = fmaf(seg_a[item], P, agg[item * 4096 + e]);
+    }
+}
+
+// The retention scan of 64 x 64 bf16 maps on the tensor cores.  With p.n_seg > 1
+// every unit is cut into segments of p.seg_len tokens: an aggregate pass over all
+// but the last segment of each unit (p.agg, p.seg_a), the carry of the start states
+// (p.incl), then the scan of every (segment, unit) item from its start state.
 cudaError_t launch_tc_decay(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
                             const CUtensorMap& o, const TcScanParams& p, bool costate, int grid,
                             cudaStream_t stream) {
     if (p.dq != 64 || p.dv != 64 || !p.g_eta) return cudaErrorInvalidValue;
-    return costate ? dec::launch_dec<true>(q, k, v, o, p, grid, stream)
-                   : dec::launch_dec<false>(q, k, v, o, p, grid, stream);
+    if (p.n_seg > 1) {
+        if (!p.agg || !p.incl || !p.seg_a) return cudaErrorInvalidValue;
+        TcScanParams pa = p;
+        pa.n_items = (p.n_seg - 1) * p.n_ut;
+        const int ga = pa.n_items < grid ? pa.n_items : grid;
+        cudaError_t e = costate ? dec::launch_dec<true, true>(q, k, v, o, pa, ga, stream)
+                                : dec::launch_dec<false, true>(q, k, v, o, pa, ga, stream);
+        if (e != cudaSuccess) return e;
+        const long long n = (long long)p.n_ut * 4096;
+        decay_carry_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(p.agg, p.seg_a, p.incl,
+                                                                                 p.n_ut, p.n_seg);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        // a fresh work ticket for the scan (the error word stays)
+        if ((e = cudaMemsetAsync(p.ctrl, 0, sizeof(unsigned int), stream)) != cudaSuccess) return e;
+    }
+    return costate ? dec::launch_dec<true, false>(q, k, v, o, p, grid, stream)
+                   : dec::launch_dec<false, false>(q, k, v, o, p, grid, stream);
 }
 
 }  // namespace gl

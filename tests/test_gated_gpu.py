@@ -3,8 +3,9 @@ sizes eta_t and retention alpha_t, decay centred at W0) against the fp64 oracle,
 which runs the same recurrence token by token.
 
 Per-token eta_t alone takes the chunked kernels on eta-scaled proposals;
-with alpha_t, bf16 64 x 64 maps run the chunked retention kernel and every
-other shape the token-serial kernels.  alpha_t = 0 marks resets (the fast
+with alpha_t, bf16 64 x 64 maps run the tensor-core retention kernel (chunks of
+128 tokens; few long units cut into segments whose states are carried) and
+every other shape the token-serial kernels.  alpha_t = 0 marks resets (the fast
 weights return to W0, as at a document boundary).
 """
 import numpy as np
@@ -123,18 +124,19 @@ def test_constant_gates_match_plain_scan():
     assert err <= TOL["bf16"], f"serial vs chunked rel-L2 {err:.3e}"
 
 
-# The retention path for bf16 64 x 64 maps runs in chunks of 64 tokens.  These
-# cases put the chunk boundaries, resets and odd gates where a chunked form of
-# Eq. 2 could go wrong: T below, at and just past one chunk; resets on the last
-# and first token of a chunk and two in a row; a negative alpha; many units.
-CHUNK_T = [1, 37, 64, 65, 128, 191, 1000]
+# The retention path for bf16 64 x 64 maps runs in chunks of 128 tokens, built
+# from 8-token pieces.  These cases put the chunk and piece boundaries, resets and
+# odd gates where a chunked form of Eq. 2 could go wrong: T below, at and just past
+# one and two chunks; resets on the last and first token of a piece and of a chunk
+# and two in a row; a negative alpha; many units.
+CHUNK_T = [1, 37, 64, 65, 127, 128, 129, 191, 255, 256, 257, 1000]
 
 
-def _chunk_gates(shape, T, seed):
+def _chunk_gates(shape, T, seed, resets=(7, 8, 63, 64, 127, 128, 130, 131, 500)):
     g = torch.Generator().manual_seed(seed)
     eta = torch.rand(shape, generator=g, dtype=torch.float64) * 0.04
     alpha = 0.85 + 0.15 * torch.rand(shape, generator=g, dtype=torch.float64)
-    for t in (63, 64, 127, 130, 131, 500):
+    for t in resets:
         if t < T:
             alpha[:, :, t, :] = 0.0
     if T > 20:
@@ -199,3 +201,43 @@ def test_retention_strided_views(offset):
     yr, gr = _oracle(inputs, eta, alpha, wl)
     _check("forward", y, yr, TOL["bf16"])
     _check("costate", gin, gr, TOL["bf16"])
+
+
+@pytest.mark.parametrize("T", [1500, 5000])
+def test_retention_segments(T):
+    """Few long units: the sequence is cut into segments (512 tokens here, the last
+    one ragged) whose start states come from an aggregate pass and the affine carry
+    (a, U) then (a', U') = (a' a, a' U + U').  Resets sit on, before and after
+    segment boundaries, and a negative alpha inside a segment."""
+    wl = W.workload("c4").resized(B=1, H=2, T=T)
+    inputs = W.make_linear(wl)
+    eta, alpha = _chunk_gates((wl.L, wl.B, wl.T, wl.H), T, 300 + T,
+                              resets=(511, 512, 1023, 1025, 2047, 4095, 4096))
+    if T > 3000:
+        alpha[:, :, 3000, :] = -0.7
+    dev = {k: (v.cuda() if isinstance(v, torch.Tensor) else v) for k, v in inputs.items()}
+    y = gl.forward_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), alpha=alpha.cuda())
+    gin = gl.costate_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), dev["g_out"],
+                          alpha=alpha.cuda())
+    torch.cuda.synchronize()
+    yr, gr = _oracle(inputs, eta, alpha, wl)
+    _check(f"T={T} segmented forward", y, yr, TOL["bf16"])
+    _check(f"T={T} segmented costate", gin, gr, TOL["bf16"])
+
+
+def test_retention_full_size_c4_every_unit():
+    """The long-context workload at full size with retention (the bench's gated
+    configuration): every unit and token row against the oracle."""
+    import bench
+    wl = W.workload("c4")
+    inputs = W.make_linear(wl)
+    gates = bench.make_gates(wl, "alpha", "cpu")
+    eta, alpha = gates["eta_t"], gates["alpha_t"]
+    dev = {k: (v.cuda() if isinstance(v, torch.Tensor) else v) for k, v in inputs.items()}
+    y = gl.forward_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), alpha=alpha.cuda())
+    gin = gl.costate_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), dev["g_out"],
+                          alpha=alpha.cuda())
+    torch.cuda.synchronize()
+    yr, gr = _oracle(inputs, eta, alpha, wl)
+    _check("c4 retention forward", y, yr, TOL["bf16"])
+    _check("c4 retention costate", gin, gr, TOL["bf16"])
