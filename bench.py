@@ -200,8 +200,14 @@ class LinearJob:
         self.ws = torch.empty(max(256, nb), dtype=torch.uint8, device=device)
         self.tokens = wl.tokens
         # one chunk-kernel launch per scan; eta_t adds the prescale launch to each,
-        # documents the gate-folding launch
-        self.launches_per_step = 4 if gates in ("eta", "docs") else 2
+        # documents the gate-folding launch.  The retention kernel cuts few long units
+        # (fewer than two per SM, more than 1024 tokens) into segments: an aggregate
+        # launch and a carry launch precede its scan.
+        units = wl.L * wl.B * wl.H
+        sms = torch.cuda.get_device_properties(device).multi_processor_count if str(device).startswith("cuda") else 152
+        segmented = gates in ("alpha", "docs") and units < 2 * sms and wl.T > 1024
+        per_scan = (3 if segmented else 1) + (1 if gates in ("eta", "docs") else 0)
+        self.launches_per_step = 2 * per_scan
         self.in_keys = ("x", "g_hat", "g_out", "W0") + (
             ("eta_t",) if gates in ("eta", "alpha") else ()) + (
             ("alpha_t",) if gates == "alpha" else ()) + (("doc_start",) if gates == "docs" else ())
@@ -209,8 +215,8 @@ class LinearJob:
         self.kernel = {"fwd": "tc_scan_kernel<64, false> (forward scan)",
                        "costate": "tc_scan_kernel<64, true> (costate scan)"}
         if gates in ("alpha", "docs"):
-            self.kernel = {"fwd": "chunk_decay_kernel<false> (forward scan, retention)",
-                           "costate": "chunk_decay_kernel<true> (costate scan, retention)"}
+            self.kernel = {"fwd": "decay_scan_kernel<false, false> (forward scan, retention)",
+                           "costate": "decay_scan_kernel<true, false> (costate scan, retention)"}
 
     def input_bytes(self):
         return _bytes(self.inp["x"], self.inp["g_hat"], self.inp["g_out"])
@@ -318,9 +324,9 @@ class LinearJob:
              "eta": wl.eta}
         if self.gates:
             c["gates"] = {"eta": "per-token eta_t",
-                          "alpha": "per-token eta_t and retention alpha_t (chunked retention kernel)",
+                          "alpha": "per-token eta_t and retention alpha_t (tensor-core retention kernel)",
                           "docs": "document resets, documents of 512-1535 tokens, scalar eta "
-                                  "(gate folding + chunked retention kernel)"}[self.gates]
+                                  "(gate folding + tensor-core retention kernel)"}[self.gates]
         return c
 
     def oracle_run(self, inp, n_units, cores, t_tokens=None):

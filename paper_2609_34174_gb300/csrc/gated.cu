@@ -7,14 +7,12 @@
 // read before each write: y_t = W_t x_t (Eq. 3), gin_t = W_t^T gout_t (Eq. 4).
 // alpha_t = 0 resets the fast weights to W0 (a document boundary).
 //
-// Two kernels:
+// Two kernels (bf16 64 x 64 maps with alpha_t run the tensor-core kernel of
+// scan_decay_tc.cu):
 //   prescale_kernel  eta_t only (alpha = 1): the writes eta_t ghat_t x_t^T are the
 //                    plain writes of ghat'_t = eta_t ghat_t, so the chunked kernels
 //                    run on ghat' with eta = 1.  One elementwise pass into the
 //                    workspace (rounded to the input dtype, like ghat itself).
-//   chunk_decay_kernel  with alpha_t, bf16 64 x 64 maps: the recurrence in chunks
-//                    of 64 tokens, the within-chunk decays as plain products of
-//                    the alphas, contractions on bf16 mma.sync fragments.
 //   serial_kernel    with alpha_t, any other shape: the recurrence token by token,
 //                    exactly as Eq. 2 states it.  Each CTA holds a 64-wide slice of
 //                    W - W0 and of W0 for one unit; the forward slices W by rows
@@ -408,387 +406,6 @@ __global__ void __launch_bounds__(kThreads)
     }
 }
 
-// ---------------------------------------------------------------------------
-// Chunked retention scan for bf16 maps of 64 x 64.  In the orientation shared by
-// both reads (o_t = (B0 + S_t) q_t with writes S <- alpha_s S - eta_s v_s k_s^T):
-//   forward  q = k = x, v = ghat, B0 = W0,   S = W - W0
-//   costate  q = gout, k = ghat, v = x, B0 = W0^T, S = (W - W0)^T
-// Eq. 2 unrolled over a chunk of kC tokens from the state S at its first token:
-//
-//   o_t = B0 q_t + a_t S q_t - sum_{s<t} E_ts (k_s . q_t) v_s
-//   S'  = a_end S - sum_s w_s v_s k_s^T
-//
-// with a_t = prod_{r<t} alpha_r, E_ts = eta_s prod_{s<r<t} alpha_r, w_s = eta_s
-// prod_{r>s} alpha_r and a_end the product of all the chunk's alphas (indices
-// local to the chunk; tokens past T carry alpha = 1, eta = 0).  The decays are
-// products of alphas, never ratios, so a reset (alpha = 0) and underflow give
-// exact zeros.  They are assembled from 8-token pieces: sig_s (alphas after s to
-// the end of its piece), pi_t (alphas from the start of t's piece up to t) and
-// the piece products tp_j.
-//
-// One CTA per unit walks its chunks in order.  Warp w reads tokens [16w, 16w+16)
-// of the chunk and owns rows [16w, 16w+16) of S, which stay in fp32 accumulator
-// registers from chunk to chunk; a bf16 copy in shared memory is the B operand of
-// the next chunk's read.  Tiles are 64 rows of 128 bytes, 16-byte pieces swizzled
-// by the row (piece ^ (row & 7)) so that every ldmatrix phase is conflict free.
-namespace cdec {
-
-constexpr int kC = 64;                 // tokens per chunk
-constexpr int kThr = 128;              // 4 warps
-constexpr int kTileB = kC * 64 * 2;    // one bf16 tile [64][64]
-
-template <bool COSTATE>
-__host__ __device__ constexpr int buf_bytes() {            // q, v (, k) tiles and alpha, eta of one chunk
-    return (COSTATE ? 3 : 2) * kTileB + 2 * kC * 4;
-}
-template <bool COSTATE>
-__host__ __device__ constexpr size_t smem_bytes() {        // B0, S copy, two chunk buffers, decay tables
-    return 2 * kTileB + 2 * buf_bytes<COSTATE>() + (2 * kC + 8) * 4;
-}
-
-__device__ __forceinline__ uint32_t swz(int row, int piece) {
-    return (uint32_t)(row * 128 + ((piece ^ (row & 7)) << 4));
-}
-// The fragment loads read shared memory (memory clobber: they stay between the
-// barriers and stores around them); the MMAs are pure register operations, free
-// to be scheduled between the loads.
-__device__ __forceinline__ void ldsm4(uint32_t a, uint32_t (&r)[4]) {
-    asm("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-        : "r"(a)
-        : "memory");
-}
-__device__ __forceinline__ void ldsm4t(uint32_t a, uint32_t (&r)[4]) {
-    asm("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-        : "r"(a)
-        : "memory");
-}
-// d += a b: a 16 x 16 (row), b 16 x 8 (col), bf16 in, fp32 accumulate
-__device__ __forceinline__ void mma(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-    asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-        "{%8,%9}, {%0,%1,%2,%3};"
-        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ uint32_t pack(float lo, float hi) {
-    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<uint32_t*>(&v);
-}
-__device__ __forceinline__ uint32_t scale2(uint32_t u, float a, float b) {
-    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u));
-    return pack(f.x * a, f.y * b);
-}
-// B fragments of two 8-column tiles [n0, n0+16) for the k-step [k0, k0+16):
-// from a tile stored [n][k] (k contiguous) ...
-__device__ __forceinline__ void ld_b_nk(uint32_t tile, int n0, int k0, int lane, uint32_t (&r)[4]) {
-    ldsm4(tile + swz(n0 + (lane & 7) + ((lane >> 4) << 3), (k0 >> 3) + ((lane >> 3) & 1)), r);
-}
-// ... or stored [k][n] (n contiguous)
-__device__ __forceinline__ void ld_b_kn(uint32_t tile, int n0, int k0, int lane, uint32_t (&r)[4]) {
-    ldsm4t(tile + swz(k0 + (lane & 7) + (((lane >> 3) & 1) << 3), (n0 >> 3) + (lane >> 4)), r);
-}
-
-template <bool COSTATE>
-__global__ void __launch_bounds__(kThr, 3) chunk_decay_kernel(GatedParams p) {
-    extern __shared__ __align__(128) unsigned char smc[];
-    constexpr int kBufB = buf_bytes<COSTATE>();
-    constexpr int kGateOff = (COSTATE ? 3 : 2) * kTileB;
-    unsigned char* B0s = smc;                          // B0 [v][q], bf16
-    unsigned char* Sbs = smc + kTileB;                 // S [v][k], bf16 copy
-    unsigned char* bufs = smc + 2 * kTileB;            // 2 x { q, v (, k), alpha, eta }
-    float* sig = reinterpret_cast<float*>(bufs + 2 * kBufB);
-    float* pim = sig + kC;
-    float* tpr = pim + kC;
-    const uint32_t sB0 = (uint32_t)__cvta_generic_to_shared(B0s);
-    const uint32_t sS = (uint32_t)__cvta_generic_to_shared(Sbs);
-
-    const int unit = blockIdx.x;
-    const int h = unit % p.H;
-    const int b = (unit / p.H) % p.B;
-    const int l = unit / (p.H * p.B);
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, cq = lane & 3;
-
-    using bf = __nv_bfloat16;
-    const bf* X = static_cast<const bf*>(p.x) + tok_off(p.x_s, l, b, 0, h);
-    const bf* G = static_cast<const bf*>(p.g) + tok_off(p.g_s, l, b, 0, h);
-    const bf* Qp = static_cast<const bf*>(p.q) + tok_off(p.q_s, l, b, 0, h);
-    const bf* Vp = COSTATE ? X : G;
-    const bf* Kp = COSTATE ? G : X;
-    const long long qst = p.q_s[2], vst = COSTATE ? p.x_s[2] : p.g_s[2], kst = COSTATE ? p.g_s[2] : p.x_s[2];
-    const long long gate0 = ((long long)l * p.B + b) * p.T * p.H + h;
-
-    // B0 as bf16 [v][q]; S starts at zero (the fast weights begin at W0)
-    const float* w0 = p.W0 + (size_t)(l * p.H + h) * 64 * 64;  // [dout][din]
-    for (int e = tid; e < 64 * 32; e += kThr) {
-        const int m = e >> 5, k = (e & 31) * 2;
-        const float v0 = COSTATE ? w0[k * 64 + m] : w0[m * 64 + k];
-        const float v1 = COSTATE ? w0[(k + 1) * 64 + m] : w0[m * 64 + k + 1];
-        const uint32_t off = swz(m, k >> 3) + (k & 7) * 2;
-        *reinterpret_cast<uint32_t*>(B0s + off) = pack(v0, v1);
-        *reinterpret_cast<uint32_t*>(Sbs + off) = 0u;
-    }
-
-    // chunk c's rows and gates into buffer c & 1 (zeros, alpha = 1, eta = 0 past T)
-    auto stage = [&](int c) {
-        unsigned char* bb = bufs + (c & 1) * kBufB;
-        const uint32_t sb = (uint32_t)__cvta_generic_to_shared(bb);
-        const int c0 = c * kC;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int pc = tid + i * kThr;
-            const int row = pc >> 3, piece = pc & 7;
-            const bool ok = c0 + row < p.T;
-            const long long t = ok ? c0 + row : 0;
-            const uint32_t off = swz(row, piece);
-            cpa16(sb + off, Qp + t * qst + piece * 8, ok);
-            cpa16(sb + kTileB + off, Vp + t * vst + piece * 8, ok);
-            if (COSTATE) cpa16(sb + 2 * kTileB + off, Kp + t * kst + piece * 8, ok);
-        }
-        const int t = c0 + (tid & 63);
-        if (t < p.T)
-            cpa4(sb + kGateOff + tid * 4, (tid < 64 ? p.alpha : p.eta) + gate0 + (long long)t * p.H, true);
-        else
-            reinterpret_cast<float*>(bb + kGateOff)[tid] = tid < 64 ? 1.0f : 0.0f;
-        cpa_commit();
-    };
-
-    float sacc[8][4];
-#pragma unroll
-    for (int n = 0; n < 8; ++n) sacc[n][0] = sacc[n][1] = sacc[n][2] = sacc[n][3] = 0.0f;
-    const int n_chunks = (p.T + kC - 1) / kC;
-    stage(0);
-    for (int c = 0; c < n_chunks; ++c) {
-        cpa_wait<0>();
-        __syncthreads();  // chunk c staged, the S copy of chunk c-1 written, chunk c-1 read
-        if (c + 1 < n_chunks) stage(c + 1);
-        unsigned char* bb = bufs + (c & 1) * kBufB;
-        const uint32_t sQ = (uint32_t)__cvta_generic_to_shared(bb);
-        const uint32_t sV = sQ + kTileB;
-        const uint32_t sK = COSTATE ? sQ + 2 * kTileB : sQ;
-        const float* al = reinterpret_cast<const float*>(bb + kGateOff);
-        const float* et = al + kC;
-
-        if (tid < kC) {  // decay pieces
-            float sg = 1.0f, pp = 1.0f;
-            for (int r = tid + 1; r <= (tid | 7); ++r) sg *= al[r];
-            for (int r = tid & ~7; r < tid; ++r) pp *= al[r];
-            sig[tid] = sg;
-            pim[tid] = pp;
-        } else if (tid < kC + 8) {
-            const int j = tid - kC;
-            float tp = 1.0f;
-            for (int r = 0; r < 8; ++r) tp *= al[8 * j + r];
-            tpr[j] = tp;
-        }
-
-        // this warp's Q fragments, reloaded where used (fewer live registers)
-        auto ldq = [&](int kk, uint32_t (&q)[4]) { ldsm4(sQ + swz(16 * warp + (lane & 15), 2 * kk + (lane >> 4)), q); };
-        // P = Q K^T over the column tiles at or before this warp's tokens
-        float pacc[8][4];
-#pragma unroll
-        for (int n = 0; n < 8; ++n) pacc[n][0] = pacc[n][1] = pacc[n][2] = pacc[n][3] = 0.0f;
-        // (k-steps outside, column tiles inside: consecutive MMAs use different
-        // accumulators)
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-            uint32_t q[4];
-            ldq(kk, q);
-#pragma unroll
-            for (int jp = 0; jp < 4; ++jp) {
-                if (jp <= warp) {
-                    uint32_t r[4];
-                    ld_b_nk(sK, 16 * jp, 16 * kk, lane, r);
-                    mma(pacc[2 * jp], q, r[0], r[1]);
-                    mma(pacc[2 * jp + 1], q, r[2], r[3]);
-                }
-            }
-        }
-        // the carried fast weights: o = Q S^T (scaled by a_t below)
-        float oacc[8][4];
-#pragma unroll
-        for (int n = 0; n < 8; ++n) oacc[n][0] = oacc[n][1] = oacc[n][2] = oacc[n][3] = 0.0f;
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-            uint32_t q[4];
-            ldq(kk, q);
-#pragma unroll
-            for (int jp = 0; jp < 4; ++jp) {
-                uint32_t r[4];
-                ld_b_nk(sS, 16 * jp, 16 * kk, lane, r);
-                mma(oacc[2 * jp], q, r[0], r[1]);
-                mma(oacc[2 * jp + 1], q, r[2], r[3]);
-            }
-        }
-        __syncthreads();  // decay pieces ready; every read of the S copy done
-
-        float tp[8];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) tp[j] = tpr[j];
-        // eta_s sig_s for this thread's columns s = 8j + 2cq + e (reads and write)
-        float se[8][2];
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-#pragma unroll
-            for (int e = 0; e < 2; ++e) se[j][e] = et[8 * j + 2 * cq + e] * sig[8 * j + 2 * cq + e];
-        // P'_ts = -E_ts P_ts (zero for s >= t); a_t for this thread's two tokens
-        float a_row[2];
-#pragma unroll
-        for (int hr = 0; hr < 2; ++hr) {
-            const int t = 16 * warp + g + 8 * hr;
-            const int jt = t >> 3;
-            float dd[2];  // columns in t's own piece: the alphas strictly between s and t
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const int s = 8 * jt + 2 * cq + e;
-                float d = s < t ? et[s] : 0.0f;
-                for (int r = s + 1; r < t; ++r) d *= al[r];
-                dd[e] = d;
-            }
-            float tau = pim[t];  // alphas in [8j + 8, t) for the piece j being scaled
-#pragma unroll
-            for (int j = 7; j >= 0; --j) {
-                const bool below = j < jt;
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const float dec = below ? se[j][e] * tau : (j == jt ? dd[e] : 0.0f);
-                    pacc[j][2 * hr + e] *= -dec;
-                }
-                tau = below ? tau * tp[j] : tau;
-            }
-            a_row[hr] = tau;
-        }
-#pragma unroll
-        for (int n = 0; n < 8; ++n) {
-            oacc[n][0] *= a_row[0];
-            oacc[n][1] *= a_row[0];
-            oacc[n][2] *= a_row[1];
-            oacc[n][3] *= a_row[1];
-        }
-        // + B0 q_t
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-            uint32_t q[4];
-            ldq(kk, q);
-#pragma unroll
-            for (int jp = 0; jp < 4; ++jp) {
-                uint32_t r[4];
-                ld_b_nk(sB0, 16 * jp, 16 * kk, lane, r);
-                mma(oacc[2 * jp], q, r[0], r[1]);
-                mma(oacc[2 * jp + 1], q, r[2], r[3]);
-            }
-        }
-        // + P' V (P' carries the minus sign)
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-            if (kk <= warp) {
-                const uint32_t pa[4] = {pack(pacc[2 * kk][0], pacc[2 * kk][1]),
-                                        pack(pacc[2 * kk][2], pacc[2 * kk][3]),
-                                        pack(pacc[2 * kk + 1][0], pacc[2 * kk + 1][1]),
-                                        pack(pacc[2 * kk + 1][2], pacc[2 * kk + 1][3])};
-#pragma unroll
-                for (int jp = 0; jp < 4; ++jp) {
-                    uint32_t r[4];
-                    ld_b_kn(sV, 16 * jp, 16 * kk, lane, r);
-                    mma(oacc[2 * jp], pa, r[0], r[1]);
-                    mma(oacc[2 * jp + 1], pa, r[2], r[3]);
-                }
-            }
-        }
-        // epilogue: rows of this thread's two tokens, two adjacent columns per tile
-        const EpiParams& ep = p.epi;
-        if (!ep.out2 && !ep.zin) {
-#pragma unroll
-            for (int hr = 0; hr < 2; ++hr) {
-                const int t = c * kC + 16 * warp + g + 8 * hr;
-                if (t < p.T) {
-                    bf* orow = static_cast<bf*>(ep.out) + tok_off(ep.out_str, l, b, t, h) + 2 * cq;
-#pragma unroll
-                    for (int n = 0; n < 8; ++n)
-                        *reinterpret_cast<uint32_t*>(orow + 8 * n) = pack(oacc[n][2 * hr], oacc[n][2 * hr + 1]);
-                }
-            }
-        } else {
-#pragma unroll
-        for (int hr = 0; hr < 2; ++hr) {
-            const int t = c * kC + 16 * warp + g + 8 * hr;
-            if (t < p.T) {
-                bf* orow = static_cast<bf*>(ep.out) + tok_off(ep.out_str, l, b, t, h);
-                bf* o2row = ep.out2 ? static_cast<bf*>(ep.out2) + tok_off(ep.out2_str, l, b, t, h) : nullptr;
-                const bf* zrow = ep.zin ? static_cast<const bf*>(ep.zin) + tok_off(ep.z_str, l, b, t, h) : nullptr;
-#pragma unroll
-                for (int n = 0; n < 8; ++n) {
-                    const int col = 8 * n + 2 * cq;
-                    float v0 = oacc[n][2 * hr], v1 = oacc[n][2 * hr + 1];
-                    if (o2row)
-                        *reinterpret_cast<__nv_bfloat162*>(o2row + col) =
-                            __floats2bfloat162_rn(act_f(ep.act, v0), act_f(ep.act, v1));
-                    if (zrow) {
-                        const float2 z = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(zrow + col));
-                        v0 *= act_df(ep.act, z.x);
-                        v1 *= act_df(ep.act, z.y);
-                    }
-                    *reinterpret_cast<__nv_bfloat162*>(orow + col) = __floats2bfloat162_rn(v0, v1);
-                }
-            }
-        }
-        }
-        // the write: S <- a_end S - sum_s w_s v_s k_s^T, w_s = eta_s sig_s prod_{pieces after s} tp
-        float sfx[8];
-        sfx[7] = 1.0f;
-#pragma unroll
-        for (int j = 6; j >= 0; --j) sfx[j] = sfx[j + 1] * tp[j + 1];
-        const float a_end = sfx[0] * tp[0];
-#pragma unroll
-        for (int n = 0; n < 8; ++n) {
-            sacc[n][0] *= a_end;
-            sacc[n][1] *= a_end;
-            sacc[n][2] *= a_end;
-            sacc[n][3] *= a_end;
-        }
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-            // A = (w o V)^T rows [16 warp, +16), tokens [16 kk, +16), from V stored [s][v]
-            uint32_t va[4];
-            ldsm4t(sV + swz(16 * kk + (lane & 7) + ((lane >> 4) << 3), 2 * warp + ((lane >> 3) & 1)), va);
-            const float w00 = -se[2 * kk][0] * sfx[2 * kk], w01 = -se[2 * kk][1] * sfx[2 * kk];
-            const float w10 = -se[2 * kk + 1][0] * sfx[2 * kk + 1], w11 = -se[2 * kk + 1][1] * sfx[2 * kk + 1];
-            va[0] = scale2(va[0], w00, w01);
-            va[1] = scale2(va[1], w00, w01);
-            va[2] = scale2(va[2], w10, w11);
-            va[3] = scale2(va[3], w10, w11);
-#pragma unroll
-            for (int jp = 0; jp < 4; ++jp) {
-                uint32_t r[4];
-                ld_b_kn(sK, 16 * jp, 16 * kk, lane, r);
-                mma(sacc[2 * jp], va, r[0], r[1]);
-                mma(sacc[2 * jp + 1], va, r[2], r[3]);
-            }
-        }
-        // bf16 copy of this warp's rows of S for the next chunk's read
-        const int m = 16 * warp + g;
-#pragma unroll
-        for (int n = 0; n < 8; ++n) {
-            *reinterpret_cast<uint32_t*>(Sbs + swz(m, n) + cq * 4) = pack(sacc[n][0], sacc[n][1]);
-            *reinterpret_cast<uint32_t*>(Sbs + swz(m + 8, n) + cq * 4) = pack(sacc[n][2], sacc[n][3]);
-        }
-    }
-}
-
-template <bool COSTATE>
-cudaError_t launch(const GatedParams& p, int blocks, cudaStream_t stream) {
-    auto kern = chunk_decay_kernel<COSTATE>;
-    const size_t smem = smem_bytes<COSTATE>();
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e == cudaSuccess)  // room for the CTAs the registers allow
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
-    if (e != cudaSuccess) return e;
-    kern<<<blocks, kThr, smem, stream>>>(p);
-    return cudaGetLastError();
-}
-
-}  // namespace cdec
-
 template <bool COSTATE>
 cudaError_t launch_serial_reg(const GatedParams& p, int blocks, cudaStream_t stream) {
     serial_reg_kernel<COSTATE><<<blocks, kThreads, 0, stream>>>(p);
@@ -826,35 +443,15 @@ static bool serial_reg_ok(const GatedParams& p, bool costate, bool bf16) {
     return true;
 }
 
-// The chunked kernel stages 16-byte pieces of 64-wide bf16 token rows and stores
-// pairs of bf16 outputs: W 64 x 64, alpha_t given, rows 16-byte aligned, the
-// epilogue tensors 4-byte aligned with even strides.
-static bool chunk_decay_ok(const GatedParams& p, bool costate, bool bf16) {
-    if (!bf16 || p.din != 64 || p.dout != 64 || !p.alpha || !p.eta || p.T <= 0) return false;
-    if (!serial_reg_ok(p, costate, bf16)) return false;
-    const void* ep[3] = {p.epi.out, p.epi.out2, p.epi.zin};
-    const long long* es[3] = {p.epi.out_str, p.epi.out2_str, p.epi.z_str};
-    for (int k = 0; k < 3; ++k) {
-        if (!ep[k]) continue;
-        if ((reinterpret_cast<uintptr_t>(ep[k]) & 3u) != 0) return false;
-        for (int i = 0; i < 4; ++i)
-            if (es[k][i] % 2 != 0) return false;
-    }
-    return true;
-}
-
-// Retention scans (alpha_t given): the chunked kernel where the shape allows it,
-// else a token-serial kernel (registers for bf16 reads of at most 64 inputs,
-// shared memory otherwise).
+// Retention scans (alpha_t given) that the tensor-core kernel (scan_decay_tc.cu)
+// does not take: a token-serial kernel (registers for bf16 reads of at most 64
+// inputs, shared memory otherwise).
 cudaError_t launch_gated_serial(const GatedParams& p, bool costate, bool bf16, cudaStream_t stream) {
     const int NO = costate ? p.din : p.dout;
     const int tiles = (NO + gated::kTile - 1) / gated::kTile;
     const long long blocks = (long long)p.L * p.B * p.H * tiles;
     const size_t smem = gated_serial_smem(p.din, p.dout, costate);
     if (blocks <= 0) return cudaSuccess;
-    if (chunk_decay_ok(p, costate, bf16))  // one CTA per unit (tiles == 1)
-        return costate ? gated::cdec::launch<true>(p, (int)blocks, stream)
-                       : gated::cdec::launch<false>(p, (int)blocks, stream);
     if (serial_reg_ok(p, costate, bf16))  // the state fits in registers
         return costate ? gated::launch_serial_reg<true>(p, (int)blocks, stream)
                        : gated::launch_serial_reg<false>(p, (int)blocks, stream);
