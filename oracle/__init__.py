@@ -1,7 +1,9 @@
 """The parity oracle for the GradLev scans (test infrastructure).
 
 A plain fp64 CPU implementation of the sequential online learner
-(GradLev Sec. 3, Eqs. 2-4, and the online MLP of Appendix A), written in C
+(GradLev Sec. 3, Eqs. 2-4, and the online MLP of Appendix A), its suffix read and
+the derivatives of an outer objective with respect to the per-token gates
+(Sec. 3, practical architecture and training), written in C
 (``gradlev_oracle.c``) and loaded through ctypes, plus the per-token consistency
 term of the training objective (Eq. 5) written out in numpy.  Only ``tests/``,
 ``__graft_entry__.smoke()`` and the ``cpu_baseline`` / ``--impl reference``
@@ -63,6 +65,8 @@ def _load():
     lib.oracle_act_deriv.restype = ctypes.c_double
     lib.oracle_suffix_batch.argtypes = [I, I, I, I, P, P, P, P, I]
     lib.oracle_suffix_batch.restype = I
+    lib.oracle_gate_grads_batch.argtypes = [I, I, I, I, P, P, P, P, P, P, P, P, I]
+    lib.oracle_gate_grads_batch.restype = I
     lib.oracle_max_threads.argtypes = []
     lib.oracle_max_threads.restype = I
     _lib = lib
@@ -225,6 +229,38 @@ def suffix_scan(q, k, v, nthreads=0):
     if lib.oracle_suffix_batch(U, T, dq, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(r), int(nthreads)):
         raise MemoryError("oracle_suffix_batch could not allocate scratch")
     return r
+
+
+def gate_grads(x, ghat, eta, alpha, a, b, nthreads=0):
+    """Derivatives of an outer objective with respect to the per-token gates of the
+    learner (Sec. 3, practical architecture and training: the gates are learned and
+    their derivatives kept, the writes detached).  Each read of W_t adds
+    a_t^T W_t b_t: the forward read with outer gradient u takes a = u, b = x; the
+    costate read with outer gradient w takes a = gout, b = w.
+
+    x [U,T,d], ghat [U,T,m], eta and alpha scalar, [T] or [U,T], a [U,T,m], b [U,T,d].
+    Returns (alpha_j dL/dalpha_j, dL/deta_j), each [U,T]: the first is the derivative
+    in log alpha_j, <W_j - W0, R_j> alpha_j with R_j = sum_{s>j} prod_{j<r<s} alpha_r
+    a_s b_s^T; the second -ghat_j^T R_j x_j."""
+    lib = _load()
+    x, ghat, a, b = _f64(x), _f64(ghat), _f64(a), _f64(b)
+    U, T, d = x.shape
+    m = ghat.shape[2]
+    if ghat.shape != (U, T, m) or a.shape != (U, T, m) or b.shape != (U, T, d):
+        raise ValueError("gate_grads shape mismatch")
+
+    def gates(v):
+        v = np.asarray(v, dtype=np.float64)
+        return np.ascontiguousarray(np.broadcast_to(v, (T,)) if v.ndim == 0 else np.broadcast_to(v, (U, T)))
+
+    eta_a = np.ascontiguousarray(np.broadcast_to(gates(eta), (U, T)))
+    alpha_a = np.ascontiguousarray(np.broadcast_to(gates(1.0 if alpha is None else alpha), (U, T)))
+    ga = np.empty((U, T))
+    ge = np.empty((U, T))
+    if lib.oracle_gate_grads_batch(U, T, d, m, _ptr(x), _ptr(ghat), _ptr(eta_a), _ptr(alpha_a),
+                                   _ptr(a), _ptr(b), _ptr(ga), _ptr(ge), int(nthreads)):
+        raise MemoryError("oracle_gate_grads_batch could not allocate scratch")
+    return ga, ge
 
 
 def consistency(proposal, target):

@@ -323,6 +323,112 @@ int oracle_suffix_batch(int U, int T, int dq, int dv, const double* q, const dou
     return err;
 }
 
+/*
+ * oracle_gate_grads -- derivatives of an outer objective with respect to the gates
+ * of one unit (Sec. 3, practical architecture and training: the gates are learned
+ * and their derivatives kept, the writes detached).  The fast weights minus W0,
+ * D_t = W_t - W0, follow Eq. 2:  D_0 = 0,  D_{t+1} = alpha_t D_t - eta_t ghat_t x_t^T.
+ * Each read of W_t adds a_t^T W_t b_t to the objective: for the forward read
+ * y_t = W_t x_t with outer gradient u_t, a = u and b = x; for the costate read
+ * gin_t = W_t^T gout_t with outer gradient w_t, a = gout and b = w.  With
+ *     R_j = sum_{s>j} (prod_{j<r<s} alpha_r) a_s b_s^T               (m x d)
+ * the derivatives are
+ *     dL/dalpha_j = <D_j, R_j>  (Frobenius),     dL/deta_j = -ghat_j^T R_j x_j,
+ * and the function returns alpha_j dL/dalpha_j (the derivative in log alpha_j) in
+ * g_alpha and dL/deta_j in g_eta.  W0 does not enter.
+ * R is walked backwards (R_{T-1} = 0, R_{j-1} = alpha_j R_j + a_j b_j^T) and kept at
+ * the last token of every block of GG_BLK tokens; inside a block it is recomputed
+ * backwards from that copy while D_j is walked forwards.
+ *   x [T][d], ghat [T][m], eta, alpha [T], a [T][m], b [T][d]; scratch holds
+ *   (ceil(T / GG_BLK) + GG_BLK + 1) m d doubles.
+ */
+#define GG_BLK 64
+void oracle_gate_grads(int T, int d, int m, const double* x, const double* ghat, const double* eta,
+                       const double* alpha, const double* a, const double* b, double* g_alpha,
+                       double* g_eta, double* scratch) {
+    const size_t md = (size_t)m * d;
+    const int nb = (T + GG_BLK - 1) / GG_BLK;
+    double* ck = scratch;                   /* [nb][m][d] R at each block's last token */
+    double* blk = ck + (size_t)nb * md;     /* [GG_BLK][m][d] R inside one block */
+    double* D = blk + (size_t)GG_BLK * md;  /* [m][d] */
+    /* backward: R_j for j = T-1 .. 0 in D (as scratch), copied at block ends */
+    memset(D, 0, sizeof(double) * md);
+    for (int j = T - 1; j >= 0; --j) {
+        if (j == T - 1 || (j + 1) % GG_BLK == 0) memcpy(ck + (size_t)(j / GG_BLK) * md, D, sizeof(double) * md);
+        if (j > 0) {
+            const double* aj = a + (size_t)j * m;
+            const double* bj = b + (size_t)j * d;
+            for (int i = 0; i < m; ++i)
+                for (int k = 0; k < d; ++k) D[(size_t)i * d + k] = alpha[j] * D[(size_t)i * d + k] + aj[i] * bj[k];
+        }
+    }
+    /* forward: D_j, with R_j of the block recomputed backwards from its last token */
+    memset(D, 0, sizeof(double) * md);
+    for (int q = 0; q < nb; ++q) {
+        const int j0 = q * GG_BLK;
+        const int e = (j0 + GG_BLK < T ? j0 + GG_BLK : T) - 1;
+        memcpy(blk + (size_t)(e - j0) * md, ck + (size_t)q * md, sizeof(double) * md);
+        for (int j = e; j > j0; --j) {
+            const double* Rj = blk + (size_t)(j - j0) * md;
+            double* Rp = blk + (size_t)(j - 1 - j0) * md;
+            const double* aj = a + (size_t)j * m;
+            const double* bj = b + (size_t)j * d;
+            for (int i = 0; i < m; ++i)
+                for (int k = 0; k < d; ++k) Rp[(size_t)i * d + k] = alpha[j] * Rj[(size_t)i * d + k] + aj[i] * bj[k];
+        }
+        for (int j = j0; j <= e; ++j) {
+            const double* Rj = blk + (size_t)(j - j0) * md;
+            const double* xj = x + (size_t)j * d;
+            const double* gj = ghat + (size_t)j * m;
+            double f = 0.0, ge = 0.0;
+            for (int i = 0; i < m; ++i) {
+                double rx = 0.0;
+                for (int k = 0; k < d; ++k) {
+                    f += D[(size_t)i * d + k] * Rj[(size_t)i * d + k];
+                    rx += Rj[(size_t)i * d + k] * xj[k];
+                }
+                ge += gj[i] * rx;
+            }
+            g_alpha[j] = alpha[j] * f;
+            g_eta[j] = -ge;
+            for (int i = 0; i < m; ++i)
+                for (int k = 0; k < d; ++k)
+                    D[(size_t)i * d + k] = alpha[j] * D[(size_t)i * d + k] - eta[j] * gj[i] * xj[k];
+        }
+    }
+}
+
+/* oracle_gate_grads over U independent units ([U][...] contiguous, gates [U][T]). */
+int oracle_gate_grads_batch(int U, int T, int d, int m, const double* x, const double* ghat,
+                            const double* eta, const double* alpha, const double* a, const double* b,
+                            double* g_alpha, double* g_eta, int nthreads) {
+    int err = 0;
+    const size_t md = (size_t)m * d;
+    const size_t ns = ((size_t)(T + GG_BLK - 1) / GG_BLK + GG_BLK + 1) * md;
+#ifdef _OPENMP
+    if (nthreads > 0) omp_set_num_threads(nthreads);
+#else
+    (void)nthreads;
+#endif
+#pragma omp parallel
+    {
+        double* scratch = (double*)malloc(sizeof(double) * ns);
+        if (!scratch) {
+#pragma omp atomic write
+            err = -1;
+        } else {
+#pragma omp for schedule(dynamic, 1)
+            for (int u = 0; u < U; ++u)
+                oracle_gate_grads(T, d, m, x + (size_t)u * T * d, ghat + (size_t)u * T * m,
+                                  eta + (size_t)u * T, alpha + (size_t)u * T, a + (size_t)u * T * m,
+                                  b + (size_t)u * T * d, g_alpha + (size_t)u * T, g_eta + (size_t)u * T,
+                                  scratch);
+            free(scratch);
+        }
+    }
+    return err;
+}
+
 /* Threads the OpenMP runtime would use (for reporting the CPU baseline). */
 int oracle_max_threads(void) {
 #ifdef _OPENMP

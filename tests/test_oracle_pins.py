@@ -562,6 +562,96 @@ def test_eta_gradient_of_costate_read_is_a_suffix_read():
     assert np.abs(fd - an).max() < 1e-7 * max(1.0, np.abs(an).max())
 
 
+# ------------------------------------------------------ gate derivatives
+def _gate_case(seed, T, d, m):
+    r = _rng(seed)
+    x, gh = r.standard_normal((1, T, d)), r.standard_normal((1, T, m))
+    go, u, w = r.standard_normal((1, T, m)), r.standard_normal((1, T, m)), r.standard_normal((1, T, d))
+    W0 = r.standard_normal((m, d)) * 0.3
+    eta = r.uniform(0.01, 0.3, T)
+    alpha = r.uniform(0.5, 1.0, T)
+    alpha[T // 3] = 0.0     # a reset
+    alpha[T // 2] = -0.6    # a negative retention
+    return x, gh, go, u, w, W0, eta, alpha
+
+
+def _fd(loss, v, h=1e-4):
+    g = np.empty_like(v)
+    for s in range(v.shape[0]):
+        v1, v2 = v.copy(), v.copy()
+        v1[s] += h
+        v2[s] -= h
+        g[s] = (loss(v1) - loss(v2)) / (2 * h)
+    return g
+
+
+@pytest.mark.parametrize("read", ["forward", "costate"])
+def test_gate_grads_match_central_differences(read):
+    """Every read is affine in each single alpha_j and eta_j (each decay product holds
+    alpha_j at most once), so central differences of the sequential learner give
+    dL/dalpha_j and dL/deta_j up to rounding.  Non-square maps catch a transposed
+    operand; a reset and a negative retention are included."""
+    T, d, m = 26, 5, 3
+    x, gh, go, u, w, W0, eta, alpha = _gate_case(404 if read == "forward" else 405, T, d, m)
+    if read == "forward":
+        loss = lambda e, a: float(np.sum(u * oracle.linear_scan(x, gh, W0, e, alpha=a)[0]))
+        ga, ge = oracle.gate_grads(x, gh, eta, alpha, u, x)
+    else:
+        loss = lambda e, a: float(np.sum(
+            w * oracle.linear_scan(x, gh, W0, e, alpha=a, gout=go, want_y=False)[1]))
+        ga, ge = oracle.gate_grads(x, gh, eta, alpha, go, w)
+    fd_a = _fd(lambda a: loss(eta, a), alpha) * alpha
+    fd_e = _fd(lambda e: loss(e, alpha), eta)
+    scale = max(1.0, np.abs(fd_a).max(), np.abs(fd_e).max())
+    assert np.abs(ga[0] - fd_a).max() < 1e-8 * scale
+    assert np.abs(ge[0] - fd_e).max() < 1e-8 * scale
+
+
+def test_gate_grads_brute_force_pairs():
+    """alpha_j dL/dalpha_j is the sum, over every write i and later read s with
+    i < j < s, of that pair's contribution -eta_i prod_{i<r<s} alpha_r
+    (u_s . ghat_i)(x_i . x_s) to L = sum_s u_s . y_s; dL/deta_i is the sum of the
+    same contributions over s > i, divided by eta_i."""
+    T, d, m = 7, 3, 2
+    x, gh, go, u, w, W0, eta, alpha = _gate_case(406, T, d, m)
+    ga, ge = oracle.gate_grads(x, gh, eta, alpha, u, x)
+    c = np.zeros((T, T))
+    for i in range(T):
+        for s_ in range(i + 1, T):
+            c[i, s_] = -eta[i] * np.prod(alpha[i + 1:s_]) * np.dot(u[0, s_], gh[0, i]) * np.dot(x[0, i], x[0, s_])
+    ref_a = np.array([sum(c[i, s_] for i in range(j) for s_ in range(j + 1, T)) for j in range(T)])
+    ref_e = np.array([c[i, i + 1:].sum() / eta[i] for i in range(T)])
+    assert np.abs(ga[0] - ref_a).max() < 1e-12 * max(1.0, np.abs(ref_a).max())
+    assert np.abs(ge[0] - ref_e).max() < 1e-12 * max(1.0, np.abs(ref_e).max())
+    assert ga[0, 0] == 0.0 and ga[0, -1] == 0.0 and ge[0, -1] == 0.0
+
+
+def test_gate_grads_at_unit_retention_are_the_suffix_read():
+    """With alpha = 1 the decayed suffix read is the plain suffix read: dL/deta_j =
+    -ghat_j . r_j with r = suffix_scan(x, x, u) (a separate routine)."""
+    T, d, m = 30, 4, 6
+    x, gh, go, u, w, W0, eta, alpha = _gate_case(407, T, d, m)
+    ga, ge = oracle.gate_grads(x, gh, eta, np.ones(T), u, x)
+    rs = oracle.suffix_scan(x, x, u)[0]
+    an = -np.sum(gh[0] * rs, axis=1)
+    assert np.abs(ge[0] - an).max() < 1e-12 * max(1.0, np.abs(an).max())
+
+
+def test_gate_grads_telescoping_identity():
+    """alpha_j dL/dalpha_j = sum_{t>j} (A_t - B_t) - B_j with A_t = u_t . (y_t - W0 x_t)
+    (the pairs ending at read t) and B_t = eta_t dL/deta_t (the pairs starting at
+    write t): the pairs that straddle j, counted another way."""
+    T, d, m = 40, 5, 4
+    x, gh, go, u, w, W0, eta, alpha = _gate_case(408, T, d, m)
+    ga, ge = oracle.gate_grads(x, gh, eta, alpha, u, x)
+    y = oracle.linear_scan(x, gh, W0, eta, alpha=alpha)[0][0]
+    A = np.sum(u[0] * (y - x[0] @ W0.T), axis=1)
+    B = eta * ge[0]
+    D = A - B
+    ref = np.array([D[j + 1:].sum() - B[j] for j in range(T)])
+    assert np.abs(ga[0] - ref).max() < 1e-11 * max(1.0, np.abs(ref).max())
+
+
 def test_gated_learner_property_sweep():
     """Random shapes and gates (zeros, negative retention, document cuts) against the
     closed form of Eq. 2, restricted to each document."""
