@@ -648,14 +648,106 @@ class MLPJob:
                 f"tokens, both layers forward and costate in one sequential walk, fp64")
 
 
+class GateGradsJob(GradsJob):
+    """Derivatives with respect to the per-token gates (eta_t and retention alpha_t)
+    of both reads of one linear map per unit, writes detached (Sec. 3, practical
+    architecture and training; Eq. 2): alpha_t dL/dalpha_t and dL/deta_t of the
+    forward read for an upstream u = dL/dy and of the costate read for w = dL/dg_in.
+    Each call runs the retention scan twice (the state at every chunk start,
+    forwards and over reversed inputs) and one per-chunk kernel."""
+
+    kind = "gate_grads"
+
+    def __init__(self, gl, wl, device, rank):
+        LinearJob.__init__(self, gl, wl, device, rank, "alpha")
+        gen = torch.Generator(device=device)
+        gen.manual_seed(wl.seed * 1000 + 31)
+        dt = self.inp["x"].dtype
+        self.inp["u"] = torch.randn(self.inp["g_hat"].shape, generator=gen, device=device).to(dt)
+        self.inp["w"] = torch.randn(self.inp["x"].shape, generator=gen, device=device).to(dt)
+        shape = (wl.L, wl.B, wl.T, wl.H)
+        self.outs = {k: torch.empty(shape, device=device) for k in ("dla_f", "deta_f", "dla_c", "deta_c")}
+        from paper_2609_34174_gb300 import _binding as _B
+        d = _B._Desc(wl.L, wl.B, wl.T, wl.H, wl.d_in, wl.d_out, 1 if wl.dtype == "bf16" else 0, 0)
+        lib = _B.load_library()
+        nb = max(lib.gradlev_gate_grads_workspace_bytes(ctypes.byref(d), 0),
+                 lib.gradlev_gate_grads_workspace_bytes(ctypes.byref(d), 1))
+        self.ws = torch.empty(max(256, int(nb)), dtype=torch.uint8, device=device)
+        self.in_keys = ("x", "g_hat", "g_out", "u", "w", "eta_t", "alpha_t")
+        self.out_keys = ("dla_f", "deta_f", "dla_c", "deta_c")
+        # two retention scans with state dumps, their reversed input copies and one
+        # per-chunk kernel per read
+        units = wl.L * wl.B * wl.H
+        sms = torch.cuda.get_device_properties(device).multi_processor_count if str(device).startswith("cuda") else 152
+        seg = 2 if (units < 2 * sms and wl.T > 1024) else 0
+        self.launches_per_step = 2 * (2 + 2 + 2 * (1 + seg) + 1)
+        self.kernel = {"fwd": "decay_scan_kernel (state dumps) + gate_chunk_kernel, forward read",
+                       "costate": "decay_scan_kernel (state dumps) + gate_chunk_kernel, costate read"}
+
+    def _run(self, src, cut, ws):
+        gl, o = self.gl, self.outs
+        with nvtx("gradlev gate_grads forward read"):
+            gl.gate_grads(cut(src["x"]), cut(src["g_hat"]), cut(src["eta_t"]), cut(src["u"]),
+                          alpha=cut(src["alpha_t"]), dlog_alpha=cut(o["dla_f"]), deta=cut(o["deta_f"]),
+                          workspace=ws)
+        yield
+        with nvtx("gradlev gate_grads costate read"):
+            gl.gate_grads(cut(src["x"]), cut(src["g_hat"]), cut(src["eta_t"]), cut(src["w"]),
+                          alpha=cut(src["alpha_t"]), read="costate", g_out=cut(src["g_out"]),
+                          dlog_alpha=cut(o["dla_c"]), deta=cut(o["deta_c"]), workspace=ws)
+        yield
+
+    def counts(self, scan):
+        """Per token and unit: two retention scans (each that of the chunk kernel) and the
+        per-chunk kernel's C*(d+m) + 4*d*m flops; compulsory bytes e*(d + 2m) + 16 for the
+        forward read's derivatives (x, ghat, u, eta_t, alpha_t in; two fp32 outputs) and
+        e*(2d + 2m) + 16 for the costate read's (g_out too)."""
+        wl = self.wl
+        e = 2 if wl.dtype == "bf16" else 4
+        d, m = wl.d_in, wl.d_out
+        tu = wl.L * wl.B * wl.T * wl.H
+        flops = tu * (2 * (4 * d * m + COUNT_CHUNK * (d + m)) + 2 * COUNT_CHUNK * (d + m) + 4 * d * m)
+        if scan == "fwd":
+            return flops, tu * (e * (d + 2 * m) + 16)
+        return flops, tu * (e * (2 * d + 2 * m) + 16)
+
+    def config(self):
+        c = LinearJob.config(self)
+        c["computes"] = ("alpha_t dL/dalpha_t and dL/deta_t of the forward and costate reads "
+                         "(state dumps of the retention scan + per-chunk expansion)")
+        return c
+
+    def oracle_run(self, inp, n_units, cores, t_tokens=None):
+        """The fp64 oracle's gate derivatives of both reads for the first n_units units."""
+        import numpy as np
+        import oracle
+        wl = self.wl
+        units = [(l, b, h) for l in range(wl.L) for b in range(wl.B) for h in range(wl.H)]
+        units = units[:n_units]
+        f = lambda k: W.units_fp64(inp[k], units)
+        x, g, go, u, w = f("x"), f("g_hat"), f("g_out"), f("u"), f("w")
+        gates = lambda k: np.stack([inp[k][l, b, :, h].double().cpu().numpy() for (l, b, h) in units])
+        et, al = gates("eta_t"), gates("alpha_t")
+        t = time.perf_counter()
+        oracle.gate_grads(x, g, et, al, u, x, nthreads=cores)
+        oracle.gate_grads(x, g, et, al, go, w, nthreads=cores)
+        return time.perf_counter() - t, len(units) * wl.T / wl.H
+
+    def sample_text(self, n, t_tokens=None):
+        return (f"{n} of {self.n_units()} (layer, batch, head) units at full T={self.wl.T}: "
+                f"gate derivatives of both reads, fp64")
+
+
 def make_job(gl, wl, device, rank, gates=None, grads=False, fused=False):
     if fused:
         if isinstance(wl, W.MLPWorkload) or gates or grads:
             raise SystemExit("--fused applies to the ungated linear workloads")
         return FusedJob(gl, wl, device, rank)
     if grads:
-        if isinstance(wl, W.MLPWorkload) or gates:
-            raise SystemExit("--grads applies to the ungated linear workloads")
+        if isinstance(wl, W.MLPWorkload) or gates not in (None, "alpha"):
+            raise SystemExit("--grads applies to the linear workloads, ungated or with --gates alpha")
+        if gates == "alpha":
+            return GateGradsJob(gl, wl, device, rank)
         return GradsJob(gl, wl, device, rank)
     if isinstance(wl, W.MLPWorkload):
         if gates:
@@ -845,6 +937,20 @@ def run_reference(args, wl, rank, world):
 
         sample = f"{wl.B} sequences x {t_tok} tokens of the deployed MLP per step, fp64"
         metric = DECODE_METRIC
+    elif args.grads and args.gates == "alpha":
+        job = GateGradsJob.__new__(GateGradsJob)
+        job.wl = wl
+        inp = W.make_linear(wl, device="cpu")
+        inp.update(make_gates(wl, "alpha", "cpu"))
+        gen = torch.Generator()
+        gen.manual_seed(wl.seed * 1000 + 31)
+        dt = inp["x"].dtype
+        inp["u"] = torch.randn(inp["g_hat"].shape, generator=gen).to(dt)
+        inp["w"] = torch.randn(inp["x"].shape, generator=gen).to(dt)
+        n = min(job.n_units(), cores)
+        run = lambda: job.oracle_run(inp, n, cores)
+        sample = job.sample_text(n) + " per step"
+        metric = GATE_GRADS_METRIC
     elif args.grads:
         job = GradsJob.__new__(GradsJob)
         job.wl = wl
@@ -899,6 +1005,8 @@ def run_reference(args, wl, rank, world):
 
 GRADS_METRIC = ("tokens/s of dL/deta_t per read (forward read, costate read) at 1 GB300; "
                 "% of roofline")
+GATE_GRADS_METRIC = ("tokens/s of the gate derivatives (alpha_t dL/dalpha_t, dL/deta_t) per read "
+                     "(forward read, costate read) at 1 GB300; % of HBM roofline")
 DECODE_METRIC = "deployment tokens/s (one token per sequence per step) at 1 GB300; % of HBM roofline"
 
 
@@ -1237,7 +1345,8 @@ def run_gradlev(args, wl, rank, world, local_rank):
            "l2": "inputs larger than L2" if flush is None else "L2 flushed between steps"}
     if job.kind == "fused":
         cfg["step"] = "forward and costate reads in one pass (gradlev_fused_scan)"
-    line = {"metric": GRADS_METRIC if args.grads else METRIC, "value": round(value, 1),
+    line = {"metric": (GATE_GRADS_METRIC if args.gates == "alpha" else GRADS_METRIC) if args.grads else METRIC,
+            "value": round(value, 1),
             "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms, 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,

@@ -186,10 +186,11 @@ int gradlev_fused_scan(const gradlev_desc* desc, const gradlev_tensor* x,
  * Without alpha_t the proposals are scaled by eta_t into the workspace (one
  * elementwise pass, rounded to the input dtype) and the chunked scan runs with
  * eta = 1.  With alpha_t:
- *   - bf16 64 x 64 maps whose token rows are 16-byte aligned (the outputs 4-byte
- *     aligned with even strides) run in chunks of 64 tokens on the tensor cores,
- *     with the decays formed as products of the alphas (exact zeros at resets;
- *     any real alpha_t is accepted);
+ *   - bf16 64 x 64 maps whose tensors a TMA map can describe (16-byte aligned
+ *     rows and strides) run in chunks of 128 tokens on the tensor cores, with the
+ *     decays formed as products of the alphas (exact zeros at resets; any real
+ *     alpha_t is accepted); fewer than two units per SM over more than 1024 tokens
+ *     are cut into segments whose states are carried (an aggregate pass first);
  *   - every other shape runs the recurrence token by token, the state W - W0 in
  *     fp32.  The read width (d_in forward, d_out costate) must be at most 256,
  *     else GRADLEV_ERR_UNSUPPORTED.
@@ -336,6 +337,41 @@ int gradlev_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x
                      const gradlev_tensor* upstream, float* deta, void* workspace,
                      size_t workspace_bytes, gradlev_stream_t stream);
 size_t gradlev_eta_grad_workspace_bytes(const gradlev_desc* desc, int read);
+
+/*
+ * gradlev_gate_grads -- derivatives of one adapted map's read with respect to its
+ * per-token gates, eta_t and retention alpha_t (Sec. 3, practical architecture and
+ * training: the gates are learned and their derivatives kept, the writes detached;
+ * Eq. 2 with decay centred at W0).  With D_t = W_t - W0 and u the read's upstream
+ * gradient, a write i and a later read s > i contribute
+ *     c_is = -eta_i (prod_{i<r<s} alpha_r) (u_s . ghat_i)(x_i . x_s)         (read 0)
+ *     c_is = -eta_i (prod_{i<r<s} alpha_r) (g_out_s . ghat_i)(u_s . x_i)     (read 1)
+ * and the outputs are
+ *     deta_i       = dL/deta_i = sum_{s>i} c_is / eta_i
+ *     dlog_alpha_j = alpha_j dL/dalpha_j = sum_{i<j<s} c_is = <D_j, R_j> alpha_j,
+ * the derivative in log alpha_j (for alpha_t = sigmoid(a_t), dL/da_t =
+ * (1 - alpha_t) dlog_alpha_t; no division, so a reset alpha_t = 0 is allowed).
+ *   read 0 (forward, y = W x): u = dL/dy [L][B][T][H][d_out]; read 1 (costate,
+ *            gin = W^T g_out): u = dL/dgin [L][B][T][H][d_in], g_out required
+ *   x, g_hat, g_out  the map's tensors as for the scans (read); token rows 16-byte
+ *            aligned with 16-byte strides, else GRADLEV_ERR_UNSUPPORTED
+ *   eta_t    fp32 [L][B][T][H] contiguous (read); alpha_t the same or NULL (= 1)
+ *   dlog_alpha, deta  fp32 [L][B][T][H], contiguous (written)
+ *   workspace/workspace_bytes  at least gradlev_gate_grads_workspace_bytes(desc, read),
+ *            256-byte aligned
+ * W0 does not enter.  The decayed suffix read R_j x (read 0) is the forward gated
+ * read of the inputs reversed in time with every step -1 and no base matrix; it
+ * and the read with W0 = 0 run through the gated scans (the tensor-core retention
+ * kernel for 64 x 64 bf16 maps), on reversed copies in the workspace; dlog_alpha
+ * then follows from the identity sum_{t>j} (A_t - B_t) - B_j with A_t = u_t . (read
+ * with W0 = 0)_t and B_t = eta_t deta_t, accumulated in fp64 per unit.  Returns
+ * the gated scans' codes; asynchronous on `stream`.
+ */
+int gradlev_gate_grads(const gradlev_desc* desc, int read, const gradlev_tensor* x,
+                       const gradlev_tensor* g_hat, const float* eta_t, const float* alpha_t,
+                       const gradlev_tensor* g_out, const gradlev_tensor* upstream, float* dlog_alpha,
+                       float* deta, void* workspace, size_t workspace_bytes, gradlev_stream_t stream);
+size_t gradlev_gate_grads_workspace_bytes(const gradlev_desc* desc, int read);
 
 /* Size of the fixed device array used by gradlev_forward_scan_noalloc (4 MiB). */
 #define GRADLEV_NOALLOC_SCRATCH_BYTES (4u << 20)

@@ -102,6 +102,11 @@ def load_library():
         lib.gradlev_eta_grad.restype = ctypes.c_int
         lib.gradlev_eta_grad_workspace_bytes.argtypes = [D, ctypes.c_int]
         lib.gradlev_eta_grad_workspace_bytes.restype = ctypes.c_size_t
+        lib.gradlev_gate_grads.argtypes = [D, ctypes.c_int, Tp, Tp, P, P, Tp, Tp, P, P, P,
+                                           ctypes.c_size_t, P]
+        lib.gradlev_gate_grads.restype = ctypes.c_int
+        lib.gradlev_gate_grads_workspace_bytes.argtypes = [D, ctypes.c_int]
+        lib.gradlev_gate_grads_workspace_bytes.restype = ctypes.c_size_t
         lib.gradlev_workspace_bytes.argtypes = [D]
         lib.gradlev_workspace_bytes.restype = ctypes.c_size_t
         lib.gradlev_workspace_status.argtypes = [P, P]
@@ -682,3 +687,60 @@ def eta_grad(x, g_hat, upstream, read="forward", g_out=None, deta=None, workspac
                                   ws.numel(), ctypes.c_void_p(stream))
     _call(rc, "gradlev_eta_grad")
     return deta
+
+
+def gate_grads(x, g_hat, eta, upstream, alpha=None, read="forward", g_out=None, dlog_alpha=None,
+               deta=None, workspace=None):
+    """Derivatives of one map's read with respect to its per-token gates (writes
+    detached, gates learned: Sec. 3, practical architecture and training; Eq. 2).
+
+    eta: per-token step sizes (tensor of the token shape of x, or a scalar); alpha:
+    per-token retention or None (= 1).  read="forward": upstream = dL/dy ([.., d_out]);
+    read="costate": upstream = dL/dg_in ([.., d_in]) and g_out is required.
+    Returns (dlog_alpha, deta), fp32 [L,B,T,H]: alpha_t dL/dalpha_t (the derivative in
+    log alpha_t) and dL/deta_t (written into dlog_alpha / deta when given: contiguous
+    float32 of that shape).  64 x 64 bf16 maps.
+    """
+    lib = load_library()
+    x5, g5, u5 = _as5(x), _as5(g_hat), _as5(upstream)
+    go5 = _as5(g_out) if g_out is not None else None
+    _check_same(x5, g5, u5, go5)
+    if not x5.is_cuda:
+        raise ValueError("tensors must be on a CUDA device")
+    rd = {"forward": 0, "costate": 1}[read]
+    if rd == 1 and go5 is None:
+        raise ValueError("the costate read needs g_out")
+    L, B, T, H, d_in = x5.shape
+    d_out = g5.shape[4]
+    shape = (L, B, T, H)
+
+    def per_token(v):
+        if isinstance(v, torch.Tensor):
+            return v.to(device=x5.device, dtype=torch.float32).reshape(shape).contiguous()
+        return torch.full(shape, float(v), dtype=torch.float32, device=x5.device)
+
+    et = per_token(eta)
+    at = per_token(alpha) if alpha is not None else None
+    desc = _desc(x5, d_out, _dtype_code(x5))
+    def out(t):
+        if t is None:
+            return torch.empty(shape, dtype=torch.float32, device=x5.device)
+        if t.dtype != torch.float32 or not t.is_contiguous() or t.numel() != L * B * T * H:
+            raise ValueError("gate_grads outputs must be contiguous float32 [L,B,T,H] tensors")
+        return t
+
+    dla = out(dlog_alpha)
+    deta = out(deta)
+    nbytes = int(lib.gradlev_gate_grads_workspace_bytes(ctypes.byref(desc), rd))
+    ws = workspace if workspace is not None else _workspace(nbytes, x5.device)
+    tx, tg, tu = _tensor(x5), _tensor(g5), _tensor(u5)
+    tgo = _tensor(go5) if go5 is not None else None
+    stream = torch.cuda.current_stream(x5.device).cuda_stream
+    ptr = lambda t: ctypes.c_void_p(t.data_ptr()) if t is not None else None
+    with torch.cuda.device(x5.device):
+        rc = lib.gradlev_gate_grads(ctypes.byref(desc), rd, ctypes.byref(tx), ctypes.byref(tg),
+                                    ptr(et), ptr(at), ctypes.byref(tgo) if tgo is not None else None,
+                                    ctypes.byref(tu), ptr(dla), ptr(deta),
+                                    ctypes.c_void_p(ws.data_ptr()), ws.numel(), ctypes.c_void_p(stream))
+    _call(rc, "gradlev_gate_grads")
+    return dla, deta

@@ -28,6 +28,15 @@ cudaError_t launch_rowdot(const void* a, const TokStr& as, const void* r, const 
 cudaError_t launch_tc_decay(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
                             const CUtensorMap& o, const TcScanParams& p, bool costate, int grid,
                             cudaStream_t stream);
+cudaError_t launch_flip_rows(const void* in, const TokStr& s, void* out, int L, int B, int T, int T_pad,
+                             int H, int w, int elem, cudaStream_t stream);
+cudaError_t launch_flip_gates(const float* in, float fill, float pad, float* out, int L, int B, int T,
+                              int T_pad, int H, cudaStream_t stream);
+cudaError_t launch_gate_chunks(const void* x, const TokStr& xs, const void* gh, const TokStr& gs,
+                               const void* a, const TokStr& as, const void* b, const TokStr& bs,
+                               const float* eta, const float* alpha, const float* Sd, const float* Rd,
+                               float* dlog_alpha, float* deta, int L, int B, int T, int H,
+                               cudaStream_t stream);
 cudaError_t launch_tc_fused(const CUtensorMap& x, const CUtensorMap& ghat, const CUtensorMap& gout,
                             const CUtensorMap& y, const CUtensorMap& gin, const TcScanParams& p,
                             int grid, cudaStream_t stream);
@@ -620,6 +629,78 @@ size_t gated_ws_bytes(const gradlev_desc& d, int sms) {
     return base + (size_t)d.L * d.B * d.T * d.H * d.d_out * elem;
 }
 
+// The retention scan of 64 x 64 bf16 maps on the tensor cores (scan_decay_tc.cu): one
+// work item per unit, or per segment of a few long units.  q, k, v are the read's
+// orientation (forward: x, x, ghat; costate: g_out, ghat, x); state_out, when given,
+// receives the state at every chunk start.
+int run_decay_tc(const gradlev_desc& d, bool costate, const Tok& tq, const Tok& tk, const Tok& tv,
+                 const Tok& to, const Tok& to2, const Tok& tz, int act, const float* W0,
+                 const float* eta_t, const float* alpha_t, float* state_out, void* ws, size_t ws_bytes,
+                 int sms, cudaStream_t stream) {
+    CUtensorMap mq, mk, mv, mo;
+    if (!make_tmap(&mq, d, tq, 64) || !make_tmap(&mk, d, tk, 64) || !make_tmap(&mv, d, tv, 64) ||
+        !make_tmap(&mo, d, to, 64))
+        return GRADLEV_ERR_UNSUPPORTED;
+    const long long units = (long long)d.L * d.B * d.H;
+    gl::TcScanParams p;
+    memset(&p, 0, sizeof(p));
+    p.L = d.L;
+    p.B = d.B;
+    p.T = d.T;
+    p.H = d.H;
+    p.dq = 64;
+    p.dv = 64;
+    p.n_tiles = 1;
+    // Few long units: cut each into segments (multiples of 128 tokens, at least
+    // 512) so that about four waves of items fill the SMs; the segments' states
+    // are carried through an aggregate pass (scan_decay_tc.cu).
+    int n_seg = 1;
+    long long seg_len = d.T;
+    if (units < 2ll * sms && d.T > 1024) {
+        const long long want = (4ll * sms + units - 1) / units;
+        seg_len = (((d.T + want - 1) / want) + 127) / 128 * 128;
+        if (seg_len < 512) seg_len = 512;
+        n_seg = (int)((d.T + seg_len - 1) / seg_len);
+        if (n_seg < 2) {
+            n_seg = 1;
+            seg_len = d.T;
+        }
+    }
+    p.seg_len = (int)seg_len;
+    p.n_seg = n_seg;
+    p.n_items = (int)(units * n_seg);
+    p.n_ut = (int)units;
+    if (n_seg > 1) {
+        // the segment states go where the eta-only path keeps its scaled proposals
+        // (d_out * elem >= 128 bytes per token-unit, against at most 64 here)
+        const size_t a = ws_bytes_for(d, d.d_in, d.d_out, sms);
+        const size_t bb = ws_bytes_for(d, d.d_out, d.d_in, sms);
+        uint8_t* base = static_cast<uint8_t*>(ws) + round_up(a > bb ? a : bb, 256);
+        const size_t blk = (size_t)p.n_items * 64 * 64 * sizeof(float);
+        p.agg = reinterpret_cast<float*>(base);
+        p.incl = reinterpret_cast<float*>(base + blk);
+        p.seg_a = reinterpret_cast<float*>(base + 2 * blk);
+        if (static_cast<size_t>(base - static_cast<uint8_t*>(ws)) + 2 * blk +
+                round_up((size_t)p.n_items * sizeof(float), 256) > ws_bytes)
+            return GRADLEV_ERR_WORKSPACE;
+    }
+    p.lam = 1.0f;
+    p.inv_lam = 1.0f;
+    p.mu = 1.0f;
+    p.w0_transposed = costate ? 1 : 0;
+    p.W0 = W0;
+    p.g_eta = eta_t;
+    p.g_alpha = alpha_t;
+    p.state_out = state_out;
+    fill_epi(&p.epi, to, to2, tz, act);
+    p.ctrl = static_cast<unsigned int*>(ws);
+    if (cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
+    const int grid = p.n_items < sms ? p.n_items : sms;
+    if (gl::launch_tc_decay(mq, mk, mv, mo, p, costate, grid, stream) != cudaSuccess)
+        return GRADLEV_ERR_CUDA;
+    return GRADLEV_OK;
+}
+
 int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
               const gradlev_tensor* g_hat, const float* W0, const float* eta_t,
               const float* alpha_t, const gradlev_tensor* g_out, int act, const gradlev_tensor* out,
@@ -682,72 +763,9 @@ int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
     if (bf16 && d.d_in == 64 && d.d_out == 64 && tc_layout_ok(tx, 2) && tc_layout_ok(tg, 2) &&
         (!costate || tc_layout_ok(tgo, 2)) && tc_layout_ok(to, 2) && tc_layout_ok(to2, 2) &&
         tc_layout_ok(tz, 2)) {
-        // 64 x 64 bf16 maps: the chunked retention scan on the tensor cores, one work
-        // item per unit (scan_decay_tc.cu)
-        const Tok& tq = costate ? tgo : tx;
-        const Tok& tk = costate ? tg : tx;
-        const Tok& tv = costate ? tx : tg;
-        CUtensorMap mq, mk, mv, mo;
-        if (!make_tmap(&mq, d, tq, 64) || !make_tmap(&mk, d, tk, 64) || !make_tmap(&mv, d, tv, 64) ||
-            !make_tmap(&mo, d, to, 64))
-            return GRADLEV_ERR_UNSUPPORTED;
-        const long long units = (long long)d.L * d.B * d.H;
-        gl::TcScanParams p;
-        memset(&p, 0, sizeof(p));
-        p.L = d.L;
-        p.B = d.B;
-        p.T = d.T;
-        p.H = d.H;
-        p.dq = 64;
-        p.dv = 64;
-        p.n_tiles = 1;
-        // Few long units: cut each into segments (multiples of 128 tokens, at least
-        // 512) so that about four waves of items fill the SMs; the segments' states
-        // are carried through an aggregate pass (scan_decay_tc.cu).
-        int n_seg = 1;
-        long long seg_len = d.T;
-        if (units < 2ll * dev.sms && d.T > 1024) {
-            const long long want = (4ll * dev.sms + units - 1) / units;
-            seg_len = (((d.T + want - 1) / want) + 127) / 128 * 128;
-            if (seg_len < 512) seg_len = 512;
-            n_seg = (int)((d.T + seg_len - 1) / seg_len);
-            if (n_seg < 2) {
-                n_seg = 1;
-                seg_len = d.T;
-            }
-        }
-        p.seg_len = (int)seg_len;
-        p.n_seg = n_seg;
-        p.n_items = (int)(units * n_seg);
-        p.n_ut = (int)units;
-        if (n_seg > 1) {
-            // the segment states go where the eta-only path keeps its scaled proposals
-            // (d_out * elem >= 128 bytes per token-unit, against at most 64 here)
-            const size_t a = ws_bytes_for(d, d.d_in, d.d_out, dev.sms);
-            const size_t bb = ws_bytes_for(d, d.d_out, d.d_in, dev.sms);
-            uint8_t* base = static_cast<uint8_t*>(ws) + round_up(a > bb ? a : bb, 256);
-            const size_t blk = (size_t)p.n_items * 64 * 64 * sizeof(float);
-            p.agg = reinterpret_cast<float*>(base);
-            p.incl = reinterpret_cast<float*>(base + blk);
-            p.seg_a = reinterpret_cast<float*>(base + 2 * blk);
-            if (static_cast<size_t>(base - static_cast<uint8_t*>(ws)) + 2 * blk +
-                    round_up((size_t)p.n_items * sizeof(float), 256) > ws_bytes)
-                return GRADLEV_ERR_WORKSPACE;
-        }
-        p.lam = 1.0f;
-        p.inv_lam = 1.0f;
-        p.mu = 1.0f;
-        p.w0_transposed = costate ? 1 : 0;
-        p.W0 = W0;
-        p.g_eta = eta_t;
-        p.g_alpha = alpha_t;
-        fill_epi(&p.epi, to, to2, tz, act);
-        p.ctrl = static_cast<unsigned int*>(ws);
-        if (cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
-        const int grid = p.n_items < dev.sms ? p.n_items : dev.sms;
-        if (gl::launch_tc_decay(mq, mk, mv, mo, p, costate, grid, stream) != cudaSuccess)
-            return GRADLEV_ERR_CUDA;
-        return GRADLEV_OK;
+        // 64 x 64 bf16 maps: the chunked retention scan on the tensor cores
+        return run_decay_tc(d, costate, costate ? tgo : tx, costate ? tg : tx, costate ? tx : tg, to, to2,
+                            tz, act, W0, eta_t, alpha_t, nullptr, ws, ws_bytes, dev.sms, stream);
     }
     if (cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
     gl::GatedParams p;
@@ -970,6 +988,118 @@ int run_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x,
     }
     if (gl::launch_rowdot(ta.data, as, trr.data, rs, deta, d.L, d.B, d.T, d.H, sd.d_out, -1.0f,
                           d.dtype == GRADLEV_BF16, stream) != cudaSuccess)
+        return GRADLEV_ERR_CUDA;
+    return GRADLEV_OK;
+}
+
+// Gate derivatives of one map's read with per-token eta_t and retention alpha_t (Sec. 3,
+// practical architecture and training), for 64 x 64 bf16 maps.  With D_t = W_t - W0
+// and the read's upstream gradient u (read 0: y = W x, a = u, b = x; read 1:
+// gin = W^T g_out, a = g_out, b = u):
+//   dlog_alpha_j = alpha_j <D_j, R_j>,  deta_j = -ghat_j^T R_j x_j,
+//   R_j = sum_{s>j} prod_{j<r<s} alpha_r a_s b_s^T.
+// D at every chunk start comes from the retention scan over (x, ghat, eta_t, alpha_t);
+// R at every chunk's last token from the same scan over (b, a) reversed in time with
+// every step -1 (its state at a reversed chunk start); gate_chunk_kernel expands
+// both inside each chunk of 128 tokens.
+size_t gate_grads_ws_bytes(const gradlev_desc& d, int sms) {
+    const long long T_pad = ((long long)d.T + 127) / 128 * 128;
+    gradlev_desc dp = d;
+    dp.T = (int32_t)T_pad;
+    const size_t units = (size_t)d.L * d.B * d.H;
+    const size_t tokens_pad = units * (size_t)T_pad;
+    const size_t g1 = gated_ws_bytes(d, sms), g2 = gated_ws_bytes(dp, sms);
+    return round_up(g1 > g2 ? g1 : g2, 256) + round_up((size_t)d.L * d.H * 64 * 64 * sizeof(float), 256) +
+           2 * round_up(units * (size_t)(T_pad / 128) * 64 * 64 * sizeof(float), 256) +
+           3 * round_up(tokens_pad * 64 * 2, 256) + 2 * round_up(tokens_pad * sizeof(float), 256);
+}
+
+int run_gate_grads(const gradlev_desc* desc, int read, const gradlev_tensor* x,
+                   const gradlev_tensor* g_hat, const float* eta_t, const float* alpha_t,
+                   const gradlev_tensor* g_out, const gradlev_tensor* upstream, float* dlog_alpha,
+                   float* deta, void* ws, size_t ws_bytes, cudaStream_t stream) {
+    if (!desc_ok(desc) || (read != 0 && read != 1)) return GRADLEV_ERR_INVALID_ARG;
+    const gradlev_desc& d = *desc;
+    if (d.T > 0 && (!eta_t || !dlog_alpha || !deta)) return GRADLEV_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(eta_t) | reinterpret_cast<uintptr_t>(alpha_t) |
+         reinterpret_cast<uintptr_t>(dlog_alpha) | reinterpret_cast<uintptr_t>(deta)) & 3u)
+        return GRADLEV_ERR_INVALID_ARG;
+    if (d.dtype != GRADLEV_BF16 || d.d_in != 64 || d.d_out != 64) return GRADLEV_ERR_UNSUPPORTED;
+    DevInfo dev;
+    if (!device_info(&dev)) return GRADLEV_ERR_CUDA;
+    if (!(dev.major == 10 && dev.minor == 3)) return GRADLEV_ERR_UNSUPPORTED;
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < gate_grads_ws_bytes(d, dev.sms))
+        return GRADLEV_ERR_WORKSPACE;
+    Tok tx, tg, tu, tgo;
+    if (!resolve(d, x, 64, &tx, true) || !resolve(d, g_hat, 64, &tg, true) ||
+        !resolve(d, upstream, 64, &tu, true) || !resolve(d, g_out, 64, &tgo, read == 1))
+        return GRADLEV_ERR_INVALID_ARG;
+    if (d.T == 0) return GRADLEV_OK;
+    // 16-byte pieces of every token row (reversed copies, TMA tiles, the chunk kernel)
+    const Tok* rows[4] = {&tx, &tg, &tu, &tgo};
+    for (const Tok* t : rows)
+        if (t->data && !tc_layout_ok(*t, 2)) return GRADLEV_ERR_UNSUPPORTED;
+    const int T_pad = (d.T + 127) / 128 * 128;
+    gradlev_desc dp = d;
+    dp.T = T_pad;
+    const size_t units = (size_t)d.L * d.B * d.H;
+    const size_t tokens_pad = units * (size_t)T_pad;
+    const size_t g1 = gated_ws_bytes(d, dev.sms), g2 = gated_ws_bytes(dp, dev.sms);
+    const size_t gws = round_up(g1 > g2 ? g1 : g2, 256);
+    uint8_t* p = static_cast<uint8_t*>(ws) + gws;
+    auto take = [&](size_t bytes) {
+        uint8_t* q = p;
+        p += round_up(bytes, 256);
+        return q;
+    };
+    const size_t w0_bytes = (size_t)d.L * d.H * 64 * 64 * sizeof(float);
+    const size_t st_bytes = units * (size_t)(T_pad / 128) * 64 * 64 * sizeof(float);
+    float* zero_w0 = reinterpret_cast<float*>(take(w0_bytes));
+    float* Sd = reinterpret_cast<float*>(take(st_bytes));
+    float* Rd = reinterpret_cast<float*>(take(st_bytes));
+    uint8_t* rb = take(tokens_pad * 64 * 2);   // b reversed
+    uint8_t* ra = take(tokens_pad * 64 * 2);   // a reversed
+    uint8_t* junk = take(tokens_pad * 64 * 2);  // the scans' unused outputs
+    float* eta_rev = reinterpret_cast<float*>(take(tokens_pad * sizeof(float)));
+    float* alpha_rev = reinterpret_cast<float*>(take(tokens_pad * sizeof(float)));
+    const Tok& ta = read == 0 ? tu : tgo;
+    const Tok& tb = read == 0 ? tx : tu;
+    auto strides = [](const Tok& t) {
+        gl::TokStr st;
+        for (int i = 0; i < 4; ++i) st.s[i] = t.s[i];
+        return st;
+    };
+    auto contiguous = [&](void* data, const gradlev_desc& dd) {
+        gradlev_tensor g;
+        g.data = data;
+        for (int i = 0; i < 4; ++i) g.stride[i] = 0;
+        Tok t;
+        resolve(dd, &g, 64, &t, true);
+        return t;
+    };
+    if (cudaMemsetAsync(zero_w0, 0, w0_bytes, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
+    if (T_pad != d.T && (cudaMemsetAsync(rb, 0, tokens_pad * 64 * 2, stream) != cudaSuccess ||
+                         cudaMemsetAsync(ra, 0, tokens_pad * 64 * 2, stream) != cudaSuccess))
+        return GRADLEV_ERR_CUDA;
+    if (gl::launch_flip_rows(tb.data, strides(tb), rb, d.L, d.B, d.T, T_pad, d.H, 64, 2, stream) != cudaSuccess ||
+        gl::launch_flip_rows(ta.data, strides(ta), ra, d.L, d.B, d.T, T_pad, d.H, 64, 2, stream) != cudaSuccess ||
+        gl::launch_flip_gates(nullptr, -1.0f, 0.0f, eta_rev, d.L, d.B, d.T, T_pad, d.H, stream) != cudaSuccess ||
+        gl::launch_flip_gates(alpha_t, 1.0f, 1.0f, alpha_rev, d.L, d.B, d.T, T_pad, d.H, stream) != cudaSuccess)
+        return GRADLEV_ERR_CUDA;
+    const Tok none;
+    // D at every chunk start: the forward-orientation scan of the writes
+    const Tok tj = contiguous(junk, d);
+    int rc = run_decay_tc(d, false, tx, tx, tg, tj, none, none, GRADLEV_ACT_NONE, zero_w0, eta_t, alpha_t, Sd,
+                          ws, gws, dev.sms, stream);
+    if (rc != GRADLEV_OK) return rc;
+    // R at every chunk's last token: the same scan over (b, a) reversed, steps -1
+    const Tok trb = contiguous(rb, dp), tra = contiguous(ra, dp), tjp = contiguous(junk, dp);
+    rc = run_decay_tc(dp, false, trb, trb, tra, tjp, none, none, GRADLEV_ACT_NONE, zero_w0, eta_rev, alpha_rev,
+                      Rd, ws, gws, dev.sms, stream);
+    if (rc != GRADLEV_OK) return rc;
+    if (gl::launch_gate_chunks(tx.data, strides(tx), tg.data, strides(tg), ta.data, strides(ta), tb.data,
+                               strides(tb), eta_t, alpha_t, Sd, Rd, dlog_alpha, deta, d.L, d.B, d.T, d.H,
+                               stream) != cudaSuccess)
         return GRADLEV_ERR_CUDA;
     return GRADLEV_OK;
 }
@@ -1213,6 +1343,19 @@ int gradlev_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x
 size_t gradlev_eta_grad_workspace_bytes(const gradlev_desc* desc, int read) {
     if (!desc_ok(desc) || (read != 0 && read != 1)) return 0;
     return eta_grad_ws_bytes(*desc, read, dev_sms_or_default());
+}
+
+int gradlev_gate_grads(const gradlev_desc* desc, int read, const gradlev_tensor* x,
+                       const gradlev_tensor* g_hat, const float* eta_t, const float* alpha_t,
+                       const gradlev_tensor* g_out, const gradlev_tensor* upstream, float* dlog_alpha,
+                       float* deta, void* workspace, size_t workspace_bytes, gradlev_stream_t stream) {
+    return run_gate_grads(desc, read, x, g_hat, eta_t, alpha_t, g_out, upstream, dlog_alpha, deta,
+                          workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t gradlev_gate_grads_workspace_bytes(const gradlev_desc* desc, int read) {
+    if (!desc_ok(desc) || (read != 0 && read != 1)) return 0;
+    return gate_grads_ws_bytes(*desc, dev_sms_or_default());
 }
 
 int gradlev_decode_read(const gradlev_desc* desc, const gradlev_tensor* x, const float* W0,
