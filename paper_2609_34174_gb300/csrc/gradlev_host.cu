@@ -32,11 +32,10 @@ cudaError_t launch_flip_rows(const void* in, const TokStr& s, void* out, int L, 
                              int H, int w, int elem, cudaStream_t stream);
 cudaError_t launch_flip_gates(const float* in, float fill, float pad, float* out, int L, int B, int T,
                               int T_pad, int H, cudaStream_t stream);
-cudaError_t launch_gate_chunks(const void* x, const TokStr& xs, const void* gh, const TokStr& gs,
-                               const void* a, const TokStr& as, const void* b, const TokStr& bs,
-                               const float* eta, const float* alpha, const float* Sd, const float* Rd,
-                               float* dlog_alpha, float* deta, int L, int B, int T, int H,
-                               cudaStream_t stream);
+cudaError_t launch_gate_chunks_tc(const CUtensorMap& x, const CUtensorMap& g, const CUtensorMap& a,
+                                  const CUtensorMap& b, const float* eta, const float* alpha, const float* Sd,
+                                  const float* Rd, float* dlog_alpha, float* deta, int L, int B, int T, int H,
+                                  unsigned int* err, cudaStream_t stream);
 cudaError_t launch_tc_fused(const CUtensorMap& x, const CUtensorMap& ghat, const CUtensorMap& gout,
                             const CUtensorMap& y, const CUtensorMap& gin, const TcScanParams& p,
                             int grid, cudaStream_t stream);
@@ -1000,8 +999,8 @@ int run_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x,
 //   R_j = sum_{s>j} prod_{j<r<s} alpha_r a_s b_s^T.
 // D at every chunk start comes from the retention scan over (x, ghat, eta_t, alpha_t);
 // R at every chunk's last token from the same scan over (b, a) reversed in time with
-// every step -1 (its state at a reversed chunk start); gate_chunk_kernel expands
-// both inside each chunk of 128 tokens.
+// every step -1 (its state at a reversed chunk start); gate_chunk_tc_kernel expands
+// both inside each chunk of 128 tokens on the tensor cores (gate_grads_tc.cu).
 size_t gate_grads_ws_bytes(const gradlev_desc& d, int sms) {
     const long long T_pad = ((long long)d.T + 127) / 128 * 128;
     gradlev_desc dp = d;
@@ -1097,9 +1096,12 @@ int run_gate_grads(const gradlev_desc* desc, int read, const gradlev_tensor* x,
     rc = run_decay_tc(dp, false, trb, trb, tra, tjp, none, none, GRADLEV_ACT_NONE, zero_w0, eta_rev, alpha_rev,
                       Rd, ws, gws, dev.sms, stream);
     if (rc != GRADLEV_OK) return rc;
-    if (gl::launch_gate_chunks(tx.data, strides(tx), tg.data, strides(tg), ta.data, strides(ta), tb.data,
-                               strides(tb), eta_t, alpha_t, Sd, Rd, dlog_alpha, deta, d.L, d.B, d.T, d.H,
-                               stream) != cudaSuccess)
+    CUtensorMap mx, mg, ma, mb;
+    if (!make_tmap(&mx, d, tx, 64) || !make_tmap(&mg, d, tg, 64) || !make_tmap(&ma, d, ta, 64) ||
+        !make_tmap(&mb, d, tb, 64))
+        return GRADLEV_ERR_UNSUPPORTED;
+    if (gl::launch_gate_chunks_tc(mx, mg, ma, mb, eta_t, alpha_t, Sd, Rd, dlog_alpha, deta, d.L, d.B, d.T, d.H,
+                                  static_cast<unsigned int*>(ws) + 1, stream) != cudaSuccess)
         return GRADLEV_ERR_CUDA;
     return GRADLEV_OK;
 }
