@@ -38,7 +38,8 @@ constexpr int kS = 4 * kTile;            // S^T, then Rt^T (bf16); afterwards N^
 constexpr int kR = kS + kStT;
 constexpr int kN = kS;                   // N^T bf16 [128][128], written after the state products
 constexpr int kV = kN + kC * kC * 2;     // v, w, eta, alpha fp32 [128] each, red[4]
-constexpr int kBar = kV + 4 * kC * 4 + 16;
+constexpr int kScan = kV + 4 * kC * 4 + 16;  // two affine scans, (A, B) [2][128] each
+constexpr int kBar = kScan + 4 * kC * 4;
 constexpr int kSmem = kBar + 64 + 1024;  // + slack for the 1024-byte alignment
 constexpr uint32_t kTmemCols = 256;
 
@@ -226,23 +227,46 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     tc_fence_before();
     __syncthreads();
-    // ---- token j: the four terms
+    // ---- token j: the four terms.  Two scans of affine maps x -> A x + B over the
+    // chunk (Hillis-Steele, 7 steps): the prefix of g_i = (alpha_i, -eta_i w_i) gives
+    // P_j and t3_j = sum_{i<j} (-eta_i) E(i,j) w_i; the suffix of f_s = (alpha_s, v_s)
+    // gives Q_j and t2_j = sum_{s>j} G(j,s) v_s.
     {
         const int j = tid;
         const float kappa = (red[0] + red[1]) + (red[2] + red[3]);
-        float P = 1.0f, Q = 1.0f;
-        for (int r = 0; r < j; ++r) P *= al[r];
-        for (int r = j + 1; r < kC; ++r) Q *= al[r];
-        float t2 = 0.0f, g = 1.0f;
-        for (int s = j + 1; s < kC; ++s) {
-            t2 = fmaf(g, v[s], t2);
-            g *= al[s];
+        float* pa = reinterpret_cast<float*>(smem + kScan);
+        float* pb = pa + kC;
+        float* sa = pb + kC;
+        float* sbv = sa + kC;
+        float ap = al[j], bp = -et[j] * w[j];  // inclusive prefix g_j o ... o g_0
+        float as = al[j], bs = v[j];           // inclusive suffix f_j o ... o f_127
+#pragma unroll 1
+        for (int o = 1; o < kC; o <<= 1) {
+            pa[j] = ap;
+            pb[j] = bp;
+            sa[j] = as;
+            sbv[j] = bs;
+            __syncthreads();
+            if (j >= o) {  // (A, B) o (A', B') = (A A', A B' + B)
+                bp = fmaf(ap, pb[j - o], bp);
+                ap *= pa[j - o];
+            }
+            if (j + o < kC) {
+                bs = fmaf(as, sbv[j + o], bs);
+                as *= sa[j + o];
+            }
+            __syncthreads();
         }
-        float t3 = 0.0f, t4 = 0.0f, e = 1.0f;
+        pa[j] = ap;
+        pb[j] = bp;
+        sa[j] = as;
+        sbv[j] = bs;
+        __syncthreads();
+        const float P = j > 0 ? pa[j - 1] : 1.0f, t3 = j > 0 ? pb[j - 1] : 0.0f;
+        const float Q = j + 1 < kC ? sa[j + 1] : 1.0f, t2 = j + 1 < kC ? sbv[j + 1] : 0.0f;
+        float t4 = 0.0f, e = 1.0f;
         for (int i = j - 1; i >= 0; --i) {
-            const float ne = -et[i] * e;
-            t3 = fmaf(ne, w[i], t3);
-            t4 = fmaf(ne, __bfloat162float(NT[nidx(j, i)]), t4);
+            t4 = fmaf(-et[i] * e, __bfloat162float(NT[nidx(j, i)]), t4);
             e *= al[i];
         }
         const int t = c0 + j;
