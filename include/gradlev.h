@@ -359,13 +359,13 @@ size_t gradlev_eta_grad_workspace_bytes(const gradlev_desc* desc, int read);
  *   dlog_alpha, deta  fp32 [L][B][T][H], contiguous (written)
  *   workspace/workspace_bytes  at least gradlev_gate_grads_workspace_bytes(desc, read),
  *            256-byte aligned
- * W0 does not enter.  The decayed suffix read R_j x (read 0) is the forward gated
- * read of the inputs reversed in time with every step -1 and no base matrix; it
- * and the read with W0 = 0 run through the gated scans (the tensor-core retention
- * kernel for 64 x 64 bf16 maps), on reversed copies in the workspace; dlog_alpha
- * then follows from the identity sum_{t>j} (A_t - B_t) - B_j with A_t = u_t . (read
- * with W0 = 0)_t and B_t = eta_t deta_t, accumulated in fp64 per unit.  Returns
- * the gated scans' codes; asynchronous on `stream`.
+ * W0 does not enter.  Only bf16 maps of 64 x 64 (else GRADLEV_ERR_UNSUPPORTED).
+ * Per chunk of 128 tokens: aggregates of the writes and of the pairs (a, b) on the
+ * tensor cores; D at every chunk start and R at every chunk end carried over the
+ * chunks in fp32; then the exact expansion of alpha_j <D_j, R_j> and
+ * -ghat_j^T R_j x_j inside each chunk (four local terms, no cancellation).  A
+ * timed-out device wait is reported by gradlev_workspace_status(workspace).
+ * Asynchronous on `stream`.
  */
 int gradlev_gate_grads(const gradlev_desc* desc, int read, const gradlev_tensor* x,
                        const gradlev_tensor* g_hat, const float* eta_t, const float* alpha_t,

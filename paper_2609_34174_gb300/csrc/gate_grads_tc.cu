@@ -20,7 +20,9 @@
 //   G1 = Ghat A^T, G2 = X B^T             (M = G1 (.) G2, elementwise)
 // with S and Rt rounded to bf16 for their products.  One CTA of 128 threads per
 // (unit, chunk); thread r owns token row r (TMEM lane r).  Tokens past T are zero
-// rows (TMA fill) with alpha = 1 and eta = 0.
+// rows (TMA fill) with alpha = 1 and eta = 0.  S and Rt of every chunk come from
+// per-chunk aggregates (gate_agg_tc_kernel) carried over the chunks by
+// gate_state_scan_kernel (grads.cu).
 #include <cuda.h>
 
 #include "scan_common.cuh"
@@ -110,7 +112,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     // ---- the states as bf16 K-major tiles (S^T rows k by threads 0-63, Rt^T by 64-127)
     const float* s_src = Sd + (unit * nch + c) * (long long)(64 * 64);
-    const float* r_src = Rd + (unit * nch + (nch - 1 - c)) * (long long)(64 * 64);
+    const float* r_src = Rd + (unit * nch + c) * (long long)(64 * 64);
     {
         const int k = tid & 63;
         const float* src = (tid < 64 ? s_src : r_src) + k * 64;
@@ -288,7 +290,174 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
 }
 
+// Chunk aggregates (one CTA of 128 threads per (unit, chunk)), in the S^T layout
+// [k][l] of the states (k: x index, l: ghat index):
+//   Vt_c = X^T (w (.) Ghat),  w_i = -eta_i prod_{i<r<c1} alpha_r   (D_{c+1} = A_c D_c + V_c)
+//   Ut_c = B^T (p (.) A),     p_s = prod_{c0<=r<s} alpha_r          (R_c = U_{c+1} + A_{c+1} R_{c+1})
+// and A_c, the product of the chunk's alphas.  Both products run with M = 128 over
+// an MN-major A operand whose second 64-row block is the next tile in shared
+// memory; those accumulator rows (TMEM lanes 64..127) are never read.
+constexpr int kAggSmem = 6 * kTile + 4 * kC * 4 + 64 + 1024;
+
+__global__ void __launch_bounds__(kThreads, 2)
+    gate_agg_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_g,
+                       const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
+                       const float* __restrict__ eta, const float* __restrict__ alpha, float* __restrict__ Vd,
+                       float* __restrict__ Ud, float* __restrict__ Ad, int B, int T, int H, int nch,
+                       unsigned int* err) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~static_cast<uintptr_t>(1023));
+    const uint32_t sb = smem_u32(smem);
+    // tiles: X | Ghat | B | A | w Ghat | p A  (X and B are each followed by a tile)
+    constexpr int oX = 0, oG = kTile, oB = 2 * kTile, oA = 3 * kTile, oWG = 4 * kTile, oPA = 5 * kTile;
+    float* sp = reinterpret_cast<float*>(smem + 6 * kTile);  // prefix products [128]
+    float* ss = sp + kC;                                      // suffix products [128]
+    float* sal = ss + kC;
+    float* set = sal + kC;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(set + kC);
+    uint64_t* tma_bar = bars;
+    uint64_t* mma_bar = bars + 1;
+    uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 3);
+
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const long long unit = blockIdx.x / nch;
+    const int c = (int)(blockIdx.x % nch);
+    const int h = (int)(unit % H);
+    const long long lb = unit / H;
+    const int b = (int)(lb % B);
+    const int l = (int)(lb / B);
+    const int c0 = c * kC;
+    if (warp == 0) {
+        tmem_alloc(tslot, 128);
+        tmem_relinquish();
+    }
+    if (tid == 0) {
+        mbar_init(tma_bar, 1);
+        mbar_init(mma_bar, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+    if (tid == 0) {
+        mbar_arrive_expect_tx(tma_bar, 4 * kTile);
+        tma_load_5d(smem + oX, &tm_x, tma_bar, 0, h, c0, b, l);
+        tma_load_5d(smem + oG, &tm_g, tma_bar, 0, h, c0, b, l);
+        tma_load_5d(smem + oB, &tm_b, tma_bar, 0, h, c0, b, l);
+        tma_load_5d(smem + oA, &tm_a, tma_bar, 0, h, c0, b, l);
+    }
+    // ---- prefix / suffix products of the chunk's alphas (Hillis-Steele, 7 steps)
+    const int t = c0 + tid;
+    const long long gi = (lb * T + t) * H + h;
+    const float a_own = t < T ? (alpha ? alpha[gi] : 1.0f) : 1.0f;
+    set[tid] = t < T ? eta[gi] : 0.0f;
+    float pr = a_own, su = a_own;  // inclusive
+#pragma unroll 1
+    for (int o = 1; o < kC; o <<= 1) {
+        sp[tid] = pr;
+        ss[tid] = su;
+        __syncthreads();
+        if (tid >= o) pr *= sp[tid - o];
+        if (tid + o < kC) su *= ss[tid + o];
+        __syncthreads();
+    }
+    sp[tid] = pr;
+    ss[tid] = su;
+    __syncthreads();
+    const float p_ex = tid > 0 ? sp[tid - 1] : 1.0f;       // alphas before tid
+    const float q_ex = tid + 1 < kC ? ss[tid + 1] : 1.0f;  // alphas after tid
+    const float wgt = -set[tid] * q_ex;
+    // ---- the scaled rows w Ghat and p A (thread = token row)
+    bool ok = wait_bar(tma_bar, 0, abort_flag, err);
+#pragma unroll 1
+    for (int q = 0; q < 8; ++q) {
+        const uint4 g4 = ld_shared_v4(sb + oG + sw128_off(tid, q));
+        const uint4 a4 = ld_shared_v4(sb + oA + sw128_off(tid, q));
+        const __nv_bfloat162* gh2 = reinterpret_cast<const __nv_bfloat162*>(&g4);
+        const __nv_bfloat162* ah2 = reinterpret_cast<const __nv_bfloat162*>(&a4);
+        uint32_t og[4], oa[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 gf = __bfloat1622float2(gh2[e]);
+            const float2 af = __bfloat1622float2(ah2[e]);
+            og[e] = pack_bf16x2(wgt * gf.x, wgt * gf.y);
+            oa[e] = pack_bf16x2(p_ex * af.x, p_ex * af.y);
+        }
+        st_shared_v4(sb + oWG + sw128_off(tid, q), og[0], og[1], og[2], og[3]);
+        st_shared_v4(sb + oPA + sw128_off(tid, q), oa[0], oa[1], oa[2], oa[3]);
+    }
+    fence_proxy_async_smem();
+    __syncthreads();
+    if (tid == 0 && ok) {
+        tc_fence_after();
+        constexpr uint32_t ID = idesc_bf16(128, 64, true, true);
+        const uint32_t x_lo = sdesc_lo(sb + oX, kTile), b_lo = sdesc_lo(sb + oB, kTile);
+        const uint32_t wg_lo = sdesc_lo(sb + oWG, kTile), pa_lo = sdesc_lo(sb + oPA, kTile);
+#pragma unroll
+        for (int kk = 0; kk < kC / 16; ++kk)  // Vt = X^T (w Ghat) into columns 0..63
+            mma_bf16_ss(tmem, sdesc_from_lo(x_lo + kk * 128), sdesc_from_lo(wg_lo + kk * 128), ID, kk > 0 ? 1u : 0u);
+#pragma unroll
+        for (int kk = 0; kk < kC / 16; ++kk)  // Ut = B^T (p A) into columns 64..127
+            mma_bf16_ss(tmem + 64, sdesc_from_lo(b_lo + kk * 128), sdesc_from_lo(pa_lo + kk * 128), ID,
+                        kk > 0 ? 1u : 0u);
+        mma_commit(mma_bar);
+    }
+    ok = wait_bar(mma_bar, 0, abort_flag, err) && ok;
+    tc_fence_after();
+    if (warp < 2) {  // rows k = 0..63 of both accumulators
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+        const long long blk = (unit * nch + c) * (long long)(64 * 64) + tid * 64;
+#pragma unroll 1
+        for (int hf = 0; hf < 2; ++hf) {
+            float vv[32], uu[32];
+            tmem_ld32(lane_base + 32 * hf, vv);
+            tmem_ld32(lane_base + 64 + 32 * hf, uu);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                reinterpret_cast<float4*>(Vd + blk + 32 * hf)[q] =
+                    make_float4(vv[4 * q], vv[4 * q + 1], vv[4 * q + 2], vv[4 * q + 3]);
+                reinterpret_cast<float4*>(Ud + blk + 32 * hf)[q] =
+                    make_float4(uu[4 * q], uu[4 * q + 1], uu[4 * q + 2], uu[4 * q + 3]);
+            }
+        }
+    } else {
+        // keep the warps' TMEM access shape uniform: nothing to read in lanes 64..127
+    }
+    if (tid == kC - 1) Ad[unit * nch + c] = sp[kC - 1];
+    tc_fence_before();
+    __syncthreads();
+    if (tid == 0 && *abort_flag) {  // no copy in flight at exit (bounded: 0.2 s)
+        const uint64_t t0 = globaltimer_ns();
+        while (!mbar_try_wait(tma_bar, 0) && globaltimer_ns() - t0 < 200000000ull) {
+        }
+    }
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 128);
+    }
+}
+
 }  // namespace ggtc
+
+cudaError_t launch_gate_aggregates_tc(const CUtensorMap& x, const CUtensorMap& g, const CUtensorMap& a,
+                                      const CUtensorMap& b, const float* eta, const float* alpha, float* Vd,
+                                      float* Ud, float* Ad, int L, int B, int T, int H, unsigned int* err,
+                                      cudaStream_t stream) {
+    const int nch = (T + ggtc::kC - 1) / ggtc::kC;
+    const long long blocks = (long long)L * B * H * nch;
+    if (blocks <= 0) return cudaSuccess;
+    if (blocks > 0x7FFFFFFF) return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(ggtc::gate_agg_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         ggtc::kAggSmem);
+    if (e != cudaSuccess) return e;
+    ggtc::gate_agg_tc_kernel<<<(int)blocks, ggtc::kThreads, ggtc::kAggSmem, stream>>>(
+        x, g, a, b, eta, alpha, Vd, Ud, Ad, B, T, H, nch, err);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_gate_chunks_tc(const CUtensorMap& x, const CUtensorMap& g, const CUtensorMap& a,
                                   const CUtensorMap& b, const float* eta, const float* alpha, const float* Sd,

@@ -28,10 +28,12 @@ cudaError_t launch_rowdot(const void* a, const TokStr& as, const void* r, const 
 cudaError_t launch_tc_decay(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
                             const CUtensorMap& o, const TcScanParams& p, bool costate, int grid,
                             cudaStream_t stream);
-cudaError_t launch_flip_rows(const void* in, const TokStr& s, void* out, int L, int B, int T, int T_pad,
-                             int H, int w, int elem, cudaStream_t stream);
-cudaError_t launch_flip_gates(const float* in, float fill, float pad, float* out, int L, int B, int T,
-                              int T_pad, int H, cudaStream_t stream);
+cudaError_t launch_gate_state_scan(float* VS, float* UR, const float* Ad, long long units, int nch,
+                                   cudaStream_t stream);
+cudaError_t launch_gate_aggregates_tc(const CUtensorMap& x, const CUtensorMap& g, const CUtensorMap& a,
+                                      const CUtensorMap& b, const float* eta, const float* alpha, float* Vd,
+                                      float* Ud, float* Ad, int L, int B, int T, int H, unsigned int* err,
+                                      cudaStream_t stream);
 cudaError_t launch_gate_chunks_tc(const CUtensorMap& x, const CUtensorMap& g, const CUtensorMap& a,
                                   const CUtensorMap& b, const float* eta, const float* alpha, const float* Sd,
                                   const float* Rd, float* dlog_alpha, float* deta, int L, int B, int T, int H,
@@ -630,12 +632,11 @@ size_t gated_ws_bytes(const gradlev_desc& d, int sms) {
 
 // The retention scan of 64 x 64 bf16 maps on the tensor cores (scan_decay_tc.cu): one
 // work item per unit, or per segment of a few long units.  q, k, v are the read's
-// orientation (forward: x, x, ghat; costate: g_out, ghat, x); state_out, when given,
-// receives the state at every chunk start.
+// orientation (forward: x, x, ghat; costate: g_out, ghat, x).
 int run_decay_tc(const gradlev_desc& d, bool costate, const Tok& tq, const Tok& tk, const Tok& tv,
                  const Tok& to, const Tok& to2, const Tok& tz, int act, const float* W0,
-                 const float* eta_t, const float* alpha_t, float* state_out, void* ws, size_t ws_bytes,
-                 int sms, cudaStream_t stream) {
+                 const float* eta_t, const float* alpha_t, void* ws, size_t ws_bytes, int sms,
+                 cudaStream_t stream) {
     CUtensorMap mq, mk, mv, mo;
     if (!make_tmap(&mq, d, tq, 64) || !make_tmap(&mk, d, tk, 64) || !make_tmap(&mv, d, tv, 64) ||
         !make_tmap(&mo, d, to, 64))
@@ -690,7 +691,6 @@ int run_decay_tc(const gradlev_desc& d, bool costate, const Tok& tq, const Tok& 
     p.W0 = W0;
     p.g_eta = eta_t;
     p.g_alpha = alpha_t;
-    p.state_out = state_out;
     fill_epi(&p.epi, to, to2, tz, act);
     p.ctrl = static_cast<unsigned int*>(ws);
     if (cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
@@ -764,7 +764,7 @@ int run_gated(const gradlev_desc* desc, bool costate, const gradlev_tensor* x,
         tc_layout_ok(tz, 2)) {
         // 64 x 64 bf16 maps: the chunked retention scan on the tensor cores
         return run_decay_tc(d, costate, costate ? tgo : tx, costate ? tg : tx, costate ? tx : tg, to, to2,
-                            tz, act, W0, eta_t, alpha_t, nullptr, ws, ws_bytes, dev.sms, stream);
+                            tz, act, W0, eta_t, alpha_t, ws, ws_bytes, dev.sms, stream);
     }
     if (cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
     gl::GatedParams p;
@@ -997,20 +997,15 @@ int run_eta_grad(const gradlev_desc* desc, int read, const gradlev_tensor* x,
 // gin = W^T g_out, a = g_out, b = u):
 //   dlog_alpha_j = alpha_j <D_j, R_j>,  deta_j = -ghat_j^T R_j x_j,
 //   R_j = sum_{s>j} prod_{j<r<s} alpha_r a_s b_s^T.
-// D at every chunk start comes from the retention scan over (x, ghat, eta_t, alpha_t);
-// R at every chunk's last token from the same scan over (b, a) reversed in time with
-// every step -1 (its state at a reversed chunk start); gate_chunk_tc_kernel expands
-// both inside each chunk of 128 tokens on the tensor cores (gate_grads_tc.cu).
-size_t gate_grads_ws_bytes(const gradlev_desc& d, int sms) {
-    const long long T_pad = ((long long)d.T + 127) / 128 * 128;
-    gradlev_desc dp = d;
-    dp.T = (int32_t)T_pad;
+// Three launches: per-chunk aggregates of the writes and of the pairs (a, b)
+// (gate_agg_tc_kernel); D at every chunk start and R at every chunk end, carried over
+// the chunks (gate_state_scan_kernel); the expansion inside each chunk of 128
+// tokens (gate_chunk_tc_kernel).
+size_t gate_grads_ws_bytes(const gradlev_desc& d, int /*sms*/) {
     const size_t units = (size_t)d.L * d.B * d.H;
-    const size_t tokens_pad = units * (size_t)T_pad;
-    const size_t g1 = gated_ws_bytes(d, sms), g2 = gated_ws_bytes(dp, sms);
-    return round_up(g1 > g2 ? g1 : g2, 256) + round_up((size_t)d.L * d.H * 64 * 64 * sizeof(float), 256) +
-           2 * round_up(units * (size_t)(T_pad / 128) * 64 * 64 * sizeof(float), 256) +
-           3 * round_up(tokens_pad * 64 * 2, 256) + 2 * round_up(tokens_pad * sizeof(float), 256);
+    const size_t nch = ((size_t)d.T + 127) / 128;
+    return 256 + 2 * round_up(units * nch * 64 * 64 * sizeof(float), 256) +
+           round_up(units * nch * sizeof(float), 256);
 }
 
 int run_gate_grads(const gradlev_desc* desc, int read, const gradlev_tensor* x,
@@ -1034,74 +1029,29 @@ int run_gate_grads(const gradlev_desc* desc, int read, const gradlev_tensor* x,
         !resolve(d, upstream, 64, &tu, true) || !resolve(d, g_out, 64, &tgo, read == 1))
         return GRADLEV_ERR_INVALID_ARG;
     if (d.T == 0) return GRADLEV_OK;
-    // 16-byte pieces of every token row (reversed copies, TMA tiles, the chunk kernel)
     const Tok* rows[4] = {&tx, &tg, &tu, &tgo};
     for (const Tok* t : rows)
         if (t->data && !tc_layout_ok(*t, 2)) return GRADLEV_ERR_UNSUPPORTED;
-    const int T_pad = (d.T + 127) / 128 * 128;
-    gradlev_desc dp = d;
-    dp.T = T_pad;
-    const size_t units = (size_t)d.L * d.B * d.H;
-    const size_t tokens_pad = units * (size_t)T_pad;
-    const size_t g1 = gated_ws_bytes(d, dev.sms), g2 = gated_ws_bytes(dp, dev.sms);
-    const size_t gws = round_up(g1 > g2 ? g1 : g2, 256);
-    uint8_t* p = static_cast<uint8_t*>(ws) + gws;
-    auto take = [&](size_t bytes) {
-        uint8_t* q = p;
-        p += round_up(bytes, 256);
-        return q;
-    };
-    const size_t w0_bytes = (size_t)d.L * d.H * 64 * 64 * sizeof(float);
-    const size_t st_bytes = units * (size_t)(T_pad / 128) * 64 * 64 * sizeof(float);
-    float* zero_w0 = reinterpret_cast<float*>(take(w0_bytes));
-    float* Sd = reinterpret_cast<float*>(take(st_bytes));
-    float* Rd = reinterpret_cast<float*>(take(st_bytes));
-    uint8_t* rb = take(tokens_pad * 64 * 2);   // b reversed
-    uint8_t* ra = take(tokens_pad * 64 * 2);   // a reversed
-    uint8_t* junk = take(tokens_pad * 64 * 2);  // the scans' unused outputs
-    float* eta_rev = reinterpret_cast<float*>(take(tokens_pad * sizeof(float)));
-    float* alpha_rev = reinterpret_cast<float*>(take(tokens_pad * sizeof(float)));
     const Tok& ta = read == 0 ? tu : tgo;
     const Tok& tb = read == 0 ? tx : tu;
-    auto strides = [](const Tok& t) {
-        gl::TokStr st;
-        for (int i = 0; i < 4; ++i) st.s[i] = t.s[i];
-        return st;
-    };
-    auto contiguous = [&](void* data, const gradlev_desc& dd) {
-        gradlev_tensor g;
-        g.data = data;
-        for (int i = 0; i < 4; ++i) g.stride[i] = 0;
-        Tok t;
-        resolve(dd, &g, 64, &t, true);
-        return t;
-    };
-    if (cudaMemsetAsync(zero_w0, 0, w0_bytes, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
-    if (T_pad != d.T && (cudaMemsetAsync(rb, 0, tokens_pad * 64 * 2, stream) != cudaSuccess ||
-                         cudaMemsetAsync(ra, 0, tokens_pad * 64 * 2, stream) != cudaSuccess))
-        return GRADLEV_ERR_CUDA;
-    if (gl::launch_flip_rows(tb.data, strides(tb), rb, d.L, d.B, d.T, T_pad, d.H, 64, 2, stream) != cudaSuccess ||
-        gl::launch_flip_rows(ta.data, strides(ta), ra, d.L, d.B, d.T, T_pad, d.H, 64, 2, stream) != cudaSuccess ||
-        gl::launch_flip_gates(nullptr, -1.0f, 0.0f, eta_rev, d.L, d.B, d.T, T_pad, d.H, stream) != cudaSuccess ||
-        gl::launch_flip_gates(alpha_t, 1.0f, 1.0f, alpha_rev, d.L, d.B, d.T, T_pad, d.H, stream) != cudaSuccess)
-        return GRADLEV_ERR_CUDA;
-    const Tok none;
-    // D at every chunk start: the forward-orientation scan of the writes
-    const Tok tj = contiguous(junk, d);
-    int rc = run_decay_tc(d, false, tx, tx, tg, tj, none, none, GRADLEV_ACT_NONE, zero_w0, eta_t, alpha_t, Sd,
-                          ws, gws, dev.sms, stream);
-    if (rc != GRADLEV_OK) return rc;
-    // R at every chunk's last token: the same scan over (b, a) reversed, steps -1
-    const Tok trb = contiguous(rb, dp), tra = contiguous(ra, dp), tjp = contiguous(junk, dp);
-    rc = run_decay_tc(dp, false, trb, trb, tra, tjp, none, none, GRADLEV_ACT_NONE, zero_w0, eta_rev, alpha_rev,
-                      Rd, ws, gws, dev.sms, stream);
-    if (rc != GRADLEV_OK) return rc;
     CUtensorMap mx, mg, ma, mb;
     if (!make_tmap(&mx, d, tx, 64) || !make_tmap(&mg, d, tg, 64) || !make_tmap(&ma, d, ta, 64) ||
         !make_tmap(&mb, d, tb, 64))
         return GRADLEV_ERR_UNSUPPORTED;
-    if (gl::launch_gate_chunks_tc(mx, mg, ma, mb, eta_t, alpha_t, Sd, Rd, dlog_alpha, deta, d.L, d.B, d.T, d.H,
-                                  static_cast<unsigned int*>(ws) + 1, stream) != cudaSuccess)
+    const size_t units = (size_t)d.L * d.B * d.H;
+    const int nch = (d.T + 127) / 128;
+    const size_t st_bytes = units * (size_t)nch * 64 * 64 * sizeof(float);
+    uint8_t* base = static_cast<uint8_t*>(ws);
+    unsigned int* ctrl = reinterpret_cast<unsigned int*>(base);
+    float* VS = reinterpret_cast<float*>(base + 256);
+    float* UR = reinterpret_cast<float*>(base + 256 + round_up(st_bytes, 256));
+    float* Ad = reinterpret_cast<float*>(base + 256 + 2 * round_up(st_bytes, 256));
+    if (cudaMemsetAsync(ws, 0, 256, stream) != cudaSuccess) return GRADLEV_ERR_CUDA;
+    if (gl::launch_gate_aggregates_tc(mx, mg, ma, mb, eta_t, alpha_t, VS, UR, Ad, d.L, d.B, d.T, d.H, ctrl + 1,
+                                      stream) != cudaSuccess ||
+        gl::launch_gate_state_scan(VS, UR, Ad, (long long)units, nch, stream) != cudaSuccess ||
+        gl::launch_gate_chunks_tc(mx, mg, ma, mb, eta_t, alpha_t, VS, UR, dlog_alpha, deta, d.L, d.B, d.T, d.H,
+                                  ctrl + 1, stream) != cudaSuccess)
         return GRADLEV_ERR_CUDA;
     return GRADLEV_OK;
 }

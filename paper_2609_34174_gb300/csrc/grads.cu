@@ -7,9 +7,9 @@
 // gin_t = W_t^T g_t the same holds with dL/deta_s = -x_s . r_s and
 // r_s = sum_{t>s} (g_t . ghat_s) dL/dgin_t.  The suffix read runs in the scan
 // kernels (reverse mode); this file holds the final row dot.  With retention alpha_t
-// the gate derivatives take the state of the retention scan at every chunk start,
-// forwards and over the inputs reversed in time; the reversed copies are here, the
-// per-chunk expansion in gate_grads_tc.cu.
+// the gate derivatives take the states at every chunk boundary, carried here from
+// per-chunk aggregates; the aggregates and the per-chunk expansion are in
+// gate_grads_tc.cu.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -103,72 +103,53 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 // ---------------------------------------------------------------------------
-// Gate derivatives with retention (alpha_t).  The decayed suffix state is the state
-// of the forward retention scan over the inputs reversed in time; its inputs are
-// copied reversed, after T_pad - T zero rows, so that the reversed chunks of 128
-// tokens are the original chunks in reverse order.
-
-// out[l][b][T_pad-1-t][h][:] = in[l][b][t][h][:], in with element strides s, out
-// contiguous with T_pad tokens; one thread per 16-byte piece.
+// Gate derivatives with retention (alpha_t): the states at every chunk boundary from
+// the per-chunk aggregates, in place (fp32 [unit][nch][64][64], one thread per entry
+// and unit):
+//   VS[c] <- D at chunk c's first token:  D_0 = 0,  D_{c+1} = A_c D_c + Vt_c
+//   UR[c] <- R at chunk c's last token:   R_{nch-1} = 0,  R_c = Ut_{c+1} + A_{c+1} R_{c+1}
+// (the chunk map of Eq. 2, S -> a S + U, carried forwards and, for the decayed suffix
+// state, backwards).
 __global__ void __launch_bounds__(kThreads)
-    flip_rows_kernel(const void* __restrict__ in, TokStr s, void* __restrict__ out, int L, int B,
-                     int T, int T_pad, int H, int pieces, int elem) {
-    const long long n = (long long)L * B * T * H * pieces;
-    for (long long v = (long long)blockIdx.x * kThreads + threadIdx.x; v < n;
-         v += (long long)gridDim.x * kThreads) {
-        const int pc = (int)(v % pieces);
-        long long r = v / pieces;
-        const int h = (int)(r % H);
-        r /= H;
-        const int t = (int)(r % T);
-        r /= T;
-        const int b = (int)(r % B);
-        const int l = (int)(r / B);
-        const long long src = tok_off(s.s, l, b, t, h) * elem + (long long)pc * 16;
-        const long long dst = ((((long long)l * B + b) * T_pad + (T_pad - 1 - t)) * H + h) * pieces * 16 +
-                              (long long)pc * 16;
-        *reinterpret_cast<uint4*>(static_cast<char*>(out) + dst) =
-            *reinterpret_cast<const uint4*>(static_cast<const char*>(in) + src);
+    gate_state_scan_kernel(float* __restrict__ VS, float* __restrict__ UR, const float* __restrict__ Ad,
+                           long long units, int nch) {
+    // one thread: 4 consecutive entries (a float4) of one unit; the next chunk's
+    // values are loaded before the current ones are used
+    const long long e4 = (long long)blockIdx.x * kThreads + threadIdx.x;
+    if (e4 >= units * 1024) return;
+    const long long unit = e4 >> 10;
+    float4* V = reinterpret_cast<float4*>(VS) + unit * nch * 1024ll + (e4 & 1023);
+    float4* U = reinterpret_cast<float4*>(UR) + unit * nch * 1024ll + (e4 & 1023);
+    const float* a = Ad + unit * nch;
+    float4 S = make_float4(0.f, 0.f, 0.f, 0.f);
+    float4 nxt = V[0];
+    for (int c = 0; c < nch; ++c) {
+        const float4 cur = nxt;
+        if (c + 1 < nch) nxt = V[(long long)(c + 1) * 1024];
+        V[(long long)c * 1024] = S;
+        const float ac = a[c];
+        S = make_float4(fmaf(ac, S.x, cur.x), fmaf(ac, S.y, cur.y), fmaf(ac, S.z, cur.z), fmaf(ac, S.w, cur.w));
     }
-}
-
-// Per-token gates [L][B][T][H] reversed into [L][B][T_pad][H]: the T_pad - T leading
-// entries are pad, the others in (or fill where in == nullptr).
-__global__ void __launch_bounds__(kThreads)
-    flip_gates_kernel(const float* __restrict__ in, float fill, float pad, float* __restrict__ out,
-                      int LB, int T, int T_pad, int H) {
-    const long long n = (long long)LB * T_pad * H;
-    for (long long v = (long long)blockIdx.x * kThreads + threadIdx.x; v < n;
-         v += (long long)gridDim.x * kThreads) {
-        const int h = (int)(v % H);
-        const long long r = v / H;
-        const int tau = (int)(r % T_pad);
-        const long long lb = r / T_pad;
-        const int t = T_pad - 1 - tau;
-        out[v] = t >= T ? pad : (in ? in[(lb * T + t) * H + h] : fill);
+    float4 R = make_float4(0.f, 0.f, 0.f, 0.f);
+    nxt = U[(long long)(nch - 1) * 1024];
+    for (int c = nch - 1; c >= 0; --c) {
+        const float4 cur = nxt;
+        if (c > 0) nxt = U[(long long)(c - 1) * 1024];
+        U[(long long)c * 1024] = R;
+        const float ac = a[c];
+        R = make_float4(fmaf(ac, R.x, cur.x), fmaf(ac, R.y, cur.y), fmaf(ac, R.z, cur.z), fmaf(ac, R.w, cur.w));
     }
 }
 
 }  // namespace grads
 
-cudaError_t launch_flip_rows(const void* in, const TokStr& s, void* out, int L, int B, int T, int T_pad,
-                             int H, int w, int elem, cudaStream_t stream) {
-    const int pieces = w * elem / 16;
-    const long long n = (long long)L * B * T * H * pieces;
-    if (n <= 0) return cudaSuccess;
+cudaError_t launch_gate_state_scan(float* VS, float* UR, const float* Ad, long long units, int nch,
+                                   cudaStream_t stream) {
+    const long long n = units * 1024;  // float4 entries
+    if (n <= 0 || nch <= 0) return cudaSuccess;
     const long long grid = (n + grads::kThreads - 1) / grads::kThreads;
-    grads::flip_rows_kernel<<<(int)(grid < 152 * 16 ? grid : 152 * 16), grads::kThreads, 0, stream>>>(
-        in, s, out, L, B, T, T_pad, H, pieces, elem);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_flip_gates(const float* in, float fill, float pad, float* out, int L, int B, int T,
-                              int T_pad, int H, cudaStream_t stream) {
-    const long long n = (long long)L * B * T_pad * H;
-    if (n <= 0) return cudaSuccess;
-    const long long grid = (n + grads::kThreads - 1) / grads::kThreads;
-    grads::flip_gates_kernel<<<(int)(grid < 152 * 16 ? grid : 152 * 16), grads::kThreads, 0, stream>>>(
-        in, fill, pad, out, L * B, T, T_pad, H);
+    if (grid > 0x7FFFFFFF) return cudaErrorInvalidValue;
+    grads::gate_state_scan_kernel<<<(int)grid, grads::kThreads, 0, stream>>>(VS, UR, Ad, units, nch);
     return cudaGetLastError();
 }
 

@@ -108,9 +108,6 @@ struct TcScanParams {
     const float* g_eta;
     const float* g_alpha;  // null: alpha = 1
     float* seg_a;
-    // optional: the state at every chunk start, fp32 [unit][ceil(T / 128)][64][64]
-    // (row q of S^T, as the state warps hold it)
-    float* state_out;
 };
 
 // Parameters of the wide-layer passes (bf16, dq % 128 == 0, dv % 64 == 0): the

@@ -962,14 +962,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             for (int c = 0; c < I.nch; ++c, ++c2) {
                 const uint32_t sb = c2 & 1, ph = (c2 >> 1) & 1;
-                if (p.state_out) {  // the state at this chunk's first token
-                    const long long chunk = I.t_begin / kChunk + c;
-                    float* dst = p.state_out +
-                                 (((long long)(item % p.n_ut) * ((p.T + kChunk - 1) / kChunk) + chunk) * 64 + row) * 64;
-#pragma unroll
-                    for (int i = 0; i < 64; i += 4)
-                        *reinterpret_cast<float4*>(dst + i) = make_float4(st[i], st[i + 1], st[i + 2], st[i + 3]);
-                }
                 if (!warp_wait(&st_free[sb], ph ^ 1, abort_flag)) {
                     raise_error(p, kErrWaitTimeout, abort_flag);
                     ok = false;
