@@ -68,14 +68,15 @@ def _run(L, B, T, H, read, seed, resets=True, with_alpha=True):
 
 
 CASES = {
-    # (L, B, T, H): one token, below / at / past one chunk, several units, a long
-    # sequence whose scans are cut into segments
+    # (L, B, T, H): one token, below / at / past one chunk of 128, several units, a
+    # long sequence whose chunk states are carried over 24 chunks (resets on and next
+    # to chunk boundaries, a negative alpha)
     "T1": (1, 1, 1, 2),
     "T100": (1, 2, 100, 2),
     "T128": (1, 1, 128, 3),
     "T129": (2, 1, 129, 2),
     "T700": (1, 2, 700, 2),
-    "T3000-segmented": (1, 1, 3000, 2),
+    "T3000": (1, 1, 3000, 2),
 }
 
 
@@ -132,23 +133,29 @@ def test_gate_grads_full_size_c4_every_unit():
     assert_parity("c4 deta", lbthw_units(de.cpu()), re, "bf16")
 
 
-def test_gate_grads_full_size_c5_sampled_units():
-    """The layer-sweep workload at full size (1152 units of 8192 tokens), costate read;
-    three units checked against the oracle."""
+def test_gate_grads_full_size_c5_every_unit():
+    """The layer-sweep workload at full size (1152 units of 8192 tokens), costate read,
+    in the configuration the bench times: every unit and token against the oracle,
+    one layer at a time."""
     import bench
     wl = W.workload("c5")
-    inp = W.make_linear(wl, device="cuda")
-    g = bench.make_gates(wl, "alpha", "cuda")
-    u = _bench_upstream(wl, 92).cuda()
-    dla, de = gl.gate_grads(inp["x"], inp["g_hat"], g["eta_t"], u, alpha=g["alpha_t"], read="costate",
-                            g_out=inp["g_out"])
+    inp = W.make_linear(wl)
+    g = bench.make_gates(wl, "alpha", "cpu")
+    u = _rand((wl.L, wl.B, wl.T, wl.H, wl.d_in), 92)
+    dla, de = gl.gate_grads(inp["x"].cuda(), inp["g_hat"].cuda(), g["eta_t"].cuda(), u.cuda(),
+                            alpha=g["alpha_t"].cuda(), read="costate", g_out=inp["g_out"].cuda())
     torch.cuda.synchronize()
-    for (l, b, h) in [(0, 0, 0), (5, 3, 7), (11, 7, 11)]:
-        sl = lambda t: t[l:l + 1, b:b + 1, :, h:h + 1].cpu()
+    dla, de = dla.cpu(), de.cpu()
+    from parity_util import Parity
+    pa, pe = Parity("c5 dlog_alpha", "bf16"), Parity("c5 deta", "bf16")
+    for l in range(wl.L):
+        sl = lambda t: t[l:l + 1]
         ra, re = _oracle(sl(inp["x"]), sl(inp["g_hat"]), sl(inp["g_out"]), sl(u), sl(g["eta_t"]),
                          sl(g["alpha_t"]), "costate")
-        assert_parity(f"c5 unit {(l, b, h)} dlog_alpha", lbthw_units(sl(dla)), ra, "bf16")
-        assert_parity(f"c5 unit {(l, b, h)} deta", lbthw_units(sl(de)), re, "bf16")
+        pa.add(lbthw_units(sl(dla)), ra)
+        pe.add(lbthw_units(sl(de)), re)
+    pa.check()
+    pe.check()
 
 
 def test_gate_grads_rejects_other_shapes():
