@@ -212,8 +212,10 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int i = tid;
         NT[nidx(kC - 1, i)] = __float2bfloat16_rn(0.0f);  // N_{i,127}: no later token
         float nrun = 0.0f;
+        // blocks of 32 columns s; none after a row of this warp below blk = warp
+        // (warp-uniform, so the TMEM loads stay collective)
 #pragma unroll 1
-        for (int blk = 3; blk >= 0; --blk) {
+        for (int blk = 3; blk >= warp; --blk) {
             float g1[32], g2[32];
             tmem_ld32(lane_base + 32 * blk, g1);
             tmem_ld32(lane_base + 128 + 32 * blk, g2);

@@ -110,42 +110,49 @@ __global__ void __launch_bounds__(kThreads)
 //   UR[c] <- R at chunk c's last token:   R_{nch-1} = 0,  R_c = Ut_{c+1} + A_{c+1} R_{c+1}
 // (the chunk map of Eq. 2, S -> a S + U, carried forwards and, for the decayed suffix
 // state, backwards).
+// One thread: two float4s of one unit (entries 4e..4e+3 and 4e+2048..4e+2051), with
+// loads two chunks ahead: four 16-byte loads in flight per thread.
 __global__ void __launch_bounds__(kThreads)
     gate_state_scan_kernel(float* __restrict__ VS, float* __restrict__ UR, const float* __restrict__ Ad,
                            long long units, int nch) {
-    // one thread: 4 consecutive entries (a float4) of one unit; the next chunk's
-    // values are loaded before the current ones are used
-    const long long e4 = (long long)blockIdx.x * kThreads + threadIdx.x;
-    if (e4 >= units * 1024) return;
-    const long long unit = e4 >> 10;
-    float4* V = reinterpret_cast<float4*>(VS) + unit * nch * 1024ll + (e4 & 1023);
-    float4* U = reinterpret_cast<float4*>(UR) + unit * nch * 1024ll + (e4 & 1023);
+    const long long e = (long long)blockIdx.x * kThreads + threadIdx.x;  // one of 512 per unit
+    if (e >= units * 512) return;
+    const long long unit = e >> 9;
+    const long long off = unit * nch * 1024ll + (e & 511);
     const float* a = Ad + unit * nch;
-    float4 S = make_float4(0.f, 0.f, 0.f, 0.f);
-    float4 nxt = V[0];
-    for (int c = 0; c < nch; ++c) {
-        const float4 cur = nxt;
-        if (c + 1 < nch) nxt = V[(long long)(c + 1) * 1024];
-        V[(long long)c * 1024] = S;
-        const float ac = a[c];
-        S = make_float4(fmaf(ac, S.x, cur.x), fmaf(ac, S.y, cur.y), fmaf(ac, S.z, cur.z), fmaf(ac, S.w, cur.w));
-    }
-    float4 R = make_float4(0.f, 0.f, 0.f, 0.f);
-    nxt = U[(long long)(nch - 1) * 1024];
-    for (int c = nch - 1; c >= 0; --c) {
-        const float4 cur = nxt;
-        if (c > 0) nxt = U[(long long)(c - 1) * 1024];
-        U[(long long)c * 1024] = R;
-        const float ac = a[c];
-        R = make_float4(fmaf(ac, R.x, cur.x), fmaf(ac, R.y, cur.y), fmaf(ac, R.z, cur.z), fmaf(ac, R.w, cur.w));
-    }
+    auto carry = [&](float4* P, bool forward) {
+        float4 s0 = make_float4(0.f, 0.f, 0.f, 0.f), s1 = s0;
+        auto at = [&](int c) { return (long long)(forward ? c : nch - 1 - c) * 1024; };
+        float4 n0 = P[at(0)], n1 = P[at(0) + 512];
+        float4 m0 = s0, m1 = s0;
+        if (nch > 1) {
+            m0 = P[at(1)];
+            m1 = P[at(1) + 512];
+        }
+        for (int c = 0; c < nch; ++c) {
+            const float4 c0 = n0, c1 = n1;
+            n0 = m0;
+            n1 = m1;
+            if (c + 2 < nch) {
+                m0 = P[at(c + 2)];
+                m1 = P[at(c + 2) + 512];
+            }
+            P[at(c)] = s0;
+            P[at(c) + 512] = s1;
+            const float ac = a[forward ? c : nch - 1 - c];
+            s0 = make_float4(fmaf(ac, s0.x, c0.x), fmaf(ac, s0.y, c0.y), fmaf(ac, s0.z, c0.z), fmaf(ac, s0.w, c0.w));
+            s1 = make_float4(fmaf(ac, s1.x, c1.x), fmaf(ac, s1.y, c1.y), fmaf(ac, s1.z, c1.z), fmaf(ac, s1.w, c1.w));
+        }
+    };
+    carry(reinterpret_cast<float4*>(VS) + off, true);
+    carry(reinterpret_cast<float4*>(UR) + off, false);
 }
 
 }  // namespace grads
 
 cudaError_t launch_gate_state_scan(float* VS, float* UR, const float* Ad, long long units, int nch,
                                    cudaStream_t stream) {
-    const long long n = units * 1024;  // float4 entries
+    const long long n = units * 512;  // pairs of float4 entries
     if (n <= 0 || nch <= 0) return cudaSuccess;
     const long long grid = (n + grads::kThreads - 1) / grads::kThreads;
     if (grid > 0x7FFFFFFF) return cudaErrorInvalidValue;
