@@ -26,7 +26,7 @@
 // All three terms of o land in one TMEM accumulator:
 //   O  = Q B0^T                 (B0^T tile in shared memory, per unit)
 //   O += P' V                   P'_ts = -E_ts (q_t . k_s), built over the score
-//   O += Q' S^T                 Q' = diag(a) Q, written by the P warps into the
+//   O += Q' S^T                 Q' = diag(a) Q, written by the epilogue warps into the
 //                               free columns of the score buffer (TS product)
 // and the state update is dZ = K^T (W V), with the rows of V scaled by -w_s into a
 // shared-memory tile, then S' = a_end S + dZ in the state warps (fp32 rows).
@@ -40,10 +40,11 @@
 //   warp 14     back MMA issuer: Q B0^T, then (P' ready) P' V, then (S ready) Q' S^T
 //   warp 15     gate factors of each chunk from alpha_t and eta_t, in registers and
 //               shuffles, into a ring of three blocks one or two chunks ahead
-//   warps 2-5   P' over score columns 0..63 and Q' (rows 0..63 also zero 64..127)
+//   warps 2-5   P' over score columns 0..63 (rows 0..63 also zero 64..127)
 //   warps 10-11 P' over columns 64..127 of rows 64..127
 //   (warps 2-3 and 10-11 then write the chunk's W V rows, 0..63 and 64..127)
-//   warps 6-9   epilogue (TMEM -> bf16 staging -> TMA store), as in scan_tc.cu
+//   warps 6-9   Q' of the next chunk into the score columns the P warps have read,
+//               then the epilogue (TMEM -> bf16 staging -> TMA store) as in scan_tc.cu
 //   warps 12-13 state rows, B0^T and S^T tiles, S' = a_end S + dZ
 // One work item is one unit (the chunks of a unit run in order in one CTA).
 #include <cuda.h>
@@ -303,6 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     volatile int* abort_flag = misc + 0;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(misc + 1);
     volatile int* item_slot = misc + 4;    // [kRing]
+    uint64_t* sr_done = bars + 61;         // [2] P warps done reading score columns 0..63
     float* gfb = reinterpret_cast<float*>(smem + Lay::kGfOff);  // [kGbRing][kGbFloats]
 
     const int warp = threadIdx.x >> 5;
@@ -316,7 +318,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(&sc_full[i], 1);
             mbar_init(&sc_free[i], 1);
-            mbar_init(&p_ready[i], 6);   // warps 2-5 and the two helpers
+            mbar_init(&p_ready[i], 10);  // warps 2-5, the two helpers, the four epilogue warps (Q')
+            mbar_init(&sr_done[i], 4);   // warps 2-5
             mbar_init(&o_staged[i], 4);
             mbar_init(&o_full[i], 1);
             mbar_init(&o_free[i], 4);
@@ -331,7 +334,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < kGbRing; ++i) {
             mbar_init(&gf_full[i], 1);
-            mbar_init(&gf_free[i], 4 + 2 + 2);  // warps 2-5, the helpers, the state warps
+            // warps 2-5, the helpers, the state warps and (outputs only) the epilogue
+            mbar_init(&gf_free[i], AGG ? 4 + 2 + 2 : 4 + 2 + 2 + 4);
         }
         mbar_init(wv_ready, 4);  // warps 2-3 and the two helpers
         mbar_init(wv_free, 1);
@@ -642,9 +646,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
     } else if (warp < kWarpO0 || warp == kWarpZ0 || warp == kWarpZ0 + 1) {
-        // ------------------------------------------------ P', Q' and the W V rows
+        // ---------------------------------------------------- P' and the W V rows
         // Warps 2-5 own token rows row = 32 (warp & 3) + lane of each chunk: P' over
-        // columns 0..63 (rows < 64 also zero columns 64..127) and Q' = a_t q_t.  The
+        // columns 0..63 (rows < 64 also zero columns 64..127); the epilogue warps then
+        // write Q' = a_t q_t into columns 32..63.  The
         // two helpers build P' over columns 64..127 of rows 64..127.  Then warps 2-3
         // (whose P' has no masked column) and the helpers write the chunk's W V rows
         // -w_t v_t (rows 0..63 and 64..127), which the front issuer's state update
@@ -686,21 +691,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                         build_p64<0, false>(base, gb, row, pim_t);
                         tmem_zero32_async(base + 64);  // tokens >= 64 all masked
                     }
-                    // ---- Q' = a_t q_t into columns 32..63 (read after the score above)
-                    const float a_t = gb[kGbA + row];
-                    const uint32_t qt = st + Lay::kQOff;
-#pragma unroll 1
-                    for (int q = 0; q < 8; ++q) {
-                        const uint4 a = ld_shared_v4(qt + sw128_off(row, q));
-                        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&a);
-                        uint32_t o[4];
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            const float2 f = __bfloat1622float2(h[i]);
-                            o[i] = pack_bf16x2(a_t * f.x, a_t * f.y);
-                        }
-                        tmem_st4_async(base + kQpCol + 4 * q, o[0], o[1], o[2], o[3]);
-                    }
+                    // the score columns 0..63 are read: the epilogue warps of the same
+                    // lanes may write Q' into columns 32..63
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&sr_done[sb]);
                 } else {
                     // ---- P'_ts for s >= 64 (rows 64..127)
                     build_p64<8, false>(base + 64, gb, row, pim_t);
@@ -756,12 +751,55 @@ __global__ void __launch_bounds__(kThreads, 1)
         const EpiParams& e = p.epi;
         uint32_t c2 = 0;
         bool ok = true;
+        // Q' = a_t q_t of the chunk with CTA chunk counter cc into columns 32..63 of its
+        // score buffer, once the P warps of these lanes have read them
+        auto write_qp = [&](uint32_t cc) -> bool {
+            const uint32_t qb = cc & 1, gk = cc % kGbRing;
+            const int s = static_cast<int>(cc % NS);
+            if (!warp_wait(&gf_full[gk], (cc / kGbRing) & 1, abort_flag) ||
+                !warp_wait(&full[s], (cc / NS) & 1, abort_flag) ||
+                !warp_wait(&sr_done[qb], (cc >> 1) & 1, abort_flag))
+                return false;
+            tc_fence_after();
+            const float a_t = gfb[gk * kGbFloats + kGbA + row];
+            const uint32_t qt = sbase + s * Lay::kStageBytes + Lay::kQOff;
+            const uint32_t dst = tmem + col_sc(qb) + lane_off + kQpCol;
+#pragma unroll 1
+            for (int q = 0; q < 8; ++q) {
+                const uint4 a = ld_shared_v4(qt + sw128_off(row, q));
+                const __nv_bfloat162* hq = reinterpret_cast<const __nv_bfloat162*>(&a);
+                uint32_t o[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const float2 f = __bfloat1622float2(hq[i]);
+                    o[i] = pack_bf16x2(a_t * f.x, a_t * f.y);
+                }
+                tmem_st4_async(dst + 4 * q, o[0], o[1], o[2], o[3]);
+            }
+            tmem_wait_st();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(&p_ready[qb]);
+                mbar_arrive(&gf_free[gk]);
+            }
+            return true;
+        };
         for (int it = 0; ok; ++it) {
             int item;
             if (!take_item(it, item) || item < 0) break;
             if (AGG) continue;  // no outputs in the aggregate pass
             const Item I = decode_unit(item, p);
+            if (!write_qp(c2)) {  // the item's first chunk
+                raise_error(p, kErrWaitTimeout, abort_flag);
+                break;
+            }
             for (int c = 0; c < I.nch; ++c, ++c2) {
+                if (c + 1 < I.nch && !write_qp(c2 + 1)) {  // the next chunk's Q' before this output
+                    raise_error(p, kErrWaitTimeout, abort_flag);
+                    ok = false;
+                    break;
+                }
                 const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
                 if (!warp_wait(&o_full[ob], oph, abort_flag)) {
                     raise_error(p, kErrWaitTimeout, abort_flag);
