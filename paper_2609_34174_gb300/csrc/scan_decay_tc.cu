@@ -37,7 +37,7 @@
 //   warp 1      front MMA issuer: the score Q K^T of chunk c, then the state update
 //               dZ of chunk c - 1 (one chunk behind, so that the score never waits
 //               for the W V tile)
-//   warp 14     back MMA issuer: Q B0^T, then (P' ready) P' V, then (S ready) Q' S^T
+//   warp 14     back MMA issuer: Q B0^T, then (S^T and P' ready) P' V and Q' S^T
 //   warp 15     gate factors of each chunk from alpha_t and eta_t, in registers and
 //               shuffles, into a ring of three blocks one or two chunks ahead
 //   warps 2-5   P' over score columns 0..63 (rows 0..63 also zero 64..127)
@@ -122,8 +122,12 @@ __device__ __forceinline__ Item decode_unit(int item, const TcScanParams& p) {
     return I;
 }
 
-__device__ __forceinline__ void raise_error(const TcScanParams& p, unsigned int bits,
-                                            volatile int* abort_flag) {
+// Out of line, like the slow half of every wait: sixteen warps run different role
+// loops, instruction fetch is the first stall, and cold code inside a hot loop spreads
+// it over more cache lines.  For the same reason the MMA issuers keep their K steps as
+// rolled loops.
+__device__ __noinline__ void raise_error(const TcScanParams& p, unsigned int bits,
+                                         volatile int* abort_flag) {
     atomicOr(p.ctrl + 1, bits);
     if (abort_flag) *abort_flag = 1;
 }
@@ -157,7 +161,7 @@ __device__ __noinline__ bool wait_slow(uint64_t* bar, uint32_t parity, volatile 
     return mbar_wait(bar, parity, abort_flag);
 }
 __device__ __forceinline__ bool bwait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
-    return test_probe(bar, parity) || wait_slow(bar, parity, abort_flag);
+    return __builtin_expect(test_probe(bar, parity), 1) || wait_slow(bar, parity, abort_flag);
 }
 
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
@@ -227,16 +231,15 @@ __device__ __forceinline__ void tmem_st4_async(uint32_t taddr, uint32_t a, uint3
 // lane's row: the fp32 scores at TMEM columns taddr .. taddr+63 become 32 packed bf16
 // columns at taddr (stores issued, not waited).  Two pieces per step, in increasing
 // order, so that no packed store reaches a score column still to be read.
-// ALL_BEFORE: every one of these pieces precedes t's own piece.
-template <int PB, bool ALL_BEFORE>
-__device__ __forceinline__ void build_p64(uint32_t taddr, const float* gb, int row, float pim) {
+// One copy of the code serves every P warp (pb = 0 or 8).
+__device__ __forceinline__ void build_p64(uint32_t taddr, const float* gb, int row, float pim, int pb) {
     const int jt = row >> 3;
     const int jmax = (row | 31) >> 3;  // the last piece of this warp's rows
     float ndd[8];
-    if (!ALL_BEFORE) same_piece_decays(gb, row, ndd);
+    same_piece_decays(gb, row, ndd);
 #pragma unroll 1
     for (int m = 0; m < 4; ++m) {
-        if (!ALL_BEFORE && PB + 2 * m > jmax) {  // after every row of the warp: masked
+        if (pb + 2 * m > jmax) {  // after every row of the warp: masked
             const uint32_t z[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
             tmem_st8_async(taddr + 8 * m, z);
             continue;
@@ -246,17 +249,15 @@ __device__ __forceinline__ void build_p64(uint32_t taddr, const float* gb, int r
         uint32_t w[8];
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-            const int j = PB + 2 * m + h;
+            const int j = pb + 2 * m + h;
             const float tau = pim * gb[kGbTpm + 16 * j + jt];  // 0 unless j < jt
             const float4 s0 = lds4(gb + kGbNse + 8 * j);
             const float4 s1 = lds4(gb + kGbNse + 8 * j + 4);
             float e[8] = {s0.x * tau, s0.y * tau, s0.z * tau, s0.w * tau,
                           s1.x * tau, s1.y * tau, s1.z * tau, s1.w * tau};
-            if (!ALL_BEFORE) {
-                const bool same = j == jt;
+            const bool same = j == jt;
 #pragma unroll
-                for (int i = 0; i < 8; ++i) e[i] = same ? ndd[i] : e[i];
-            }
+            for (int i = 0; i < 8; ++i) e[i] = same ? ndd[i] : e[i];
 #pragma unroll
             for (int i = 0; i < 4; ++i)
                 w[4 * h + i] = pack_bf16x2(e[2 * i] * v[8 * h + 2 * i], e[2 * i + 1] * v[8 * h + 2 * i + 1]);
@@ -426,7 +427,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t n = 0, c2 = 0, dzc = 0;
             bool ok = true;
             auto wait_or_fail = [&](uint64_t* bar, uint32_t par) -> bool {
-                if (bwait(bar, par, abort_flag)) return true;
+                if (__builtin_expect(bwait(bar, par, abort_flag), 1)) return true;
                 raise_error(p, kErrWaitTimeout, abort_flag);
                 return false;
             };
@@ -447,7 +448,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc_fence_after();
                     const uint32_t a_lo = sdesc_lo(sbase + sp * Lay::kStageBytes + Lay::kKOff, kTile);
                     const uint32_t b_lo = sdesc_lo(wv, kTile);
-#pragma unroll
+#pragma unroll 1
                     for (int kk = 0; kk < kChunk / 16; ++kk)
                         mma_bf16_ss(tmem + col_dz(b), sdesc_from_lo(a_lo + mnmaj_step(kk)),
                                     sdesc_from_lo(b_lo + mnmaj_step(kk)), ID_DZ, kk > 0 ? 1u : 0u);
@@ -470,7 +471,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t st = sbase + s * Lay::kStageBytes;
                     const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
                     const uint32_t k_lo = sdesc_lo(st + Lay::kKOff, 16);
-#pragma unroll
+#pragma unroll 1
                     for (int kk = 0; kk < 4; ++kk)
                         mma_bf16_ss(tmem + col_sc(sb), sdesc_from_lo(q_lo + kmaj_step(kk)),
                                     sdesc_from_lo(k_lo + kmaj_step(kk)), ID_SC, kk > 0 ? 1u : 0u);
@@ -490,7 +491,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t n = 0, c2 = 0, ucnt = 0;
             bool ok = true;
             auto wait_or_fail = [&](uint64_t* bar, uint32_t par) -> bool {
-                if (bwait(bar, par, abort_flag)) return true;
+                if (__builtin_expect(bwait(bar, par, abort_flag), 1)) return true;
                 raise_error(p, kErrWaitTimeout, abort_flag);
                 return false;
             };
@@ -513,27 +514,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t st = sbase + s * Lay::kStageBytes;
                     // O = Q B0^T
                     const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
-#pragma unroll
+#pragma unroll 1
                     for (int kk = 0; kk < 4; ++kk)
                         mma_bf16_ss(tmem + col_o(ob), sdesc_from_lo(q_lo + kmaj_step(kk)),
                                     sdesc_from_lo(b0_lo + mnmaj_step(kk)), ID_O, kk > 0 ? 1u : 0u);
+                    if (!(ok = wait_or_fail(&st_ready[ob], oph))) break;
                     if (!(ok = wait_or_fail(&p_ready[ob], oph))) break;
                     tc_fence_after();
-                    // O += P' V  (P' over the score buffer: tokens s < 64 in columns 0..31,
-                    // s >= 64 in columns 64..95)
+                    // O += P' V + Q' S^T: A from the score buffer (P' for tokens s < 64 in
+                    // columns 0..31, s >= 64 in 64..95; Q' in 32..63), B = V then S^T
                     const uint32_t v_lo = sdesc_lo(st + Lay::kVOff, kTile);
-#pragma unroll
-                    for (int kk = 0; kk < kChunk / 16; ++kk)
-                        mma_bf16_ts(tmem + col_o(ob), tmem + col_sc(ob) + (kk < 4 ? kk * 8 : 64 + (kk - 4) * 8),
-                                    sdesc_from_lo(v_lo + mnmaj_step(kk)), ID_O, 1u);
-                    // O += Q' S^T  (A = a_t q_t from TMEM columns 32..63 of the score buffer)
-                    if (!(ok = wait_or_fail(&st_ready[ob], oph))) break;
-                    tc_fence_after();
                     const uint32_t s_lo = sdesc_lo(sbase + Lay::kStOff + ob * kStTile, kTile);
-#pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
-                        mma_bf16_ts(tmem + col_o(ob), tmem + col_sc(ob) + kQpCol + kk * 8,
-                                    sdesc_from_lo(s_lo + mnmaj_step(kk)), ID_O, 1u);
+#pragma unroll 1
+                    for (int kk = 0; kk < kChunk / 16 + 4; ++kk) {
+                        const uint32_t acol = kk < 4 ? kk * 8 : (kk < 8 ? 64 + (kk - 4) * 8 : kQpCol + (kk - 8) * 8);
+                        const uint32_t blo = kk < 8 ? v_lo + mnmaj_step(kk) : s_lo + mnmaj_step(kk - 8);
+                        mma_bf16_ts(tmem + col_o(ob), tmem + col_sc(ob) + acol, sdesc_from_lo(blo), ID_O, 1u);
+                    }
                     mma_commit(&st_free[ob]);
                     mma_commit(&o_full[ob]);
                     mma_commit(&sc_free[ob]);
@@ -683,22 +680,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_after();
                 const uint32_t base = tmem + col_sc(sb) + lane_off;
                 const float pim_t = gb[kGbPim + row];
+                // ---- P'_ts = -E_ts (q_t . k_s): warps 2-5 for s < 64, the helpers for
+                // s >= 64 (rows 64..127)
+                build_p64(helper ? base + 64 : base, gb, row, pim_t, helper ? 8 : 0);
                 if (!helper) {
-                    // ---- P'_ts = -E_ts (q_t . k_s) for s < 64
-                    if (q4 >= 2) {
-                        build_p64<0, true>(base, gb, row, pim_t);
-                    } else {
-                        build_p64<0, false>(base, gb, row, pim_t);
-                        tmem_zero32_async(base + 64);  // tokens >= 64 all masked
-                    }
+                    if (q4 < 2) tmem_zero32_async(base + 64);  // tokens >= 64 all masked
                     // the score columns 0..63 are read: the epilogue warps of the same
                     // lanes may write Q' into columns 32..63
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&sr_done[sb]);
-                } else {
-                    // ---- P'_ts for s >= 64 (rows 64..127)
-                    build_p64<8, false>(base + 64, gb, row, pim_t);
                 }
                 tmem_wait_st();
                 tc_fence_before();
