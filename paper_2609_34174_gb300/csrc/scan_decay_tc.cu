@@ -23,28 +23,30 @@
 // from the start of t's piece up to t) and the piece products tp_j, so that for s in
 // an earlier piece than t, E_ts = (eta_s sig_s) * pim_t * prod_{js<i<jt} tp_i.
 //
-// All three terms of o land in one TMEM accumulator:
-//   O  = Q B0^T                 (B0^T tile in shared memory, per unit)
-//   O += P' V                   P'_ts = -E_ts (q_t . k_s), built over the score
-//   O += Q' S^T                 Q' = diag(a) Q, written by the epilogue warps into the
-//                               free columns of the score buffer (TS product)
-// and the state update is dZ = K^T (W V), with the rows of V scaled by -w_s into a
-// shared-memory tile, then S' = a_end S + dZ in the state warps (fp32 rows).
+// The read lands in one 128-column TMEM accumulator X:
+//   X  = Q [B0^T | S^T]         one N = 128 product: B0^T (per unit) and the chunk's
+//                               S^T are the two 64-wide halves of the B operand
+//   X[:, 0:64] += P' V          P'_ts = -E_ts (q_t . k_s), built over the score
+// and the epilogue forms o_t = X_t[0:64] + a_t X_t[64:128] in fp32.  The state
+// update is dZ = K^T (W V), with the rows of V scaled by -w_s into a shared-memory
+// tile, then S' = a_end S + dZ in the state warps (fp32 rows).  TMEM holds two chunk
+// buffers (score, then P' and dZ in its columns) and two X accumulators, so the
+// issuer works on chunk c + 1 while the epilogue drains chunk c.
 //
 // Warp roles (16 warps), with the rings and bounded waits of the chunk kernel of
 // scan_tc.cu:
 //   warp 0      TMA producer (stage = [q | k | v], or [qk | v] forward)
-//   warp 1      front MMA issuer: the score Q K^T of chunk c, then the state update
-//               dZ of chunk c - 1 (one chunk behind, so that the score never waits
-//               for the W V tile)
-//   warp 14     back MMA issuer: Q B0^T, then (S^T and P' ready) P' V and Q' S^T
+//   warp 1      front MMA issuer: the score Q K^T of chunk c + 1, then (P' of chunk
+//               c built, so its score columns are free) dZ of chunk c into them
+//   warp 14     back MMA issuer: X of chunk c, then (P' ready) P' V
+//               (each group's K steps back to back on one accumulator)
 //   warp 15     gate factors of each chunk from alpha_t and eta_t, in registers and
 //               shuffles, into a ring of three blocks one or two chunks ahead
 //   warps 2-5   P' over score columns 0..63 (rows 0..63 also zero 64..127)
 //   warps 10-11 P' over columns 64..127 of rows 64..127
-//   (warps 2-3 and 10-11 then write the chunk's W V rows, 0..63 and 64..127)
-//   warps 6-9   Q' of the next chunk into the score columns the P warps have read,
-//               then the epilogue (TMEM -> bf16 staging -> TMA store) as in scan_tc.cu
+//   (warps 4-5 and 10-11, whose P' rows are the shorter ones, then write the chunk's
+//   W V rows 0..63 and 64..127)
+//   warps 6-9   the epilogue (TMEM -> o_t -> bf16 staging -> TMA store)
 //   warps 12-13 state rows, B0^T and S^T tiles, S' = a_end S + dZ
 // One work item is one unit (the chunks of a unit run in order in one CTA).
 #include <cuda.h>
@@ -64,10 +66,12 @@ constexpr int kWarpO0 = 6, kWarpZ0 = 10, kWarpBack = 14, kWarpGate = 15;
 constexpr int kRing = 4;
 constexpr int kItemConsumers = 2 + 4 + 4 + 2 + 2 + 1;
 constexpr uint32_t kTmemCols = 512;
+// TMEM columns: two chunk buffers of 128 (the fp32 score; then P' packed in columns
+// 0..31 (tokens s < 64) and 96..127 (s >= 64), and the state update dZ of the same
+// chunk in columns 32..95) and two X accumulators of 128.
 __host__ __device__ constexpr uint32_t col_sc(uint32_t i) { return i * 128u; }
-__host__ __device__ constexpr uint32_t col_o(uint32_t i) { return 256u + i * 64u; }
-__host__ __device__ constexpr uint32_t col_dz(uint32_t i) { return 384u + i * 64u; }
-constexpr uint32_t kQpCol = 32;  // Q' in columns 32..63 of the score buffer
+constexpr uint32_t kDzCol = 32, kPhiCol = 96;
+__host__ __device__ constexpr uint32_t col_x(uint32_t i) { return 256u + i * 128u; }
 
 // Gate block of one chunk (floats), written by the gate warp: per token alpha, eta,
 // -eta_s sig_s, pim_t, a_t and w_t; the products between pieces
@@ -84,20 +88,21 @@ struct DLayout {
     static constexpr int kKOff = COSTATE ? kTile : 0;
     static constexpr int kVOff = COSTATE ? 2 * kTile : kTile;
     static constexpr int kStageBytes = (COSTATE ? 3 : 2) * kTile;
-    // fixed regions: the output staging tile, two S^T tiles, the B0^T tile, the W V
-    // tile, the ring of gate blocks, barriers
+    // fixed regions: the output staging tile, the B0^T tile followed by the two S^T
+    // tiles (the N = 128 operand [B0^T | S^T] of buffer i has its halves
+    // (i + 1) * kStTile apart), the W V tile, the ring of gate blocks, barriers
     static constexpr int kFixed = kTile + 2 * kStTile + kStTile + kTile + kGbRing * kGbBytes;
     static constexpr int kAvail = 232448 - kFixed - 1024 - 1024;
     static constexpr int kStages0 = kAvail / kStageBytes;
     static constexpr int kStages = kStages0 > 6 ? 6 : kStages0;
     static constexpr int kOOff = kStages * kStageBytes;
-    static constexpr int kStOff = kOOff + kTile;
-    static constexpr int kB0Off = kStOff + 2 * kStTile;
-    static constexpr int kWvOff = kB0Off + kStTile;
+    static constexpr int kB0Off = kOOff + kTile;
+    static constexpr int kStOff = kB0Off + kStTile;
+    static constexpr int kWvOff = kStOff + 2 * kStTile;
     static constexpr int kGfOff = kWvOff + kTile;
     static constexpr int kBarOff = kGfOff + kGbRing * kGbBytes;
     static constexpr int kSmemBytes = kBarOff + 1024 + 1024;
-    static_assert(kStages >= 3, "the lagged state update holds two stages");
+    static_assert(kStages >= 3, "a chunk and the next chunk's score hold two stages");
     static_assert(kSmemBytes <= 232448, "shared memory budget exceeded");
     static_assert(kGfOff % 32 == 0 && kBarOff % 8 == 0, "alignment");
 };
@@ -219,33 +224,60 @@ __device__ __forceinline__ void same_piece_decays(const float* gb, int row, floa
     }
 }
 
-// Store 4 consecutive 32-bit columns of this thread's TMEM lane without waiting.
-__device__ __forceinline__ void tmem_st4_async(uint32_t taddr, uint32_t a, uint32_t b, uint32_t c,
-                                               uint32_t d) {
-    asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr), "r"(a),
-                 "r"(b), "r"(c), "r"(d)
-                 : "memory");
+// Two 32-column loads of this thread's TMEM lane (32x32b shape, as tmem_ld32) with
+// one wait: columns ta .. ta+31 into a, tb .. tb+31 into b.
+__device__ __forceinline__ void tmem_ld32_pair(uint32_t ta, uint32_t tb, float (&a)[32], float (&b)[32]) {
+    uint32_t r[64];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%64];\n\t"
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, "
+        "%48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%65];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]),
+          "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]),
+          "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]),
+          "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]),
+          "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]),
+          "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+        : "r"(ta), "r"(tb)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+        a[i] = __uint_as_float(r[i]);
+        b[i] = __uint_as_float(r[32 + i]);
+    }
 }
 
-// P'_ts = -E_ts (q_t . k_s) over the 64 score columns of pieces PB .. PB+7 of this
-// lane's row: the fp32 scores at TMEM columns taddr .. taddr+63 become 32 packed bf16
-// columns at taddr (stores issued, not waited).  Two pieces per step, in increasing
-// order, so that no packed store reaches a score column still to be read.
-// One copy of the code serves every P warp (pb = 0 or 8).
-__device__ __forceinline__ void build_p64(uint32_t taddr, const float* gb, int row, float pim, int pb) {
+// P'_ts = -E_ts (q_t . k_s) over the 64 score columns of pieces pb .. pb+7 of this
+// lane's row: the fp32 scores at TMEM columns rd .. rd+63 become 32 packed bf16
+// columns at wr (stores issued, not waited), two pieces per step.  Pieces 0..7
+// (wr = rd) go in increasing order, pieces 8..15 (wr = rd + 32) in decreasing
+// order, so that no packed store reaches a score column still to be read.  One copy
+// of the code serves every P warp.
+__device__ __forceinline__ void build_p64(uint32_t rd, uint32_t wr, const float* gb, int row, float pim,
+                                          int pb) {
     const int jt = row >> 3;
     const int jmax = (row | 31) >> 3;  // the last piece of this warp's rows
     float ndd[8];
     same_piece_decays(gb, row, ndd);
 #pragma unroll 1
-    for (int m = 0; m < 4; ++m) {
+    for (int mi = 0; mi < 4; ++mi) {
+        const int m = pb == 0 ? mi : 3 - mi;
         if (pb + 2 * m > jmax) {  // after every row of the warp: masked
             const uint32_t z[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-            tmem_st8_async(taddr + 8 * m, z);
+            tmem_st8_async(wr + 8 * m, z);
             continue;
         }
         float v[16];
-        tmem_ld16(taddr + 16 * m, v);
+        tmem_ld16(rd + 16 * m, v);
         uint32_t w[8];
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
@@ -262,7 +294,7 @@ __device__ __forceinline__ void build_p64(uint32_t taddr, const float* gb, int r
             for (int i = 0; i < 4; ++i)
                 w[4 * h + i] = pack_bf16x2(e[2 * i] * v[8 * h + 2 * i], e[2 * i + 1] * v[8 * h + 2 * i + 1]);
         }
-        tmem_st8_async(taddr + 8 * m, w);
+        tmem_st8_async(wr + 8 * m, w);
     }
 }
 
@@ -282,19 +314,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* empty = bars + 8;            // [NS] stage read by both MMA issuers
     uint64_t* sc_full = bars + 16;         // [2] score in TMEM
     uint64_t* sc_free = bars + 18;         // [2] score/P' buffer reusable
-    uint64_t* o_full = bars + 20;          // [2]
-    uint64_t* o_free = bars + 22;          // [2]
-    uint64_t* dz_full = bars + 24;         // [2]
-    uint64_t* dz_free = bars + 26;         // [2]
+    uint64_t* o_full = bars + 20;          // [2] X of the chunk complete
+    uint64_t* o_free = bars + 22;          // [2] X read by the epilogue
+    uint64_t* dz_full = bars + 24;         // [2] dZ of the chunk in its buffer (or none)
+    uint64_t* dz_free = bars + 26;         // [2] dZ read by the state warps
     uint64_t* st_ready = bars + 28;        // [2]
     uint64_t* st_free = bars + 30;         // [2]
     uint64_t* gf_full = bars + 32;         // [3] gate block of a chunk written
     uint64_t* gf_free = bars + 35;         // [3] gate block read by every user
-    uint64_t* p_ready = bars + 38;         // [2] P' (and Q') in TMEM
+    uint64_t* p_ready = bars + 38;         // [2] P' in TMEM
     uint64_t* b0_ready = bars + 40;        // B0^T tile of the current unit written
     uint64_t* b0_free = bars + 41;         // B0^T tile no longer read
-    uint64_t* drain = bars + 42;
-    uint64_t* drain2 = bars + 43;
+    uint64_t* drain = bars + 42;           // [2]
     uint64_t* o_staged = bars + 44;        // [2]
     uint64_t* o_buf_free = bars + 46;      // the staging tile read by its store
     uint64_t* wv_ready = bars + 47;        // the W V tile written
@@ -305,7 +336,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     volatile int* abort_flag = misc + 0;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(misc + 1);
     volatile int* item_slot = misc + 4;    // [kRing]
-    uint64_t* sr_done = bars + 61;         // [2] P warps done reading score columns 0..63
     float* gfb = reinterpret_cast<float*>(smem + Lay::kGfOff);  // [kGbRing][kGbFloats]
 
     const int warp = threadIdx.x >> 5;
@@ -314,13 +344,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < NS; ++i) {
             mbar_init(&full[i], 1);
-            mbar_init(&empty[i], AGG ? 1 : 2);  // both MMA issuers (the front one alone in AGG)
+            mbar_init(&empty[i], AGG ? 1 : 2);  // both issuers (the front one alone in AGG)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&sc_full[i], 1);
             mbar_init(&sc_free[i], 1);
-            mbar_init(&p_ready[i], 10);  // warps 2-5, the two helpers, the four epilogue warps (Q')
-            mbar_init(&sr_done[i], 4);   // warps 2-5
+            mbar_init(&p_ready[i], 6);  // warps 2-5 and the two helpers
             mbar_init(&o_staged[i], 4);
             mbar_init(&o_full[i], 1);
             mbar_init(&o_free[i], 4);
@@ -338,13 +367,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             // warps 2-5, the helpers, the state warps and (outputs only) the epilogue
             mbar_init(&gf_free[i], AGG ? 4 + 2 + 2 : 4 + 2 + 2 + 4);
         }
-        mbar_init(wv_ready, 4);  // warps 2-3 and the two helpers
+        mbar_init(wv_ready, 4);  // warps 4-5 and the two helpers
         mbar_init(wv_free, 1);
         mbar_init(o_buf_free, 1);
         mbar_init(b0_ready, 2);
         mbar_init(b0_free, 1);
-        mbar_init(drain, 1);
-        mbar_init(drain2, 1);
+        mbar_init(drain, 1);  // [2] one per issuer
+        mbar_init(drain + 1, 1);
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -418,18 +447,59 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
-    } else if (warp == 1) {
-        // ------------------------------------------------- front MMA issuer
+    } else if (warp == 1 || warp == kWarpBack) {
+        // ------------------------------------------- MMA issuers: warp 1 the score
+        // of chunk c + 1 and dZ of chunk c, warp 14 X and P' V of chunk c
+        const bool front = warp == 1;
         if (lane == 0) {
             constexpr uint32_t ID_SC = idesc_bf16(128, 128, false, false);  // Q K^T
             constexpr uint32_t ID_DZ = idesc_bf16(128, 64, true, true);     // K^T (W V)
+            constexpr uint32_t ID_X = idesc_bf16(128, 128, false, true);    // Q [B0^T | S^T]
+            constexpr uint32_t ID_PV = idesc_bf16(128, 64, false, true);    // P' V
             const uint32_t wv = sbase + Lay::kWvOff;
-            uint32_t n = 0, c2 = 0, dzc = 0;
+            uint32_t n = 0, c2 = 0, dzc = 0, ucnt = 0;
             bool ok = true;
             auto wait_or_fail = [&](uint64_t* bar, uint32_t par) -> bool {
                 if (__builtin_expect(bwait(bar, par, abort_flag), 1)) return true;
                 raise_error(p, kErrWaitTimeout, abort_flag);
                 return false;
+            };
+            // dZ = K^T (W V) of the chunk in stage sp (chunk counter cc) into columns
+            // 32..95 of its buffer, which its P warps have read: A = K^T (MN-major,
+            // 64-wide M blocks 16 KB apart; the second block's rows land in TMEM lanes
+            // 64..127, unread)
+            auto issue_dz = [&](int sp, uint32_t cc) -> bool {
+                if (!wait_or_fail(wv_ready, dzc & 1)) return false;
+                tc_fence_after();
+                const uint32_t a_lo = sdesc_lo(sbase + sp * Lay::kStageBytes + Lay::kKOff, kTile);
+                const uint32_t b_lo = sdesc_lo(wv, kTile);
+#pragma unroll 1
+                for (int kk = 0; kk < kChunk / 16; ++kk)
+                    mma_bf16_ss(tmem + col_sc(cc & 1) + kDzCol, sdesc_from_lo(a_lo + mnmaj_step(kk)),
+                                sdesc_from_lo(b_lo + mnmaj_step(kk)), ID_DZ, kk > 0 ? 1u : 0u);
+                mma_commit(&dz_full[cc & 1]);
+                mma_commit(wv_free);
+                ++dzc;
+                return true;
+            };
+            // the score Q K^T of the chunk with stage counter nn and chunk counter cc,
+            // once its buffer's previous chunk is done (P' V read, dZ taken)
+            auto issue_score = [&](uint32_t nn, uint32_t cc) -> bool {
+                const int s = static_cast<int>(nn % NS);
+                const uint32_t sb = cc & 1;
+                if (!wait_or_fail(&full[s], (nn / NS) & 1)) return false;
+                if (!wait_or_fail(&sc_free[sb], ((cc >> 1) & 1) ^ 1)) return false;
+                if (!wait_or_fail(&dz_free[sb], ((cc >> 1) & 1) ^ 1)) return false;
+                tc_fence_after();
+                const uint32_t st = sbase + s * Lay::kStageBytes;
+                const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
+                const uint32_t k_lo = sdesc_lo(st + Lay::kKOff, 16);
+#pragma unroll 1
+                for (int kk = 0; kk < 4; ++kk)
+                    mma_bf16_ss(tmem + col_sc(sb), sdesc_from_lo(q_lo + kmaj_step(kk)),
+                                sdesc_from_lo(k_lo + kmaj_step(kk)), ID_SC, kk > 0 ? 1u : 0u);
+                mma_commit(&sc_full[sb]);
+                return true;
             };
             for (int it = 0; ok; ++it) {
                 const int slot = it % kRing;
@@ -438,110 +508,73 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_arrive(&item_empty[slot]);
                 if (item < 0) break;
                 const Item I = decode_unit(item, p);
-                // dZ = K^T (W V) of the chunk in stage sp: A = K^T (MN-major, 64-wide M
-                // blocks 16 KB apart; the second block's rows land in TMEM lanes 64..127,
-                // unread)
-                auto issue_dz = [&](int sp) -> bool {
-                    const uint32_t b = dzc & 1;
-                    if (!wait_or_fail(&dz_free[b], ((dzc >> 1) & 1) ^ 1)) return false;
-                    if (!wait_or_fail(wv_ready, dzc & 1)) return false;
-                    tc_fence_after();
-                    const uint32_t a_lo = sdesc_lo(sbase + sp * Lay::kStageBytes + Lay::kKOff, kTile);
-                    const uint32_t b_lo = sdesc_lo(wv, kTile);
-#pragma unroll 1
-                    for (int kk = 0; kk < kChunk / 16; ++kk)
-                        mma_bf16_ss(tmem + col_dz(b), sdesc_from_lo(a_lo + mnmaj_step(kk)),
-                                    sdesc_from_lo(b_lo + mnmaj_step(kk)), ID_DZ, kk > 0 ? 1u : 0u);
-                    mma_commit(&dz_full[b]);
-                    mma_commit(wv_free);
-                    mma_commit(&empty[sp]);
-                    ++dzc;
-                    return true;
-                };
-                for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
-                    const int s = n % NS;
-                    const uint32_t sb = c2 & 1;
-                    if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
-                    if (AGG) {  // the segment's aggregate: the state update of every chunk
-                        if (!(ok = issue_dz(s))) break;
-                        continue;
+                if (AGG) {  // the segment's aggregate: the state update of every chunk
+                    if (!front) continue;
+                    for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
+                        const int s = n % NS;
+                        if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
+                        if (!(ok = wait_or_fail(&dz_free[c2 & 1], ((c2 >> 1) & 1) ^ 1))) break;
+                        if (!(ok = issue_dz(s, c2))) break;
+                        mma_commit(&empty[s]);
                     }
-                    if (!(ok = wait_or_fail(&sc_free[sb], ((c2 >> 1) & 1) ^ 1))) break;
-                    tc_fence_after();
-                    const uint32_t st = sbase + s * Lay::kStageBytes;
-                    const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
-                    const uint32_t k_lo = sdesc_lo(st + Lay::kKOff, 16);
-#pragma unroll 1
-                    for (int kk = 0; kk < 4; ++kk)
-                        mma_bf16_ss(tmem + col_sc(sb), sdesc_from_lo(q_lo + kmaj_step(kk)),
-                                    sdesc_from_lo(k_lo + kmaj_step(kk)), ID_SC, kk > 0 ? 1u : 0u);
-                    mma_commit(&sc_full[sb]);
-                    // the previous chunk's state update, one chunk behind its score
-                    if (c > 0 && !(ok = issue_dz(static_cast<int>((n - 1) % NS)))) break;
-                    if (c == I.nch - 1) mma_commit(&empty[s]);  // no state update reads it
+                    continue;
                 }
-            }
-            mma_commit(drain);
-            mbar_drain(drain, 0);
-        }
-    } else if (warp == kWarpBack) {
-        // -------------------------------------------------- back MMA issuer
-        if (lane == 0) {
-            constexpr uint32_t ID_O = idesc_bf16(128, 64, false, true);  // [Q|P'|Q'] x [B0^T|V|S^T]
-            uint32_t n = 0, c2 = 0, ucnt = 0;
-            bool ok = true;
-            auto wait_or_fail = [&](uint64_t* bar, uint32_t par) -> bool {
-                if (__builtin_expect(bwait(bar, par, abort_flag), 1)) return true;
-                raise_error(p, kErrWaitTimeout, abort_flag);
-                return false;
-            };
-            const uint32_t b0_lo = sdesc_lo(sbase + Lay::kB0Off, kTile);
-            for (int it = 0; ok; ++it) {
-                const int slot = it % kRing;
-                if (!wait_or_fail(&item_full[slot], (it / kRing) & 1)) break;
-                const int item = item_slot[slot];
-                mbar_arrive(&item_empty[slot]);
-                if (item < 0) break;
-                if (AGG) continue;  // no outputs in the aggregate pass
-                const Item I = decode_unit(item, p);
+                if (front) {
+                    if (!(ok = issue_score(n, c2))) break;
+                    for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
+                        const int s = n % NS;
+                        const uint32_t sb = c2 & 1, ph = (c2 >> 1) & 1;
+                        // the next chunk's score, then this chunk's state update (an
+                        // item's last chunk has none: its barrier completes empty)
+                        if (c + 1 < I.nch && !(ok = issue_score(n + 1, c2 + 1))) break;
+                        if (!(ok = wait_or_fail(&p_ready[sb], ph))) break;
+                        if (c + 1 < I.nch) {
+                            if (!(ok = issue_dz(s, c2))) break;
+                        } else {
+                            mma_commit(&dz_full[sb]);
+                        }
+                        mma_commit(&empty[s]);
+                    }
+                    continue;
+                }
                 if (!(ok = wait_or_fail(b0_ready, ucnt & 1))) break;
                 for (int c = 0; c < I.nch; ++c, ++n, ++c2) {
                     const int s = n % NS;
-                    const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
-                    if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
-                    if (!(ok = wait_or_fail(&o_free[ob], oph ^ 1))) break;
-                    tc_fence_after();
+                    const uint32_t sb = c2 & 1, ph = (c2 >> 1) & 1;
                     const uint32_t st = sbase + s * Lay::kStageBytes;
-                    // O = Q B0^T
+                    if (!(ok = wait_or_fail(&full[s], (n / NS) & 1))) break;
+                    // X = Q [B0^T | S^T]: an MN-major B whose two 64-wide N blocks are
+                    // the B0^T tile and this chunk's S^T tile, (sb + 1) * kStTile apart
+                    if (!(ok = wait_or_fail(&o_free[sb], ph ^ 1))) break;
+                    if (!(ok = wait_or_fail(&st_ready[sb], ph))) break;
+                    tc_fence_after();
                     const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
+                    const uint32_t b_lo = sdesc_lo(sbase + Lay::kB0Off, kStTile * (sb + 1));
 #pragma unroll 1
                     for (int kk = 0; kk < 4; ++kk)
-                        mma_bf16_ss(tmem + col_o(ob), sdesc_from_lo(q_lo + kmaj_step(kk)),
-                                    sdesc_from_lo(b0_lo + mnmaj_step(kk)), ID_O, kk > 0 ? 1u : 0u);
-                    if (!(ok = wait_or_fail(&st_ready[ob], oph))) break;
-                    if (!(ok = wait_or_fail(&p_ready[ob], oph))) break;
+                        mma_bf16_ss(tmem + col_x(sb), sdesc_from_lo(q_lo + kmaj_step(kk)),
+                                    sdesc_from_lo(b_lo + mnmaj_step(kk)), ID_X, kk > 0 ? 1u : 0u);
+                    mma_commit(&st_free[sb]);
+                    // X[:, 0:64] += P' V  (P' in the chunk buffer: tokens s < 64 in
+                    // columns 0..31, s >= 64 in columns 96..127)
+                    if (!(ok = wait_or_fail(&p_ready[sb], ph))) break;
                     tc_fence_after();
-                    // O += P' V + Q' S^T: A from the score buffer (P' for tokens s < 64 in
-                    // columns 0..31, s >= 64 in 64..95; Q' in 32..63), B = V then S^T
                     const uint32_t v_lo = sdesc_lo(st + Lay::kVOff, kTile);
-                    const uint32_t s_lo = sdesc_lo(sbase + Lay::kStOff + ob * kStTile, kTile);
 #pragma unroll 1
-                    for (int kk = 0; kk < kChunk / 16 + 4; ++kk) {
-                        const uint32_t acol = kk < 4 ? kk * 8 : (kk < 8 ? 64 + (kk - 4) * 8 : kQpCol + (kk - 8) * 8);
-                        const uint32_t blo = kk < 8 ? v_lo + mnmaj_step(kk) : s_lo + mnmaj_step(kk - 8);
-                        mma_bf16_ts(tmem + col_o(ob), tmem + col_sc(ob) + acol, sdesc_from_lo(blo), ID_O, 1u);
-                    }
-                    mma_commit(&st_free[ob]);
-                    mma_commit(&o_full[ob]);
-                    mma_commit(&sc_free[ob]);
+                    for (int kk = 0; kk < kChunk / 16; ++kk)
+                        mma_bf16_ts(tmem + col_x(sb),
+                                    tmem + col_sc(sb) + (kk < 4 ? kk * 8 : kPhiCol + (kk - 4) * 8),
+                                    sdesc_from_lo(v_lo + mnmaj_step(kk)), ID_PV, 1u);
+                    mma_commit(&o_full[sb]);
+                    mma_commit(&sc_free[sb]);
                     mma_commit(&empty[s]);
                 }
                 if (!ok) break;
                 mma_commit(b0_free);  // every product of this unit that reads B0^T issued
                 ++ucnt;
             }
-            mma_commit(drain2);
-            mbar_drain(drain2, 0);
+            mma_commit(front ? drain : drain + 1);
+            mbar_drain(front ? drain : drain + 1, 0);
         }
     } else if (warp == kWarpGate) {
         // ------------------------------------------------------- gate factors
@@ -645,18 +678,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp < kWarpO0 || warp == kWarpZ0 || warp == kWarpZ0 + 1) {
         // ---------------------------------------------------- P' and the W V rows
         // Warps 2-5 own token rows row = 32 (warp & 3) + lane of each chunk: P' over
-        // columns 0..63 (rows < 64 also zero columns 64..127); the epilogue warps then
-        // write Q' = a_t q_t into columns 32..63.  The
-        // two helpers build P' over columns 64..127 of rows 64..127.  Then warps 2-3
-        // (whose P' has no masked column) and the helpers write the chunk's W V rows
-        // -w_t v_t (rows 0..63 and 64..127), which the front issuer's state update
-        // reads one chunk later.
+        // columns 0..63 (rows < 64 also zero columns 64..127).  The two helpers build
+        // P' over columns 64..127 of rows 64..127.  Then warps 4-5 (whose P' rows are
+        // half masked) and the helpers write the chunk's W V rows -w_t v_t (rows
+        // 0..63 and 64..127), which the state update dZ of the same chunk reads.
         const bool helper = warp >= kWarpZ0;
         const int q4 = warp & 3;
         const int row = q4 * 32 + lane;
         const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
-        const bool wv_writer = helper || q4 >= 2;
-        const int wv_row = helper ? row : row - 64;
+        const bool wv_writer = helper || q4 < 2;  // W V row wv_row = row
+        const int wv_row = row;
         uint32_t c2 = 0, wvn = 0;
         bool ok = true;
         for (int it = 0; ok; ++it) {
@@ -682,15 +713,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const float pim_t = gb[kGbPim + row];
                 // ---- P'_ts = -E_ts (q_t . k_s): warps 2-5 for s < 64, the helpers for
                 // s >= 64 (rows 64..127)
-                build_p64(helper ? base + 64 : base, gb, row, pim_t, helper ? 8 : 0);
-                if (!helper) {
-                    if (q4 < 2) tmem_zero32_async(base + 64);  // tokens >= 64 all masked
-                    // the score columns 0..63 are read: the epilogue warps of the same
-                    // lanes may write Q' into columns 32..63
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&sr_done[sb]);
-                }
+                build_p64(helper ? base + 64 : base, helper ? base + kPhiCol : base, gb, row, pim_t,
+                          helper ? 8 : 0);
+                if (!helper && q4 < 2) tmem_zero32_async(base + kPhiCol);  // tokens >= 64 all masked
                 tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
@@ -742,62 +767,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         const EpiParams& e = p.epi;
         uint32_t c2 = 0;
         bool ok = true;
-        // Q' = a_t q_t of the chunk with CTA chunk counter cc into columns 32..63 of its
-        // score buffer, once the P warps of these lanes have read them
-        auto write_qp = [&](uint32_t cc) -> bool {
-            const uint32_t qb = cc & 1, gk = cc % kGbRing;
-            const int s = static_cast<int>(cc % NS);
-            if (!warp_wait(&gf_full[gk], (cc / kGbRing) & 1, abort_flag) ||
-                !warp_wait(&full[s], (cc / NS) & 1, abort_flag) ||
-                !warp_wait(&sr_done[qb], (cc >> 1) & 1, abort_flag))
-                return false;
-            tc_fence_after();
-            const float a_t = gfb[gk * kGbFloats + kGbA + row];
-            const uint32_t qt = sbase + s * Lay::kStageBytes + Lay::kQOff;
-            const uint32_t dst = tmem + col_sc(qb) + lane_off + kQpCol;
-#pragma unroll 1
-            for (int q = 0; q < 8; ++q) {
-                const uint4 a = ld_shared_v4(qt + sw128_off(row, q));
-                const __nv_bfloat162* hq = reinterpret_cast<const __nv_bfloat162*>(&a);
-                uint32_t o[4];
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const float2 f = __bfloat1622float2(hq[i]);
-                    o[i] = pack_bf16x2(a_t * f.x, a_t * f.y);
-                }
-                tmem_st4_async(dst + 4 * q, o[0], o[1], o[2], o[3]);
-            }
-            tmem_wait_st();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(&p_ready[qb]);
-                mbar_arrive(&gf_free[gk]);
-            }
-            return true;
-        };
         for (int it = 0; ok; ++it) {
             int item;
             if (!take_item(it, item) || item < 0) break;
             if (AGG) continue;  // no outputs in the aggregate pass
             const Item I = decode_unit(item, p);
-            if (!write_qp(c2)) {  // the item's first chunk
-                raise_error(p, kErrWaitTimeout, abort_flag);
-                break;
-            }
             for (int c = 0; c < I.nch; ++c, ++c2) {
-                if (c + 1 < I.nch && !write_qp(c2 + 1)) {  // the next chunk's Q' before this output
-                    raise_error(p, kErrWaitTimeout, abort_flag);
-                    ok = false;
-                    break;
-                }
                 const uint32_t ob = c2 & 1, oph = (c2 >> 1) & 1;
-                if (!warp_wait(&o_full[ob], oph, abort_flag)) {
+                const uint32_t gk = c2 % kGbRing;
+                if (!warp_wait(&o_full[ob], oph, abort_flag) ||
+                    !warp_wait(&gf_full[gk], (c2 / kGbRing) & 1, abort_flag)) {
                     raise_error(p, kErrWaitTimeout, abort_flag);
                     ok = false;
                     break;
                 }
                 tc_fence_after();
+                // o_t = X_t[0:64] + a_t X_t[64:128]
+                const float a_t = gfb[gk * kGbFloats + kGbA + row];
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&gf_free[gk]);
+                const uint32_t xt = tmem + col_x(ob) + lane_off;
                 const int t0 = I.t_begin + c * kChunk;
                 const int t = t0 + row;
                 const bool valid = t < p.T;
@@ -810,12 +799,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                         break;
                     }
 #pragma unroll 1
-                    for (int m = 0; m < 4; ++m) {
-                        float u[16];
-                        tmem_ld16(tmem + col_o(ob) + lane_off + 16 * m, u);
+                    for (int m = 0; m < 2; ++m) {  // 32 output columns per TMEM round trip
+                        float u[32], z[32];
+                        tmem_ld32_pair(xt + 32 * m, xt + 64 + 32 * m, u, z);
 #pragma unroll
-                        for (int h = 0; h < 2; ++h)
-                            st_shared_v4(otile + sw128_off(row, 2 * m + h), pack_bf16x2(u[8 * h], u[8 * h + 1]),
+                        for (int i = 0; i < 32; ++i) u[i] = fmaf(a_t, z[i], u[i]);
+#pragma unroll
+                        for (int h = 0; h < 4; ++h)
+                            st_shared_v4(otile + sw128_off(row, 4 * m + h), pack_bf16x2(u[8 * h], u[8 * h + 1]),
                                          pack_bf16x2(u[8 * h + 2], u[8 * h + 3]),
                                          pack_bf16x2(u[8 * h + 4], u[8 * h + 5]),
                                          pack_bf16x2(u[8 * h + 6], u[8 * h + 7]));
@@ -825,7 +816,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (lane == 0) mbar_arrive(&o_free[ob]);
                 } else {
                 float v[64];
-                tmem_ld64(tmem + col_o(ob) + lane_off, v);
+                tmem_ld64(xt, v);
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    float z[32];
+                    tmem_ld32(xt + 64 + 32 * h, z);
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[32 * h + i] = fmaf(a_t, z[i], v[32 * h + i]);
+                }
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&o_free[ob]);
@@ -888,7 +886,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int q4 = warp & 3;
         const int row = q4 * 32 + lane;
         const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
-        uint32_t c2 = 0, dzc = 0, ucnt = 0;
+        uint32_t c2 = 0, ucnt = 0;
         float st[64];
         bool ok = true;
         auto put_row = [&](uint32_t tile) {
@@ -901,22 +899,25 @@ __global__ void __launch_bounds__(kThreads, 1)
             fence_proxy_async_smem();
             __syncwarp();
         };
-        // S' = a_end S + dZ with the next product from TMEM
-        auto advance = [&](float a_end) -> bool {
-            const uint32_t b = dzc & 1;
-            if (!warp_wait(&dz_full[b], (dzc >> 1) & 1, abort_flag)) return false;
-            tc_fence_after();
-            float a[32];
+        // S' = a_end S + dZ with the chunk's product from its TMEM buffer (chunk
+        // counter cc); an item's last chunk has no product (use = false) but its
+        // barriers still turn
+        auto advance = [&](uint32_t cc, float a_end, bool use) -> bool {
+            const uint32_t b = cc & 1;
+            if (!warp_wait(&dz_full[b], (cc >> 1) & 1, abort_flag)) return false;
+            if (use) {
+                tc_fence_after();
+                float a[32];
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                tmem_ld32(tmem + col_dz(b) + lane_off + h * 32, a);
+                for (int h = 0; h < 2; ++h) {
+                    tmem_ld32(tmem + col_sc(b) + kDzCol + lane_off + h * 32, a);
 #pragma unroll
-                for (int i = 0; i < 32; ++i) st[h * 32 + i] = fmaf(a_end, st[h * 32 + i], a[i]);
+                    for (int i = 0; i < 32; ++i) st[h * 32 + i] = fmaf(a_end, st[h * 32 + i], a[i]);
+                }
+                tc_fence_before();
             }
-            tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&dz_free[b]);
-            ++dzc;
             return true;
         };
         for (int it = 0; ok; ++it) {
@@ -934,7 +935,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         break;
                     }
                     const float a_end = gfb[gk * kGbFloats + kGbEnd];
-                    if (!advance(a_end)) {
+                    if (!advance(c2, a_end, true)) {
                         ok = false;
                         break;
                     }
@@ -1005,7 +1006,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 const float a_end = gfb[gk * kGbFloats + kGbEnd];
-                if (c < I.nch - 1 && !advance(a_end)) {
+                if (!advance(c2, a_end, c < I.nch - 1)) {
                     raise_error(p, kErrWaitTimeout, abort_flag);
                     ok = false;
                     break;
