@@ -35,10 +35,10 @@
 //
 // Warp roles (16 warps), with the rings and bounded waits of the chunk kernel of
 // scan_tc.cu:
-//   warp 0      TMA producer (stage = [q | k | v], or [qk | v] forward)
+//   warp 14     TMA producer (stage = [q | k | v], or [qk | v] forward)
 //   warp 1      front MMA issuer: the score Q K^T of chunk c + 1, then (P' of chunk
 //               c built, so its score columns are free) dZ of chunk c into them
-//   warp 14     back MMA issuer: X of chunk c, then (P' ready) P' V
+//   warp 0      back MMA issuer: X of chunk c, then (P' ready) P' V
 //               (each group's K steps back to back on one accumulator)
 //   warp 15     gate factors of each chunk from alpha_t and eta_t, in registers and
 //               shuffles, into a ring of three blocks one or two chunks ahead
@@ -62,7 +62,11 @@ constexpr int kTile = 16384;   // [128 rows][64 bf16], 128-byte swizzle
 constexpr int kStTile = 8192;  // [64 rows][64 bf16]
 constexpr int kWarps = 16;
 constexpr int kThreads = kWarps * 32;
-constexpr int kWarpO0 = 6, kWarpZ0 = 10, kWarpBack = 14, kWarpGate = 15;
+// Both MMA issuers sit on sub-partitions 0 and 1 (warp % 4), whose P warps build the
+// half-masked rows: a warp issuing ALU work every cycle on an issuer's sub-partition
+// slows its MMAs by 1.7x, one on another sub-partition not at all.  The TMA producer
+// issues a few instructions a chunk and takes sub-partition 2.
+constexpr int kWarpO0 = 6, kWarpZ0 = 10, kWarpBack = 0, kWarpProd = 14, kWarpGate = 15;
 constexpr int kRing = 4;
 constexpr int kItemConsumers = 2 + 4 + 4 + 2 + 2 + 1;
 constexpr uint32_t kTmemCols = 512;
@@ -382,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_relinquish();
         tc_fence_before();
     }
-    if (warp == 0 && lane == 0) {
+    if (warp == kWarpProd && lane == 0) {
         prefetch_tmap(&tm_q);
         prefetch_tmap(&tm_k);
         prefetch_tmap(&tm_v);
@@ -405,7 +409,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         return true;
     };
 
-    if (warp == 0) {
+    if (warp == kWarpProd) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
             uint32_t n = 0;
@@ -449,7 +453,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp == 1 || warp == kWarpBack) {
         // ------------------------------------------- MMA issuers: warp 1 the score
-        // of chunk c + 1 and dZ of chunk c, warp 14 X and P' V of chunk c
+        // of chunk c + 1 and dZ of chunk c, warp 0 X and P' V of chunk c
         const bool front = warp == 1;
         if (lane == 0) {
             constexpr uint32_t ID_SC = idesc_bf16(128, 128, false, false);  // Q K^T
