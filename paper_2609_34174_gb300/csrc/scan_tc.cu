@@ -21,10 +21,10 @@
 // taken and successors in other CTAs rarely wait in their look-back.
 //
 // Warp roles (15 warps, one CTA per SM):
-//   warp 0      TMA producer: tickets, item queue, chunk tiles into a stage ring
+//   warp 14     TMA producer: tickets, item queue, chunk tiles into a stage ring
 //   warp 1      TMEM allocator; its lane 0 issues the "front" MMAs of every chunk
 //               (score Q K^T and state increment K^T V), up to two chunks ahead
-//   warp 14     lane 0 issues the "back" MMAs (O = Q S^T, then O += P V); the two
+//   warp 0      lane 0 issues the "back" MMAs (O = Q S^T, then O += P V); the two
 //               issuers run independent in-order loops, so the output product of
 //               chunk c never waits behind the score of chunk c+1
 //   warps 2-5   score -> P: TMEM score tile, causal mask, bf16 P written back over
@@ -57,7 +57,9 @@ constexpr int kTile = 16384;  // one [128 rows][64 bf16] 128B-swizzled tile
 constexpr int kWarps = 15;
 constexpr int kThreads = kWarps * 32;
 constexpr int kWarpO0 = 6, kWarpZ0 = 10;  // score->P warps are 2..5
-constexpr int kWarpBack = 14;             // back-MMA issuer
+// The back issuer sits on sub-partition 0 (warp % 4), with the forward read's
+// half-masked P rows; the producer, a few instructions a chunk, on sub-partition 2.
+constexpr int kWarpBack = 0, kWarpProd = 14;  // back-MMA issuer, TMA producer
 constexpr int kItemConsumers = 2 + 4 + 4 + 4;  // two MMA issuers + lane 0 of every other role warp
 constexpr int kRing = 4;                        // item queue depth
 
@@ -344,7 +346,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_relinquish();
         tc_fence_before();
     }
-    if (warp == 0 && lane == 0) {
+    if (warp == kWarpProd && lane == 0) {
         prefetch_tmap(&tm_q);
         prefetch_tmap(&tm_k);
         prefetch_tmap(&tm_v);
@@ -355,7 +357,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 0) {
+    if (warp == kWarpProd) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
             uint32_t n = 0, an = 0;
