@@ -241,3 +241,39 @@ def test_retention_full_size_c4_every_unit():
     yr, gr = _oracle(inputs, eta, alpha, wl)
     _check("c4 retention forward", y, yr, TOL["bf16"])
     _check("c4 retention costate", gin, gr, TOL["bf16"])
+
+
+def test_retention_many_items_per_cta_odd_chunks():
+    """More units than SMs, each of three chunks (257 tokens, the last ragged): every
+    CTA runs several items whose chunk counts are odd, so the two chunk buffers
+    (score, then P' and the state update) and the two output accumulators, with their
+    barrier phases, alternate from one item to the next."""
+    wl = W.workload("c5").resized(L=1, B=4, H=100, T=257)
+    inputs = W.make_linear(wl)
+    eta, alpha = _chunk_gates((wl.L, wl.B, wl.T, wl.H), wl.T, 4001)
+    dev = {k: (v.cuda() if isinstance(v, torch.Tensor) else v) for k, v in inputs.items()}
+    y = gl.forward_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), alpha=alpha.cuda())
+    gin = gl.costate_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), dev["g_out"],
+                          alpha=alpha.cuda())
+    torch.cuda.synchronize()
+    yr, gr = _oracle(inputs, eta, alpha, wl)
+    _check("400 units x 3 chunks forward", y, yr, TOL["bf16"])
+    _check("400 units x 3 chunks costate", gin, gr, TOL["bf16"])
+
+
+def test_retention_segmented_many_items():
+    """Segmented units with more items than SMs: 100 units of 1300 tokens cut into
+    512 + 512 + 276 (four, four and three chunks), 300 items, so the aggregate pass
+    and the scan each run several items of mixed chunk counts per CTA."""
+    wl = W.workload("c4").resized(B=4, H=25, T=1300)
+    inputs = W.make_linear(wl)
+    eta, alpha = _chunk_gates((wl.L, wl.B, wl.T, wl.H), wl.T, 4002,
+                              resets=(511, 512, 1023, 1024, 1299))
+    dev = {k: (v.cuda() if isinstance(v, torch.Tensor) else v) for k, v in inputs.items()}
+    y = gl.forward_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), alpha=alpha.cuda())
+    gin = gl.costate_scan(dev["x"], dev["g_hat"], dev["W0"], eta.cuda(), dev["g_out"],
+                          alpha=alpha.cuda())
+    torch.cuda.synchronize()
+    yr, gr = _oracle(inputs, eta, alpha, wl)
+    _check("segmented 100 x 1300 forward", y, yr, TOL["bf16"])
+    _check("segmented 100 x 1300 costate", gin, gr, TOL["bf16"])
