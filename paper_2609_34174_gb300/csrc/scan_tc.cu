@@ -164,8 +164,9 @@ __device__ __noinline__ void epi_store_row(const EpiParams& e, long long o_off, 
     }
 }
 
-__device__ __forceinline__ void raise_error(const TcScanParams& p, unsigned int bits,
-                                            volatile int* abort_flag) {
+// Out of line: cold code inside the role loops spreads their instruction fetch.
+__device__ __noinline__ void raise_error(const TcScanParams& p, unsigned int bits,
+                                         volatile int* abort_flag) {
     atomicOr(p.ctrl + 1, bits);
     if (abort_flag) *abort_flag = 1;
 }
@@ -254,6 +255,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     using Lay = TcLayout<DQ, COSTATE, REV, FUSED>;
     static_assert(!FUSED || (DQ == 64 && !COSTATE && !REV), "the fused pass is built for 64-wide maps");
     constexpr int kJobs = FUSED ? 2 : 1;  // reads per chunk
+    // The suffix read and the fused pass carry more code (the per-row dot, two reads'
+    // epilogues): their MMA K steps stay rolled loops, which eases instruction fetch
+    // (c5: suffix read with dot 1.24 -> 1.10 ms, fused 1.29 -> 1.26 ms); the plain
+    // causal reads measured faster fully unrolled.
+    constexpr int kMmaUnroll = (REV || FUSED) ? 1 : 8;
     constexpr int NS = Lay::kStages;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -452,7 +458,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t n = 0, c2 = 0, dzc = 0;
             bool ok = true;
             auto wait_or_fail = [&](uint64_t* bar, uint32_t par) -> bool {
-                if (mbar_wait(bar, par, abort_flag)) return true;
+                if (__builtin_expect(mbar_wait(bar, par, abort_flag), 1)) return true;
                 raise_error(p, kErrWaitTimeout, abort_flag);
                 return false;
             };
@@ -463,7 +469,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // REV: A starts one block before k, so K^T lands in lanes 64..127
                 const uint32_t a_lo = sdesc_lo(st + (REV ? Lay::kKOff - kTile : Lay::kKOff), kTile);
                 const uint32_t b_lo = sdesc_lo(st + Lay::kVOff, kTile);
-#pragma unroll
+#pragma unroll kMmaUnroll
                 for (int kk = 0; kk < kChunk / 16; ++kk)
                     mma_bf16_ss(tmem + dcol, sdesc_from_lo(a_lo + mnmaj_step(kk)),
                                 sdesc_from_lo(b_lo + mnmaj_step(kk)), ID_DZ,
@@ -513,7 +519,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t st = sbase + s * Lay::kStageBytes;
                         const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
                         const uint32_t k_lo = sdesc_lo(st + Lay::kKOff, 16);
-#pragma unroll
+#pragma unroll kMmaUnroll
                         for (int kk = 0; kk < DQ / 16; ++kk)
                             mma_bf16_ss(tmem + col_sc(sb), sdesc_from_lo(q_lo + kmaj_step(kk)),
                                         sdesc_from_lo(k_lo + kmaj_step(kk)), ID_SC, kk > 0 ? 1u : 0u);
@@ -526,7 +532,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             tc_fence_after();
                             const uint32_t g_lo = sdesc_lo(st + Lay::kGOff, 16);
                             const uint32_t h_lo = sdesc_lo(st + Lay::kVOff, 16);
-#pragma unroll
+#pragma unroll kMmaUnroll
                             for (int kk = 0; kk < DQ / 16; ++kk)
                                 mma_bf16_ss(tmem + col_sc(sb2), sdesc_from_lo(g_lo + kmaj_step(kk)),
                                             sdesc_from_lo(h_lo + kmaj_step(kk)), ID_SC, kk > 0 ? 1u : 0u);
@@ -557,7 +563,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t n = 0, c2 = 0, p1c = 0;
             bool ok = true;
             auto wait_or_fail = [&](uint64_t* bar, uint32_t par) -> bool {
-                if (mbar_wait(bar, par, abort_flag)) return true;
+                if (__builtin_expect(mbar_wait(bar, par, abort_flag), 1)) return true;
                 raise_error(p, kErrWaitTimeout, abort_flag);
                 return false;
             };
@@ -610,7 +616,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (dir == 0) {
                                 const uint32_t x_lo = sdesc_lo(st + Lay::kQOff, 16);
                                 const uint32_t s_mn = sdesc_lo(tile, kTile);
-#pragma unroll
+#pragma unroll kMmaUnroll
                                 for (int kk = 0; kk < DQ / 16; ++kk)
                                     mma_bf16_ss(tmem + col_o(0), sdesc_from_lo(x_lo + kmaj_step(kk)),
                                                 sdesc_from_lo(s_mn + mnmaj_step(kk)), ID_O,
@@ -618,7 +624,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             } else {
                                 const uint32_t g_lo = sdesc_lo(st + Lay::kGOff, 16);
                                 const uint32_t s_k = sdesc_lo(tile, 16);
-#pragma unroll
+#pragma unroll kMmaUnroll
                                 for (int kk = 0; kk < DQ / 16; ++kk)
                                     mma_bf16_ss(tmem + col_o(1), sdesc_from_lo(g_lo + kmaj_step(kk)),
                                                 sdesc_from_lo(s_k + kmaj_step(kk)), ID_OK,
@@ -629,7 +635,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             tc_fence_after();
                             // forward: V = ghat; costate: V = x (both MN-major [128 t][64])
                             const uint32_t v_lo = sdesc_lo(st + (dir == 0 ? Lay::kVOff : Lay::kQOff), kTile);
-#pragma unroll
+#pragma unroll kMmaUnroll
                             for (int kk = 0; kk < kChunk / 16; ++kk)
                                 mma_bf16_ts(tmem + col_o(dir),
                                             tmem + col_sc(dir) + (kk < 4 ? kk * 8 : 64 + (kk - 4) * 8),
@@ -653,7 +659,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         // O = Q S^T  (B = S^T tile [dq][64]: MN-major)
                         const uint32_t q_lo = sdesc_lo(st + Lay::kQOff, 16);
                         const uint32_t s_lo = sdesc_lo(sbase + Lay::kStOff + ob * Lay::kStBytes, kTile);
-#pragma unroll
+#pragma unroll kMmaUnroll
                         for (int kk = 0; kk < DQ / 16; ++kk)
                             mma_bf16_ss(tmem + col_o(ob), sdesc_from_lo(q_lo + kmaj_step(kk)),
                                         sdesc_from_lo(s_lo + mnmaj_step(kk)), ID_O, kk > 0 ? 1u : 0u);
@@ -663,7 +669,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         // O += P V  (A = P in TMEM over the score buffer: tokens s < 64 in
                         // columns 0..31, s >= 64 in columns 64..95; B = V [128 t][64]: MN-major)
                         const uint32_t v_lo = sdesc_lo(st + Lay::kVOff, kTile);
-#pragma unroll
+#pragma unroll kMmaUnroll
                         for (int kk = 0; kk < kChunk / 16; ++kk)
                             mma_bf16_ts(tmem + col_o(ob),
                                         tmem + col_sc(ob) + (kk < 4 ? kk * 8 : 64 + (kk - 4) * 8),
