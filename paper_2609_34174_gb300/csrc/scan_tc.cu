@@ -20,13 +20,14 @@
 // its previous item, so an aggregate is published right after its ticket is
 // taken and successors in other CTAs rarely wait in their look-back.
 //
-// Warp roles (15 warps, one CTA per SM):
-//   warp 14     TMA producer: tickets, item queue, chunk tiles into a stage ring
-//   warp 1      TMEM allocator; its lane 0 issues the "front" MMAs of every chunk
-//               (score Q K^T and state increment K^T V), up to two chunks ahead
-//   warp 0      lane 0 issues the "back" MMAs (O = Q S^T, then O += P V); the two
-//               issuers run independent in-order loops, so the output product of
-//               chunk c never waits behind the score of chunk c+1
+// Warp roles (15 warps, 16 for the suffix read, whose numbers are in brackets;
+// one CTA per SM):
+//   warp 14 [0]   TMA producer: tickets, item queue, chunk tiles into a stage ring
+//   warp 1 [14]   lane 0 issues the "front" MMAs of every chunk (score Q K^T and
+//                 state increment K^T V), up to two chunks ahead; warp 1 allocates TMEM
+//   warp 0 [15]   lane 0 issues the "back" MMAs (O = Q S^T, then O += P V); the two
+//                 issuers run independent in-order loops, so the output product of
+//                 chunk c never waits behind the score of chunk c+1
 //   warps 2-5   score -> P: TMEM score tile, causal mask, bf16 P written back over
 //               the same TMEM columns (the PV product reads its A operand from
 //               tensor memory, so P never touches shared memory).  P is left
@@ -57,9 +58,15 @@ constexpr int kTile = 16384;  // one [128 rows][64 bf16] 128B-swizzled tile
 constexpr int kWarps = 15;
 constexpr int kThreads = kWarps * 32;
 constexpr int kWarpO0 = 6, kWarpZ0 = 10;  // score->P warps are 2..5
-// The back issuer sits on sub-partition 0 (warp % 4), with the forward read's
-// half-masked P rows; the producer, a few instructions a chunk, on sub-partition 2.
-constexpr int kWarpBack = 0, kWarpProd = 14;  // back-MMA issuer, TMA producer
+// The MMA issuers sit on the SM sub-partitions (warp % 4) whose P warps build the
+// half-masked rows: 0 and 1 for the causal reads, 2 and 3 for the suffix read (REV),
+// which adds a 16th warp for its back issuer; warp 1 then only allocates tensor memory.
+// The producer, a few instructions a chunk, takes a sub-partition left over.  A warp
+// issuing ALU work every cycle on an issuer's sub-partition slows its MMAs.
+template <bool REV> struct Roles {
+    static constexpr int kProd = REV ? 0 : 14, kFront = REV ? 14 : 1, kBack = REV ? 15 : 0;
+    static constexpr int kThreads = (REV ? 16 : 15) * 32;
+};
 constexpr int kItemConsumers = 2 + 4 + 4 + 4;  // two MMA issuers + lane 0 of every other role warp
 constexpr int kRing = 4;                        // item queue depth
 
@@ -248,7 +255,7 @@ __host__ __device__ constexpr uint32_t mnmaj_step(int kk) { return (uint32_t)((k
 // 1, stored through tm_o2), one S'^T tile and one state update.  Maps: tm_q = x,
 // tm_k = ghat, tm_v = g_out.
 template <int DQ, bool COSTATE, bool REV, bool FUSED>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(Roles<REV>::kThreads, 1)
     tc_scan_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
                    const __grid_constant__ CUtensorMap tm_o2, const TcScanParams p) {
@@ -352,7 +359,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_relinquish();
         tc_fence_before();
     }
-    if (warp == kWarpProd && lane == 0) {
+    if (warp == Roles<REV>::kProd && lane == 0) {
         prefetch_tmap(&tm_q);
         prefetch_tmap(&tm_k);
         prefetch_tmap(&tm_v);
@@ -363,7 +370,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == kWarpProd) {
+    if (warp == Roles<REV>::kProd) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
             uint32_t n = 0, an = 0;
@@ -450,7 +457,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
-    } else if (warp == 1) {
+    } else if (warp == Roles<REV>::kFront) {
         // ------------------------------------------------- front MMA issuer
         if (lane == 0) {
             constexpr uint32_t ID_SC = idesc_bf16(128, 128, false, false);  // Q K^T
@@ -556,7 +563,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_commit(drain);
             mbar_drain(drain, 0);
         }
-    } else if (warp == kWarpBack) {
+    } else if (warp == Roles<REV>::kBack) {
         // -------------------------------------------------- back MMA issuer
         if (lane == 0) {
             constexpr uint32_t ID_O = idesc_bf16(128, 64, false, true);  // Q S^T, P V
@@ -685,6 +692,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_commit(drain2);
             mbar_drain(drain2, 0);
         }
+    } else if (REV && warp == 1) {
+        // the suffix read's issuers are warps 14 and 15: this warp only allocates TMEM
     } else if (warp < kWarpO0 ||
                (warp >= kWarpZ0 && (REV ? (warp & 3) < 2 : (warp & 3) >= kZActiveWarps))) {
         // ------------------------------------------------------ score -> P
@@ -1182,7 +1191,7 @@ static cudaError_t launch_one(const CUtensorMap& q, const CUtensorMap& k, const 
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          Lay::kSmemBytes);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kThreads, Lay::kSmemBytes, stream>>>(q, k, v, o, o2 ? *o2 : o, p);
+    kern<<<grid, Roles<REV>::kThreads, Lay::kSmemBytes, stream>>>(q, k, v, o, o2 ? *o2 : o, p);
     return cudaGetLastError();
 }
 
