@@ -809,8 +809,13 @@ __global__ void __launch_bounds__(Roles<REV>::kThreads, 1)
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&o_free[ob]);
+                // O = lam * (Q S'^T + L(Q K^T) V); a suffix read reduced to its per-row dot
+                // alone takes lam into the dot's scale instead
+                const bool dot_only = REV && e.dot_out && !e.zin && !e.out2 && e.out == nullptr;
+                if (!dot_only) {
 #pragma unroll
-                for (int i = 0; i < 64; ++i) v[i] *= p.lam;  // O = lam * (Q S'^T + L(Q K^T) V)
+                    for (int i = 0; i < 64; ++i) v[i] *= p.lam;
+                }
                 const int t0 = chunk_t0<REV>(I, c);
                 const int t = t0 + row;
                 const int col0 = I.j * 64;
@@ -878,9 +883,9 @@ __global__ void __launch_bounds__(Roles<REV>::kThreads, 1)
                         if (valid) {
                             float* dst = e.dot_out + (((long long)I.l * p.B + I.b) * p.T + t) * p.H + I.h;
                             if (p.n_tiles > 1)
-                                atomicAdd(dst, e.dot_scale * acc);
+                                atomicAdd(dst, (dot_only ? e.dot_scale * p.lam : e.dot_scale) * acc);
                             else
-                                *dst = e.dot_scale * acc;
+                                *dst = (dot_only ? e.dot_scale * p.lam : e.dot_scale) * acc;
                         }
                     }
                 }
