@@ -675,14 +675,10 @@ class GateGradsJob(GradsJob):
         self.ws = torch.empty(max(256, int(nb)), dtype=torch.uint8, device=device)
         self.in_keys = ("x", "g_hat", "g_out", "u", "w", "eta_t", "alpha_t")
         self.out_keys = ("dla_f", "deta_f", "dla_c", "deta_c")
-        # two retention scans with state dumps, their reversed input copies and one
-        # per-chunk kernel per read
-        units = wl.L * wl.B * wl.H
-        sms = torch.cuda.get_device_properties(device).multi_processor_count if str(device).startswith("cuda") else 152
-        seg = 2 if (units < 2 * sms and wl.T > 1024) else 0
-        self.launches_per_step = 2 * (2 + 2 + 2 * (1 + seg) + 1)
-        self.kernel = {"fwd": "decay_scan_kernel (state dumps) + gate_chunk_kernel, forward read",
-                       "costate": "decay_scan_kernel (state dumps) + gate_chunk_kernel, costate read"}
+        # per read: the chunk aggregates, the carried chunk states, the per-chunk expansion
+        self.launches_per_step = 2 * 3
+        self.kernel = {"fwd": "gate_agg_tc_kernel + gate_state_scan_kernel + gate_chunk_tc_kernel, forward read",
+                       "costate": "gate_agg_tc_kernel + gate_state_scan_kernel + gate_chunk_tc_kernel, costate read"}
 
     def _run(self, src, cut, ws):
         gl, o = self.gl, self.outs
