@@ -332,8 +332,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* drain = bars + 42;           // [2]
     uint64_t* o_staged = bars + 44;        // [2]
     uint64_t* o_buf_free = bars + 46;      // the staging tile read by its store
-    uint64_t* wv_ready = bars + 47;        // the W V tile written
-    uint64_t* wv_free = bars + 48;         // the W V tile read by the dZ product
+    uint64_t* wv_ready = bars + 61;        // [2] a W V tile written
+    uint64_t* wv_free = bars + 63;         // [2] a W V tile read by the dZ product
     uint64_t* item_full = bars + 49;       // [kRing]
     uint64_t* item_empty = bars + 53;      // [kRing]
     int* misc = reinterpret_cast<int*>(bars + 57);
@@ -344,6 +344,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
+    // The n-th W V tile: the aggregate pass, which stores no outputs, alternates it
+    // with the output staging tile, so that W V of chunk c + 1 is written while the
+    // state update of chunk c reads the other; the scan keeps one tile.
+    auto wv_buf = [](uint32_t n) -> uint32_t { return AGG ? (n & 1) : 0u; };
+    auto wv_par = [](uint32_t n) -> uint32_t { return AGG ? ((n >> 1) & 1) : (n & 1); };
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < NS; ++i) {
@@ -371,8 +376,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             // warps 2-5, the helpers, the state warps and (outputs only) the epilogue
             mbar_init(&gf_free[i], AGG ? 4 + 2 + 2 : 4 + 2 + 2 + 4);
         }
-        mbar_init(wv_ready, 4);  // warps 4-5 and the two helpers
-        mbar_init(wv_free, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&wv_ready[i], 4);  // warps 4-5 and the two helpers
+            mbar_init(&wv_free[i], 1);
+        }
         mbar_init(o_buf_free, 1);
         mbar_init(b0_ready, 2);
         mbar_init(b0_free, 1);
@@ -473,16 +480,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             // 64-wide M blocks 16 KB apart; the second block's rows land in TMEM lanes
             // 64..127, unread)
             auto issue_dz = [&](int sp, uint32_t cc) -> bool {
-                if (!wait_or_fail(wv_ready, dzc & 1)) return false;
+                const uint32_t wb = wv_buf(dzc);
+                if (!wait_or_fail(&wv_ready[wb], wv_par(dzc))) return false;
                 tc_fence_after();
                 const uint32_t a_lo = sdesc_lo(sbase + sp * Lay::kStageBytes + Lay::kKOff, kTile);
-                const uint32_t b_lo = sdesc_lo(wv, kTile);
+                const uint32_t b_lo = sdesc_lo(wb ? sbase + Lay::kOOff : wv, kTile);
 #pragma unroll 1
                 for (int kk = 0; kk < kChunk / 16; ++kk)
                     mma_bf16_ss(tmem + col_sc(cc & 1) + kDzCol, sdesc_from_lo(a_lo + mnmaj_step(kk)),
                                 sdesc_from_lo(b_lo + mnmaj_step(kk)), ID_DZ, kk > 0 ? 1u : 0u);
                 mma_commit(&dz_full[cc & 1]);
-                mma_commit(wv_free);
+                mma_commit(&wv_free[wb]);
                 ++dzc;
                 return true;
             };
@@ -728,14 +736,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (wv_writer && (AGG || c < I.nch - 1)) {
                     // ---- the chunk's W V row -w_t v_t (an item's last chunk needs none
                     // unless its state at the segment end is the aggregate)
-                    if (!warp_wait(wv_free, (wvn & 1) ^ 1, abort_flag)) {
+                    const uint32_t wb = wv_buf(wvn);
+                    if (!warp_wait(&wv_free[wb], wv_par(wvn) ^ 1, abort_flag)) {
                         raise_error(p, kErrWaitTimeout, abort_flag);
                         ok = false;
                         break;
                     }
                     const float w = -gb[kGbW + wv_row];
                     const uint32_t vt = st + Lay::kVOff;
-                    const uint32_t wvt = sbase + Lay::kWvOff;
+                    const uint32_t wvt = sbase + (wb ? Lay::kOOff : Lay::kWvOff);
 #pragma unroll 1
                     for (int q = 0; q < 8; q += 2) {
                         const uint4 a0 = ld_shared_v4(vt + sw128_off(wv_row, q));
@@ -755,7 +764,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     fence_proxy_async_smem();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(wv_ready);
+                    if (lane == 0) mbar_arrive(&wv_ready[wb]);
                     ++wvn;
                 }
                 __syncwarp();
