@@ -31,7 +31,7 @@
 // update is dZ = K^T (W V), with the rows of V scaled by -w_s into a shared-memory
 // tile, then S' = a_end S + dZ in the state warps (fp32 rows).  TMEM holds two chunk
 // buffers (score, then P' and dZ in its columns) and two X accumulators, so the
-// issuer works on chunk c + 1 while the epilogue drains chunk c.
+// issuers work on chunk c + 1 while the epilogue drains chunk c.
 //
 // Warp roles (16 warps), with the rings and bounded waits of the chunk kernel of
 // scan_tc.cu:
@@ -48,7 +48,9 @@
 //   W V rows 0..63 and 64..127)
 //   warps 6-9   the epilogue (TMEM -> o_t -> bf16 staging -> TMA store)
 //   warps 12-13 state rows, B0^T and S^T tiles, S' = a_end S + dZ
-// One work item is one unit (the chunks of a unit run in order in one CTA).
+// One work item is one unit, or one segment of a few long units (its chunks run in
+// order in one CTA; the segments' start states come from an aggregate pass and the
+// carry kernel below).
 #include <cuda.h>
 
 #include "scan_common.cuh"
