@@ -254,7 +254,7 @@ __host__ __device__ constexpr uint32_t mnmaj_step(int kk) { return (uint32_t)((k
 // read (score, P and O buffers 0, stored through tm_o) and the costate read (buffers
 // 1, stored through tm_o2), one S'^T tile and one state update.  Maps: tm_q = x,
 // tm_k = ghat, tm_v = g_out.
-template <int DQ, bool COSTATE, bool REV, bool FUSED>
+template <int DQ, bool COSTATE, bool REV, bool FUSED, bool DOT>
 __global__ void __launch_bounds__(Roles<REV>::kThreads, 1)
     tc_scan_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
@@ -267,6 +267,9 @@ __global__ void __launch_bounds__(Roles<REV>::kThreads, 1)
     // (c5: suffix read with dot 1.24 -> 1.10 ms, fused 1.29 -> 1.26 ms); the plain
     // causal reads measured faster fully unrolled.
     constexpr int kMmaUnroll = (REV || FUSED) ? 1 : 8;
+    // DOT: a suffix read reduced to its per-row dot alone (no rows stored, no
+    // activation): its epilogue compiles to the dot, with no staging or store code.
+    constexpr bool kDotOnly = REV && DOT;
     constexpr int NS = Lay::kStages;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -811,7 +814,7 @@ __global__ void __launch_bounds__(Roles<REV>::kThreads, 1)
                 if (lane == 0) mbar_arrive(&o_free[ob]);
                 // O = lam * (Q S'^T + L(Q K^T) V); a suffix read reduced to its per-row dot
                 // alone takes lam into the dot's scale instead
-                const bool dot_only = REV && e.dot_out && !e.zin && !e.out2 && e.out == nullptr;
+                constexpr bool dot_only = kDotOnly;
                 if (!dot_only) {
 #pragma unroll
                     for (int i = 0; i < 64; ++i) v[i] *= p.lam;
@@ -822,7 +825,7 @@ __global__ void __launch_bounds__(Roles<REV>::kThreads, 1)
                 const bool valid = REV ? (t >= I.t_begin && t < I.t_end) : t < I.t_end;
                 // The activation paths (MLP layers only) run out of line, so the hot
                 // loop of the plain scans stays small in the instruction cache.
-                if (e.zin && valid) {
+                if (!kDotOnly && e.zin && valid) {
                     float tmp[64];
 #pragma unroll
                     for (int i = 0; i < 64; ++i) tmp[i] = v[i];
@@ -830,7 +833,7 @@ __global__ void __launch_bounds__(Roles<REV>::kThreads, 1)
 #pragma unroll
                     for (int i = 0; i < 64; ++i) v[i] = tmp[i];
                 }
-                if (e.out2 && valid) {
+                if (!kDotOnly && e.out2 && valid) {
                     float tmp[64];
 #pragma unroll
                     for (int i = 0; i < 64; ++i) tmp[i] = v[i];
@@ -846,6 +849,44 @@ __global__ void __launch_bounds__(Roles<REV>::kThreads, 1)
                                         (((long long)I.l * p.B + I.b) * p.T + t) * p.H + I.h);
                     }
                 }
+                // (REV) dot_out[t] (+)= dot_scale * (row . a row) over this 64-wide tile.
+                // The tile of a (TMA, 128B-swizzled like an output tile) lets each lane
+                // read its own row without bank conflicts.
+                auto row_dot = [&]() -> bool {
+                    const uint32_t ak = ae % 3;
+                    if (!warp_wait(&a_full[ak], (ae / 3) & 1, abort_flag)) {
+                        raise_error(p, kErrWaitTimeout, abort_flag);
+                        return false;
+                    }
+                    const uint32_t atile = smem_u32(a_tile(ak));
+                    float acc = 0.f;
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) {
+                        const uint4 a4 = ld_shared_v4(atile + sw128_off(row, q));
+                        const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&a4);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) acc = fmaf(v[8 * q + i], __bfloat162float(hb[i]), acc);
+                    }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&a_empty[ak]);
+                    ++ae;
+                    if (valid) {
+                        float* dst = e.dot_out + (((long long)I.l * p.B + I.b) * p.T + t) * p.H + I.h;
+                        const float sc = dot_only ? e.dot_scale * p.lam : e.dot_scale;
+                        if (p.n_tiles > 1)
+                            atomicAdd(dst, sc * acc);
+                        else
+                            *dst = sc * acc;
+                    }
+                    return true;
+                };
+                if constexpr (kDotOnly) {
+                    if (!row_dot()) {
+                        ok = false;
+                        break;
+                    }
+                    continue;  // no rows staged or stored
+                }
                 // Stage the bf16 row in the 128B-swizzled output tile (the TMA store
                 // clips rows past the end of the sequence).
                 if (!warp_wait(&o_buf_free[ob], oph ^ 1, abort_flag)) {
@@ -858,35 +899,9 @@ __global__ void __launch_bounds__(Roles<REV>::kThreads, 1)
                 // suffix read reduced to a per-token dot stores no rows at all
                 const bool direct = REV && (t0 < 0 || e.out == nullptr);
                 if constexpr (REV) {
-                    if (e.dot_out) {
-                        // dot_out[t] (+)= dot_scale * (row . a row) over this 64-wide tile.
-                        // The tile of a (TMA, 128B-swizzled like an output tile) lets each
-                        // lane read its own row without bank conflicts.
-                        const uint32_t ak = ae % 3;
-                        if (!warp_wait(&a_full[ak], (ae / 3) & 1, abort_flag)) {
-                            raise_error(p, kErrWaitTimeout, abort_flag);
-                            ok = false;
-                            break;
-                        }
-                        const uint32_t atile = smem_u32(a_tile(ak));
-                        float acc = 0.f;
-#pragma unroll
-                        for (int q = 0; q < 8; ++q) {
-                            const uint4 a4 = ld_shared_v4(atile + sw128_off(row, q));
-                            const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&a4);
-#pragma unroll
-                            for (int i = 0; i < 8; ++i) acc = fmaf(v[8 * q + i], __bfloat162float(hb[i]), acc);
-                        }
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(&a_empty[ak]);
-                        ++ae;
-                        if (valid) {
-                            float* dst = e.dot_out + (((long long)I.l * p.B + I.b) * p.T + t) * p.H + I.h;
-                            if (p.n_tiles > 1)
-                                atomicAdd(dst, (dot_only ? e.dot_scale * p.lam : e.dot_scale) * acc);
-                            else
-                                *dst = (dot_only ? e.dot_scale * p.lam : e.dot_scale) * acc;
-                        }
+                    if (e.dot_out && !row_dot()) {
+                        ok = false;
+                        break;
                     }
                 }
                 if (direct) {
@@ -1187,12 +1202,12 @@ __global__ void __launch_bounds__(Roles<REV>::kThreads, 1)
 }
 
 // ------------------------------------------------------------------ host side
-template <int DQ, bool COSTATE, bool REV, bool FUSED = false>
+template <int DQ, bool COSTATE, bool REV, bool FUSED = false, bool DOT = false>
 static cudaError_t launch_one(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
                               const CUtensorMap& o, const TcScanParams& p, int grid,
                               cudaStream_t stream, const CUtensorMap* o2 = nullptr) {
     using Lay = TcLayout<DQ, COSTATE, REV, FUSED>;
-    auto kern = tc_scan_kernel<DQ, COSTATE, REV, FUSED>;
+    auto kern = tc_scan_kernel<DQ, COSTATE, REV, FUSED, DOT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          Lay::kSmemBytes);
     if (e != cudaSuccess) return e;
@@ -1226,6 +1241,10 @@ cudaError_t launch_tc_suffix(const CUtensorMap& q, const CUtensorMap& k, const C
                              const CUtensorMap& o, const TcScanParams& p, bool shared_qk, int grid,
                              cudaStream_t stream) {
     if (p.dq != 64) return cudaErrorInvalidValue;
+    const bool dot_only = p.epi.dot_out && !p.epi.out && !p.epi.zin && !p.epi.out2;
+    if (dot_only)
+        return shared_qk ? launch_one<64, false, true, false, true>(q, k, v, o, p, grid, stream)
+                         : launch_one<64, true, true, false, true>(q, k, v, o, p, grid, stream);
     return shared_qk ? launch_one<64, false, true>(q, k, v, o, p, grid, stream)
                      : launch_one<64, true, true>(q, k, v, o, p, grid, stream);
 }
