@@ -451,8 +451,8 @@ class GradsJob(LinearJob):
         self.ws = torch.empty(max(256, int(nb)), dtype=torch.uint8, device=device)
         self.in_keys = ("x", "g_hat", "g_out", "u", "w")
         self.out_keys = ("deta_f", "deta_c")
-        self.kernel = {"fwd": "tc_scan_kernel<64, false, REV> (suffix read, q = k = x, dot with ghat)",
-                       "costate": "tc_scan_kernel<64, true, REV> (suffix read, q = ghat, k = g_out, dot with x)"}
+        self.kernel = {"fwd": "tc_scan_kernel<64, false, REV, DOT> (suffix read, q = k = x, dot with ghat)",
+                       "costate": "tc_scan_kernel<64, true, REV, DOT> (suffix read, q = ghat, k = g_out, dot with x)"}
 
     def input_bytes(self):
         return _bytes(*(self.inp[k] for k in self.in_keys))
